@@ -1,0 +1,215 @@
+"""Pins of the oracle's AL codec against what the paper fixes.
+
+Sec. 4.1-4.2, Eq. (3)-(6). None of these tests re-derives the oracle's formula:
+they check the exact-zero invariant (Eq. (6)), the endpoint codes that Eq. (4)
+forces at z = 0 and z = 1, monotone codes, the half-log-step round trip that
+Eq. (5) implies, idempotence, the degenerate cases of Sec. 4.1, and a brute
+force at 4 bits (L = 16) where every code tuple is built and re-encoded.
+"""
+import itertools
+import math
+
+import numpy as np
+import pytest
+
+import oracle as ora
+from paper_2608_22322_gb300 import workloads as wl
+
+FLOOR = float(np.float32(math.log2(1e-16)))  # log2(eps^2) for eps = 1e-8
+
+
+def _blocks(x, block):
+    for lo in range(0, x.size, block):
+        yield lo, x[lo:lo + block]
+
+
+def _random_state(n, seed, zero_frac=0.1, spread=20.0):
+    """Positive log-uniform values over `spread` octaves with exact zeros."""
+    r = wl.rng(seed)
+    x = np.exp2(r.uniform(-30.0, -30.0 + spread, n)).astype(np.float32)
+    x[r.random(n) < zero_frac] = 0.0
+    return x
+
+
+@pytest.mark.parametrize("bits", [8, 16])
+@pytest.mark.parametrize("block", [32, 128, 256, 2048])
+def test_exact_zero_invariant(bits, block):
+    """Eq. (6): q = 0 exactly when x = 0, including all-zero blocks."""
+    n = 5 * block + 17  # ragged tail
+    x = _random_state(n, 1 + block + bits)
+    x[block:2 * block] = 0.0  # one all-zero block
+    x[3 * block + 5] = -0.0   # negative zero counts as zero
+    codes, meta = ora.al_encode(x, block, bits, FLOOR)
+    np.testing.assert_array_equal(codes == 0, x == 0)
+    assert meta[2] == 0 and meta[3] == 0  # all-zero block stores (0, 0)
+    xh = ora.al_decode(codes, meta, block, bits)
+    np.testing.assert_array_equal(xh == 0, x == 0)
+    assert np.all(xh[x > 0] > 0)
+
+
+def test_dormant_rows_stay_zero():
+    """A dormant state (all-zero rows) keeps only zero codes (Sec. 4.2)."""
+    x = _random_state(256 * 1024, 5).reshape(256, 1024)
+    x[[3, 100, 200]] = 0.0
+    codes, meta = ora.al_encode(x, 256, 8, FLOOR)
+    c = codes.reshape(256, 1024)
+    assert not c[[3, 100, 200]].any()
+
+
+@pytest.mark.parametrize("bits", [4, 8, 16])
+def test_endpoint_codes(bits):
+    """Eq. (4) at z = 0 and z = 1: min positive -> 1, max -> L-1."""
+    L = 1 << bits
+    for seed in range(40):
+        x = _random_state(256, 100 + seed, spread=float(wl.rng(seed).uniform(0.5, 60)))
+        if (x > 0).sum() < 2 or x[x > 0].min() == x.max():
+            continue
+        codes, meta = ora.al_encode(x, 256, bits, FLOOR)
+        pos = x > 0
+        assert codes[np.argmin(np.where(pos, x, np.inf))] == 1
+        assert codes[np.argmax(x)] == L - 1
+
+
+@pytest.mark.parametrize("bits", [8, 16])
+def test_monotone_codes(bits):
+    """Within a block, x <= y implies q(x) <= q(y)."""
+    x = _random_state(64 * 256, 7, spread=40.0)
+    codes, _ = ora.al_encode(x, 256, bits, FLOOR)
+    for lo, xb in _blocks(x, 256):
+        cb = codes[lo:lo + 256].astype(np.int64)
+        order = np.argsort(xb, kind="stable")
+        assert np.all(np.diff(cb[order]) >= 0)
+
+
+@pytest.mark.parametrize("bits", [8, 16])
+def test_round_trip_half_log_step(bits):
+    """Eq. (5): |log2 x_hat - log2 x| <= Delta / (2 (L-2)) inside the interval,
+    up to the fp32 rounding of l_min, Delta and x_hat."""
+    L = 1 << bits
+    x = _random_state(200 * 256, 11, spread=35.0)
+    codes, meta = ora.al_encode(x, 256, bits, FLOOR)
+    xh = ora.al_decode(codes, meta, 256, bits)
+    for b, (lo, xb) in enumerate(_blocks(x, 256)):
+        lmin, delta = float(meta[2 * b]), float(meta[2 * b + 1])
+        pos = xb > 0
+        if not pos.any():
+            continue
+        lx = np.log2(xb[pos].astype(np.float64))
+        lh = np.log2(xh[lo:lo + 256][pos].astype(np.float64))
+        slack = 4 * np.spacing(np.float32(abs(lmin) + delta)) + 2e-7
+        assert np.max(np.abs(lh - lx)) <= delta / (2 * (L - 2)) + slack
+
+
+def test_below_floor_and_constant_blocks():
+    """Sec. 4.1 degenerate cases: a block of equal values is widened by one
+    unit (all codes 1, decoded value ~ the constant); values below l_floor sit
+    on the floor level."""
+    c = np.float32(3.7e-5)
+    x = np.full(256, c, np.float32)
+    x[::3] = 0.0
+    codes, meta = ora.al_encode(x, 256, 8, FLOOR)
+    assert set(np.unique(codes)) == {0, 1}
+    assert meta[1] == 1.0
+    xh = ora.al_decode(codes, meta, 256, 8)
+    rel = abs(float(xh[1]) - float(c)) / float(c)
+    assert rel <= abs(math.log2(c)) * 2.0 ** -24 * math.log(2) * 2 + 2.0 ** -24
+    # every positive value below the floor -> code 1, decodes to 2^l_floor
+    y = np.array([0, 1e-20, 2e-19, 5e-18], np.float32)
+    codes, meta = ora.al_encode(y, 4, 8, FLOOR)
+    np.testing.assert_array_equal(codes, [0, 1, 1, 1])
+    assert meta[0] == np.float32(FLOOR) and meta[1] == 1.0
+    yh = ora.al_decode(codes, meta, 4, 8)
+    assert yh[1] == np.float32(2.0 ** float(np.float32(FLOOR)))
+
+
+def test_floor_clips_small_values_to_level_one():
+    """l_min = max(l_floor, log2 min): values below the floor share code 1 and
+    the interval starts at the floor (Eq. (3))."""
+    y = np.array([1e-30, 1e-20, 1e-10, 1e-3], np.float32)
+    codes, meta = ora.al_encode(y, 4, 8, FLOOR)
+    assert meta[0] == np.float32(FLOOR)
+    assert codes[0] == 1 and codes[1] == 1 and codes[3] == 255
+    assert 1 < codes[2] < 255
+
+
+def test_lmax_cap_126():
+    """Sec. 4.1: l_max is capped at 126."""
+    y = np.array([2.0 ** 120, 2.0 ** 127.5], np.float32)
+    _, meta = ora.al_encode(y, 2, 8, FLOOR)
+    assert float(meta[0]) == 120.0 and float(meta[0] + meta[1]) == 126.0
+
+
+@pytest.mark.parametrize("bits", [8, 16])
+def test_idempotent(bits):
+    """Encoding a decoded code with the same (l_min, Delta) returns it."""
+    L = 1 << bits
+    r = wl.rng(3)
+    for _ in range(20):
+        lmin = np.float32(r.uniform(-60, 10))
+        delta = np.float32(r.uniform(0.05, 60))
+        qs = range(1, L) if bits == 8 else r.integers(1, L, 3000)
+        for q in qs:
+            xh = ora.al_dequantize(int(q), lmin, delta, bits)
+            assert ora.al_quantize(xh, lmin, delta, bits) == q
+
+
+def test_brute_force_4bit_every_code_tuple():
+    """b = 4 (L = 16, 15 positive levels) on blocks of 4: build every code
+    tuple that contains both endpoint codes, place each value within a third
+    of a log step of its level, re-encode with fresh block bounds and recover
+    the tuple; also check the decoded value sits on its level."""
+    bits, L = 4, 16
+    lmin0, step = -20.0, 0.5  # levels 2^(-20 + 0.5 (q-1)), Delta = 7
+    r = wl.rng(4)
+    checked = 0
+    for tup in itertools.product(range(L), repeat=4):
+        if 1 not in tup or L - 1 not in tup:
+            continue
+        x = np.zeros(4, np.float32)
+        for i, q in enumerate(tup):
+            if q == 0:
+                continue
+            jit = 0.0 if q in (1, L - 1) else r.uniform(-step / 3, step / 3)
+            x[i] = np.float32(2.0 ** (lmin0 + step * (q - 1) + jit))
+        codes, meta = ora.al_encode(x, 4, bits, FLOOR)
+        assert tuple(int(c) for c in codes) == tup
+        assert meta[0] == np.float32(lmin0) and meta[1] == np.float32(7.0)
+        xh = ora.al_decode(codes, meta, 4, bits)
+        for q, v in zip(tup, xh):
+            want = 0.0 if q == 0 else np.float32(2.0 ** (lmin0 + step * (q - 1)))
+            assert v == want
+        checked += 1
+    assert checked == 16 ** 4 - 2 * 15 ** 4 + 14 ** 4  # tuples holding codes 1 and 15
+
+
+def test_brute_force_4bit_nearest_level():
+    """b = 4: for random blocks, each code is the nearest of the 15 log levels
+    (brute-force argmin, clipped to the interval)."""
+    bits, L = 4, 16
+    r = wl.rng(5)
+    for _ in range(3000):
+        x = np.exp2(r.uniform(-40, -20, 4)).astype(np.float32)
+        x[r.random(4) < 0.2] = 0.0
+        if not (x > 0).any():
+            continue
+        codes, meta = ora.al_encode(x, 4, bits, FLOOR)
+        lmin, delta = float(meta[0]), float(meta[1])
+        levels = lmin + np.arange(L - 1) * delta / (L - 2)
+        for v, q in zip(x, codes):
+            if v == 0:
+                assert q == 0
+                continue
+            d = np.abs(levels - math.log2(float(v)))
+            best = np.sort(d)
+            if best[1] - best[0] < 1e-9:
+                continue  # numerical tie
+            assert q == 1 + int(np.argmin(d))
+
+
+def test_ragged_tail_excludes_padding():
+    """Elements past n never enter a block statistic."""
+    x = _random_state(300, 9)
+    c1, m1 = ora.al_encode(x, 256, 8, FLOOR)
+    c2, m2 = ora.al_encode(x[256:], 256, 8, FLOOR)
+    np.testing.assert_array_equal(m1[2:], m2)
+    np.testing.assert_array_equal(c1[256:], c2)
