@@ -27,7 +27,7 @@
  *  - Quantization blocks are consecutive runs of `block` elements of one
  *    tensor; the last block of a tensor may be partial, and elements past the
  *    end never enter a block statistic. `block` must be a power of two in
- *    [32, 4096].
+ *    [128, 4096].
  *  - AL metadata is two fp32 values per block, interleaved:
  *    meta[2b] = l_min, meta[2b+1] = Delta (Sec. 4.1, "each block also stores
  *    l_min and Delta"). An all-zero block stores (0, 0) and all-zero codes.
@@ -89,7 +89,7 @@ int64_t al_state_bytes(int64_t n, int block, int bits);
  * paragraph of Sec. 4.1.
  *   x         [n] fp32, non-negative, finite (negative values are outside the
  *             contract and are not checked; -0.0 counts as zero).
- *   block     elements per block (power of two, 32..4096).
+ *   block     elements per block (power of two, 128..4096).
  *   bits      8 (AL8, L = 256, codes uint8_t) or 16 (AL16, L = 65536,
  *             codes uint16_t).
  *   log_floor l_floor of Eq. (3), the lower bound of l_min.

@@ -1,0 +1,239 @@
+"""ctypes binding of libalq.so (the C ABI of include/alq.h).
+
+Argument marshalling only: every function takes torch CUDA tensors, passes
+their device pointers, sizes and the current CUDA stream to the library entry
+point of the same name, and raises AlqError on a non-zero status. All the
+arithmetic runs in the library's kernels; there is no fallback. If the
+library has not been built (paper_2608_22322_gb300.build_lib.build()), loading
+this module raises.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import torch
+
+from . import build_lib
+
+_LIB_PATH = build_lib.LIB
+if not os.path.exists(_LIB_PATH):
+    raise ImportError(
+        f"CUDA library {_LIB_PATH} is missing: build it with "
+        "paper_2608_22322_gb300.build_lib.build() (or __graft_entry__.build())")
+lib = C.CDLL(_LIB_PATH)
+
+ALQ_OK = 0
+AL_OP_ADAFACTOR, AL_OP_CAME, AL_OP_APOLLO = 1, 2, 3
+
+
+class AlqError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        name = lib.alq_status_string(status).decode()
+        extra = lib.alq_last_cuda_error().decode()
+        super().__init__(f"{fn} failed: {name}" + (f" ({extra})" if extra else ""))
+        self.status = status
+
+
+class AdamWHP(C.Structure):
+    _fields_ = [(k, C.c_float) for k in
+                ("lr", "beta1", "beta2", "eps", "weight_decay", "log_floor")]
+
+
+class AdafactorHP(C.Structure):
+    _fields_ = [(k, C.c_float) for k in
+                ("lr", "eps1", "clip_d", "decay_rate", "beta1", "weight_decay",
+                 "log_floor")]
+
+
+class CameHP(C.Structure):
+    _fields_ = [(k, C.c_float) for k in
+                ("lr", "beta1", "beta2", "beta3", "eps1", "eps2", "clip_d",
+                 "weight_decay", "log_floor_v", "log_floor_c")]
+
+
+class ApolloHP(C.Structure):
+    _fields_ = ([(k, C.c_float) for k in
+                 ("lr", "beta1", "beta2", "eps", "alpha", "weight_decay",
+                  "norm_growth_gamma", "log_floor")] + [("rank", C.c_int32)])
+
+
+class AdamWTensor(C.Structure):
+    _fields_ = [("p", C.c_void_p), ("g", C.c_void_p), ("m_codes", C.c_void_p),
+                ("m_absmax", C.c_void_p), ("v_codes", C.c_void_p),
+                ("v_meta", C.c_void_p), ("n", C.c_int64)]
+
+
+class MultiInfo(C.Structure):
+    _fields_ = [("ntensors", C.c_int32), ("m_block", C.c_int32),
+                ("v_block", C.c_int32), ("v_bits", C.c_int32),
+                ("total_tiles", C.c_int64), ("total_elems", C.c_int64)]
+
+
+_vp, _i64, _int, _flt = C.c_void_p, C.c_int64, C.c_int, C.c_float
+
+
+def _sig(name, res, *args):
+    f = getattr(lib, name)
+    f.restype = res
+    f.argtypes = list(args)
+
+
+_sig("alq_status_string", C.c_char_p, _int)
+_sig("alq_last_cuda_error", C.c_char_p)
+_sig("alq_version", _int)
+_sig("al_num_blocks", _i64, _i64, _int)
+_sig("al_state_bytes", _i64, _i64, _int, _int)
+_sig("al_encode", _int, _vp, _i64, _int, _int, _flt, _vp, _vp, _vp)
+_sig("al_decode", _int, _vp, _vp, _i64, _int, _int, _vp, _vp)
+_sig("uf8_encode", _int, _vp, _i64, _int, _vp, _vp, _vp)
+_sig("uf8_decode", _int, _vp, _vp, _i64, _int, _vp, _vp)
+_sig("al_adamw_step", _int, _vp, _vp, _vp, _vp, _vp, _vp, _i64, _int, _int, _int,
+     C.POINTER(AdamWHP), _i64, _vp)
+_sig("al_adamw_plan_bytes", _int, _int, C.POINTER(C.c_size_t))
+_sig("al_adamw_plan", _int, C.POINTER(AdamWTensor), _int, _int, _int, _int, _vp,
+     C.c_size_t, C.POINTER(MultiInfo))
+_sig("al_adamw_step_multi", _int, _vp, C.POINTER(MultiInfo), C.POINTER(AdamWHP), _i64, _vp)
+_sig("al_workspace_size", _int, _int, _i64, _i64, _int, C.POINTER(C.c_size_t))
+_sig("al_adafactor_step", _int, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _vp, _int, _int,
+     _vp, _vp, _int, C.POINTER(AdafactorHP), _i64, _vp, C.c_size_t, _vp)
+_sig("al_came_step", _int, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _vp, _int, _int,
+     _vp, _vp, _vp, _vp, _int, _int, _vp, _vp, _int, C.POINTER(CameHP), _i64, _vp,
+     C.c_size_t, _vp)
+_sig("al_apollo_step", _int, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _int, _vp, _vp,
+     _int, _int, _vp, C.POINTER(ApolloHP), _i64, _vp, C.c_size_t, _vp)
+
+
+# ------------------------------------------------------------------ helpers --
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream=None):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _check(fn, st):
+    if st != ALQ_OK:
+        raise AlqError(fn, st)
+
+
+def _hp(cls, d):
+    return cls(**{k: d[k] for k, _ in cls._fields_})
+
+
+# ------------------------------------------------------------------- sizes --
+def version() -> int:
+    return lib.alq_version()
+
+
+def al_num_blocks(n: int, block: int) -> int:
+    return lib.al_num_blocks(n, block)
+
+
+def al_state_bytes(n: int, block: int, bits: int) -> int:
+    return lib.al_state_bytes(n, block, bits)
+
+
+def al_workspace_size(op: int, rows: int, cols: int, rank: int = 0) -> int:
+    b = C.c_size_t(0)
+    _check("al_workspace_size", lib.al_workspace_size(op, rows, cols, rank, C.byref(b)))
+    return b.value
+
+
+# ------------------------------------------------------------------- codec --
+def al_encode(x, block, bits, log_floor, codes, meta, stream=None):
+    _check("al_encode", lib.al_encode(_ptr(x), x.numel(), block, bits, log_floor,
+                                      _ptr(codes), _ptr(meta), _stream(stream)))
+
+
+def al_decode(codes, meta, block, bits, out, stream=None):
+    _check("al_decode", lib.al_decode(_ptr(codes), _ptr(meta), out.numel(), block, bits,
+                                      _ptr(out), _stream(stream)))
+
+
+def uf8_encode(m, block, codes, absmax, stream=None):
+    _check("uf8_encode", lib.uf8_encode(_ptr(m), m.numel(), block, _ptr(codes),
+                                        _ptr(absmax), _stream(stream)))
+
+
+def uf8_decode(codes, absmax, block, out, stream=None):
+    _check("uf8_decode", lib.uf8_decode(_ptr(codes), _ptr(absmax), out.numel(), block,
+                                        _ptr(out), _stream(stream)))
+
+
+# ------------------------------------------------------------------- AdamW --
+def al_adamw_step(p, g, m_codes, m_absmax, v_codes, v_meta, m_block, v_block, v_bits,
+                  hp: dict, t: int, stream=None):
+    h = _hp(AdamWHP, hp)
+    _check("al_adamw_step", lib.al_adamw_step(
+        _ptr(p), _ptr(g), _ptr(m_codes), _ptr(m_absmax), _ptr(v_codes), _ptr(v_meta),
+        p.numel(), m_block, v_block, v_bits, C.byref(h), t, _stream(stream)))
+
+
+class AdamWPlan:
+    """Device copy of a multi-tensor AdamW plan (al_adamw_plan) and its host
+    summary. `tensors` is a list of dicts with keys p, g, m_codes, m_absmax,
+    v_codes, v_meta (torch CUDA tensors)."""
+
+    def __init__(self, tensors, m_block, v_block, v_bits, device=None):
+        nt = len(tensors)
+        arr = (AdamWTensor * nt)()
+        for i, t in enumerate(tensors):
+            arr[i] = AdamWTensor(_ptr(t["p"]), _ptr(t["g"]), _ptr(t["m_codes"]),
+                                 _ptr(t["m_absmax"]), _ptr(t["v_codes"]),
+                                 _ptr(t["v_meta"]), t["p"].numel())
+        nbytes = C.c_size_t(0)
+        _check("al_adamw_plan_bytes", lib.al_adamw_plan_bytes(nt, C.byref(nbytes)))
+        host = torch.zeros(nbytes.value, dtype=torch.uint8)
+        self.info = MultiInfo()
+        _check("al_adamw_plan", lib.al_adamw_plan(arr, nt, m_block, v_block, v_bits,
+                                                  host.data_ptr(), nbytes.value,
+                                                  C.byref(self.info)))
+        dev = device if device is not None else tensors[0]["p"].device
+        self.dev = host.to(dev)
+        self.tensors = tensors  # keep the arrays alive while the plan is used
+
+    def step(self, hp: dict, t: int, stream=None):
+        h = _hp(AdamWHP, hp)
+        _check("al_adamw_step_multi", lib.al_adamw_step_multi(
+            _ptr(self.dev), C.byref(self.info), C.byref(h), t, _stream(stream)))
+
+
+# --------------------------------------------------------------- factored --
+def al_adafactor_step(p, g, rows, cols, r_codes, r_meta, c_codes, c_meta, fac_bits,
+                      fac_block, m_codes, m_absmax, m_block, hp: dict, t: int,
+                      workspace, stream=None):
+    h = _hp(AdafactorHP, hp)
+    _check("al_adafactor_step", lib.al_adafactor_step(
+        _ptr(p), _ptr(g), rows, cols, _ptr(r_codes), _ptr(r_meta), _ptr(c_codes),
+        _ptr(c_meta), fac_bits, fac_block, _ptr(m_codes), _ptr(m_absmax), m_block,
+        C.byref(h), t, _ptr(workspace), workspace.numel() * workspace.element_size(),
+        _stream(stream)))
+
+
+def al_came_step(p, g, rows, cols, vr_codes, vr_meta, vc_codes, vc_meta, v_bits,
+                 v_block, cr_codes, cr_meta, cc_codes, cc_meta, c_bits, c_block,
+                 m_codes, m_absmax, m_block, hp: dict, t: int, workspace, stream=None):
+    h = _hp(CameHP, hp)
+    _check("al_came_step", lib.al_came_step(
+        _ptr(p), _ptr(g), rows, cols, _ptr(vr_codes), _ptr(vr_meta), _ptr(vc_codes),
+        _ptr(vc_meta), v_bits, v_block, _ptr(cr_codes), _ptr(cr_meta), _ptr(cc_codes),
+        _ptr(cc_meta), c_bits, c_block, _ptr(m_codes), _ptr(m_absmax), m_block,
+        C.byref(h), t, _ptr(workspace), workspace.numel() * workspace.element_size(),
+        _stream(stream)))
+
+
+def al_apollo_step(p, g, rows, cols, proj, m_codes, m_absmax, m_block, v_codes, v_meta,
+                   v_bits, v_block, prev_norm, hp: dict, t: int, workspace, stream=None):
+    h = _hp(ApolloHP, hp)
+    _check("al_apollo_step", lib.al_apollo_step(
+        _ptr(p), _ptr(g), rows, cols, _ptr(proj), _ptr(m_codes), _ptr(m_absmax), m_block,
+        _ptr(v_codes), _ptr(v_meta), v_bits, v_block, _ptr(prev_norm), C.byref(h), t,
+        _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))

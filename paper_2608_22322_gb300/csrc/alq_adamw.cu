@@ -1,0 +1,312 @@
+// alq_adamw.cu -- fused AdamW step with UF8 momentum and AL-coded second
+// moment (Sec. 3.1 Eq. (1); Sec. 6.2; fused as in Sec. 7.1).
+//
+// One HBM pass per element: read p, g (fp32), the momentum and second-moment
+// codes and their per-block metadata; decode; update m, v and p in fp32; write
+// p; reduce each block's absmax (momentum) and minimum-positive / maximum
+// (second moment) with warp reductions; derive the new block constants; encode
+// and write the codes and metadata. 16.09 bytes per parameter for AL8/UF8
+// with 256-element blocks.
+//
+// The same kernel serves one tensor (descriptor passed by value) or a plan of
+// many tensors (descriptor table in device memory, tiles never crossing a
+// tensor boundary). The grid is persistent: each CTA walks tiles with a
+// stride of gridDim.x and a forward-only cursor into the descriptor table.
+#include "alq_kernels.cuh"
+
+namespace alq {
+
+template <int CPBV, int CPBM, int VBITS>
+__global__ void __launch_bounds__(kThreads, 2)
+adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t total_tiles,
+                   PlanEntry single, int v_block, int m_block, AdamWScalars s) {
+    constexpr int NBV = 4 / CPBV;
+    constexpr int NBM = 4 / CPBM;
+    constexpr float Lm2 = VBITS == 8 ? 254.0f : 65534.0f;
+    __shared__ float2 s_tab[kThreads / 32][NBV * 32];
+    __shared__ uint32_t s_part[3][kThreads / 32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int wpbv = v_block > kSeg ? v_block / kSeg : 1;
+    const int wpbm = m_block > kSeg ? m_block / kSeg : 1;
+    int cur = 0;
+    for (int64_t tile = blockIdx.x; tile < total_tiles; tile += gridDim.x) {
+        PlanEntry d;
+        if (table) {
+            while (cur + 1 < ntensors && table[cur + 1].first_tile <= tile) ++cur;
+            d = table[cur];
+        } else {
+            d = single;
+        }
+        const int64_t n = d.n;
+        const int64_t seg0 = (tile - d.first_tile) * kTile + (int64_t)warp * kSeg;
+
+        // ---- stream in p, g and the codes of this lane's four chunks
+        float4 g[4], p[4];
+        uint32_t mw[4], vw[4 * VBITS / 8];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int64_t idx = chunk_index(seg0, c, lane);
+            g[c] = load4f(d.g, idx, n);
+            p[c] = load4f(d.p, idx, n);
+            mw[c] = load4b((const uint8_t*)d.m_codes, idx, n);
+            if (VBITS == 8) {
+                vw[c] = load4b((const uint8_t*)d.v_codes, idx, n);
+            } else {
+                const uint2 h = load4h((const uint16_t*)d.v_codes, idx, n);
+                vw[2 * c] = h.x;
+                vw[2 * c + 1] = h.y;
+            }
+        }
+
+        // ---- previous block constants
+        const int64_t nvb = blocks_of_dev(n, v_block), nmb = blocks_of_dev(n, m_block);
+        const int64_t vb0 = seg0 / v_block, mb0 = seg0 / m_block;
+        float olmin[NBV], odelta[NBV], dm[NBM];
+#pragma unroll
+        for (int b = 0; b < NBV; ++b) {
+            float2 mt = make_float2(0.f, 0.f);
+            if (vb0 + b < nvb) mt = __ldg(reinterpret_cast<const float2*>(d.v_meta) + vb0 + b);
+            olmin[b] = mt.x;
+            odelta[b] = mt.y;
+        }
+#pragma unroll
+        for (int b = 0; b < NBM; ++b)
+            dm[b] = (mb0 + b < nmb) ? __ldg(d.m_absmax + mb0 + b) / 127.0f : 0.0f;
+        if (VBITS == 8) al8_build_tables<NBV>(s_tab[warp], olmin, odelta);
+
+        // ---- decode, update, write p; keep the fresh m and v
+        float mf[16], vf[16];
+        uint32_t cvmin[4], cvmax[4], cmabs[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int bv = c / CPBV, bm = c / CPBM;
+            const bool fast = al8_fast_ok(olmin[bv], odelta[bv]);
+            float pn[4];
+            cvmin[c] = 0xFFFFFFFFu;
+            cvmax[c] = 0u;
+            cmabs[c] = 0u;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t qv = code_of<VBITS>(vw, c, i);
+                const float vh = VBITS == 8
+                                     ? al8_decode(qv, s_tab[warp] + 32 * bv, fast, olmin[bv], odelta[bv])
+                                     : al16_decode(qv, olmin[bv], odelta[bv]);
+                const float mh = s8_to_float((mw[c] >> (8 * i)) & 0xFFu) * dm[bm];
+                const float gi = f4get(g[c], i);
+                const float p1 = f4get(p[c], i) * s.decay;
+                const float mm = s.beta1 * mh + s.omb1 * gi;
+                const float vv = s.beta2 * vh + s.omb2 * (gi * gi);
+                const float den = sqrtf(vv) * s.c2 + s.eps;
+                pn[i] = p1 - s.step * (mm / den);
+                mf[4 * c + i] = mm;
+                vf[4 * c + i] = vv;
+                const uint32_t vb = f2u(vv);
+                cvmin[c] = umix<false>(cvmin[c], vb - 1u);  // 0 -> max: min positive
+                cvmax[c] = umix<true>(cvmax[c], vb);
+                cmabs[c] = umix<true>(cmabs[c], f2u(mm) & 0x7FFFFFFFu);
+            }
+            store4f(d.p, chunk_index(seg0, c, lane), n, make_float4(pn[0], pn[1], pn[2], pn[3]));
+        }
+
+        // ---- new block statistics
+        uint32_t bvmin[NBV], bvmax[NBV], bmabs[NBM];
+        warp_blocks_reduce<CPBV, false>(cvmin, bvmin);
+        warp_blocks_reduce<CPBV, true>(cvmax, bvmax);
+        warp_blocks_reduce<CPBM, true>(cmabs, bmabs);
+        if (wpbv > 1) {
+            bvmin[0] = cta_group_reduce<false>(bvmin[0], s_part[0], wpbv);
+            bvmax[0] = cta_group_reduce<true>(bvmax[0], s_part[1], wpbv);
+        }
+        if (wpbm > 1) bmabs[0] = cta_group_reduce<true>(bmabs[0], s_part[2], wpbm);
+
+        float vmn[NBV], vmx[NBV], nlmin[NBV], ndelta[NBV], K[NBV], E[NBV];
+#pragma unroll
+        for (int b = 0; b < NBV; ++b) {
+            vmn[b] = u2f(bvmin[b] + 1u);
+            vmx[b] = u2f(bvmax[b]);
+        }
+        al_blocks_params<NBV>(vmn, vmx, s.log_floor, nlmin, ndelta);
+#pragma unroll
+        for (int b = 0; b < NBV; ++b) al_encode_consts(ndelta[b], Lm2, K[b], E[b]);
+        float ms[NBM], msc[NBM], minv[NBM];
+#pragma unroll
+        for (int b = 0; b < NBM; ++b) {
+            ms[b] = u2f(bmabs[b]);
+            msc[b] = 1.0f;
+            minv[b] = 0.0f;
+            if (ms[b] > 0.0f) uf8_encode_consts(ms[b], msc[b], minv[b]);
+        }
+
+        // ---- encode and write the codes and block constants
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int bv = c / CPBV, bm = c / CPBM;
+            const int64_t idx = chunk_index(seg0, c, lane);
+            uint32_t qm = 0, qv[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                if (ms[bm] > 0.0f)
+                    qm |= ((uint32_t)uf8_quantize(mf[4 * c + i], msc[bm], minv[bm]) & 0xFFu) << (8 * i);
+                qv[i] = al_encode_elem<VBITS>(vf[4 * c + i], nlmin[bv], ndelta[bv], K[bv], E[bv]);
+            }
+            store4b((uint8_t*)d.m_codes, idx, n, qm);
+            if (VBITS == 8)
+                store4b((uint8_t*)d.v_codes, idx, n, qv[0] | (qv[1] << 8) | (qv[2] << 16) | (qv[3] << 24));
+            else
+                store4h((uint16_t*)d.v_codes, idx, n,
+                        make_uint2(qv[0] | (qv[1] << 16), qv[2] | (qv[3] << 16)));
+        }
+        if (lane == 0) {
+            if ((warp % wpbv) == 0) {
+#pragma unroll
+                for (int b = 0; b < NBV; ++b)
+                    if (vb0 + b < nvb)
+                        reinterpret_cast<float2*>(d.v_meta)[vb0 + b] = make_float2(nlmin[b], ndelta[b]);
+            }
+            if ((warp % wpbm) == 0) {
+#pragma unroll
+                for (int b = 0; b < NBM; ++b)
+                    if (mb0 + b < nmb) d.m_absmax[mb0 + b] = ms[b];
+            }
+        }
+        __syncwarp();
+    }
+}
+
+// ------------------------------------------------------------- dispatch --
+static int cpb_of(int block) { return block >= 512 ? 4 : block / 128; }
+
+template <int CPBV, int CPBM, int VBITS>
+static int launch_adamw_t(const PlanEntry* table, int ntensors, int64_t total_tiles,
+                          const PlanEntry& single, int v_block, int m_block,
+                          const AdamWScalars& s, cudaStream_t stream) {
+    auto k = adamw_fused_kernel<CPBV, CPBM, VBITS>;
+    const int grid = persistent_grid((const void*)k, kThreads, 0, total_tiles);
+    k<<<grid, kThreads, 0, stream>>>(table, ntensors, total_tiles, single, v_block, m_block, s);
+    return check_launch();
+}
+
+template <int VBITS>
+static int launch_adamw_v(int cv, int cm, const PlanEntry* table, int ntensors,
+                          int64_t total_tiles, const PlanEntry& single, int v_block,
+                          int m_block, const AdamWScalars& s, cudaStream_t st) {
+#define ALQ_CASE(A, B)                                                                      \
+    if (cv == A && cm == B)                                                                 \
+        return launch_adamw_t<A, B, VBITS>(table, ntensors, total_tiles, single, v_block, \
+                                           m_block, s, st);
+    ALQ_CASE(1, 1) ALQ_CASE(1, 2) ALQ_CASE(1, 4)
+    ALQ_CASE(2, 1) ALQ_CASE(2, 2) ALQ_CASE(2, 4)
+    ALQ_CASE(4, 1) ALQ_CASE(4, 2) ALQ_CASE(4, 4)
+#undef ALQ_CASE
+    return ALQ_ERR_UNSUPPORTED;
+}
+
+static int launch_adamw(const PlanEntry* table, int ntensors, int64_t total_tiles,
+                        const PlanEntry& single, int v_block, int m_block, int v_bits,
+                        const al_adamw_hp* hp, int64_t t, cudaStream_t st) {
+    const AdamWScalars s = adamw_scalars(hp, t);
+    const int cv = cpb_of(v_block), cm = cpb_of(m_block);
+    if (v_bits == 8)
+        return launch_adamw_v<8>(cv, cm, table, ntensors, total_tiles, single, v_block, m_block, s, st);
+    return launch_adamw_v<16>(cv, cm, table, ntensors, total_tiles, single, v_block, m_block, s, st);
+}
+
+static int check_hp(const al_adamw_hp* hp) {
+    if (!hp) return ALQ_ERR_INVALID_ARG;
+    if (!(hp->beta1 >= 0.0f && hp->beta1 < 1.0f) || !(hp->beta2 >= 0.0f && hp->beta2 < 1.0f) ||
+        !(hp->eps > 0.0f) || !(hp->lr >= 0.0f))
+        return ALQ_ERR_INVALID_ARG;
+    return ALQ_OK;
+}
+
+static int check_tensor(const PlanEntry& e, int v_bits) {
+    if (e.n < 0) return ALQ_ERR_INVALID_ARG;
+    if (e.n == 0) return ALQ_OK;
+    if (!e.p || !e.g || !e.m_codes || !e.m_absmax || !e.v_codes || !e.v_meta)
+        return ALQ_ERR_INVALID_ARG;
+    if (!aligned(e.p, 16) || !aligned(e.g, 16) || !aligned(e.m_codes, 16) ||
+        !aligned(e.v_codes, 16) || !aligned(e.v_meta, 8) || !aligned(e.m_absmax, 4))
+        return ALQ_ERR_ALIGN;
+    (void)v_bits;
+    return ALQ_OK;
+}
+
+}  // namespace alq
+
+using namespace alq;
+
+extern "C" {
+
+int al_adamw_step(float* p, const float* g, int8_t* m_codes, float* m_absmax, void* v_codes,
+                  float* v_meta, int64_t n, int m_block, int v_block, int v_bits,
+                  const al_adamw_hp* hp, int64_t t, void* stream) {
+    if (!valid_block(m_block) || !valid_block(v_block) || (v_bits != 8 && v_bits != 16))
+        return ALQ_ERR_UNSUPPORTED;
+    if (t < 1) return ALQ_ERR_INVALID_ARG;
+    int st = check_hp(hp);
+    if (st) return st;
+    PlanEntry e{p, g, m_codes, m_absmax, v_codes, v_meta, n, 0};
+    st = check_tensor(e, v_bits);
+    if (st) return st;
+    if (n == 0) return ALQ_OK;
+    return launch_adamw(nullptr, 1, blocks_of(n, kTile), e, v_block, m_block, v_bits, hp, t,
+                        (cudaStream_t)stream);
+}
+
+int al_adamw_plan(const al_adamw_tensor* tensors, int ntensors, int m_block, int v_block,
+                  int v_bits, void* plan_host, size_t plan_bytes, al_multi_info* info) {
+    if (!tensors || ntensors <= 0 || !plan_host || !info) return ALQ_ERR_INVALID_ARG;
+    if (!valid_block(m_block) || !valid_block(v_block) || (v_bits != 8 && v_bits != 16))
+        return ALQ_ERR_UNSUPPORTED;
+    size_t need = 0;
+    al_adamw_plan_bytes(ntensors, &need);
+    if (plan_bytes < need) return ALQ_ERR_INVALID_ARG;
+    PlanHeader* h = (PlanHeader*)plan_host;
+    PlanEntry* ent = (PlanEntry*)((char*)plan_host + sizeof(PlanHeader));
+    int64_t tiles = 0, elems = 0;
+    for (int i = 0; i < ntensors; ++i) {
+        const al_adamw_tensor& t = tensors[i];
+        PlanEntry e{t.p, t.g, t.m_codes, t.m_absmax, t.v_codes, t.v_meta, t.n, tiles};
+        int st = check_tensor(e, v_bits);
+        if (st) return st;
+        ent[i] = e;
+        tiles += blocks_of(t.n, kTile);
+        elems += t.n;
+    }
+    memset(h, 0, sizeof(PlanHeader));
+    h->magic = kPlanMagic;
+    h->ntensors = ntensors;
+    h->m_block = m_block;
+    h->v_block = v_block;
+    h->v_bits = v_bits;
+    h->tile = kTile;
+    h->total_tiles = tiles;
+    h->total_elems = elems;
+    info->ntensors = ntensors;
+    info->m_block = m_block;
+    info->v_block = v_block;
+    info->v_bits = v_bits;
+    info->total_tiles = tiles;
+    info->total_elems = elems;
+    return ALQ_OK;
+}
+
+int al_adamw_step_multi(const void* plan_dev, const al_multi_info* info, const al_adamw_hp* hp,
+                        int64_t t, void* stream) {
+    if (!plan_dev || !info || t < 1) return ALQ_ERR_INVALID_ARG;
+    if (!aligned(plan_dev, 16)) return ALQ_ERR_ALIGN;
+    if (info->ntensors <= 0 || info->total_tiles < 0) return ALQ_ERR_INVALID_ARG;
+    if (!valid_block(info->m_block) || !valid_block(info->v_block) ||
+        (info->v_bits != 8 && info->v_bits != 16))
+        return ALQ_ERR_UNSUPPORTED;
+    int st = check_hp(hp);
+    if (st) return st;
+    if (info->total_tiles == 0) return ALQ_OK;
+    const PlanEntry* table =
+        (const PlanEntry*)((const char*)plan_dev + sizeof(PlanHeader));
+    PlanEntry none{};
+    return launch_adamw(table, info->ntensors, info->total_tiles, none, info->v_block,
+                        info->m_block, info->v_bits, hp, t, (cudaStream_t)stream);
+}
+
+}  // extern "C"

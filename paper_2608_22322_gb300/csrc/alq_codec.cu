@@ -1,0 +1,296 @@
+// alq_codec.cu -- stand-alone AL (Sec. 4.1, Eq. (3)-(5)) and UF8 (Sec. 4.3)
+// codec kernels and their C-ABI entry points. One HBM pass each: the encoder
+// reduces each block's minimum positive value and maximum with warp
+// reductions, derives (l_min, Delta) once per block and writes codes and
+// metadata; the decoder rebuilds each block's level tables and writes fp32.
+#include "alq_kernels.cuh"
+
+namespace alq {
+
+template <typename Kernel>
+static int grid_for(Kernel kernel, int64_t ntiles) {
+    return persistent_grid((const void*)kernel, kThreads, 0, ntiles);
+}
+
+// ------------------------------------------------------------- AL encode --
+template <int CPB, int BITS>
+__global__ void __launch_bounds__(kThreads)
+al_encode_kernel(const float* __restrict__ x, int64_t n, int block, float log_floor,
+                 void* __restrict__ codes, float* __restrict__ meta, int64_t ntiles) {
+    constexpr int NB = 4 / CPB;
+    constexpr float Lm2 = BITS == 8 ? 254.0f : 65534.0f;
+    __shared__ uint32_t s_part[2][kThreads / 32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int wpb = block > kSeg ? block / kSeg : 1;
+    const int64_t nblk = blocks_of_dev(n, block);
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
+        float4 v[4];
+        uint32_t cmin[4], cmax[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            v[c] = load4f(x, chunk_index(seg0, c, lane), n);
+            cmin[c] = 0xFFFFFFFFu;
+            cmax[c] = 0u;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t b = f2u(f4get(v[c], i)) & 0x7FFFFFFFu;  // -0 -> 0
+                cmin[c] = umix<false>(cmin[c], b - 1u);               // 0 -> max
+                cmax[c] = umix<true>(cmax[c], b);
+            }
+        }
+        uint32_t bmin[NB], bmax[NB];
+        warp_blocks_reduce<CPB, false>(cmin, bmin);
+        warp_blocks_reduce<CPB, true>(cmax, bmax);
+        if (wpb > 1) {
+            bmin[0] = cta_group_reduce<false>(bmin[0], s_part[0], wpb);
+            bmax[0] = cta_group_reduce<true>(bmax[0], s_part[1], wpb);
+        }
+        float mn[NB], mx[NB], lmin[NB], delta[NB], K[NB], E[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            mn[b] = u2f(bmin[b] + 1u);
+            mx[b] = u2f(bmax[b]);
+        }
+        al_blocks_params<NB>(mn, mx, log_floor, lmin, delta);
+#pragma unroll
+        for (int b = 0; b < NB; ++b) al_encode_consts(delta[b], Lm2, K[b], E[b]);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int b = c / CPB;
+            uint32_t q[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                q[i] = al_encode_elem<BITS>(f4get(v[c], i), lmin[b], delta[b], K[b], E[b]);
+            const int64_t idx = chunk_index(seg0, c, lane);
+            if (BITS == 8)
+                store4b((uint8_t*)codes, idx, n, q[0] | (q[1] << 8) | (q[2] << 16) | (q[3] << 24));
+            else
+                store4h((uint16_t*)codes, idx, n, make_uint2(q[0] | (q[1] << 16), q[2] | (q[3] << 16)));
+        }
+        if (lane == 0 && (warp % wpb) == 0) {
+            const int64_t gb0 = seg0 / block;
+#pragma unroll
+            for (int b = 0; b < NB; ++b)
+                if (gb0 + b < nblk)
+                    reinterpret_cast<float2*>(meta)[gb0 + b] = make_float2(lmin[b], delta[b]);
+        }
+    }
+}
+
+// ------------------------------------------------------------- AL decode --
+template <int CPB, int BITS>
+__global__ void __launch_bounds__(kThreads)
+al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta, int64_t n,
+                 int block, float* __restrict__ out, int64_t ntiles) {
+    constexpr int NB = 4 / CPB;
+    __shared__ float2 s_tab[kThreads / 32][NB * 32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t nblk = blocks_of_dev(n, block);
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
+        uint32_t w[4 * BITS / 8];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int64_t idx = chunk_index(seg0, c, lane);
+            if (BITS == 8) {
+                w[c] = load4b((const uint8_t*)codes, idx, n);
+            } else {
+                const uint2 h = load4h((const uint16_t*)codes, idx, n);
+                w[2 * c] = h.x;
+                w[2 * c + 1] = h.y;
+            }
+        }
+        float lmin[NB], delta[NB];
+        const int64_t gb0 = seg0 / block;
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            float2 mt = make_float2(0.f, 0.f);
+            if (gb0 + b < nblk) mt = __ldg(reinterpret_cast<const float2*>(meta) + gb0 + b);
+            lmin[b] = mt.x;
+            delta[b] = mt.y;
+        }
+        if (BITS == 8) al8_build_tables<NB>(s_tab[warp], lmin, delta);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int b = c / CPB;
+            const bool fast = al8_fast_ok(lmin[b], delta[b]);
+            float r[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t q = code_of<BITS>(w, c, i);
+                r[i] = BITS == 8 ? al8_decode(q, s_tab[warp] + 32 * b, fast, lmin[b], delta[b])
+                                 : al16_decode(q, lmin[b], delta[b]);
+            }
+            store4f(out, chunk_index(seg0, c, lane), n, make_float4(r[0], r[1], r[2], r[3]));
+        }
+        __syncwarp();
+    }
+}
+
+// ------------------------------------------------------------ UF8 encode --
+template <int CPB>
+__global__ void __launch_bounds__(kThreads)
+uf8_encode_kernel(const float* __restrict__ m, int64_t n, int block, int8_t* __restrict__ codes,
+                  float* __restrict__ absmax, int64_t ntiles) {
+    constexpr int NB = 4 / CPB;
+    __shared__ uint32_t s_part[kThreads / 32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int wpb = block > kSeg ? block / kSeg : 1;
+    const int64_t nblk = blocks_of_dev(n, block);
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
+        float4 v[4];
+        uint32_t ca[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            v[c] = load4f(m, chunk_index(seg0, c, lane), n);
+            ca[c] = 0u;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) ca[c] = umix<true>(ca[c], f2u(f4get(v[c], i)) & 0x7FFFFFFFu);
+        }
+        uint32_t ba[NB];
+        warp_blocks_reduce<CPB, true>(ca, ba);
+        if (wpb > 1) ba[0] = cta_group_reduce<true>(ba[0], s_part, wpb);
+        float s[NB], sc[NB], inv[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            s[b] = u2f(ba[b]);
+            sc[b] = 1.0f;
+            inv[b] = 0.0f;
+            if (s[b] > 0.0f) uf8_encode_consts(s[b], sc[b], inv[b]);
+        }
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int b = c / CPB;
+            uint32_t wd = 0;
+            if (s[b] > 0.0f) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    wd |= ((uint32_t)uf8_quantize(f4get(v[c], i), sc[b], inv[b]) & 0xFFu) << (8 * i);
+            }
+            store4b((uint8_t*)codes, chunk_index(seg0, c, lane), n, wd);
+        }
+        if (lane == 0 && (warp % wpb) == 0) {
+            const int64_t gb0 = seg0 / block;
+#pragma unroll
+            for (int b = 0; b < NB; ++b)
+                if (gb0 + b < nblk) absmax[gb0 + b] = s[b];
+        }
+    }
+}
+
+// ------------------------------------------------------------ UF8 decode --
+template <int CPB>
+__global__ void __launch_bounds__(kThreads)
+uf8_decode_kernel(const int8_t* __restrict__ codes, const float* __restrict__ absmax, int64_t n,
+                  int block, float* __restrict__ out, int64_t ntiles) {
+    constexpr int NB = 4 / CPB;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t nblk = blocks_of_dev(n, block);
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
+        float d[NB];
+        const int64_t gb0 = seg0 / block;
+#pragma unroll
+        for (int b = 0; b < NB; ++b)
+            d[b] = (gb0 + b < nblk) ? __ldg(absmax + gb0 + b) / 127.0f : 0.0f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int64_t idx = chunk_index(seg0, c, lane);
+            const uint32_t w = load4b((const uint8_t*)codes, idx, n);
+            const int b = c / CPB;
+            float4 r;
+            r.x = s8_to_float(w & 0xFFu) * d[b];
+            r.y = s8_to_float((w >> 8) & 0xFFu) * d[b];
+            r.z = s8_to_float((w >> 16) & 0xFFu) * d[b];
+            r.w = s8_to_float(w >> 24) * d[b];
+            store4f(out, idx, n, r);
+        }
+    }
+}
+
+// ------------------------------------------------------------- launchers --
+static int cpb_of(int block) { return block >= 512 ? 4 : block / 128; }
+
+#define ALQ_DISPATCH_CPB(block, KERNEL_TMPL, ...)                 \
+    switch (cpb_of(block)) {                                      \
+        case 1: { auto k = KERNEL_TMPL<1 __VA_ARGS__>; LAUNCH(k); } break; \
+        case 2: { auto k = KERNEL_TMPL<2 __VA_ARGS__>; LAUNCH(k); } break; \
+        default: { auto k = KERNEL_TMPL<4 __VA_ARGS__>; LAUNCH(k); } break; \
+    }
+
+}  // namespace alq
+
+using namespace alq;
+
+extern "C" {
+
+int al_encode(const float* x, int64_t n, int block, int bits, float log_floor, void* codes,
+              float* meta, void* stream) {
+    if (n < 0) return ALQ_ERR_INVALID_ARG;
+    if (!valid_block(block) || (bits != 8 && bits != 16)) return ALQ_ERR_UNSUPPORTED;
+    if (n == 0) return ALQ_OK;
+    if (!x || !codes || !meta) return ALQ_ERR_INVALID_ARG;
+    if (!aligned(x, 16) || !aligned(codes, 16) || !aligned(meta, 8)) return ALQ_ERR_ALIGN;
+    const int64_t ntiles = blocks_of(n, kTile);
+    cudaStream_t s = (cudaStream_t)stream;
+#define LAUNCH(k) k<<<grid_for(k, ntiles), kThreads, 0, s>>>(x, n, block, log_floor, codes, meta, ntiles)
+    if (bits == 8) {
+        ALQ_DISPATCH_CPB(block, al_encode_kernel, , 8)
+    } else {
+        ALQ_DISPATCH_CPB(block, al_encode_kernel, , 16)
+    }
+#undef LAUNCH
+    return check_launch();
+}
+
+int al_decode(const void* codes, const float* meta, int64_t n, int block, int bits, float* out,
+              void* stream) {
+    if (n < 0) return ALQ_ERR_INVALID_ARG;
+    if (!valid_block(block) || (bits != 8 && bits != 16)) return ALQ_ERR_UNSUPPORTED;
+    if (n == 0) return ALQ_OK;
+    if (!codes || !meta || !out) return ALQ_ERR_INVALID_ARG;
+    if (!aligned(out, 16) || !aligned(codes, 16) || !aligned(meta, 8)) return ALQ_ERR_ALIGN;
+    const int64_t ntiles = blocks_of(n, kTile);
+    cudaStream_t s = (cudaStream_t)stream;
+#define LAUNCH(k) k<<<grid_for(k, ntiles), kThreads, 0, s>>>(codes, meta, n, block, out, ntiles)
+    if (bits == 8) {
+        ALQ_DISPATCH_CPB(block, al_decode_kernel, , 8)
+    } else {
+        ALQ_DISPATCH_CPB(block, al_decode_kernel, , 16)
+    }
+#undef LAUNCH
+    return check_launch();
+}
+
+int uf8_encode(const float* m, int64_t n, int block, int8_t* codes, float* absmax, void* stream) {
+    if (n < 0) return ALQ_ERR_INVALID_ARG;
+    if (!valid_block(block)) return ALQ_ERR_UNSUPPORTED;
+    if (n == 0) return ALQ_OK;
+    if (!m || !codes || !absmax) return ALQ_ERR_INVALID_ARG;
+    if (!aligned(m, 16) || !aligned(codes, 16) || !aligned(absmax, 4)) return ALQ_ERR_ALIGN;
+    const int64_t ntiles = blocks_of(n, kTile);
+    cudaStream_t s = (cudaStream_t)stream;
+#define LAUNCH(k) k<<<grid_for(k, ntiles), kThreads, 0, s>>>(m, n, block, codes, absmax, ntiles)
+    ALQ_DISPATCH_CPB(block, uf8_encode_kernel, )
+#undef LAUNCH
+    return check_launch();
+}
+
+int uf8_decode(const int8_t* codes, const float* absmax, int64_t n, int block, float* out,
+               void* stream) {
+    if (n < 0) return ALQ_ERR_INVALID_ARG;
+    if (!valid_block(block)) return ALQ_ERR_UNSUPPORTED;
+    if (n == 0) return ALQ_OK;
+    if (!codes || !absmax || !out) return ALQ_ERR_INVALID_ARG;
+    if (!aligned(out, 16) || !aligned(codes, 16) || !aligned(absmax, 4)) return ALQ_ERR_ALIGN;
+    const int64_t ntiles = blocks_of(n, kTile);
+    cudaStream_t s = (cudaStream_t)stream;
+#define LAUNCH(k) k<<<grid_for(k, ntiles), kThreads, 0, s>>>(codes, absmax, n, block, out, ntiles)
+    ALQ_DISPATCH_CPB(block, uf8_decode_kernel, )
+#undef LAUNCH
+    return check_launch();
+}
+
+}  // extern "C"

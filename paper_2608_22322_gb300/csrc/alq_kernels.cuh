@@ -1,0 +1,229 @@
+// alq_kernels.cuh -- device building blocks of the element-wise kernels:
+// masked chunk loads/stores, per-block reductions, per-block AL/UF8
+// constants, and the AL8 decode tables.
+//
+// Geometry (see alq_internal.h): a warp owns a 512-element segment; lane l
+// owns chunk c = 0..3 = elements [128 c + 4 l, 128 c + 4 l + 4) of it. For a
+// block size B = 128 * CPB (CPB = 1, 2, 4 chunks per block) a segment holds
+// NB = 4 / CPB blocks, each spanning all 32 lanes; for B > 512 a block spans
+// B / 512 consecutive warps and its statistics are combined through shared
+// memory.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "alq_internal.h"
+#include "alq_numerics.h"
+
+namespace alq {
+
+// ------------------------------------------------------------- chunk I/O --
+__device__ __forceinline__ int64_t blocks_of_dev(int64_t n, int block) {
+    return (n + block - 1) / block;
+}
+
+__device__ __forceinline__ int64_t chunk_index(int64_t seg0, int c, int lane) {
+    return seg0 + 128 * c + 4 * lane;
+}
+
+__device__ __forceinline__ float4 load4f(const float* p, int64_t i, int64_t n) {
+    if (i + 4 <= n) return __ldcs(reinterpret_cast<const float4*>(p + i));
+    float4 r = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (i < n) r.x = p[i];
+    if (i + 1 < n) r.y = p[i + 1];
+    if (i + 2 < n) r.z = p[i + 2];
+    return r;
+}
+
+__device__ __forceinline__ void store4f(float* p, int64_t i, int64_t n, float4 v) {
+    if (i + 4 <= n) {
+        __stcs(reinterpret_cast<float4*>(p + i), v);
+        return;
+    }
+    if (i < n) p[i] = v.x;
+    if (i + 1 < n) p[i + 1] = v.y;
+    if (i + 2 < n) p[i + 2] = v.z;
+}
+
+// Four 8-bit codes as one little-endian word.
+__device__ __forceinline__ uint32_t load4b(const uint8_t* p, int64_t i, int64_t n) {
+    if (i + 4 <= n) return __ldcs(reinterpret_cast<const unsigned int*>(p + i));
+    uint32_t r = 0;
+    if (i < n) r |= (uint32_t)p[i];
+    if (i + 1 < n) r |= (uint32_t)p[i + 1] << 8;
+    if (i + 2 < n) r |= (uint32_t)p[i + 2] << 16;
+    return r;
+}
+
+__device__ __forceinline__ void store4b(uint8_t* p, int64_t i, int64_t n, uint32_t w) {
+    if (i + 4 <= n) {
+        __stcs(reinterpret_cast<unsigned int*>(p + i), w);
+        return;
+    }
+    if (i < n) p[i] = (uint8_t)w;
+    if (i + 1 < n) p[i + 1] = (uint8_t)(w >> 8);
+    if (i + 2 < n) p[i + 2] = (uint8_t)(w >> 16);
+}
+
+// Four 16-bit codes as two words (w0 = codes 0,1; w1 = codes 2,3).
+__device__ __forceinline__ uint2 load4h(const uint16_t* p, int64_t i, int64_t n) {
+    if (i + 4 <= n) return __ldcs(reinterpret_cast<const uint2*>(p + i));
+    uint2 r = make_uint2(0u, 0u);
+    if (i < n) r.x |= (uint32_t)p[i];
+    if (i + 1 < n) r.x |= (uint32_t)p[i + 1] << 16;
+    if (i + 2 < n) r.y |= (uint32_t)p[i + 2];
+    return r;
+}
+
+__device__ __forceinline__ void store4h(uint16_t* p, int64_t i, int64_t n, uint2 w) {
+    if (i + 4 <= n) {
+        __stcs(reinterpret_cast<uint2*>(p + i), w);
+        return;
+    }
+    if (i < n) p[i] = (uint16_t)w.x;
+    if (i + 1 < n) p[i + 1] = (uint16_t)(w.x >> 16);
+    if (i + 2 < n) p[i + 2] = (uint16_t)w.y;
+}
+
+__device__ __forceinline__ float f4get(const float4& v, int i) {
+    return i == 0 ? v.x : (i == 1 ? v.y : (i == 2 ? v.z : v.w));
+}
+
+// Code i (0..3) of a chunk: 8-bit codes packed in one word, 16-bit in two.
+template <int BITS>
+__device__ __forceinline__ uint32_t code_of(const uint32_t* w, int c, int i) {
+    if (BITS == 8) return (w[c] >> (8 * i)) & 0xFFu;
+    return (w[2 * c + (i >> 1)] >> (16 * (i & 1))) & 0xFFFFu;
+}
+
+// --------------------------------------------------------- block reductions --
+template <bool kMax>
+__device__ __forceinline__ uint32_t umix(uint32_t a, uint32_t b) {
+    return kMax ? (a > b ? a : b) : (a < b ? a : b);
+}
+
+// Per-block warp-wide min or max of per-chunk values (unsigned order).
+template <int CPB, bool kMax>
+__device__ __forceinline__ void warp_blocks_reduce(const uint32_t (&chunk)[4],
+                                                   uint32_t (&out)[4 / CPB]) {
+#pragma unroll
+    for (int b = 0; b < 4 / CPB; ++b) {
+        uint32_t v = chunk[b * CPB];
+#pragma unroll
+        for (int c = 1; c < CPB; ++c) v = umix<kMax>(v, chunk[b * CPB + c]);
+        out[b] = kMax ? __reduce_max_sync(0xFFFFFFFFu, v) : __reduce_min_sync(0xFFFFFFFFu, v);
+    }
+}
+
+// Blocks wider than a segment: combine the per-warp results of the `wpb`
+// warps that share a block. Every thread of the CTA must call this.
+template <bool kMax>
+__device__ __forceinline__ uint32_t cta_group_reduce(uint32_t v, uint32_t* s_part,
+                                                     int wpb) {
+    const int warp = threadIdx.x >> 5;
+    if ((threadIdx.x & 31) == 0) s_part[warp] = v;
+    __syncthreads();
+    const int g0 = (warp / wpb) * wpb;
+    uint32_t r = s_part[g0];
+    for (int k = 1; k < wpb; ++k) r = umix<kMax>(r, s_part[g0 + k]);
+    __syncthreads();
+    return r;
+}
+
+// ------------------------------------------------------- AL block constants --
+// (l_min, Delta) of the NB blocks of a segment from their minimum positive
+// value mn and maximum mx (Eq. (3)). The 2 NB fp32-rounded logs are spread
+// over the lanes (one log per lane) and exchanged by shuffles.
+template <int NB>
+__device__ __forceinline__ void al_blocks_params(const float (&mn)[NB], const float (&mx)[NB],
+                                                 float log_floor, float (&lmin)[NB],
+                                                 float (&delta)[NB]) {
+    const int lane = threadIdx.x & 31;
+    const int v = lane & (2 * NB - 1);
+    float x = 0.0f;
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+        if (v == 2 * b) x = mn[b];
+        if (v == 2 * b + 1) x = mx[b];
+    }
+    const float L = (x > 0.0f) ? log2_rn(x) : 0.0f;
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+        const float l0 = __shfl_sync(0xFFFFFFFFu, L, 2 * b);
+        const float l1 = __shfl_sync(0xFFFFFFFFu, L, 2 * b + 1);
+        al_block_params_from_logs(mx[b], l0, l1, log_floor, lmin[b], delta[b]);
+    }
+}
+
+// ------------------------------------------------------ AL8 decode tables --
+// The two 16-entry level tables of each of the NB blocks of a segment
+// (Eq. (5)): entry b < 16 holds 2^((b-1) d), entry 16 + a holds
+// 2^(l_min + 16 a d), d = Delta / 254, as two-float pairs; code q decodes to
+// entry[16 + (q >> 4)] * entry[q & 15]. One entry per lane per block.
+// Blocks whose l_min is below -96 (or that are empty) take the FP64 path.
+template <int NB>
+__device__ __forceinline__ void al8_build_tables(float2* tab, const float (&lmin)[NB],
+                                                 const float (&delta)[NB]) {
+    const int lane = threadIdx.x & 31;
+    const bool hi = lane >= 16;
+    const int k = hi ? 16 * (lane - 16) : (lane - 1);
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+        float rh = 0.0f, rl = 0.0f;
+        if (delta[b] > 0.0f && lmin[b] >= -96.0f)
+            al_level_ff(hi ? lmin[b] : 0.0f, delta[b], k, 254.0f, 1.0f / 254.0f, rh, rl);
+        tab[32 * b + lane] = make_float2(rh, rl);
+    }
+    __syncwarp();
+}
+
+__device__ __forceinline__ bool al8_fast_ok(float lmin, float delta) {
+    return delta > 0.0f && lmin >= -96.0f;
+}
+
+// AL8 element decode through a block's tables; FP64 when the two-float
+// product may round differently, or the block is outside the fast range.
+__device__ __forceinline__ float al8_decode(uint32_t q, const float2* tab, bool fast,
+                                            float lmin, float delta) {
+    if (q == 0u) return 0.0f;
+    if (fast) {
+        const float2 a = tab[16 + (q >> 4)];
+        const float2 b = tab[q & 15u];
+        bool fb;
+        const float r = al8_decode_pair(a.x, a.y, b.x, b.y, fb);
+        if (!fb) return r;
+    }
+    return al_dequantize_fp64(q, lmin, delta, 254.0);
+}
+
+// AL16 element decode: the level directly in two-float form.
+__device__ __forceinline__ float al16_decode(uint32_t q, float lmin, float delta) {
+    if (q == 0u) return 0.0f;
+    if (lmin >= -96.0f) {
+        float rh, rl;
+        al_level_ff(lmin, delta, (int)q - 1, 65534.0f, 1.0f / 65534.0f, rh, rl);
+        const float hu = half_ulp_below(rh);
+        if (fabsf(rl) < hu - hu * 0x1p-16f) return rh;
+    }
+    return al_dequantize_fp64(q, lmin, delta, 65534.0);
+}
+
+// Eq. (4) element encode with the FP64 fallback near rounding boundaries.
+template <int BITS>
+__device__ __forceinline__ uint32_t al_encode_elem(float x, float lmin, float delta,
+                                                   float K, float E) {
+    if (x == 0.0f) return 0u;
+    constexpr float Lm2 = BITS == 8 ? 254.0f : 65534.0f;
+    bool fb;
+    uint32_t q = al_quantize_fast(x, lmin, K, E, Lm2, fb);
+    if (fb) q = al_quantize_fp64(x, lmin, delta, (double)Lm2);
+    return q;
+}
+
+// Signed 8-bit code (two's complement byte) to float, exactly.
+__device__ __forceinline__ float s8_to_float(uint32_t byte) {
+    return (float)(int)(int8_t)(uint8_t)byte;
+}
+
+}  // namespace alq

@@ -1,0 +1,194 @@
+"""GPU parity of the fused AdamW step (UF8 momentum, AL-coded V) with the
+oracle.
+
+Sec. 3.1 Eq. (1), Sec. 6.2, Sec. 7.1. Both sides run the same steps from the
+same seeded state and gradients; parameters, codes and block metadata must
+agree bit for bit after every step (the arithmetic contract fixes the fp32
+operation order, and the codec's fast paths fall back to the defining double
+expressions near rounding boundaries). Covered: the 256x1024 single-tensor
+workload for 10 steps (persistent and redrawn zero masks), the paper's
+B_V = 2048 setting, AL16, every block-size class, ragged lengths, a
+multi-tensor plan with tiny and ragged tensors, and the full 1.1B-parameter
+TinyLlama plan checked on sampled blocks.
+"""
+import numpy as np
+import pytest
+
+import oracle as ora
+from gpu_util import ADAMW_HP, bytes_equal, gpu_available
+from paper_2608_22322_gb300 import workloads as wl
+
+pytestmark = [pytest.mark.gpu,
+              pytest.mark.skipif(not gpu_available(), reason="needs a CUDA GPU")]
+
+
+@pytest.fixture(scope="module")
+def B():
+    from paper_2608_22322_gb300 import binding
+    return binding
+
+
+class Pair:
+    """The same AdamW state on the host (oracle) and the device (library)."""
+
+    def __init__(self, p0, m_block, v_block, v_bits):
+        import torch
+        n = p0.size
+        self.n, self.mb, self.vb, self.bits = n, m_block, v_block, v_bits
+        self.h = dict(p=p0.ravel().copy(), mc=np.zeros(n, np.int8),
+                      ma=np.zeros((n + m_block - 1) // m_block, np.float32),
+                      vc=np.zeros(n, ora.code_dtype(v_bits)),
+                      vm=np.zeros(2 * ((n + v_block - 1) // v_block), np.float32))
+        self.d = {k: torch.from_numpy(v.view(np.int16) if v.dtype == np.uint16 else v.copy()).cuda()
+                  for k, v in self.h.items()}
+
+    def host_step(self, g, t, hp=ADAMW_HP):
+        h = self.h
+        ora.adamw_step(h["p"], g, h["mc"], h["ma"], h["vc"], h["vm"], self.mb, self.vb,
+                       self.bits, hp, t)
+
+    def dev_args(self):
+        d = self.d
+        return dict(p=d["p"], m_codes=d["mc"], m_absmax=d["ma"], v_codes=d["vc"], v_meta=d["vm"])
+
+    def compare(self, what=""):
+        import torch
+        torch.cuda.synchronize()
+        for k in ("p", "mc", "ma", "vc", "vm"):
+            got = self.d[k].cpu().numpy()
+            bad = bytes_equal(self.h[k], got)
+            assert bad == 0, f"{what}: {k} differs in {bad} bytes"
+
+
+def _run_single(B, w, m_block, v_block, v_bits, steps, hp=ADAMW_HP):
+    import torch
+    pr = Pair(w.p0, m_block, v_block, v_bits)
+    for t in range(1, steps + 1):
+        g = w.grad(t).ravel()
+        pr.host_step(g, t, hp)
+        a = pr.dev_args()
+        B.al_adamw_step(a["p"], torch.from_numpy(g).cuda(), a["m_codes"], a["m_absmax"],
+                        a["v_codes"], a["v_meta"], m_block, v_block, v_bits, hp, t)
+        pr.compare(f"step {t}")
+    return pr
+
+
+def test_adamw_256x1024_ten_steps(B):
+    """The single-tensor workload: 256x1024, 10% zero mask, 2% dormant rows,
+    AL8/UF8 blocks of 256, wd 0.01, 10 steps."""
+    w = wl.AdamWSingle()
+    pr = _run_single(B, w, 256, 256, 8, 10)
+    codes = pr.h["vc"].reshape(w.shape)
+    assert not codes[w.dormant].any()
+
+
+def test_adamw_redrawn_mask(B):
+    w = wl.AdamWSingle(redraw_mask=True)
+    _run_single(B, w, 256, 256, 8, 5)
+
+
+@pytest.mark.parametrize("m_block,v_block", [(256, 2048), (128, 128), (512, 1024),
+                                             (4096, 256), (1024, 4096)])
+def test_adamw_block_sizes(B, m_block, v_block):
+    w = wl.AdamWSingle(shape=(37, 1111))  # 41107 elements: ragged tiles and blocks
+    _run_single(B, w, m_block, v_block, 8, 4)
+
+
+def test_adamw_al16(B):
+    w = wl.AdamWSingle(shape=(64, 777))
+    _run_single(B, w, 256, 256, 16, 4)
+
+
+def test_adamw_plan_many_tensors(B):
+    """Multi-tensor plan: tiny, ragged and multi-tile tensors in one launch."""
+    import torch
+    sizes = [1, 5, 4095, 4097, 300, 2 * 4096 + 511, 17, 64 * 1024]
+    pairs, gens = [], []
+    for i, n in enumerate(sizes):
+        p0 = wl.param_init((n,), 40 + i, norm_vector_value=0.5) if i % 2 else \
+            (wl.rng(40 + i).standard_normal(n) * 0.02).astype(np.float32)
+        pairs.append(Pair(p0, 256, 2048, 8))
+        gens.append(lambda t, n=n, i=i: wl.gaussian_grad((n,), 1e-3, 900 + 31 * i + t,
+                                                         wl.zero_mask((n,), 0.1, 77 + i)))
+    gdev = [torch.zeros(n, dtype=torch.float32, device="cuda") for n in sizes]
+    plan = B.AdamWPlan([dict(g=gdev[i], **pr.dev_args()) for i, pr in enumerate(pairs)],
+                       256, 2048, 8)
+    for t in range(1, 4):
+        for i, pr in enumerate(pairs):
+            g = gens[i](t)
+            pr.host_step(g, t)
+            gdev[i].copy_(torch.from_numpy(g))
+        plan.step(ADAMW_HP, t)
+        for i, pr in enumerate(pairs):
+            pr.compare(f"tensor {i} (n={sizes[i]}) step {t}")
+
+
+def test_adamw_tinyllama_full_plan_sampled(B):
+    """All 201 TinyLlama-1.1B tensors (1,100,048,384 parameters) in one plan,
+    the launch the benchmark times. Blocks are independent in AdamW, so the
+    oracle re-runs sampled blocks (first, last and random ones of every tensor)
+    from a snapshot of their state and gradient, step by step."""
+    import torch
+    cfg = wl.CONFIGS["tinyllama_adamw"]
+    mb, vb = cfg["m_block"], cfg["v_block"]
+    tens = wl.tinyllama_tensors()
+    dev = []
+    for i, (name, shape) in enumerate(tens):
+        n = wl.numel(shape)
+        p = torch.empty(n, dtype=torch.float32, device="cuda")
+        if len(shape) == 1:
+            p.fill_(1.0)
+        else:
+            wl.torch_device_normal_(p, 0.02, 1000 + i)
+        dev.append(dict(p=p, g=torch.empty(n, dtype=torch.float32, device="cuda"),
+                        m_codes=torch.zeros(n, dtype=torch.int8, device="cuda"),
+                        m_absmax=torch.zeros((n + mb - 1) // mb, dtype=torch.float32, device="cuda"),
+                        v_codes=torch.zeros(n, dtype=torch.uint8, device="cuda"),
+                        v_meta=torch.zeros(2 * ((n + vb - 1) // vb), dtype=torch.float32,
+                                           device="cuda")))
+    plan = B.AdamWPlan(dev, mb, vb, 8)
+    assert plan.info.total_elems == 1_100_048_384
+    r = wl.rng(5)
+    samples = []
+    for i, (_, shape) in enumerate(tens):
+        nb = (wl.numel(shape) + 255) // 256
+        picks = {0, nb - 1, *map(int, r.integers(0, nb, 2))}
+        samples += [(i, b) for b in sorted(picks)]
+    for t in (1, 2, 3):
+        for i, d in enumerate(dev):
+            wl.torch_device_normal_(d["g"], 1e-3, 50_000 + 1000 * t + i)
+            wl.torch_device_zero_(d["g"], 0.01, 90_000 + 1000 * t + i)
+        snap = []
+        for i, b in samples:
+            d = dev[i]
+            lo, hi = 256 * b, min(256 * (b + 1), d["p"].numel())
+            snap.append(dict(p=d["p"][lo:hi].cpu().numpy(), g=d["g"][lo:hi].cpu().numpy(),
+                             mc=d["m_codes"][lo:hi].cpu().numpy(),
+                             ma=d["m_absmax"][b:b + 1].cpu().numpy(),
+                             vc=d["v_codes"][lo:hi].cpu().numpy(),
+                             vm=d["v_meta"][2 * b:2 * b + 2].cpu().numpy()))
+        plan.step(ADAMW_HP, t)
+        torch.cuda.synchronize()
+        for (i, b), s in zip(samples, snap):
+            ora.adamw_step(s["p"], s["g"], s["mc"], s["ma"], s["vc"], s["vm"], 256, 256, 8,
+                           ADAMW_HP, t)
+            d = dev[i]
+            lo, hi = 256 * b, min(256 * (b + 1), d["p"].numel())
+            for k, got in (("p", d["p"][lo:hi]), ("mc", d["m_codes"][lo:hi]),
+                           ("ma", d["m_absmax"][b:b + 1]), ("vc", d["v_codes"][lo:hi]),
+                           ("vm", d["v_meta"][2 * b:2 * b + 2])):
+                assert bytes_equal(s[k], got.cpu().numpy()) == 0, (tens[i][0], b, k, t)
+    del dev, plan
+    torch.cuda.empty_cache()
+
+
+def test_adamw_rejects_bad_arguments(B):
+    import torch
+    x = torch.zeros(1024, device="cuda")
+    c = torch.zeros(1024, dtype=torch.int8, device="cuda")
+    with pytest.raises(B.AlqError, match="UNSUPPORTED"):
+        B.al_adamw_step(x, x, c, x, c, x, 100, 256, 8, ADAMW_HP, 1)
+    with pytest.raises(B.AlqError, match="ALIGN"):
+        B.al_adamw_step(x[1:], x[1:], c[1:], x, c[1:], x, 256, 256, 8, ADAMW_HP, 1)
+    with pytest.raises(B.AlqError, match="INVALID_ARG"):
+        B.al_adamw_step(x, x, c, x, c, x, 256, 256, 8, ADAMW_HP, 0)

@@ -1,0 +1,135 @@
+"""CPU parity of the CUDA library's codec arithmetic (host build) with the
+oracle.
+
+The library evaluates Eq. (3)-(5) with fp32/two-float fast paths and an FP64
+fallback near rounding boundaries (alq_numerics.h). Built for the host, the
+same source must reproduce the oracle's codes, bounds and decoded values bit
+for bit, with rare fallbacks. The GPU build differs only in the hardware
+log2 approximation used by the encoder's fast path (covered by the GPU
+tests).
+"""
+import ctypes as C
+import math
+import os
+import subprocess
+
+import numpy as np
+import pytest
+
+import oracle as ora
+from paper_2608_22322_gb300 import workloads as wl
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+ROOT = os.path.dirname(HERE)
+CSRC = os.path.join(ROOT, "paper_2608_22322_gb300", "csrc")
+SRC = os.path.join(HERE, "numerics_host.cpp")
+OUT = os.path.join(ROOT, "_build", "numerics_host.so")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    os.makedirs(os.path.dirname(OUT), exist_ok=True)
+    deps = [SRC, os.path.join(CSRC, "alq_numerics.h"), os.path.join(CSRC, "al_tables.inc")]
+    if not os.path.exists(OUT) or any(os.path.getmtime(d) > os.path.getmtime(OUT) for d in deps):
+        tmp = OUT + f".{os.getpid()}"
+        subprocess.run(["g++", "-O2", "-std=c++17", "-ffp-contract=off", "-fno-fast-math",
+                        "-shared", "-fPIC", "-I", CSRC, "-o", tmp, SRC], check=True)
+        os.replace(tmp, OUT)
+    L = C.CDLL(OUT)
+    f32p = np.ctypeslib.ndpointer(np.float32, flags="C_CONTIGUOUS")
+    L.alqn_log2_rn.restype = C.c_float
+    L.alqn_log2_rn.argtypes = [C.c_float]
+    L.alqn_block_params.argtypes = [C.c_float, C.c_float, C.c_float,
+                                    C.POINTER(C.c_float), C.POINTER(C.c_float)]
+    L.alqn_level.argtypes = [C.c_float, C.c_float, C.c_int, C.c_float,
+                             C.POINTER(C.c_float), C.POINTER(C.c_float)]
+    L.alqn_al8_decode.argtypes = [np.ctypeslib.ndpointer(np.uint8), C.c_int64, C.c_float,
+                                  C.c_float, f32p, C.POINTER(C.c_int64)]
+    L.alqn_al_quantize.argtypes = [f32p, C.c_int64, C.c_float, C.c_float, C.c_int,
+                                   np.ctypeslib.ndpointer(np.uint32), C.POINTER(C.c_int64)]
+    return L
+
+
+def test_log2_rn_matches_double_rounding(lib):
+    r = wl.rng(1)
+    xs = np.concatenate([
+        np.exp2(r.uniform(-126, 127, 200000)).astype(np.float32),
+        (1 + r.uniform(-1e-3, 1e-3, 20000)).astype(np.float32),  # near 1
+        np.float32(2.0) ** np.arange(-126, 127, dtype=np.float32),  # exact powers
+        np.array([1e-42, 3e-39, 1.0], np.float32),  # subnormal, tiny, exact 1
+    ])
+    for x in xs:
+        assert lib.alqn_log2_rn(float(x)) == np.float32(math.log2(float(x))), x
+
+
+def test_block_params_match_oracle(lib):
+    r = wl.rng(2)
+    floor_ = np.float32(math.log2(1e-16))
+    for _ in range(20000):
+        x = np.exp2(r.uniform(-70, 20, 8)).astype(np.float32)
+        if r.random() < 0.1:
+            x[:] = x[0]  # degenerate: all equal
+        lm, de, _ = ora.al_block_meta(x, float(floor_))
+        a, b = C.c_float(), C.c_float()
+        lib.alqn_block_params(float(x.min()), float(x.max()), float(floor_), C.byref(a), C.byref(b))
+        assert (np.float32(a.value), np.float32(b.value)) == (lm, de)
+
+
+def test_level_two_float_accuracy(lib):
+    """Table levels: |hi + lo - 2^(l_min + k Delta / 254)| < 2^-44 relative
+    (reference in Python decimal arithmetic)."""
+    from decimal import Decimal, getcontext
+    getcontext().prec = 50
+    ln2 = Decimal(2).ln()
+    r = wl.rng(3)
+    worst = 0.0
+    for _ in range(3000):
+        lmin = np.float32(r.uniform(-96, 40))
+        delta = np.float32(r.uniform(1e-3, min(222.0, 126.0 - float(lmin))))
+        k = int(r.integers(-1, 255))
+        hi, lo = C.c_float(), C.c_float()
+        lib.alqn_level(float(lmin), float(delta), k, 254.0, C.byref(hi), C.byref(lo))
+        y = Decimal(float(lmin)) + Decimal(k) * Decimal(float(delta)) / 254
+        ref = (y * ln2).exp()
+        got = Decimal(hi.value) + Decimal(lo.value)
+        worst = max(worst, float(abs(got - ref) / ref))
+    assert worst < 2.0 ** -44, worst
+
+
+def test_al8_decode_tables_match_oracle(lib):
+    r = wl.rng(4)
+    codes = np.arange(256, dtype=np.uint8)
+    fb_total = C.c_int64(0)
+    n_total = 0
+    for _ in range(4000):
+        lmin = np.float32(r.uniform(-96, 30))
+        delta = np.float32(r.choice([r.uniform(0.01, 2), r.uniform(2, 60),
+                                     r.uniform(60, 120)]))
+        if lmin + delta > 126:
+            continue
+        out = np.zeros(256, np.float32)
+        lib.alqn_al8_decode(codes, 256, float(lmin), float(delta), out, C.byref(fb_total))
+        want = np.array([ora.al_dequantize(int(q), lmin, delta, 8) for q in codes], np.float32)
+        np.testing.assert_array_equal(out.view(np.uint32), want.view(np.uint32))
+        n_total += 256
+    assert fb_total.value < n_total * 1e-4, (fb_total.value, n_total)
+
+
+@pytest.mark.parametrize("bits", [8, 16])
+def test_al_quantize_fast_matches_oracle(lib, bits):
+    r = wl.rng(5 + bits)
+    fb = C.c_int64(0)
+    n_total = 0
+    floor_ = np.float32(math.log2(1e-16))
+    for _ in range(400):
+        spread = float(r.choice([0.5, 5.0, 20.0, 60.0]))
+        x = np.exp2(r.uniform(-40, -40 + spread, 512)).astype(np.float32)
+        x[r.random(512) < 0.05] = 0.0
+        lm, de, _ = ora.al_block_meta(x, float(floor_))
+        q = np.zeros(512, np.uint32)
+        lib.alqn_al_quantize(x, 512, float(lm), float(de), bits, q, C.byref(fb))
+        want = np.array([ora.al_quantize(float(v), lm, de, bits) for v in x], np.uint32)
+        np.testing.assert_array_equal(q, want)
+        n_total += 512
+    limit = 2e-3 if bits == 8 else 0.2  # AL16's 65534 levels exceed fp32 resolution
+    assert fb.value < n_total * limit, (fb.value, n_total)
