@@ -149,6 +149,7 @@ typedef struct {
  *   p        [n] fp32 parameters (read and written).
  *   g        [n] fp32 gradient.
  *   m_codes  [n] int8 UF8 codes, m_absmax [ceil(n/m_block)] fp32.
+ *   m_block, v_block  block sizes, powers of two in [128, 2048].
  *   v_codes  [n] uint8 (v_bits = 8) or uint16 (v_bits = 16) AL codes,
  *   v_meta   [2*ceil(n/v_block)] fp32.
  *   hp       host pointer; t >= 1.

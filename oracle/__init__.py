@@ -84,6 +84,8 @@ _sig("ora_apollo_update_fp32", None, _f32p, _f32p, _i64, _i64, _u16p, _f32p,
 _sig("ora_apollo_step", None, _f32p, _f32p, _i64, _i64, _u16p, _i8p, _f32p,
      _int, _vp, _f32p, _int, _int, C.POINTER(_flt), C.POINTER(ApolloHP), _i64,
      _vp, _vp, _vp)
+_sig("ora_apollo_step_given_R", None, _f32p, _f32p, _i64, _i64, _f32p, _i8p, _f32p, _int,
+     _vp, _f32p, _int, _int, C.POINTER(_flt), C.POINTER(ApolloHP), _i64, _vp)
 _sig("ora_f32_to_bf16", C.c_uint16, _flt)
 _sig("ora_bf16_to_f32", _flt, C.c_uint16)
 _sig("ora_update_error", C.c_double, _f32p, _f32p, _i64, C.c_double)
@@ -273,6 +275,19 @@ def apollo_step(p, g, rows, cols, proj, m_codes, m_absmax, m_block, v_codes,
                          _ptr(s), _ptr(MPf), _ptr(VPf))
     if want_fresh:
         return s, np.float32(pn.value), MPf, VPf
+    return s, np.float32(pn.value)
+
+
+def apollo_step_given_R(p, g, rows, cols, R, m_codes, m_absmax, m_block, v_codes,
+                        v_meta, v_bits, v_block, prev_norm, hp: dict, t: int):
+    """Quantized APOLLO step in place for a given projection R (teacher-forced
+    parity of everything after the projection); returns (scales, prev_norm)."""
+    L = cols if rows <= cols else rows
+    s = np.zeros(L, np.float32)
+    pn = _flt(float(prev_norm))
+    _lib.ora_apollo_step_given_R(p, _f32(g), rows, cols, _f32(R), m_codes, m_absmax,
+                                 m_block, _ptr(v_codes), v_meta, v_bits, v_block,
+                                 C.byref(pn), C.byref(_hp(ApolloHP, hp)), t, _ptr(s))
     return s, np.float32(pn.value)
 
 

@@ -473,15 +473,15 @@ void ora_apollo_project(const float* g, int64_t rows, int64_t cols,
         }
 }
 
-void ora_apollo_update_fp32(float* p, const float* g, int64_t rows,
-                            int64_t cols, const uint16_t* proj, float* MP,
-                            float* VP, float* prev_norm,
-                            const ora_apollo_hp* hp, int64_t t,
-                            float* scale_out) {
+/* Everything after the projection, for a given R [c x rank]. */
+void ora_apollo_update_given_R(float* p, const float* g, int64_t rows,
+                               int64_t cols, const float* R, float* MP,
+                               float* VP, float* prev_norm,
+                               const ora_apollo_hp* hp, int64_t t,
+                               float* scale_out) {
     const int rank = hp->rank;
     const int rows_short = rows <= cols;
     const int64_t L = rows_short ? cols : rows;
-    const int64_t n = rows * cols;
     const double bc1 = 1.0 - pow((double)hp->beta1, (double)t);
     const double bc2 = 1.0 - pow((double)hp->beta2, (double)t);
     const float ic1 = (float)(1.0 / bc1);
@@ -491,10 +491,7 @@ void ora_apollo_update_fp32(float* p, const float* g, int64_t rows,
     const float decay = (float)(1.0 - (double)hp->lr * (double)hp->weight_decay);
     const float lr_a = (float)((double)hp->lr * (double)hp->alpha);
 
-    float* R = (float*)xmalloc(sizeof(float) * (size_t)(L * rank));
     float* s = (float*)xmalloc(sizeof(float) * (size_t)L);
-    ora_apollo_project(g, rows, cols, proj, rank, R);
-
     for (int64_t j = 0; j < L; ++j) {
         double nr = 0.0, ng = 0.0;
         for (int k = 0; k < rank; ++k) {
@@ -539,9 +536,39 @@ void ora_apollo_update_fp32(float* p, const float* g, int64_t rows,
             if (hp->norm_growth_gamma > 0.0f) gt = gt * lim;
             p[k] = p[k] * decay - lr_a * gt;
         }
-    (void)n;
-    free(R);
     free(s);
+}
+
+void ora_apollo_update_fp32(float* p, const float* g, int64_t rows,
+                            int64_t cols, const uint16_t* proj, float* MP,
+                            float* VP, float* prev_norm,
+                            const ora_apollo_hp* hp, int64_t t,
+                            float* scale_out) {
+    const int64_t L = rows <= cols ? cols : rows;
+    float* R = (float*)xmalloc(sizeof(float) * (size_t)(L * hp->rank));
+    ora_apollo_project(g, rows, cols, proj, hp->rank, R);
+    ora_apollo_update_given_R(p, g, rows, cols, R, MP, VP, prev_norm, hp, t, scale_out);
+    free(R);
+}
+
+/* Quantized APOLLO for a given projection R (decode, update, encode). */
+void ora_apollo_step_given_R(float* p, const float* g, int64_t rows,
+                             int64_t cols, const float* R, int8_t* m_codes,
+                             float* m_absmax, int m_block, void* v_codes,
+                             float* v_meta, int v_bits, int v_block,
+                             float* prev_norm, const ora_apollo_hp* hp,
+                             int64_t t, float* scale_out) {
+    const int64_t L = rows <= cols ? cols : rows;
+    const int64_t np = L * hp->rank;
+    float* MP = (float*)xmalloc(sizeof(float) * (size_t)np);
+    float* VP = (float*)xmalloc(sizeof(float) * (size_t)np);
+    ora_uf8_decode(m_codes, m_absmax, np, m_block, MP);
+    ora_al_decode(v_codes, v_meta, np, v_block, v_bits, VP);
+    ora_apollo_update_given_R(p, g, rows, cols, R, MP, VP, prev_norm, hp, t, scale_out);
+    ora_uf8_encode(MP, np, m_block, m_codes, m_absmax);
+    ora_al_encode(VP, np, v_block, v_bits, hp->log_floor, v_codes, v_meta);
+    free(MP);
+    free(VP);
 }
 
 void ora_apollo_step(float* p, const float* g, int64_t rows, int64_t cols,

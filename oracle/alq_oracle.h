@@ -125,6 +125,21 @@ void ora_apollo_update_fp32(float* p, const float* g, int64_t rows,
                             const ora_apollo_hp* hp, int64_t t,
                             float* scale_out);
 
+/* Everything after the projection, for a given R [c x rank] (fp32 states). */
+void ora_apollo_update_given_R(float* p, const float* g, int64_t rows,
+                               int64_t cols, const float* R, float* MP,
+                               float* VP, float* prev_norm,
+                               const ora_apollo_hp* hp, int64_t t,
+                               float* scale_out);
+
+/* Quantized APOLLO for a given projection R. */
+void ora_apollo_step_given_R(float* p, const float* g, int64_t rows,
+                             int64_t cols, const float* R, int8_t* m_codes,
+                             float* m_absmax, int m_block, void* v_codes,
+                             float* v_meta, int v_bits, int v_block,
+                             float* prev_norm, const ora_apollo_hp* hp,
+                             int64_t t, float* scale_out);
+
 /* Quantized APOLLO: UF8 M^P, AL V^P over the flattened [c x rank] arrays. */
 void ora_apollo_step(float* p, const float* g, int64_t rows, int64_t cols,
                      const uint16_t* proj, int8_t* m_codes, float* m_absmax,

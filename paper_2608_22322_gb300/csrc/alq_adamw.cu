@@ -16,18 +16,26 @@
 
 namespace alq {
 
+// Geometry of this kernel: 2 chunks per lane (8 elements), 256-element
+// segments per warp, 2048-element tiles per CTA; blocks of 128..2048.
+constexpr int kCH = 2;
+constexpr int kASeg = 128 * kCH;
+constexpr int kATile = 8 * kASeg;
+
 template <int CPBV, int CPBM, int VBITS>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, 3)
 adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t total_tiles,
                    PlanEntry single, int v_block, int m_block, AdamWScalars s) {
-    constexpr int NBV = 4 / CPBV;
-    constexpr int NBM = 4 / CPBM;
+    constexpr int NBV = kCH / CPBV;
+    constexpr int NBM = kCH / CPBM;
+    constexpr int NE = 4 * kCH;
     constexpr float Lm2 = VBITS == 8 ? 254.0f : 65534.0f;
     __shared__ float2 s_tab[kThreads / 32][NBV * 32];
     __shared__ uint32_t s_part[3][kThreads / 32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int wpbv = v_block > kSeg ? v_block / kSeg : 1;
-    const int wpbm = m_block > kSeg ? m_block / kSeg : 1;
+    const int wpbv = v_block > kASeg ? v_block / kASeg : 1;
+    const int wpbm = m_block > kASeg ? m_block / kASeg : 1;
+    const float kf = al8_table_k(lane);
     int cur = 0;
     for (int64_t tile = blockIdx.x; tile < total_tiles; tile += gridDim.x) {
         PlanEntry d;
@@ -38,21 +46,30 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
             d = single;
         }
         const int64_t n = d.n;
-        const int64_t seg0 = (tile - d.first_tile) * kTile + (int64_t)warp * kSeg;
+        const int64_t seg0 = (tile - d.first_tile) * kATile + (int64_t)warp * kASeg;
 
-        // ---- stream in p, g and the codes of this lane's four chunks
-        float4 g[4], p[4];
-        uint32_t mw[4], vw[4 * VBITS / 8];
+        // ---- stream in p, g and the codes of this lane's chunks
+        const bool full = seg0 + kASeg <= n;  // warp-uniform: unmasked I/O
+        float4 g[kCH], p[kCH];
+        uint32_t mw[kCH], vw[kCH * VBITS / 8];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+        for (int c = 0; c < kCH; ++c) {
             const int64_t idx = chunk_index(seg0, c, lane);
-            g[c] = load4f(d.g, idx, n);
-            p[c] = load4f(d.p, idx, n);
-            mw[c] = load4b((const uint8_t*)d.m_codes, idx, n);
-            if (VBITS == 8) {
-                vw[c] = load4b((const uint8_t*)d.v_codes, idx, n);
+            if (full) {
+                g[c] = __ldcs(reinterpret_cast<const float4*>(d.g + idx));
+                p[c] = __ldcs(reinterpret_cast<const float4*>(d.p + idx));
+                mw[c] = __ldcs(reinterpret_cast<const unsigned int*>(d.m_codes + idx));
             } else {
-                const uint2 h = load4h((const uint16_t*)d.v_codes, idx, n);
+                g[c] = load4f(d.g, idx, n);
+                p[c] = load4f(d.p, idx, n);
+                mw[c] = load4b((const uint8_t*)d.m_codes, idx, n);
+            }
+            if constexpr (VBITS == 8) {
+                vw[c] = full ? __ldcs(reinterpret_cast<const unsigned int*>((const uint8_t*)d.v_codes + idx))
+                             : load4b((const uint8_t*)d.v_codes, idx, n);
+            } else {
+                const uint2 h = full ? __ldcs(reinterpret_cast<const uint2*>((const uint16_t*)d.v_codes + idx))
+                                     : load4h((const uint16_t*)d.v_codes, idx, n);
                 vw[2 * c] = h.x;
                 vw[2 * c + 1] = h.y;
             }
@@ -72,30 +89,36 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
 #pragma unroll
         for (int b = 0; b < NBM; ++b)
             dm[b] = (mb0 + b < nmb) ? __ldg(d.m_absmax + mb0 + b) / 127.0f : 0.0f;
-        if (VBITS == 8) al8_build_tables<NBV>(s_tab[warp], olmin, odelta);
 
-        // ---- decode, update, write p; keep the fresh m and v
-        float mf[16], vf[16];
-        uint32_t cvmin[4], cvmax[4], cmabs[4];
+        // ---- decode the previous states
+        float vh[NE];
+        if constexpr (VBITS == 8) {
+            al8_build_tables<NBV>(s_tab[warp], olmin, odelta, kf);
+            al8_decode_chunks<CPBV, NBV, kCH>(vw, s_tab[warp], olmin, odelta, vh);
+        } else {
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            const int bv = c / CPBV, bm = c / CPBM;
-            const bool fast = al8_fast_ok(olmin[bv], odelta[bv]);
+            for (int e = 0; e < NE; ++e)
+                vh[e] = al16_decode(code_of<VBITS>(vw, e / 4, e % 4), olmin[e / 4 / CPBV],
+                                    odelta[e / 4 / CPBV]);
+        }
+
+        // ---- update, write p; keep the fresh m and v
+        float mf[NE], vf[NE];
+        uint32_t cvmin[kCH], cvmax[kCH], cmabs[kCH];
+#pragma unroll
+        for (int c = 0; c < kCH; ++c) {
+            const int bm = c / CPBM;
             float pn[4];
             cvmin[c] = 0xFFFFFFFFu;
             cvmax[c] = 0u;
             cmabs[c] = 0u;
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
-                const uint32_t qv = code_of<VBITS>(vw, c, i);
-                const float vh = VBITS == 8
-                                     ? al8_decode(qv, s_tab[warp] + 32 * bv, fast, olmin[bv], odelta[bv])
-                                     : al16_decode(qv, olmin[bv], odelta[bv]);
                 const float mh = s8_to_float((mw[c] >> (8 * i)) & 0xFFu) * dm[bm];
                 const float gi = f4get(g[c], i);
                 const float p1 = f4get(p[c], i) * s.decay;
                 const float mm = s.beta1 * mh + s.omb1 * gi;
-                const float vv = s.beta2 * vh + s.omb2 * (gi * gi);
+                const float vv = s.beta2 * vh[4 * c + i] + s.omb2 * (gi * gi);
                 const float den = sqrtf(vv) * s.c2 + s.eps;
                 pn[i] = p1 - s.step * (mm / den);
                 mf[4 * c + i] = mm;
@@ -105,7 +128,12 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
                 cvmax[c] = umix<true>(cvmax[c], vb);
                 cmabs[c] = umix<true>(cmabs[c], f2u(mm) & 0x7FFFFFFFu);
             }
-            store4f(d.p, chunk_index(seg0, c, lane), n, make_float4(pn[0], pn[1], pn[2], pn[3]));
+            const int64_t idx = chunk_index(seg0, c, lane);
+            const float4 pv = make_float4(pn[0], pn[1], pn[2], pn[3]);
+            if (full)
+                __stcs(reinterpret_cast<float4*>(d.p + idx), pv);
+            else
+                store4f(d.p, idx, n, pv);
         }
 
         // ---- new block statistics
@@ -138,23 +166,35 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
         }
 
         // ---- encode and write the codes and block constants
+        uint32_t qv[NE];
+        al_encode_chunks<VBITS, CPBV, NBV, kCH>(vf, nlmin, ndelta, K, E, qv);
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            const int bv = c / CPBV, bm = c / CPBM;
+        for (int c = 0; c < kCH; ++c) {
+            const int bm = c / CPBM;
             const int64_t idx = chunk_index(seg0, c, lane);
-            uint32_t qm = 0, qv[4];
+            uint32_t qm = 0;
+            if (ms[bm] > 0.0f) {
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                if (ms[bm] > 0.0f)
+                for (int i = 0; i < 4; ++i)
                     qm |= ((uint32_t)uf8_quantize(mf[4 * c + i], msc[bm], minv[bm]) & 0xFFu) << (8 * i);
-                qv[i] = al_encode_elem<VBITS>(vf[4 * c + i], nlmin[bv], ndelta[bv], K[bv], E[bv]);
             }
-            store4b((uint8_t*)d.m_codes, idx, n, qm);
-            if (VBITS == 8)
-                store4b((uint8_t*)d.v_codes, idx, n, qv[0] | (qv[1] << 8) | (qv[2] << 16) | (qv[3] << 24));
-            else
-                store4h((uint16_t*)d.v_codes, idx, n,
-                        make_uint2(qv[0] | (qv[1] << 16), qv[2] | (qv[3] << 16)));
+            if (full) {
+                __stcs(reinterpret_cast<unsigned int*>(d.m_codes + idx), qm);
+                if constexpr (VBITS == 8)
+                    __stcs(reinterpret_cast<unsigned int*>((uint8_t*)d.v_codes + idx),
+                           qv[4 * c] | (qv[4 * c + 1] << 8) | (qv[4 * c + 2] << 16) | (qv[4 * c + 3] << 24));
+                else
+                    __stcs(reinterpret_cast<uint2*>((uint16_t*)d.v_codes + idx),
+                           make_uint2(qv[4 * c] | (qv[4 * c + 1] << 16), qv[4 * c + 2] | (qv[4 * c + 3] << 16)));
+            } else {
+                store4b((uint8_t*)d.m_codes, idx, n, qm);
+                if constexpr (VBITS == 8)
+                    store4b((uint8_t*)d.v_codes, idx, n,
+                            qv[4 * c] | (qv[4 * c + 1] << 8) | (qv[4 * c + 2] << 16) | (qv[4 * c + 3] << 24));
+                else
+                    store4h((uint16_t*)d.v_codes, idx, n,
+                            make_uint2(qv[4 * c] | (qv[4 * c + 1] << 16), qv[4 * c + 2] | (qv[4 * c + 3] << 16)));
+            }
         }
         if (lane == 0) {
             if ((warp % wpbv) == 0) {
@@ -174,7 +214,8 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
 }
 
 // ------------------------------------------------------------- dispatch --
-static int cpb_of(int block) { return block >= 512 ? 4 : block / 128; }
+static int cpb_of(int block) { return block >= kASeg ? kCH : block / 128; }
+static bool adamw_block_ok(int block) { return valid_block(block) && block <= kATile; }
 
 template <int CPBV, int CPBM, int VBITS>
 static int launch_adamw_t(const PlanEntry* table, int ntensors, int64_t total_tiles,
@@ -194,9 +235,7 @@ static int launch_adamw_v(int cv, int cm, const PlanEntry* table, int ntensors,
     if (cv == A && cm == B)                                                                 \
         return launch_adamw_t<A, B, VBITS>(table, ntensors, total_tiles, single, v_block, \
                                            m_block, s, st);
-    ALQ_CASE(1, 1) ALQ_CASE(1, 2) ALQ_CASE(1, 4)
-    ALQ_CASE(2, 1) ALQ_CASE(2, 2) ALQ_CASE(2, 4)
-    ALQ_CASE(4, 1) ALQ_CASE(4, 2) ALQ_CASE(4, 4)
+    ALQ_CASE(1, 1) ALQ_CASE(1, 2) ALQ_CASE(2, 1) ALQ_CASE(2, 2)
 #undef ALQ_CASE
     return ALQ_ERR_UNSUPPORTED;
 }
@@ -240,7 +279,7 @@ extern "C" {
 int al_adamw_step(float* p, const float* g, int8_t* m_codes, float* m_absmax, void* v_codes,
                   float* v_meta, int64_t n, int m_block, int v_block, int v_bits,
                   const al_adamw_hp* hp, int64_t t, void* stream) {
-    if (!valid_block(m_block) || !valid_block(v_block) || (v_bits != 8 && v_bits != 16))
+    if (!adamw_block_ok(m_block) || !adamw_block_ok(v_block) || (v_bits != 8 && v_bits != 16))
         return ALQ_ERR_UNSUPPORTED;
     if (t < 1) return ALQ_ERR_INVALID_ARG;
     int st = check_hp(hp);
@@ -249,14 +288,14 @@ int al_adamw_step(float* p, const float* g, int8_t* m_codes, float* m_absmax, vo
     st = check_tensor(e, v_bits);
     if (st) return st;
     if (n == 0) return ALQ_OK;
-    return launch_adamw(nullptr, 1, blocks_of(n, kTile), e, v_block, m_block, v_bits, hp, t,
+    return launch_adamw(nullptr, 1, blocks_of(n, kATile), e, v_block, m_block, v_bits, hp, t,
                         (cudaStream_t)stream);
 }
 
 int al_adamw_plan(const al_adamw_tensor* tensors, int ntensors, int m_block, int v_block,
                   int v_bits, void* plan_host, size_t plan_bytes, al_multi_info* info) {
     if (!tensors || ntensors <= 0 || !plan_host || !info) return ALQ_ERR_INVALID_ARG;
-    if (!valid_block(m_block) || !valid_block(v_block) || (v_bits != 8 && v_bits != 16))
+    if (!adamw_block_ok(m_block) || !adamw_block_ok(v_block) || (v_bits != 8 && v_bits != 16))
         return ALQ_ERR_UNSUPPORTED;
     size_t need = 0;
     al_adamw_plan_bytes(ntensors, &need);
@@ -270,7 +309,7 @@ int al_adamw_plan(const al_adamw_tensor* tensors, int ntensors, int m_block, int
         int st = check_tensor(e, v_bits);
         if (st) return st;
         ent[i] = e;
-        tiles += blocks_of(t.n, kTile);
+        tiles += blocks_of(t.n, kATile);
         elems += t.n;
     }
     memset(h, 0, sizeof(PlanHeader));
@@ -279,7 +318,7 @@ int al_adamw_plan(const al_adamw_tensor* tensors, int ntensors, int m_block, int
     h->m_block = m_block;
     h->v_block = v_block;
     h->v_bits = v_bits;
-    h->tile = kTile;
+    h->tile = kATile;
     h->total_tiles = tiles;
     h->total_elems = elems;
     info->ntensors = ntensors;
@@ -296,7 +335,7 @@ int al_adamw_step_multi(const void* plan_dev, const al_multi_info* info, const a
     if (!plan_dev || !info || t < 1) return ALQ_ERR_INVALID_ARG;
     if (!aligned(plan_dev, 16)) return ALQ_ERR_ALIGN;
     if (info->ntensors <= 0 || info->total_tiles < 0) return ALQ_ERR_INVALID_ARG;
-    if (!valid_block(info->m_block) || !valid_block(info->v_block) ||
+    if (!adamw_block_ok(info->m_block) || !adamw_block_ok(info->v_block) ||
         (info->v_bits != 8 && info->v_bits != 16))
         return ALQ_ERR_UNSUPPORTED;
     int st = check_hp(hp);

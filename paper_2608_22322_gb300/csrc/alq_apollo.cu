@@ -1,0 +1,704 @@
+// alq_apollo.cu -- APOLLO step with quantized projected moments (Sec. 3.1:
+// moments in a low-rank projected space give a channel-wise scale applied to
+// the original gradient; rank 256, channel-wise scaling in Sec. 6.1).
+//
+// Launch sequence of one step:
+//   convert   G (fp32) -> A (bf16, round to nearest even), laid out
+//             [channels][short side] so that the projection's reduction
+//             dimension is contiguous (a tiled transpose when the rows are
+//             the short side, a plain conversion otherwise).
+//   project   R = A * P^T on the tensor cores: TMA loads 128-row tiles of A
+//             and the whole P tile (128-byte swizzle) into a 4-stage shared
+//             memory ring; one thread issues tcgen05.mma (bf16 x bf16 -> fp32)
+//             into a 128 x rank accumulator in tensor memory; the epilogue
+//             reads it back with tcgen05.ld and writes R [channels][rank].
+//   moments   per channel (one quantization block = rank values): decode
+//             UF8 M^P and AL8 V^P, Adam EMAs with bias correction, channel
+//             norms of Rt and R (exact two-float sums) -> s_j, re-encode.
+//   limiter   (optional) ||G s|| and the norm-growth cap.
+//   update    p = p (1 - lr wd) - (lr alpha) g s_j.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "alq_kernels.cuh"
+
+namespace alq {
+
+constexpr int kGM = 128;      // UMMA M (rows of A per CTA)
+constexpr int kGK = 64;       // K per stage (64 bf16 = one 128-byte swizzle row)
+constexpr int kStages = 4;
+constexpr int kAStage = kGM * kGK * 2;     // 16 KB
+constexpr int kBStage = 256 * kGK * 2;     // 32 KB (rank <= 256)
+constexpr int kGemmSmem = kStages * (kAStage + kBStage) + 1024 + 256;
+constexpr uint32_t kWaitLimit = 1u << 26;  // bounded mbarrier polls
+
+// ------------------------------------------------------------ workspace --
+struct ApWs {
+    uint16_t* A;     // [L][s] bf16
+    float* R;        // [L][rank]
+    float* scale;    // [L]
+    double* npart;   // [kMaxNormParts] limiter partials
+    float* lim;      // [2]: limiter factor
+    int* err;        // [1]: projection pipeline timeout flag
+    size_t bytes;
+};
+constexpr int kMaxNormParts = 4096;
+
+static size_t r256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+static ApWs ap_layout(void* base, int64_t rows, int64_t cols, int rank) {
+    const int64_t s = rows <= cols ? rows : cols, L = rows <= cols ? cols : rows;
+    ApWs w;
+    size_t off = 0;
+    char* p = (char*)base;
+    auto take = [&](size_t b) {
+        char* r = p ? p + off : nullptr;
+        off += r256(b);
+        return r;
+    };
+    w.A = (uint16_t*)take(2 * (size_t)L * s);
+    w.R = (float*)take(4 * (size_t)L * rank);
+    w.scale = (float*)take(4 * (size_t)L);
+    w.npart = (double*)take(8 * (size_t)kMaxNormParts);
+    w.lim = (float*)take(8);
+    w.err = (int*)take(4);
+    w.bytes = off;
+    return w;
+}
+
+int al_apollo_workspace(int64_t rows, int64_t cols, int rank, size_t* bytes) {
+    *bytes = ap_layout(nullptr, rows, cols, rank).bytes;
+    return ALQ_OK;
+}
+
+// --------------------------------------------------------------- convert --
+// rows > cols: A[j][i] = bf16(G[j][i]) (channels are rows, K = cols).
+__global__ void __launch_bounds__(kThreads)
+to_bf16_kernel(const float* __restrict__ g, int64_t n, uint16_t* __restrict__ A) {
+    for (int64_t i = 4 * ((int64_t)blockIdx.x * kThreads + threadIdx.x); i < n;
+         i += 4 * (int64_t)gridDim.x * kThreads) {
+        const float4 v = __ldcs(reinterpret_cast<const float4*>(g + i));
+        const uint32_t lo = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.x)) |
+                            ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.y)) << 16);
+        const uint32_t hi = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.z)) |
+                            ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.w)) << 16);
+        *reinterpret_cast<uint2*>(A + i) = make_uint2(lo, hi);
+    }
+}
+
+// rows <= cols: A[j][i] = bf16(G[i][j]) (channels are columns, K = rows),
+// through 32 x 32 shared-memory tiles.
+__global__ void __launch_bounds__(256)
+to_bf16_t_kernel(const float* __restrict__ g, int rows, int cols, uint16_t* __restrict__ A) {
+    __shared__ float t[32][33];
+    const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;  // 32 x 8
+    for (int k = ty; k < 32; k += 8) {
+        const int r = r0 + k, c = c0 + tx;
+        t[k][tx] = (r < rows && c < cols) ? g[(int64_t)r * cols + c] : 0.0f;
+    }
+    __syncthreads();
+    for (int k = ty; k < 32; k += 8) {
+        const int j = c0 + k, i = r0 + tx;  // A row j (channel), column i
+        if (j < cols && i < rows)
+            A[(int64_t)j * rows + i] = __bfloat16_as_ushort(__float2bfloat16_rn(t[tx][k]));
+    }
+}
+
+// ------------------------------------------------------ PTX primitives --
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+// Bounded wait on an mbarrier phase; false after kWaitLimit polls.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+    for (uint32_t i = 0; i < kWaitLimit; ++i) {
+        uint32_t done;
+        asm volatile(
+            "{\n.reg .pred p;\nmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+            "selp.b32 %0, 1, 0, p;\n}\n"
+            : "=r"(done)
+            : "r"(bar), "r"(parity)
+            : "memory");
+        if (done) return true;
+    }
+    return false;
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                            uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major operand tile stored in the
+// 128-byte-swizzled layout TMA writes: rows of 128 bytes, 8-row groups 1024
+// bytes apart (SBO), descriptor version 1, swizzle mode 128B.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
+    uint64_t d = (uint64_t)((addr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)1 << 16;            // LBO (not used by swizzled K-major layouts)
+    d |= (uint64_t)(1024 >> 4) << 32;  // SBO
+    d |= (uint64_t)1 << 46;            // descriptor version
+    d |= (uint64_t)2 << 61;            // 128-byte swizzle
+    return d;
+}
+
+__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                          uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+        "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, "
+        "%28, %29, %30, %31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Instruction descriptor of tcgen05.mma kind::f16: bf16 A and B (K-major),
+// fp32 accumulator, M x N.
+__host__ __device__ constexpr uint32_t umma_idesc_bf16(int M, int N) {
+    return (1u << 4)                         // D format: f32
+           | (1u << 7)                       // A format: bf16
+           | (1u << 10)                      // B format: bf16
+           | ((uint32_t)(N >> 3) << 17)      // N / 8
+           | ((uint32_t)(M >> 4) << 24);     // M / 16
+}
+
+// ---------------------------------------------------------- projection --
+struct GemmArgs {
+    float* R;
+    int L;
+    int rank;
+    int kblocks;
+    int* err;
+};
+
+__global__ void __launch_bounds__(128, 1)
+apollo_project_kernel(const __grid_constant__ CUtensorMap tmA,
+                      const __grid_constant__ CUtensorMap tmB, GemmArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t* sA = smem;
+    uint8_t* sB = smem + kStages * kAStage;
+    uint64_t* bars = (uint64_t*)(sB + kStages * kBStage);  // full[4], empty[4], accum
+    uint32_t* tmem_slot = (uint32_t*)(bars + 2 * kStages + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.x * kGM;
+    const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + kStages);
+    const uint32_t accum = smem_u32(bars + 2 * kStages);
+    const uint32_t ncols = a.rank <= 128 ? 128u : 256u;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(full0 + 8 * s, 1);
+            mbar_init(empty0 + 8 * s, 1);
+        }
+        mbar_init(accum, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(tmem_slot)),
+                     "r"(ncols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = *tmem_slot;
+    const uint32_t b_bytes = (uint32_t)a.rank * kGK * 2;
+
+    bool ok = true;
+    if (warp == 0 && lane == 0) {
+        // TMA producer: stage s is refilled once the MMAs that read it retire
+        for (int kb = 0; kb < a.kblocks && ok; ++kb) {
+            const int s = kb % kStages;
+            if (kb >= kStages) ok = mbar_wait(empty0 + 8 * s, ((kb / kStages) - 1) & 1);
+            if (!ok) break;
+            mbar_expect_tx(full0 + 8 * s, kAStage + b_bytes);
+            tma_load_2d(smem_u32(sA + s * kAStage), &tmA, kb * kGK, m0, full0 + 8 * s);
+            tma_load_2d(smem_u32(sB + s * kBStage), &tmB, kb * kGK, 0, full0 + 8 * s);
+        }
+    } else if (warp == 1 && lane == 0) {
+        // MMA issuer: four K = 16 steps per stage, 32 bytes apart in the row
+        const uint32_t idesc = umma_idesc_bf16(kGM, a.rank);
+        for (int kb = 0; kb < a.kblocks && ok; ++kb) {
+            const int s = kb % kStages;
+            ok = mbar_wait(full0 + 8 * s, (kb / kStages) & 1);
+            if (!ok) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const uint32_t a0 = smem_u32(sA + s * kAStage), b0 = smem_u32(sB + s * kBStage);
+#pragma unroll
+            for (int k = 0; k < kGK / 16; ++k)
+                umma_bf16(tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc,
+                          (kb | k) != 0);
+            umma_commit(empty0 + 8 * s);
+        }
+        if (ok) umma_commit(accum);
+    }
+    if (!ok) atomicExch(a.err, 1);
+    __syncwarp();
+
+    // epilogue: warp w reads TMEM lanes 32w..32w+31 (tile rows), 32 columns
+    // at a time
+    const bool have = mbar_wait(accum, 0);
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const int row = m0 + warp * 32 + lane;
+    if (!have && lane == 0) atomicExch(a.err, 1);
+    for (int c0 = 0; c0 < a.rank; c0 += 32) {
+        float v[32];
+        if (have) {
+            tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = __int_as_float(0x7FC00000);  // NaN marks a failure
+        }
+        if (row < a.L) {
+            float4* dst = reinterpret_cast<float4*>(a.R + (int64_t)row * a.rank + c0);
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+        }
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "r"(ncols)
+                     : "memory");
+}
+
+// ------------------------------------------------------------- moments --
+// Projected Adam moments, one quantization block per channel (block = rank).
+struct MomentArgs {
+    const float* R;
+    int64_t n;  // L * rank
+    int8_t* m_codes;
+    float* m_absmax;
+    void* v_codes;
+    float* v_meta;
+    int block;
+    float* scale;
+    float beta1, beta2, omb1, omb2, ic1, c2, eps, log_floor;
+};
+
+template <int CPB, int VBITS>
+__global__ void __launch_bounds__(kThreads)
+apollo_moments_kernel(MomentArgs m, int64_t ntiles) {
+    constexpr int NB = 4 / CPB;
+    constexpr float Lm2 = VBITS == 8 ? 254.0f : 65534.0f;
+    __shared__ float2 s_tab[kThreads / 32][NB * 32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const float kf = al8_table_k(lane);
+    const int64_t nblk = blocks_of_dev(m.n, m.block);
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
+        const int64_t b0 = seg0 / m.block;
+        float4 r[4];
+        uint32_t mw[4], vw[4 * VBITS / 8];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int64_t idx = chunk_index(seg0, c, lane);
+            r[c] = load4f(m.R, idx, m.n);
+            mw[c] = load4b((const uint8_t*)m.m_codes, idx, m.n);
+            if (VBITS == 8) {
+                vw[c] = load4b((const uint8_t*)m.v_codes, idx, m.n);
+            } else {
+                const uint2 h = load4h((const uint16_t*)m.v_codes, idx, m.n);
+                vw[2 * c] = h.x;
+                vw[2 * c + 1] = h.y;
+            }
+        }
+        float olmin[NB], odelta[NB], dm[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            float2 mt = make_float2(0.f, 0.f);
+            float sa = 0.0f;
+            if (b0 + b < nblk) {
+                mt = __ldg(reinterpret_cast<const float2*>(m.v_meta) + b0 + b);
+                sa = __ldg(m.m_absmax + b0 + b);
+            }
+            olmin[b] = mt.x;
+            odelta[b] = mt.y;
+            dm[b] = sa / 127.0f;
+        }
+        if (VBITS == 8) al8_build_tables<NB>(s_tab[warp], olmin, odelta, kf);
+        float mf[16], vf[16];
+        uint32_t cvmin[4], cvmax[4], cmabs[4];
+        float nrh[NB], nrl[NB], ngh[NB], ngl[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) nrh[b] = nrl[b] = ngh[b] = ngl[b] = 0.0f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int b = c / CPB;
+            const bool fast = al8_fast_ok(olmin[b], odelta[b]);
+            cvmin[c] = 0xFFFFFFFFu;
+            cvmax[c] = 0u;
+            cmabs[c] = 0u;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t qv = code_of<VBITS>(vw, c, i);
+                const float vh = VBITS == 8
+                                     ? al8_decode(qv, s_tab[warp] + 32 * b, fast, olmin[b], odelta[b])
+                                     : al16_decode(qv, olmin[b], odelta[b]);
+                const float mh = s8_to_float((mw[c] >> (8 * i)) & 0xFFu) * dm[b];
+                const float rv = f4get(r[c], i);
+                const float mq = m.beta1 * mh + m.omb1 * rv;
+                const float vq = m.beta2 * vh + m.omb2 * (rv * rv);
+                const float rt = (mq * m.ic1) / (sqrtf(vq) * m.c2 + m.eps);
+                mf[4 * c + i] = mq;
+                vf[4 * c + i] = vq;
+                float h, l;
+                two_prod(rt, rt, h, l);
+                ff_acc(nrh[b], nrl[b], h, l);
+                two_prod(rv, rv, h, l);
+                ff_acc(ngh[b], ngl[b], h, l);
+                const uint32_t vb = f2u(vq);
+                cvmin[c] = umix<false>(cvmin[c], vb - 1u);
+                cvmax[c] = umix<true>(cvmax[c], vb);
+                cmabs[c] = umix<true>(cmabs[c], f2u(mq) & 0x7FFFFFFFu);
+            }
+        }
+        uint32_t bvmin[NB], bvmax[NB], bmabs[NB];
+        warp_blocks_reduce<CPB, false>(cvmin, bvmin);
+        warp_blocks_reduce<CPB, true>(cvmax, bvmax);
+        warp_blocks_reduce<CPB, true>(cmabs, bmabs);
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            ff_warp_sum(nrh[b], nrl[b]);
+            ff_warp_sum(ngh[b], ngl[b]);
+        }
+        float vmn[NB], vmx[NB], nlmin[NB], ndelta[NB], K[NB], E[NB], ms[NB], sc[NB], inv[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            vmn[b] = u2f(bvmin[b] + 1u);
+            vmx[b] = u2f(bvmax[b]);
+            ms[b] = u2f(bmabs[b]);
+            sc[b] = 1.0f;
+            inv[b] = 0.0f;
+            if (ms[b] > 0.0f) uf8_encode_consts(ms[b], sc[b], inv[b]);
+        }
+        al_blocks_params<NB>(vmn, vmx, m.log_floor, nlmin, ndelta);
+#pragma unroll
+        for (int b = 0; b < NB; ++b) al_encode_consts(ndelta[b], Lm2, K[b], E[b]);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int b = c / CPB;
+            const int64_t idx = chunk_index(seg0, c, lane);
+            uint32_t qm = 0, qv[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                if (ms[b] > 0.0f)
+                    qm |= ((uint32_t)uf8_quantize(mf[4 * c + i], sc[b], inv[b]) & 0xFFu) << (8 * i);
+                qv[i] = al_encode_elem<VBITS>(vf[4 * c + i], nlmin[b], ndelta[b], K[b], E[b]);
+            }
+            store4b((uint8_t*)m.m_codes, idx, m.n, qm);
+            if (VBITS == 8)
+                store4b((uint8_t*)m.v_codes, idx, m.n, qv[0] | (qv[1] << 8) | (qv[2] << 16) | (qv[3] << 24));
+            else
+                store4h((uint16_t*)m.v_codes, idx, m.n,
+                        make_uint2(qv[0] | (qv[1] << 16), qv[2] | (qv[3] << 16)));
+        }
+        if (lane == 0) {
+#pragma unroll
+            for (int b = 0; b < NB; ++b) {
+                if (b0 + b >= nblk) continue;
+                reinterpret_cast<float2*>(m.v_meta)[b0 + b] = make_float2(nlmin[b], ndelta[b]);
+                m.m_absmax[b0 + b] = ms[b];
+                const double nr = (double)nrh[b] + (double)nrl[b];
+                const double ng = (double)ngh[b] + (double)ngl[b];
+                m.scale[b0 + b] = (float)(sqrt(nr) / (sqrt(ng) + 1e-8));
+            }
+        }
+        __syncwarp();
+    }
+}
+
+// ------------------------------------------------------ limiter, update --
+struct ApUpdateArgs {
+    float* p;
+    const float* g;
+    int64_t n;
+    Divider dv;
+    int rows_short;  // 1: channel = column; 0: channel = row
+    const float* scale;
+    const float* lim;  // nullptr when the limiter is off
+    float decay, lr_a;
+};
+
+__global__ void __launch_bounds__(kThreads)
+apollo_gnorm_kernel(ApUpdateArgs u, int64_t ntiles, double* __restrict__ part) {
+    __shared__ double s_w[kThreads / 32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float hi = 0.0f, lo = 0.0f;
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int64_t idx = chunk_index(seg0, c, lane);
+            if (idx >= u.n) continue;
+            const uint32_t row = divide((uint32_t)idx, u.dv);
+            const uint32_t col = (uint32_t)idx - row * u.dv.d;
+            const float4 gv = __ldcs(reinterpret_cast<const float4*>(u.g + idx));
+            float4 sv;
+            if (u.rows_short) {
+                sv = __ldg(reinterpret_cast<const float4*>(u.scale + col));
+            } else {
+                const float s = __ldg(u.scale + row);
+                sv = make_float4(s, s, s, s);
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const float gt = f4get(gv, j) * f4get(sv, j);
+                float h, l;
+                two_prod(gt, gt, h, l);
+                ff_acc(hi, lo, h, l);
+            }
+        }
+    }
+    ff_warp_sum(hi, lo);
+    if (lane == 0) s_w[warp] = (double)hi + (double)lo;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double s = 0.0;
+        for (int w = 0; w < kThreads / 32; ++w) s += s_w[w];
+        part[blockIdx.x] = s;
+    }
+}
+
+__global__ void apollo_limit_kernel(const double* __restrict__ part, int nparts, float gamma,
+                                    float* __restrict__ prev_norm, float* __restrict__ lim) {
+    if (threadIdx.x != 0) return;
+    double ss = 0.0;
+    for (int i = 0; i < nparts; ++i) ss += part[i];
+    const double nt = sqrt(ss);
+    const double prev = (double)*prev_norm;
+    const double cap = (double)gamma * prev;
+    if (prev > 0.0 && nt > cap) {
+        lim[0] = (float)(cap / nt);
+        *prev_norm = (float)cap;
+    } else {
+        lim[0] = 1.0f;
+        *prev_norm = (float)nt;
+    }
+}
+
+__global__ void __launch_bounds__(kThreads)
+apollo_update_kernel(ApUpdateArgs u, int64_t ntiles) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const float lim = u.lim ? __ldg(u.lim) : 1.0f;
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int64_t idx = chunk_index(seg0, c, lane);
+            if (idx >= u.n) continue;
+            const uint32_t row = divide((uint32_t)idx, u.dv);
+            const uint32_t col = (uint32_t)idx - row * u.dv.d;
+            const float4 gv = __ldcs(reinterpret_cast<const float4*>(u.g + idx));
+            const float4 pv = __ldcs(reinterpret_cast<const float4*>(u.p + idx));
+            float4 sv;
+            if (u.rows_short) {
+                sv = __ldg(reinterpret_cast<const float4*>(u.scale + col));
+            } else {
+                const float s = __ldg(u.scale + row);
+                sv = make_float4(s, s, s, s);
+            }
+            float pn[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                float gt = f4get(gv, j) * f4get(sv, j);
+                if (u.lim) gt = gt * lim;
+                pn[j] = f4get(pv, j) * u.decay - u.lr_a * gt;
+            }
+            __stcs(reinterpret_cast<float4*>(u.p + idx), make_float4(pn[0], pn[1], pn[2], pn[3]));
+        }
+    }
+}
+
+// ------------------------------------------------------------- host side --
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static std::mutex mu;
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (PFN_cuTensorMapEncodeTiled_v12000)p;
+    }
+    return fn;
+}
+
+// 2-D bf16 tensor map over a row-major [rows][k] matrix, box [box_rows][64],
+// 128-byte swizzle, zero fill out of bounds.
+static bool make_map(CUtensorMap* map, const void* base, uint64_t k, uint64_t rows,
+                     uint32_t box_rows) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {k, rows};
+    const cuuint64_t strides[1] = {k * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)kGK, box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+static int launch_project(const uint16_t* A, const uint16_t* P, int64_t L, int64_t s, int rank,
+                          float* R, int* err, cudaStream_t st) {
+    CUtensorMap ma, mb;
+    if (!make_map(&ma, A, (uint64_t)s, (uint64_t)L, kGM) ||
+        !make_map(&mb, P, (uint64_t)s, (uint64_t)rank, (uint32_t)rank))
+        return record_cuda(cudaErrorInvalidValue);
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [] {
+        attr_err = cudaFuncSetAttribute(apollo_project_kernel,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);
+    });
+    if (attr_err != cudaSuccess) return record_cuda(attr_err);
+    GemmArgs a{R, (int)L, rank, (int)blocks_of(s, kGK), err};
+    apollo_project_kernel<<<(unsigned)blocks_of(L, kGM), 128, kGemmSmem, st>>>(ma, mb, a);
+    return check_launch();
+}
+
+template <int CPB, int VBITS>
+static void launch_moments_t(const MomentArgs& m, cudaStream_t st) {
+    const int64_t ntiles = blocks_of(m.n, kTile);
+    auto k = apollo_moments_kernel<CPB, VBITS>;
+    k<<<persistent_grid((const void*)k, kThreads, 0, ntiles), kThreads, 0, st>>>(m, ntiles);
+}
+
+}  // namespace alq
+
+using namespace alq;
+
+extern "C" int al_apollo_step(float* p, const float* g, int64_t rows, int64_t cols,
+                              const uint16_t* proj, int8_t* m_codes, float* m_absmax, int m_block,
+                              void* v_codes, float* v_meta, int v_bits, int v_block,
+                              float* prev_norm, const al_apollo_hp* hp, int64_t t,
+                              void* workspace, size_t ws_bytes, void* stream) {
+    if (!p || !g || !proj || !m_codes || !m_absmax || !v_codes || !v_meta || !hp || t < 1 ||
+        rows < 1 || cols < 1)
+        return ALQ_ERR_INVALID_ARG;
+    const int rank = hp->rank;
+    const int64_t s = rows <= cols ? rows : cols, L = rows <= cols ? cols : rows;
+    if ((rank != 128 && rank != 256) || m_block != rank || v_block != rank ||
+        (v_bits != 8 && v_bits != 16) || cols % 4 != 0 || s % 8 != 0 ||
+        rows * cols >= (int64_t)1 << 31 || L > (1 << 30))
+        return ALQ_ERR_UNSUPPORTED;
+    if (hp->norm_growth_gamma > 0.0f && !prev_norm) return ALQ_ERR_INVALID_ARG;
+    if (!aligned(p, 16) || !aligned(g, 16) || !aligned(proj, 16) || !aligned(m_codes, 16) ||
+        !aligned(v_codes, 16) || !aligned(v_meta, 8) || !aligned(m_absmax, 4))
+        return ALQ_ERR_ALIGN;
+    const ApWs w = ap_layout(workspace, rows, cols, rank);
+    if (!workspace || ws_bytes < w.bytes || !aligned(workspace, 256)) return ALQ_ERR_WORKSPACE;
+    cudaStream_t st = (cudaStream_t)stream;
+    const int rows_short = rows <= cols;
+
+    // bf16 operand with the short side contiguous
+    if (rows_short) {
+        dim3 grid((unsigned)blocks_of(cols, 32), (unsigned)blocks_of(rows, 32));
+        to_bf16_t_kernel<<<grid, 256, 0, st>>>(g, (int)rows, (int)cols, w.A);
+    } else {
+        const int64_t n = rows * cols;
+        int grid = (int)blocks_of(n / 4, kThreads);
+        if (grid > 8 * sm_count()) grid = 8 * sm_count();
+        to_bf16_kernel<<<grid, kThreads, 0, st>>>(g, n, w.A);
+    }
+    int rc = check_launch();
+    if (rc) return rc;
+    rc = launch_project(w.A, proj, L, s, rank, w.R, w.err, st);
+    if (rc) return rc;
+
+    const double bc1 = 1.0 - pow((double)hp->beta1, (double)t);
+    const double bc2 = 1.0 - pow((double)hp->beta2, (double)t);
+    MomentArgs m;
+    m.R = w.R;
+    m.n = L * rank;
+    m.m_codes = m_codes;
+    m.m_absmax = m_absmax;
+    m.v_codes = v_codes;
+    m.v_meta = v_meta;
+    m.block = rank;
+    m.scale = w.scale;
+    m.beta1 = hp->beta1;
+    m.beta2 = hp->beta2;
+    m.omb1 = (float)(1.0 - (double)hp->beta1);
+    m.omb2 = (float)(1.0 - (double)hp->beta2);
+    m.ic1 = (float)(1.0 / bc1);
+    m.c2 = (float)(1.0 / sqrt(bc2));
+    m.eps = hp->eps;
+    m.log_floor = hp->log_floor;
+    if (rank == 128) {
+        if (v_bits == 8) launch_moments_t<1, 8>(m, st); else launch_moments_t<1, 16>(m, st);
+    } else {
+        if (v_bits == 8) launch_moments_t<2, 8>(m, st); else launch_moments_t<2, 16>(m, st);
+    }
+    rc = check_launch();
+    if (rc) return rc;
+
+    ApUpdateArgs u;
+    u.p = p;
+    u.g = g;
+    u.n = rows * cols;
+    u.dv = make_divider((uint32_t)cols);
+    u.rows_short = rows_short;
+    u.scale = w.scale;
+    u.lim = nullptr;
+    u.decay = (float)(1.0 - (double)hp->lr * (double)hp->weight_decay);
+    u.lr_a = (float)((double)hp->lr * (double)hp->alpha);
+    const int64_t ntiles = blocks_of(u.n, kTile);
+    if (hp->norm_growth_gamma > 0.0f) {
+        int grid = persistent_grid((const void*)apollo_gnorm_kernel, kThreads, 0, ntiles);
+        if (grid > kMaxNormParts) grid = kMaxNormParts;
+        apollo_gnorm_kernel<<<grid, kThreads, 0, st>>>(u, ntiles, w.npart);
+        apollo_limit_kernel<<<1, 32, 0, st>>>(w.npart, grid, hp->norm_growth_gamma, prev_norm,
+                                               w.lim);
+        u.lim = w.lim;
+    }
+    apollo_update_kernel<<<persistent_grid((const void*)apollo_update_kernel, kThreads, 0, ntiles),
+                           kThreads, 0, st>>>(u, ntiles);
+    return check_launch();
+}

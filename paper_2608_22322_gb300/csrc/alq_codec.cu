@@ -86,6 +86,7 @@ al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta,
     constexpr int NB = 4 / CPB;
     __shared__ float2 s_tab[kThreads / 32][NB * 32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const float kf = al8_table_k(lane);
     const int64_t nblk = blocks_of_dev(n, block);
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
@@ -110,7 +111,7 @@ al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta,
             lmin[b] = mt.x;
             delta[b] = mt.y;
         }
-        if (BITS == 8) al8_build_tables<NB>(s_tab[warp], lmin, delta);
+        if (BITS == 8) al8_build_tables<NB>(s_tab[warp], lmin, delta, kf);
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
             const int b = c / CPB;

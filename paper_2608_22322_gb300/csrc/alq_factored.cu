@@ -1,31 +1,636 @@
-// alq_factored.cu -- Adafactor / CAME / APOLLO steps and their workspace sizes.
-#include "alq_internal.h"
+// alq_factored.cu -- Adafactor and CAME steps with AL-coded factored states
+// (Sec. 3.1: row/column statistics reconstruct the second moment; CAME adds
+// factored confidence states tracking a residual) and UF8 momentum.
+//
+// Launch sequence of one step (all on the caller's stream, no host sync):
+//   sumsq      G read once: per 64-row x 512-column tile, exact float-float
+//              sums of g^2 per row (over the tile's columns) and per column
+//              (over its rows) -> fp64 partials in the workspace.
+//   factor     one CTA per factor block: finish r_i / c_j (fp64, fixed order),
+//              decode the old factor, EMA, AL-encode the fresh factor.
+//   scale      a_i = 1/sqrt(R_i / mean(R)), b_j = 1/sqrt(C_j).
+//   usq        G read again: u = (g a_i) b_j, exact float-float sum of u^2,
+//              one fp64 partial per CTA of a persistent grid (fixed order).
+//   clip       1 / max(1, RMS(u) / d).
+//   update     G read a third time: u_hat, optional UF8 momentum, p update.
+// CAME inserts, before its update, a second sumsq pass over the residual
+// (u_hat - m)^2 + eps2 (recomputing m from the old momentum codes), a second
+// factor pass (confidence, beta3) and a second scale pass; its update uses
+// m / sqrt(S) with S from the confidence factors.
+// Every reduction is deterministic: error-free fp32 transforms inside a
+// thread, fixed shuffle and tree orders, fp64 merges; no float atomics.
+#include "alq_kernels.cuh"
+
+namespace alq {
+
+constexpr int kFR = 64;   // rows per sumsq tile
+constexpr int kFC = 512;  // columns per sumsq tile
+constexpr int kMaxParts = 4096;
+
+// ------------------------------------------------------------ workspace --
+struct FacWs {
+    double* rowpart;  // [ncb][rows]
+    double* colpart;  // [nrb][cols]
+    double* upart;    // [kMaxParts]
+    float* fr;        // fresh row factor (V)
+    float* fc;        // fresh column factor (V)
+    float* fr2;       // fresh row factor (C)
+    float* fc2;       // fresh column factor (C)
+    float* a;         // [rows]
+    float* b;         // [cols]
+    float* a2;        // [rows]
+    float* b2;        // [cols]
+    float* scal;      // [4]: icf
+    size_t bytes;
+};
+
+static size_t round256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+static FacWs fac_layout(void* base, int64_t rows, int64_t cols) {
+    const int64_t ncb = blocks_of(cols, kFC), nrb = blocks_of(rows, kFR);
+    FacWs w;
+    size_t off = 0;
+    char* p = (char*)base;
+    auto take = [&](size_t bytes) {
+        char* r = p ? p + off : nullptr;
+        off += round256(bytes);
+        return r;
+    };
+    w.rowpart = (double*)take(sizeof(double) * ncb * rows);
+    w.colpart = (double*)take(sizeof(double) * nrb * cols);
+    w.upart = (double*)take(sizeof(double) * kMaxParts);
+    w.fr = (float*)take(sizeof(float) * rows);
+    w.fc = (float*)take(sizeof(float) * cols);
+    w.fr2 = (float*)take(sizeof(float) * rows);
+    w.fc2 = (float*)take(sizeof(float) * cols);
+    w.a = (float*)take(sizeof(float) * rows);
+    w.b = (float*)take(sizeof(float) * cols);
+    w.a2 = (float*)take(sizeof(float) * rows);
+    w.b2 = (float*)take(sizeof(float) * cols);
+    w.scal = (float*)take(sizeof(float) * 4);
+    w.bytes = off;
+    return w;
+}
+
+// ------------------------------------------------------------ residual --
+// CAME's residual inputs: old momentum codes, scales, clip factor.
+struct ResidualArgs {
+    const int8_t* m_codes;
+    const float* m_absmax;
+    int m_shift;  // log2(m_block)
+    const float* a;
+    const float* b;
+    const float* scal;  // scal[0] = 1 / max(1, RMS(u)/d)
+    float beta1, omb1, eps2;
+};
+
+// ----------------------------------------------------------------- sumsq --
+// MODE 0: terms g^2 (exact two-float squares). MODE 1: terms CAME's
+// residual (u_hat - m)^2 + eps2 rounded to fp32 as the update defines it.
+template <int MODE>
+__global__ void __launch_bounds__(kThreads)
+sumsq_kernel(const float* __restrict__ g, int rows, int cols, ResidualArgs ra,
+             double* __restrict__ rowpart, double* __restrict__ colpart) {
+    __shared__ double s_col[kThreads / 32][kFC];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int c0 = blockIdx.x * kFC, r0 = blockIdx.y * kFR;
+    float ch[16], cl[16];
+#pragma unroll
+    for (int k = 0; k < 16; ++k) ch[k] = cl[k] = 0.0f;
+    float icf = 0.0f;
+    if (MODE == 1) icf = __ldg(ra.scal);
+    for (int rr = 0; rr < kFR / 8; ++rr) {
+        const int row = r0 + warp + 8 * rr;
+        float rh = 0.0f, rl = 0.0f;
+        if (row < rows) {
+            float ai = 0.0f;
+            if (MODE == 1) ai = __ldg(ra.a + row);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int col = c0 + 128 * k + 4 * lane;
+                if (col < cols) {
+                    const int64_t idx = (int64_t)row * cols + col;
+                    const float4 gv = __ldcs(reinterpret_cast<const float4*>(g + idx));
+                    float4 bv;
+                    uint32_t mw = 0;
+                    float dm = 0.0f;
+                    if (MODE == 1) {
+                        bv = __ldg(reinterpret_cast<const float4*>(ra.b + col));
+                        mw = __ldcs(reinterpret_cast<const unsigned int*>(ra.m_codes + idx));
+                        dm = __ldg(ra.m_absmax + (idx >> ra.m_shift)) / 127.0f;
+                    }
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const float x = f4get(gv, j);
+                        float h, l;
+                        if (MODE == 0) {
+                            two_prod(x, x, h, l);
+                        } else {
+                            const float u = (x * ai) * f4get(bv, j);
+                            const float uh = u * icf;
+                            const float mh = s8_to_float((mw >> (8 * j)) & 0xFFu) * dm;
+                            const float mk = ra.beta1 * mh + ra.omb1 * uh;
+                            const float d = uh - mk;
+                            h = d * d + ra.eps2;
+                            l = 0.0f;
+                        }
+                        ff_acc(ch[4 * k + j], cl[4 * k + j], h, l);
+                        ff_acc(rh, rl, h, l);
+                    }
+                }
+            }
+        }
+        ff_warp_sum(rh, rl);
+        if (lane == 0 && row < rows)
+            rowpart[(int64_t)blockIdx.x * rows + row] = (double)rh + (double)rl;
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            s_col[warp][128 * k + 4 * lane + j] = (double)ch[4 * k + j] + (double)cl[4 * k + j];
+    __syncthreads();
+    for (int t = threadIdx.x; t < kFC; t += kThreads) {
+        if (c0 + t >= cols) continue;
+        double s = 0.0;
+#pragma unroll
+        for (int w = 0; w < kThreads / 32; ++w) s += s_col[w][t];
+        colpart[(int64_t)blockIdx.y * cols + c0 + t] = s;
+    }
+}
+
+// ---------------------------------------------------------------- factor --
+// One factor vector's update: stat_i = sum_p part[p][i] / mean_len + add_eps
+// (fp64, fixed order, rounded once), fresh = beta * decode(old) + omb * stat,
+// then AL re-encoding of each block.
+struct FactorDesc {
+    const double* part;
+    int nparts;
+    int64_t len;
+    double mean_len;
+    double add_eps;
+    float beta, omb;
+    void* codes;
+    float* meta;
+    int bits;
+    int block;
+    float log_floor;
+    float* fresh;
+};
+
+__device__ __forceinline__ uint32_t fac_code(const FactorDesc& f, int64_t i) {
+    return f.bits == 8 ? (uint32_t)((const uint8_t*)f.codes)[i] : (uint32_t)((const uint16_t*)f.codes)[i];
+}
+
+__global__ void __launch_bounds__(kThreads)
+factor_kernel(FactorDesc f0, FactorDesc f1, int nb0) {
+    __shared__ uint32_t s_part[2][kThreads / 32];
+    const bool first = (int)blockIdx.x < nb0;
+    const FactorDesc& f = first ? f0 : f1;
+    const int64_t b = first ? blockIdx.x : blockIdx.x - nb0;
+    const int64_t lo = b * f.block;
+    const int64_t hi = lo + f.block < f.len ? lo + f.block : f.len;
+    const float2 om = __ldg(reinterpret_cast<const float2*>(f.meta) + b);
+    const float Lm2 = f.bits == 8 ? 254.0f : 65534.0f;
+    float v[16];
+    uint32_t vmin = 0xFFFFFFFFu, vmax = 0u;
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+        const int64_t i = lo + threadIdx.x + (int64_t)kThreads * k;
+        v[k] = 0.0f;
+        if (i < hi) {
+            double s = 0.0;
+            for (int p = 0; p < f.nparts; ++p) s += f.part[(int64_t)p * f.len + i];
+            const float stat = (float)(s / f.mean_len + f.add_eps);
+            const float old = al_decode_direct(fac_code(f, i), om.x, om.y, Lm2);
+            v[k] = f.beta * old + f.omb * stat;
+            f.fresh[i] = v[k];
+            const uint32_t vb = f2u(v[k]);
+            vmin = umix<false>(vmin, vb - 1u);
+            vmax = umix<true>(vmax, vb);
+        }
+    }
+    vmin = __reduce_min_sync(0xFFFFFFFFu, vmin);
+    vmax = __reduce_max_sync(0xFFFFFFFFu, vmax);
+    vmin = cta_group_reduce<false>(vmin, s_part[0], kThreads / 32);
+    vmax = cta_group_reduce<true>(vmax, s_part[1], kThreads / 32);
+    float lmin, delta, K, E;
+    al_block_params(u2f(vmin + 1u), u2f(vmax), f.log_floor, lmin, delta);
+    al_encode_consts(delta, Lm2, K, E);
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+        const int64_t i = lo + threadIdx.x + (int64_t)kThreads * k;
+        if (i < hi) {
+            uint32_t q = 0;
+            if (v[k] != 0.0f) {
+                bool fb;
+                q = al_quantize_fast(v[k], lmin, K, E, Lm2, fb);
+                if (fb) q = al_quantize_fp64(v[k], lmin, delta, (double)Lm2);
+            }
+            if (f.bits == 8)
+                ((uint8_t*)f.codes)[i] = (uint8_t)q;
+            else
+                ((uint16_t*)f.codes)[i] = (uint16_t)q;
+        }
+    }
+    if (threadIdx.x == 0) reinterpret_cast<float2*>(f.meta)[b] = make_float2(lmin, delta);
+}
+
+// ----------------------------------------------------------------- scale --
+// a_i = 1/sqrt(R_i / mean(R)), b_j = 1/sqrt(C_j); mean(R) in fp64 with a fixed
+// tree order, rounded once.
+__global__ void __launch_bounds__(1024)
+scale_kernel(const float* __restrict__ R, int rows, const float* __restrict__ C, int cols,
+             float* __restrict__ a, float* __restrict__ b) {
+    __shared__ double s[1024];
+    double acc = 0.0;
+    for (int i = threadIdx.x; i < rows; i += 1024) acc += (double)R[i];
+    s[threadIdx.x] = acc;
+    __syncthreads();
+    for (int st = 512; st > 0; st >>= 1) {
+        if ((int)threadIdx.x < st) s[threadIdx.x] += s[threadIdx.x + st];
+        __syncthreads();
+    }
+    const float meanR = (float)(s[0] / (double)rows);
+    for (int i = threadIdx.x; i < rows; i += 1024) a[i] = 1.0f / sqrtf(R[i] / meanR);
+    for (int j = threadIdx.x; j < cols; j += 1024) b[j] = 1.0f / sqrtf(C[j]);
+}
+
+// ------------------------------------------------------------------- usq --
+// Sum of u^2, u = (g a_i) b_j, over the whole matrix: exact squares in
+// two-float per thread, fixed warp/CTA order, one fp64 partial per CTA.
+__global__ void __launch_bounds__(kThreads)
+usq_kernel(const float* __restrict__ g, int64_t n, Divider dv, const float* __restrict__ a,
+           const float* __restrict__ b, int64_t ntiles, double* __restrict__ upart) {
+    __shared__ double s_w[kThreads / 32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float hi = 0.0f, lo = 0.0f;
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int64_t idx = chunk_index(seg0, c, lane);
+            if (idx < n) {
+                const uint32_t row = divide((uint32_t)idx, dv);
+                const uint32_t col = (uint32_t)idx - row * dv.d;
+                const float4 gv = __ldcs(reinterpret_cast<const float4*>(g + idx));
+                const float4 bv = __ldg(reinterpret_cast<const float4*>(b + col));
+                const float ai = __ldg(a + row);
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float u = (f4get(gv, j) * ai) * f4get(bv, j);
+                    float h, l;
+                    two_prod(u, u, h, l);
+                    ff_acc(hi, lo, h, l);
+                }
+            }
+        }
+    }
+    ff_warp_sum(hi, lo);
+    if (lane == 0) s_w[warp] = (double)hi + (double)lo;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double s = 0.0;
+        for (int w = 0; w < kThreads / 32; ++w) s += s_w[w];
+        upart[blockIdx.x] = s;
+    }
+}
+
+// ------------------------------------------------------------------ clip --
+__global__ void __launch_bounds__(1024)
+clip_kernel(const double* __restrict__ upart, int nparts, double count, float clip_d,
+            float* __restrict__ scal) {
+    __shared__ double s[1024];
+    double acc = 0.0;
+    for (int i = threadIdx.x; i < nparts; i += 1024) acc += upart[i];
+    s[threadIdx.x] = acc;
+    __syncthreads();
+    for (int st = 512; st > 0; st >>= 1) {
+        if ((int)threadIdx.x < st) s[threadIdx.x] += s[threadIdx.x + st];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+        const double rms = sqrt(s[0] / count);
+        double cf = rms / (double)clip_d;
+        if (cf < 1.0) cf = 1.0;
+        scal[0] = (float)(1.0 / cf);
+    }
+}
+
+// ---------------------------------------------------------------- update --
+// MODE 0: Adafactor without momentum; 1: Adafactor with UF8 momentum;
+// 2: CAME (UF8 momentum, p -= lr (m a2_i) b2_j).
+struct UpdateArgs {
+    float* p;
+    const float* g;
+    int64_t n;
+    Divider dv;
+    const float* a;
+    const float* b;
+    const float* a2;
+    const float* b2;
+    const float* scal;
+    int8_t* m_codes;
+    float* m_absmax;
+    int m_block;
+    float beta1, omb1, decay, lr;
+};
+
+template <int MODE, int CPBM>
+__global__ void __launch_bounds__(kThreads)
+update_kernel(UpdateArgs u, int64_t ntiles) {
+    constexpr int NBM = 4 / CPBM;
+    __shared__ uint32_t s_part[kThreads / 32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int wpbm = u.m_block > kSeg ? u.m_block / kSeg : 1;
+    const float icf = __ldg(u.scal);
+    const int64_t nmb = blocks_of_dev(u.n, u.m_block);
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
+        const int64_t mb0 = seg0 / u.m_block;
+        float dm[NBM];
+#pragma unroll
+        for (int b = 0; b < NBM; ++b)
+            dm[b] = (MODE > 0 && mb0 + b < nmb) ? __ldg(u.m_absmax + mb0 + b) / 127.0f : 0.0f;
+        float mf[16];
+        uint32_t cabs[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int64_t idx = chunk_index(seg0, c, lane);
+            cabs[c] = 0u;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) mf[4 * c + j] = 0.0f;
+            if (idx >= u.n) continue;
+            const uint32_t row = divide((uint32_t)idx, u.dv);
+            const uint32_t col = (uint32_t)idx - row * u.dv.d;
+            const float4 gv = __ldcs(reinterpret_cast<const float4*>(u.g + idx));
+            const float4 pv = __ldcs(reinterpret_cast<const float4*>(u.p + idx));
+            const float4 bv = __ldg(reinterpret_cast<const float4*>(u.b + col));
+            const float ai = __ldg(u.a + row);
+            uint32_t mw = 0;
+            float4 b2v = make_float4(0.f, 0.f, 0.f, 0.f);
+            float a2i = 0.0f;
+            if (MODE > 0) mw = __ldcs(reinterpret_cast<const unsigned int*>(u.m_codes + idx));
+            if (MODE == 2) {
+                b2v = __ldg(reinterpret_cast<const float4*>(u.b2 + col));
+                a2i = __ldg(u.a2 + row);
+            }
+            float pn[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const float uu = (f4get(gv, j) * ai) * f4get(bv, j);
+                const float uh = uu * icf;
+                float upd = uh;
+                if (MODE > 0) {
+                    const float mh = s8_to_float((mw >> (8 * j)) & 0xFFu) * dm[c / CPBM];
+                    const float mk = u.beta1 * mh + u.omb1 * uh;
+                    mf[4 * c + j] = mk;
+                    cabs[c] = umix<true>(cabs[c], f2u(mk) & 0x7FFFFFFFu);
+                    upd = MODE == 2 ? (mk * a2i) * f4get(b2v, j) : mk;
+                }
+                pn[j] = f4get(pv, j) * u.decay - u.lr * upd;
+            }
+            __stcs(reinterpret_cast<float4*>(u.p + idx), make_float4(pn[0], pn[1], pn[2], pn[3]));
+        }
+        if (MODE == 0) continue;
+        uint32_t babs[NBM];
+        warp_blocks_reduce<CPBM, true>(cabs, babs);
+        if (wpbm > 1) babs[0] = cta_group_reduce<true>(babs[0], s_part, wpbm);
+        float ms[NBM], sc[NBM], inv[NBM];
+#pragma unroll
+        for (int b = 0; b < NBM; ++b) {
+            ms[b] = u2f(babs[b]);
+            sc[b] = 1.0f;
+            inv[b] = 0.0f;
+            if (ms[b] > 0.0f) uf8_encode_consts(ms[b], sc[b], inv[b]);
+        }
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int64_t idx = chunk_index(seg0, c, lane);
+            const int b = c / CPBM;
+            uint32_t qm = 0;
+            if (ms[b] > 0.0f) {
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    qm |= ((uint32_t)uf8_quantize(mf[4 * c + j], sc[b], inv[b]) & 0xFFu) << (8 * j);
+            }
+            if (idx < u.n) __stcs(reinterpret_cast<unsigned int*>(u.m_codes + idx), qm);
+        }
+        if (lane == 0 && (warp % wpbm) == 0) {
+#pragma unroll
+            for (int b = 0; b < NBM; ++b)
+                if (mb0 + b < nmb) u.m_absmax[mb0 + b] = ms[b];
+        }
+    }
+}
+
+// ------------------------------------------------------------- host side --
+static int cpb_of(int block) { return block >= 512 ? 4 : block / 128; }
+
+template <int MODE>
+static int launch_update(const UpdateArgs& u, cudaStream_t st) {
+    const int64_t ntiles = blocks_of(u.n, kTile);
+    const int cpb = MODE == 0 ? 4 : cpb_of(u.m_block);
+    const void* k = cpb == 1 ? (const void*)update_kernel<MODE, 1>
+                  : cpb == 2 ? (const void*)update_kernel<MODE, 2>
+                             : (const void*)update_kernel<MODE, 4>;
+    const int grid = persistent_grid(k, kThreads, 0, ntiles);
+    if (cpb == 1) update_kernel<MODE, 1><<<grid, kThreads, 0, st>>>(u, ntiles);
+    else if (cpb == 2) update_kernel<MODE, 2><<<grid, kThreads, 0, st>>>(u, ntiles);
+    else update_kernel<MODE, 4><<<grid, kThreads, 0, st>>>(u, ntiles);
+    return check_launch();
+}
+
+static int check_matrix(const float* p, const float* g, int64_t rows, int64_t cols) {
+    if (!p || !g || rows < 1 || cols < 1) return ALQ_ERR_INVALID_ARG;
+    if (cols % 4 != 0 || rows * cols >= (int64_t)1 << 31) return ALQ_ERR_UNSUPPORTED;
+    if (!aligned(p, 16) || !aligned(g, 16)) return ALQ_ERR_ALIGN;
+    return ALQ_OK;
+}
+
+static int check_factor(const void* codes, const float* meta, int bits, int block) {
+    if (!codes || !meta) return ALQ_ERR_INVALID_ARG;
+    if ((bits != 8 && bits != 16) || !valid_block(block)) return ALQ_ERR_UNSUPPORTED;
+    if (!aligned(codes, 16) || !aligned(meta, 8)) return ALQ_ERR_ALIGN;
+    return ALQ_OK;
+}
+
+static int check_momentum(const int8_t* codes, const float* absmax, int block) {
+    if (!codes || !absmax) return ALQ_ERR_INVALID_ARG;
+    if (!valid_block(block)) return ALQ_ERR_UNSUPPORTED;
+    if (!aligned(codes, 16) || !aligned(absmax, 4)) return ALQ_ERR_ALIGN;
+    return ALQ_OK;
+}
+
+static FactorDesc factor_desc(const double* part, int nparts, int64_t len, int64_t mean_len,
+                              double add_eps, float beta, float omb, void* codes, float* meta,
+                              int bits, int block, float floor_, float* fresh) {
+    FactorDesc f;
+    f.part = part;
+    f.nparts = nparts;
+    f.len = len;
+    f.mean_len = (double)mean_len;
+    f.add_eps = add_eps;
+    f.beta = beta;
+    f.omb = omb;
+    f.codes = codes;
+    f.meta = meta;
+    f.bits = bits;
+    f.block = block;
+    f.log_floor = floor_;
+    f.fresh = fresh;
+    return f;
+}
+
+// G pass 1 (g^2 sums), factor update, scales, G pass 2 (RMS) -> a, b, icf.
+static int second_moment_passes(const float* g, int64_t rows, int64_t cols, const FacWs& w,
+                                FactorDesc fr, FactorDesc fc, float clip_d, cudaStream_t st,
+                                float* a, float* b) {
+    const int ncb = (int)blocks_of(cols, kFC), nrb = (int)blocks_of(rows, kFR);
+    ResidualArgs none{};
+    sumsq_kernel<0><<<dim3(ncb, nrb), kThreads, 0, st>>>(g, (int)rows, (int)cols, none,
+                                                        w.rowpart, w.colpart);
+    const int nb0 = (int)blocks_of(rows, fr.block), nb1 = (int)blocks_of(cols, fc.block);
+    factor_kernel<<<nb0 + nb1, kThreads, 0, st>>>(fr, fc, nb0);
+    scale_kernel<<<1, 1024, 0, st>>>(fr.fresh, (int)rows, fc.fresh, (int)cols, a, b);
+    const int64_t n = rows * cols;
+    const int64_t ntiles = blocks_of(n, kTile);
+    int grid = persistent_grid((const void*)usq_kernel, kThreads, 0, ntiles);
+    if (grid > kMaxParts) grid = kMaxParts;
+    usq_kernel<<<grid, kThreads, 0, st>>>(g, n, make_divider((uint32_t)cols), a, b, ntiles,
+                                          w.upart);
+    clip_kernel<<<1, 1024, 0, st>>>(w.upart, grid, (double)n, clip_d, w.scal);
+    return check_launch();
+}
+
+}  // namespace alq
 
 using namespace alq;
 
 extern "C" {
 
 int al_workspace_size(int op, int64_t rows, int64_t cols, int rank, size_t* bytes) {
-    (void)op; (void)rows; (void)cols; (void)rank;
-    if (!bytes) return ALQ_ERR_INVALID_ARG;
-    *bytes = 0;
-    return ALQ_ERR_UNSUPPORTED;
+    if (!bytes || rows < 1 || cols < 1) return ALQ_ERR_INVALID_ARG;
+    if (op == AL_OP_ADAFACTOR || op == AL_OP_CAME) {
+        *bytes = fac_layout(nullptr, rows, cols).bytes;
+        return ALQ_OK;
+    }
+    if (op == AL_OP_APOLLO) {
+        if (rank < 1) return ALQ_ERR_INVALID_ARG;
+        return al_apollo_workspace(rows, cols, rank, bytes);
+    }
+    return ALQ_ERR_INVALID_ARG;
 }
 
-int al_adafactor_step(float*, const float*, int64_t, int64_t, void*, float*, void*, float*, int, int,
-                      int8_t*, float*, int, const al_adafactor_hp*, int64_t, void*, size_t, void*) {
-    return ALQ_ERR_UNSUPPORTED;
+int al_adafactor_step(float* p, const float* g, int64_t rows, int64_t cols, void* r_codes,
+                      float* r_meta, void* c_codes, float* c_meta, int fac_bits, int fac_block,
+                      int8_t* m_codes, float* m_absmax, int m_block,
+                      const al_adafactor_hp* hp, int64_t t, void* workspace, size_t ws_bytes,
+                      void* stream) {
+    int st = check_matrix(p, g, rows, cols);
+    if (st) return st;
+    if (!hp || t < 1 || !(hp->eps1 > 0.0f) || !(hp->clip_d > 0.0f)) return ALQ_ERR_INVALID_ARG;
+    st = check_factor(r_codes, r_meta, fac_bits, fac_block);
+    if (!st) st = check_factor(c_codes, c_meta, fac_bits, fac_block);
+    if (!st && m_codes) st = check_momentum(m_codes, m_absmax, m_block);
+    if (st) return st;
+    const FacWs w = fac_layout(workspace, rows, cols);
+    if (!workspace || ws_bytes < w.bytes || !aligned(workspace, 256)) return ALQ_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+
+    const double omr_d = pow((double)t, (double)hp->decay_rate);
+    const float omr = (float)omr_d, rho = (float)(1.0 - omr_d);
+    const int ncb = (int)blocks_of(cols, kFC), nrb = (int)blocks_of(rows, kFR);
+    FactorDesc fr = factor_desc(w.rowpart, ncb, rows, cols, hp->eps1, rho, omr, r_codes, r_meta,
+                                fac_bits, fac_block, hp->log_floor, w.fr);
+    FactorDesc fc = factor_desc(w.colpart, nrb, cols, rows, hp->eps1, rho, omr, c_codes, c_meta,
+                                fac_bits, fac_block, hp->log_floor, w.fc);
+    st = second_moment_passes(g, rows, cols, w, fr, fc, hp->clip_d, s, w.a, w.b);
+    if (st) return st;
+
+    UpdateArgs u{};
+    u.p = p;
+    u.g = g;
+    u.n = rows * cols;
+    u.dv = make_divider((uint32_t)cols);
+    u.a = w.a;
+    u.b = w.b;
+    u.scal = w.scal;
+    u.m_codes = m_codes;
+    u.m_absmax = m_absmax;
+    u.m_block = m_codes ? m_block : 4096;
+    u.beta1 = hp->beta1;
+    u.omb1 = (float)(1.0 - (double)hp->beta1);
+    u.decay = (float)(1.0 - (double)hp->lr * (double)hp->weight_decay);
+    u.lr = hp->lr;
+    return m_codes ? launch_update<1>(u, s) : launch_update<0>(u, s);
 }
 
-int al_came_step(float*, const float*, int64_t, int64_t, void*, float*, void*, float*, int, int, void*,
-                 float*, void*, float*, int, int, int8_t*, float*, int, const al_came_hp*, int64_t,
-                 void*, size_t, void*) {
-    return ALQ_ERR_UNSUPPORTED;
-}
+int al_came_step(float* p, const float* g, int64_t rows, int64_t cols, void* vr_codes,
+                 float* vr_meta, void* vc_codes, float* vc_meta, int v_bits, int v_block,
+                 void* cr_codes, float* cr_meta, void* cc_codes, float* cc_meta, int c_bits,
+                 int c_block, int8_t* m_codes, float* m_absmax, int m_block,
+                 const al_came_hp* hp, int64_t t, void* workspace, size_t ws_bytes,
+                 void* stream) {
+    int st = check_matrix(p, g, rows, cols);
+    if (st) return st;
+    if (!hp || t < 1 || !(hp->eps1 > 0.0f) || !(hp->eps2 > 0.0f) || !(hp->clip_d > 0.0f))
+        return ALQ_ERR_INVALID_ARG;
+    st = check_factor(vr_codes, vr_meta, v_bits, v_block);
+    if (!st) st = check_factor(vc_codes, vc_meta, v_bits, v_block);
+    if (!st) st = check_factor(cr_codes, cr_meta, c_bits, c_block);
+    if (!st) st = check_factor(cc_codes, cc_meta, c_bits, c_block);
+    if (!st) st = check_momentum(m_codes, m_absmax, m_block);
+    if (st) return st;
+    const FacWs w = fac_layout(workspace, rows, cols);
+    if (!workspace || ws_bytes < w.bytes || !aligned(workspace, 256)) return ALQ_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
 
-int al_apollo_step(float*, const float*, int64_t, int64_t, const uint16_t*, int8_t*, float*, int, void*,
-                   float*, int, int, float*, const al_apollo_hp*, int64_t, void*, size_t, void*) {
-    return ALQ_ERR_UNSUPPORTED;
+    const float omb1 = (float)(1.0 - (double)hp->beta1);
+    const float omb2 = (float)(1.0 - (double)hp->beta2);
+    const float omb3 = (float)(1.0 - (double)hp->beta3);
+    const int ncb = (int)blocks_of(cols, kFC), nrb = (int)blocks_of(rows, kFR);
+    FactorDesc fr = factor_desc(w.rowpart, ncb, rows, cols, hp->eps1, hp->beta2, omb2, vr_codes,
+                                vr_meta, v_bits, v_block, hp->log_floor_v, w.fr);
+    FactorDesc fc = factor_desc(w.colpart, nrb, cols, rows, hp->eps1, hp->beta2, omb2, vc_codes,
+                                vc_meta, v_bits, v_block, hp->log_floor_v, w.fc);
+    st = second_moment_passes(g, rows, cols, w, fr, fc, hp->clip_d, s, w.a, w.b);
+    if (st) return st;
+
+    // residual (u_hat - m)^2 + eps2 from the old momentum codes, its factored
+    // confidence (beta3) and the confidence scales
+    ResidualArgs ra{m_codes, m_absmax, 0, w.a, w.b, w.scal, hp->beta1, omb1, hp->eps2};
+    while ((1 << ra.m_shift) < m_block) ++ra.m_shift;
+    sumsq_kernel<1><<<dim3(ncb, nrb), kThreads, 0, s>>>(g, (int)rows, (int)cols, ra, w.rowpart,
+                                                       w.colpart);
+    FactorDesc cr = factor_desc(w.rowpart, ncb, rows, cols, 0.0, hp->beta3, omb3, cr_codes,
+                                cr_meta, c_bits, c_block, hp->log_floor_c, w.fr2);
+    FactorDesc cc = factor_desc(w.colpart, nrb, cols, rows, 0.0, hp->beta3, omb3, cc_codes,
+                                cc_meta, c_bits, c_block, hp->log_floor_c, w.fc2);
+    const int nb0 = (int)blocks_of(rows, c_block), nb1 = (int)blocks_of(cols, c_block);
+    factor_kernel<<<nb0 + nb1, kThreads, 0, s>>>(cr, cc, nb0);
+    scale_kernel<<<1, 1024, 0, s>>>(w.fr2, (int)rows, w.fc2, (int)cols, w.a2, w.b2);
+    st = check_launch();
+    if (st) return st;
+
+    UpdateArgs u{};
+    u.p = p;
+    u.g = g;
+    u.n = rows * cols;
+    u.dv = make_divider((uint32_t)cols);
+    u.a = w.a;
+    u.b = w.b;
+    u.a2 = w.a2;
+    u.b2 = w.b2;
+    u.scal = w.scal;
+    u.m_codes = m_codes;
+    u.m_absmax = m_absmax;
+    u.m_block = m_block;
+    u.beta1 = hp->beta1;
+    u.omb1 = omb1;
+    u.decay = (float)(1.0 - (double)hp->lr * (double)hp->weight_decay);
+    u.lr = hp->lr;
+    return launch_update<2>(u, s);
 }
 
 }  // extern "C"

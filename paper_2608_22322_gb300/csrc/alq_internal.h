@@ -67,4 +67,7 @@ int sm_count();                       // multiprocessors of the current device
 int persistent_grid(const void* kernel, int threads, size_t smem, int64_t ntiles);
 int64_t blocks_of(int64_t n, int block);
 
+// APOLLO workspace bytes (alq_apollo.cu).
+int al_apollo_workspace(int64_t rows, int64_t cols, int rank, size_t* bytes);
+
 }  // namespace alq

@@ -103,12 +103,13 @@ __device__ __forceinline__ uint32_t umix(uint32_t a, uint32_t b) {
     return kMax ? (a > b ? a : b) : (a < b ? a : b);
 }
 
-// Per-block warp-wide min or max of per-chunk values (unsigned order).
-template <int CPB, bool kMax>
-__device__ __forceinline__ void warp_blocks_reduce(const uint32_t (&chunk)[4],
-                                                   uint32_t (&out)[4 / CPB]) {
+// Per-block warp-wide min or max of per-chunk values (unsigned order): a lane
+// holds CH chunks, CPB consecutive chunks form one block.
+template <int CPB, bool kMax, int CH>
+__device__ __forceinline__ void warp_blocks_reduce(const uint32_t (&chunk)[CH],
+                                                   uint32_t (&out)[CH / CPB]) {
 #pragma unroll
-    for (int b = 0; b < 4 / CPB; ++b) {
+    for (int b = 0; b < CH / CPB; ++b) {
         uint32_t v = chunk[b * CPB];
 #pragma unroll
         for (int c = 1; c < CPB; ++c) v = umix<kMax>(v, chunk[b * CPB + c]);
@@ -162,17 +163,22 @@ __device__ __forceinline__ void al_blocks_params(const float (&mn)[NB], const fl
 // 2^(l_min + 16 a d), d = Delta / 254, as two-float pairs; code q decodes to
 // entry[16 + (q >> 4)] * entry[q & 15]. One entry per lane per block.
 // Blocks whose l_min is below -96 (or that are empty) take the FP64 path.
+// Level index of this lane's table entry: k = b - 1 for lanes b < 16,
+// k = 16 (lane - 16) for the others (as a float).
+__device__ __forceinline__ float al8_table_k(int lane) {
+    return int_to_float_small(lane >= 16 ? 16 * (lane - 16) : lane - 1);
+}
+
 template <int NB>
 __device__ __forceinline__ void al8_build_tables(float2* tab, const float (&lmin)[NB],
-                                                 const float (&delta)[NB]) {
+                                                 const float (&delta)[NB], float kf) {
     const int lane = threadIdx.x & 31;
     const bool hi = lane >= 16;
-    const int k = hi ? 16 * (lane - 16) : (lane - 1);
 #pragma unroll
     for (int b = 0; b < NB; ++b) {
         float rh = 0.0f, rl = 0.0f;
         if (delta[b] > 0.0f && lmin[b] >= -96.0f)
-            al_level_ff(hi ? lmin[b] : 0.0f, delta[b], k, 254.0f, 1.0f / 254.0f, rh, rl);
+            al_level_ff(hi ? lmin[b] : 0.0f, delta[b], kf, 254.0f, 1.0f / 254.0f, rh, rl);
         tab[32 * b + lane] = make_float2(rh, rl);
     }
     __syncwarp();
@@ -180,6 +186,65 @@ __device__ __forceinline__ void al8_build_tables(float2* tab, const float (&lmin
 
 __device__ __forceinline__ bool al8_fast_ok(float lmin, float delta) {
     return delta > 0.0f && lmin >= -96.0f;
+}
+
+// AL8 decode of the 16 codes of a lane's four chunks through their blocks'
+// tables, branch-free: the fast results are selected per element and the
+// rare elements whose two-float product lies too close to an fp32 rounding
+// boundary (or whose block is outside the fast range) are marked in a bit
+// mask and recomputed in FP64 under one warp-uniform, rarely taken branch.
+template <int CPB, int NB, int CH>
+__device__ __forceinline__ void al8_decode_chunks(const uint32_t (&w)[CH], const float2* tab,
+                                                  const float (&lmin)[NB], const float (&delta)[NB],
+                                                  float (&out)[4 * CH]) {
+    uint32_t fbm = 0;
+#pragma unroll
+    for (int c = 0; c < CH; ++c) {
+        const int b = c / CPB;
+        const bool fast = al8_fast_ok(lmin[b], delta[b]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const uint32_t q = (w[c] >> (8 * i)) & 0xFFu;
+            const float2 A = tab[32 * b + 16 + (q >> 4)];
+            const float2 Bt = tab[32 * b + (q & 15u)];
+            bool fb;
+            const float r = al8_decode_pair(A.x, A.y, Bt.x, Bt.y, fb);
+            out[4 * c + i] = q == 0u ? 0.0f : r;
+            fbm |= (uint32_t)((q != 0u) & (fb | !fast)) << (4 * c + i);
+        }
+    }
+    if (__any_sync(0xFFFFFFFFu, fbm != 0u)) {
+#pragma unroll
+        for (int e = 0; e < 4 * CH; ++e)
+            if ((fbm >> e) & 1u)
+                out[e] = al_dequantize_fp64((w[e / 4] >> (8 * (e % 4))) & 0xFFu, lmin[e / 4 / CPB],
+                                            delta[e / 4 / CPB], 254.0);
+    }
+}
+
+// Eq. (4) for the 4 CH values of a lane's chunks, branch-free with the same
+// bit-mask fixup in FP64 for values near a half-integer of t.
+template <int BITS, int CPB, int NB, int CH>
+__device__ __forceinline__ void al_encode_chunks(const float (&x)[4 * CH], const float (&lmin)[NB],
+                                                 const float (&delta)[NB], const float (&K)[NB],
+                                                 const float (&E)[NB], uint32_t (&q)[4 * CH]) {
+    constexpr float Lm2 = BITS == 8 ? 254.0f : 65534.0f;
+    uint32_t fbm = 0;
+#pragma unroll
+    for (int e = 0; e < 4 * CH; ++e) {
+        const int b = e / 4 / CPB;
+        bool fb;
+        const uint32_t v = al_quantize_fast(x[e], lmin[b], K[b], E[b], Lm2, fb);
+        const bool nz = x[e] != 0.0f;
+        q[e] = nz ? v : 0u;
+        fbm |= (uint32_t)(nz & fb) << e;
+    }
+    if (__any_sync(0xFFFFFFFFu, fbm != 0u)) {
+#pragma unroll
+        for (int e = 0; e < 4 * CH; ++e)
+            if ((fbm >> e) & 1u)
+                q[e] = al_quantize_fp64(x[e], lmin[e / 4 / CPB], delta[e / 4 / CPB], (double)Lm2);
+    }
 }
 
 // AL8 element decode through a block's tables; FP64 when the two-float
@@ -197,16 +262,22 @@ __device__ __forceinline__ float al8_decode(uint32_t q, const float2* tab, bool 
     return al_dequantize_fp64(q, lmin, delta, 254.0);
 }
 
-// AL16 element decode: the level directly in two-float form.
-__device__ __forceinline__ float al16_decode(uint32_t q, float lmin, float delta) {
+// Element decode with the level computed directly in two-float form (any
+// bit width; used for AL16 and for the small factor vectors).
+__device__ __forceinline__ float al_decode_direct(uint32_t q, float lmin, float delta,
+                                                  float Lm2) {
     if (q == 0u) return 0.0f;
-    if (lmin >= -96.0f) {
+    if (lmin >= -96.0f && delta > 0.0f) {
         float rh, rl;
-        al_level_ff(lmin, delta, (int)q - 1, 65534.0f, 1.0f / 65534.0f, rh, rl);
+        al_level_ff(lmin, delta, int_to_float_small((int)q - 1), Lm2, 1.0f / Lm2, rh, rl);
         const float hu = half_ulp_below(rh);
         if (fabsf(rl) < hu - hu * 0x1p-16f) return rh;
     }
-    return al_dequantize_fp64(q, lmin, delta, 65534.0);
+    return al_dequantize_fp64(q, lmin, delta, (double)Lm2);
+}
+
+__device__ __forceinline__ float al16_decode(uint32_t q, float lmin, float delta) {
+    return al_decode_direct(q, lmin, delta, 65534.0f);
 }
 
 // Eq. (4) element encode with the FP64 fallback near rounding boundaries.
@@ -221,9 +292,52 @@ __device__ __forceinline__ uint32_t al_encode_elem(float x, float lmin, float de
     return q;
 }
 
-// Signed 8-bit code (two's complement byte) to float, exactly.
+// Signed 8-bit code (two's complement byte) to float, exactly, without an
+// int-to-float conversion: (byte ^ 0x80) is q + 128 in [0, 255]; placed in
+// the low mantissa of 1.5 * 2^23 it reads as 1.5 * 2^23 + q + 128.
 __device__ __forceinline__ float s8_to_float(uint32_t byte) {
-    return (float)(int)(int8_t)(uint8_t)byte;
+    return __uint_as_float(0x4B400000u | ((byte & 0xFFu) ^ 0x80u)) - 12583040.0f;
+}
+
+// ------------------------------------------- division by an invariant int --
+// Unsigned 32-bit division by a run-time invariant d >= 2 through one
+// multiply-high (Granlund and Montgomery, "Division by invariant integers
+// using multiplication", PLDI 1994, Fig. 4.1).
+struct Divider {
+    uint32_t m, s1, s2, d;
+};
+
+inline Divider make_divider(uint32_t d) {
+    uint32_t l = 0;
+    while ((1ull << l) < d) ++l;
+    Divider v;
+    v.m = (uint32_t)(((1ull << 32) * ((1ull << l) - d)) / d + 1);
+    v.s1 = l > 0 ? 1 : 0;
+    v.s2 = l > 0 ? l - 1 : 0;
+    v.d = d;
+    return v;
+}
+
+__device__ __forceinline__ uint32_t divide(uint32_t n, const Divider& v) {
+    const uint32_t t1 = __umulhi(v.m, n);
+    return (t1 + ((n - t1) >> v.s1)) >> v.s2;
+}
+
+// ----------------------------------------------------- float-float add-in --
+__device__ __forceinline__ void ff_acc(float& hi, float& lo, float h, float l) {
+    float s, e;
+    two_sum(hi, h, s, e);
+    hi = s;
+    lo = lo + (e + l);
+}
+
+__device__ __forceinline__ void ff_warp_sum(float& hi, float& lo) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float oh = __shfl_xor_sync(0xFFFFFFFFu, hi, o);
+        const float ol = __shfl_xor_sync(0xFFFFFFFFu, lo, o);
+        ff_acc(hi, lo, oh, ol);
+    }
 }
 
 }  // namespace alq

@@ -15,7 +15,7 @@ void alqn_block_params(float mn, float mx, float floor_, float* lmin, float* del
 
 // Level k (two-float) of a block, as the decode tables build it.
 void alqn_level(float lmin, float delta, int k, float Lm2, float* hi, float* lo) {
-    al_level_ff(lmin, delta, k, Lm2, 1.0f / Lm2, *hi, *lo);
+    al_level_ff(lmin, delta, (float)k, Lm2, 1.0f / Lm2, *hi, *lo);
 }
 
 // AL8 decode through the two 16-entry tables; fb_count accumulates fallbacks.
@@ -23,8 +23,8 @@ void alqn_al8_decode(const uint8_t* q, int64_t n, float lmin, float delta,
                      float* out, int64_t* fb_count) {
     float th[16], tl[16], uh[16], ul[16];
     const float inv = 1.0f / 254.0f;
-    for (int a = 0; a < 16; ++a) al_level_ff(lmin, delta, 16 * a, 254.0f, inv, th[a], tl[a]);
-    for (int b = 0; b < 16; ++b) al_level_ff(0.0f, delta, b - 1, 254.0f, inv, uh[b], ul[b]);
+    for (int a = 0; a < 16; ++a) al_level_ff(lmin, delta, (float)(16 * a), 254.0f, inv, th[a], tl[a]);
+    for (int b = 0; b < 16; ++b) al_level_ff(0.0f, delta, (float)(b - 1), 254.0f, inv, uh[b], ul[b]);
     for (int64_t i = 0; i < n; ++i) {
         uint32_t c = q[i];
         if (c == 0) { out[i] = 0.0f; continue; }

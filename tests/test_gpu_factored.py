@@ -1,0 +1,145 @@
+"""GPU parity of the Adafactor and CAME steps (AL-coded factors, UF8
+momentum) with the oracle.
+
+Sec. 3.1 (factored second moment; CAME's factored confidence), Sec. 6.1
+hyperparameters. Same seeded states and gradients on both sides, several
+steps. The fp32 state arithmetic is identical on both sides; the row/column
+means and RMS are exact sums rounded once on both sides but in a different
+order (two-float partials merged in fp64 on the GPU, fp64 sequential in the
+oracle), so a factor can in principle round to a neighbouring fp32 value.
+Bar: parameters within 1e-6 of max|p| element-wise after every step (the
+spec bound is 1e-5 relative after 10 steps), factor codes and
+metadata exact except for rare +-1 code flips (<= 1e-4 of codes), momentum
+codes exact up to the same flip rate. Mismatch counts are reported.
+"""
+import math
+
+import numpy as np
+import pytest
+
+import oracle as ora
+from gpu_util import bytes_equal, gpu_available
+from paper_2608_22322_gb300 import workloads as wl
+
+pytestmark = [pytest.mark.gpu,
+              pytest.mark.skipif(not gpu_available(), reason="needs a CUDA GPU")]
+
+F1 = float(np.float32(math.log2(1e-30)))
+F2 = float(np.float32(math.log2(1e-16)))
+ADA_HP = dict(lr=1e-3, eps1=1e-30, clip_d=1.0, decay_rate=-0.8, beta1=0.9,
+              weight_decay=0.0, log_floor=F1)
+CAME_HP = dict(lr=1e-4, beta1=0.9, beta2=0.999, beta3=0.9999, eps1=1e-30, eps2=1e-16,
+               clip_d=1.0, weight_decay=0.0, log_floor_v=F1, log_floor_c=F2)
+
+
+@pytest.fixture(scope="module")
+def B():
+    from paper_2608_22322_gb300 import binding
+    return binding
+
+
+def _t(a):
+    import torch
+    if a.dtype == np.uint16:
+        a = a.view(np.int16)
+    return torch.from_numpy(a.copy()).cuda()
+
+
+def _cmp_codes(name, want, got, bits):
+    got = got.cpu().numpy()
+    if bits == 16:
+        got = got.view(np.uint16)
+    d = np.abs(want.astype(np.int64) - got.astype(np.int64))
+    flips = int(np.sum(d != 0))
+    assert d.max(initial=0) <= 1, f"{name}: code differs by {d.max()}"
+    assert flips <= max(1, 1e-4 * want.size), f"{name}: {flips} flips"
+    return flips
+
+
+def _cmp_p(want, got, what):
+    got = got.cpu().numpy()
+    err = np.max(np.abs(got.astype(np.float64) - want))
+    assert err <= 1e-6 * np.max(np.abs(want)), f"{what}: max |dp| = {err}"
+    return bytes_equal(want, got)
+
+
+def _state(n, bits, block):
+    nb = (n + block - 1) // block
+    return np.zeros(n, ora.code_dtype(bits)), np.zeros(2 * nb, np.float32)
+
+
+@pytest.mark.parametrize("rows,cols,bits,fblock,mom,steps", [
+    (512, 1024, 16, 128, True, 20),     # the Adafactor setting, smaller matrix
+    (300, 772, 16, 128, True, 6),       # ragged tiles
+    (257, 2048, 8, 256, False, 6),      # AL8 factors, no momentum
+    (4096, 4096, 16, 128, True, 3),     # the full 4096x4096 workload
+])
+def test_adafactor_matches_oracle(B, rows, cols, bits, fblock, mom, steps):
+    import torch
+    n = rows * cols
+    p = wl.param_init((rows, cols), 5).ravel()
+    rc, rm = _state(rows, bits, fblock)
+    cc, cm = _state(cols, bits, fblock)
+    mc = np.zeros(n, np.int8) if mom else None
+    ma = np.zeros((n + 255) // 256, np.float32) if mom else None
+    d = dict(p=_t(p), rc=_t(rc), rm=_t(rm), cc=_t(cc), cm=_t(cm),
+             mc=_t(mc) if mom else None, ma=_t(ma) if mom else None)
+    ws = torch.empty(B.al_workspace_size(B.AL_OP_ADAFACTOR, rows, cols), dtype=torch.uint8,
+                     device="cuda")
+    flips = 0
+    for t in range(1, steps + 1):
+        g = wl.lognormal_col_grad((rows, cols), 1e-3, 0.05, 7000 + t).ravel()
+        ora.adafactor_step(p, g, rows, cols, rc, rm, cc, cm, bits, fblock, mc, ma, 256,
+                           ADA_HP, t)
+        B.al_adafactor_step(d["p"], _t(g), rows, cols, d["rc"], d["rm"], d["cc"], d["cm"],
+                            bits, fblock, d["mc"], d["ma"], 256, ADA_HP, t, ws)
+        torch.cuda.synchronize()
+        _cmp_p(p, d["p"], f"step {t}")
+        flips += _cmp_codes("R codes", rc, d["rc"], bits) + _cmp_codes("C codes", cc, d["cc"], bits)
+        if mom:
+            flips += _cmp_codes("M codes", mc, d["mc"], 8)
+    print(f"adafactor {rows}x{cols}: code flips over {steps} steps = {flips}")
+
+
+@pytest.mark.parametrize("rows,cols,steps", [(256, 1408, 10), (130, 516, 5), (2048, 5632, 3)])
+def test_came_matches_oracle(B, rows, cols, steps):
+    import torch
+    n = rows * cols
+    p = wl.param_init((rows, cols), 8).ravel()
+    st = [_state(rows, 16, 128), _state(cols, 16, 128), _state(rows, 16, 128),
+          _state(cols, 16, 128)]
+    mc = np.zeros(n, np.int8)
+    ma = np.zeros((n + 255) // 256, np.float32)
+    dp = _t(p)
+    dst = [(_t(c), _t(m)) for c, m in st]
+    dmc, dma = _t(mc), _t(ma)
+    ws = torch.empty(B.al_workspace_size(B.AL_OP_CAME, rows, cols), dtype=torch.uint8,
+                     device="cuda")
+    flips = 0
+    for t in range(1, steps + 1):
+        g = wl.student_t_grad((rows, cols), 1e-3, 3.0, 0.05, 8000 + t).ravel()
+        ora.came_step(p, g, rows, cols, st[0][0], st[0][1], st[1][0], st[1][1], 16, 128,
+                      st[2][0], st[2][1], st[3][0], st[3][1], 16, 128, mc, ma, 256, CAME_HP, t)
+        B.al_came_step(dp, _t(g), rows, cols, dst[0][0], dst[0][1], dst[1][0], dst[1][1], 16,
+                       128, dst[2][0], dst[2][1], dst[3][0], dst[3][1], 16, 128, dmc, dma, 256,
+                       CAME_HP, t, ws)
+        torch.cuda.synchronize()
+        _cmp_p(p, dp, f"step {t}")
+        for (c, _), (dc, _) in zip(st, dst):
+            flips += _cmp_codes("factor codes", c, dc, 16)
+        flips += _cmp_codes("M codes", mc, dmc, 8)
+    print(f"came {rows}x{cols}: code flips over {steps} steps = {flips}")
+
+
+def test_factored_rejects_bad_arguments(B):
+    import torch
+    x = torch.zeros(64 * 64, device="cuda")
+    c = torch.zeros(64, dtype=torch.int16, device="cuda")
+    m = torch.zeros(2, device="cuda")
+    ws = torch.empty(B.al_workspace_size(B.AL_OP_ADAFACTOR, 64, 64), dtype=torch.uint8,
+                     device="cuda")
+    with pytest.raises(B.AlqError, match="UNSUPPORTED"):   # cols not a multiple of 4
+        B.al_adafactor_step(x, x, 64, 62, c, m, c, m, 16, 128, None, None, 256, ADA_HP, 1, ws)
+    with pytest.raises(B.AlqError, match="WORKSPACE"):
+        B.al_adafactor_step(x, x, 64, 64, c, m, c, m, 16, 128, None, None, 256, ADA_HP, 1,
+                            ws[:16])
