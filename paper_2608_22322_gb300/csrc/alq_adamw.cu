@@ -26,6 +26,7 @@ template <int CPBV, int CPBM, int VBITS>
 __global__ void __launch_bounds__(kThreads, 3)
 adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t total_tiles,
                    PlanEntry single, int v_block, int m_block, AdamWScalars s) {
+    const int v_shift = __ffs(v_block) - 1, m_shift = __ffs(m_block) - 1;  // powers of two
     constexpr int NBV = kCH / CPBV;
     constexpr int NBM = kCH / CPBM;
     constexpr int NE = 4 * kCH;
@@ -76,8 +77,8 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
         }
 
         // ---- previous block constants
-        const int64_t nvb = blocks_of_dev(n, v_block), nmb = blocks_of_dev(n, m_block);
-        const int64_t vb0 = seg0 / v_block, mb0 = seg0 / m_block;
+        const int64_t nvb = (n + v_block - 1) >> v_shift, nmb = (n + m_block - 1) >> m_shift;
+        const int64_t vb0 = seg0 >> v_shift, mb0 = seg0 >> m_shift;
         float olmin[NBV], odelta[NBV], dm[NBM];
 #pragma unroll
         for (int b = 0; b < NBV; ++b) {

@@ -329,9 +329,10 @@ apollo_moments_kernel(MomentArgs m, int64_t ntiles) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const float kf = al8_table_k(lane);
     const int64_t nblk = blocks_of_dev(m.n, m.block);
+    const int bshift = __ffs(m.block) - 1;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
-        const int64_t b0 = seg0 / m.block;
+        const int64_t b0 = seg0 >> bshift;
         float4 r[4];
         uint32_t mw[4], vw[4 * VBITS / 8];
 #pragma unroll

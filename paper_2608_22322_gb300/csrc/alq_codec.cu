@@ -23,6 +23,7 @@ al_encode_kernel(const float* __restrict__ x, int64_t n, int block, float log_fl
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int wpb = block > kSeg ? block / kSeg : 1;
     const int64_t nblk = blocks_of_dev(n, block);
+    const int bshift = __ffs(block) - 1;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
         float4 v[4];
@@ -69,7 +70,7 @@ al_encode_kernel(const float* __restrict__ x, int64_t n, int block, float log_fl
                 store4h((uint16_t*)codes, idx, n, make_uint2(q[0] | (q[1] << 16), q[2] | (q[3] << 16)));
         }
         if (lane == 0 && (warp % wpb) == 0) {
-            const int64_t gb0 = seg0 / block;
+            const int64_t gb0 = seg0 >> bshift;
 #pragma unroll
             for (int b = 0; b < NB; ++b)
                 if (gb0 + b < nblk)
@@ -88,6 +89,7 @@ al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta,
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const float kf = al8_table_k(lane);
     const int64_t nblk = blocks_of_dev(n, block);
+    const int bshift = __ffs(block) - 1;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
         uint32_t w[4 * BITS / 8];
@@ -103,7 +105,7 @@ al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta,
             }
         }
         float lmin[NB], delta[NB];
-        const int64_t gb0 = seg0 / block;
+        const int64_t gb0 = seg0 >> bshift;
 #pragma unroll
         for (int b = 0; b < NB; ++b) {
             float2 mt = make_float2(0.f, 0.f);
@@ -139,6 +141,7 @@ uf8_encode_kernel(const float* __restrict__ m, int64_t n, int block, int8_t* __r
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int wpb = block > kSeg ? block / kSeg : 1;
     const int64_t nblk = blocks_of_dev(n, block);
+    const int bshift = __ffs(block) - 1;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
         float4 v[4];
@@ -173,7 +176,7 @@ uf8_encode_kernel(const float* __restrict__ m, int64_t n, int block, int8_t* __r
             store4b((uint8_t*)codes, chunk_index(seg0, c, lane), n, wd);
         }
         if (lane == 0 && (warp % wpb) == 0) {
-            const int64_t gb0 = seg0 / block;
+            const int64_t gb0 = seg0 >> bshift;
 #pragma unroll
             for (int b = 0; b < NB; ++b)
                 if (gb0 + b < nblk) absmax[gb0 + b] = s[b];
@@ -189,10 +192,11 @@ uf8_decode_kernel(const int8_t* __restrict__ codes, const float* __restrict__ ab
     constexpr int NB = 4 / CPB;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t nblk = blocks_of_dev(n, block);
+    const int bshift = __ffs(block) - 1;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
         float d[NB];
-        const int64_t gb0 = seg0 / block;
+        const int64_t gb0 = seg0 >> bshift;
 #pragma unroll
         for (int b = 0; b < NB; ++b)
             d[b] = (gb0 + b < nblk) ? __ldg(absmax + gb0 + b) / 127.0f : 0.0f;

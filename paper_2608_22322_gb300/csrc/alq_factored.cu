@@ -345,9 +345,10 @@ update_kernel(UpdateArgs u, int64_t ntiles) {
     const int wpbm = u.m_block > kSeg ? u.m_block / kSeg : 1;
     const float icf = __ldg(u.scal);
     const int64_t nmb = blocks_of_dev(u.n, u.m_block);
+    const int mshift = __ffs(u.m_block) - 1;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
-        const int64_t mb0 = seg0 / u.m_block;
+        const int64_t mb0 = seg0 >> mshift;
         float dm[NBM];
 #pragma unroll
         for (int b = 0; b < NBM; ++b)

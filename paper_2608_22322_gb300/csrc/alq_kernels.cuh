@@ -197,7 +197,7 @@ template <int CPB, int NB, int CH>
 __device__ __forceinline__ void al8_decode_chunks(const uint32_t (&w)[CH], const float2* tab,
                                                   const float (&lmin)[NB], const float (&delta)[NB],
                                                   float (&out)[4 * CH]) {
-    uint32_t fbm = 0;
+    bool any_fb = false;
 #pragma unroll
     for (int c = 0; c < CH; ++c) {
         const int b = c / CPB;
@@ -210,15 +210,26 @@ __device__ __forceinline__ void al8_decode_chunks(const uint32_t (&w)[CH], const
             bool fb;
             const float r = al8_decode_pair(A.x, A.y, Bt.x, Bt.y, fb);
             out[4 * c + i] = q == 0u ? 0.0f : r;
-            fbm |= (uint32_t)((q != 0u) & (fb | !fast)) << (4 * c + i);
+            any_fb |= (q != 0u) & (fb | !fast);
         }
     }
-    if (__any_sync(0xFFFFFFFFu, fbm != 0u)) {
+    if (__any_sync(0xFFFFFFFFu, any_fb)) {
+        // rare: redo the boundary test per element and recompute in FP64
 #pragma unroll
-        for (int e = 0; e < 4 * CH; ++e)
-            if ((fbm >> e) & 1u)
-                out[e] = al_dequantize_fp64((w[e / 4] >> (8 * (e % 4))) & 0xFFu, lmin[e / 4 / CPB],
-                                            delta[e / 4 / CPB], 254.0);
+        for (int c = 0; c < CH; ++c) {
+            const int b = c / CPB;
+            const bool fast = al8_fast_ok(lmin[b], delta[b]);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t q = (w[c] >> (8 * i)) & 0xFFu;
+                const float2 A = tab[32 * b + 16 + (q >> 4)];
+                const float2 Bt = tab[32 * b + (q & 15u)];
+                bool fb;
+                al8_decode_pair(A.x, A.y, Bt.x, Bt.y, fb);
+                if ((q != 0u) && (fb || !fast))
+                    out[4 * c + i] = al_dequantize_fp64(q, lmin[b], delta[b], 254.0);
+            }
+        }
     }
 }
 
@@ -229,7 +240,7 @@ __device__ __forceinline__ void al_encode_chunks(const float (&x)[4 * CH], const
                                                  const float (&delta)[NB], const float (&K)[NB],
                                                  const float (&E)[NB], uint32_t (&q)[4 * CH]) {
     constexpr float Lm2 = BITS == 8 ? 254.0f : 65534.0f;
-    uint32_t fbm = 0;
+    bool any_fb = false;
 #pragma unroll
     for (int e = 0; e < 4 * CH; ++e) {
         const int b = e / 4 / CPB;
@@ -237,13 +248,16 @@ __device__ __forceinline__ void al_encode_chunks(const float (&x)[4 * CH], const
         const uint32_t v = al_quantize_fast(x[e], lmin[b], K[b], E[b], Lm2, fb);
         const bool nz = x[e] != 0.0f;
         q[e] = nz ? v : 0u;
-        fbm |= (uint32_t)(nz & fb) << e;
+        any_fb |= nz & fb;
     }
-    if (__any_sync(0xFFFFFFFFu, fbm != 0u)) {
+    if (__any_sync(0xFFFFFFFFu, any_fb)) {
 #pragma unroll
-        for (int e = 0; e < 4 * CH; ++e)
-            if ((fbm >> e) & 1u)
-                q[e] = al_quantize_fp64(x[e], lmin[e / 4 / CPB], delta[e / 4 / CPB], (double)Lm2);
+        for (int e = 0; e < 4 * CH; ++e) {
+            const int b = e / 4 / CPB;
+            bool fb;
+            al_quantize_fast(x[e], lmin[b], K[b], E[b], Lm2, fb);
+            if (x[e] != 0.0f && fb) q[e] = al_quantize_fp64(x[e], lmin[b], delta[b], (double)Lm2);
+        }
     }
 }
 
