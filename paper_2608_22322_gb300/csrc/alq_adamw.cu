@@ -32,6 +32,7 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
     constexpr int NE = 4 * kCH;
     constexpr float Lm2 = VBITS == 8 ? 254.0f : 65534.0f;
     __shared__ float2 s_tab[kThreads / 32][NBV * 32];
+    __shared__ float s_val[kThreads / 32][VBITS == 8 ? NBV * 256 : 1];
     __shared__ uint32_t s_part[3][kThreads / 32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int wpbv = v_block > kASeg ? v_block / kASeg : 1;
@@ -94,8 +95,10 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
         // ---- decode the previous states
         float vh[NE];
         if constexpr (VBITS == 8) {
-            al8_build_tables<NBV>(s_tab[warp], olmin, odelta, kf);
-            al8_decode_chunks<CPBV, NBV, kCH>(vw, s_tab[warp], olmin, odelta, vh);
+            al8_build_values<NBV>(s_val[warp], s_tab[warp], olmin, odelta, kf);
+#pragma unroll
+            for (int e = 0; e < NE; ++e)
+                vh[e] = s_val[warp][256 * (e / 4 / CPBV) + ((vw[e / 4] >> (8 * (e % 4))) & 0xFFu)];
         } else {
 #pragma unroll
             for (int e = 0; e < NE; ++e)

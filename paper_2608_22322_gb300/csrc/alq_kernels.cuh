@@ -261,6 +261,53 @@ __device__ __forceinline__ void al_encode_chunks(const float (&x)[4 * CH], const
     }
 }
 
+// The 256 decoded values of each of the NB blocks of a segment (Eq. (5), code
+// 0 -> 0), exactly as the double expression rounds them, in shared memory:
+// lane l computes codes l, l + 32, ..., l + 224 from the block's two-float
+// level tables (T_hi[q >> 4] * T_lo[q & 15]); entries whose two-float product
+// lies too close to an fp32 rounding boundary, and blocks outside the fast
+// range, are recomputed in FP64 under one warp-uniform branch. An element
+// decode is then a single shared-memory load.
+template <int NB>
+__device__ __forceinline__ void al8_build_values(float* vals, float2* tab,
+                                                 const float (&lmin)[NB],
+                                                 const float (&delta)[NB], float kf) {
+    al8_build_tables<NB>(tab, lmin, delta, kf);
+    const int lane = threadIdx.x & 31;
+    bool any_fb = false;
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+        const bool fast = al8_fast_ok(lmin[b], delta[b]);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const uint32_t q = (uint32_t)(lane + 32 * k);
+            const float2 A = tab[32 * b + 16 + (q >> 4)];
+            const float2 Bt = tab[32 * b + (q & 15u)];
+            bool fb;
+            const float r = al8_decode_pair(A.x, A.y, Bt.x, Bt.y, fb);
+            vals[256 * b + q] = q == 0u ? 0.0f : r;
+            any_fb |= (q != 0u) & (fb | !fast);
+        }
+    }
+    if (__any_sync(0xFFFFFFFFu, any_fb)) {
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            const bool fast = al8_fast_ok(lmin[b], delta[b]);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const uint32_t q = (uint32_t)(lane + 32 * k);
+                const float2 A = tab[32 * b + 16 + (q >> 4)];
+                const float2 Bt = tab[32 * b + (q & 15u)];
+                bool fb;
+                al8_decode_pair(A.x, A.y, Bt.x, Bt.y, fb);
+                if ((q != 0u) && (fb || !fast))
+                    vals[256 * b + q] = al_dequantize_fp64(q, lmin[b], delta[b], 254.0);
+            }
+        }
+    }
+    __syncwarp();
+}
+
 // AL8 element decode through a block's tables; FP64 when the two-float
 // product may round differently, or the block is outside the fast range.
 __device__ __forceinline__ float al8_decode(uint32_t q, const float2* tab, bool fast,
