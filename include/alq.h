@@ -253,6 +253,40 @@ int al_adafactor_step(float* p, const float* g, int64_t rows, int64_t cols,
                       const al_adafactor_hp* hp, int64_t t, void* workspace,
                       size_t ws_bytes, void* stream);
 
+/*
+ * al_adafactor_step_noalloc -- al_adafactor_step for callers that cannot
+ * allocate GPU memory (no counterpart in the paper; an interface addition).
+ * Some callers cannot call cudaMalloc when they step the optimizer: code
+ * running under a framework that owns all device memory, code with a fixed
+ * memory budget after start-up, or bindings without access to the CUDA
+ * allocator. This variant takes the step's scratch space from a fixed array
+ * inside the library (al_adafactor_noalloc_capacity() bytes, 4 MiB, enough
+ * for matrices up to 4096 x 4096) and allocates nothing; arguments and
+ * results are exactly those of al_adafactor_step without the workspace.
+ *   - Every GPU that loads the library reserves that array until the process
+ *     exits.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current); make that first call
+ *     before capturing any stream.
+ *   - Every call on a device shares the one array: calls that may run
+ *     concurrently on the GPU (different streams, no ordering between them)
+ *     race and corrupt each other's results. Serialise them on one stream.
+ *     The array keeps the previous call's contents; every scratch word a call
+ *     reads it has written first in the same call, so nothing needs clearing.
+ *   - Returns ALQ_ERR_WORKSPACE when the matrix needs more scratch than the
+ *     array holds (see al_workspace_size(AL_OP_ADAFACTOR, ...)), and every
+ *     status of al_adafactor_step otherwise.
+ */
+int al_adafactor_step_noalloc(float* p, const float* g, int64_t rows,
+                              int64_t cols, void* r_codes, float* r_meta,
+                              void* c_codes, float* c_meta, int fac_bits,
+                              int fac_block, int8_t* m_codes, float* m_absmax,
+                              int m_block, const al_adafactor_hp* hp,
+                              int64_t t, void* stream);
+
+/* Bytes of the fixed scratch array that al_adafactor_step_noalloc uses. */
+size_t al_adafactor_noalloc_capacity(void);
+
 /* ------------------------------------------------------------------ CAME -- */
 typedef struct {
     float lr;

@@ -97,6 +97,9 @@ _sig("al_adamw_step_multi", _int, _vp, C.POINTER(MultiInfo), C.POINTER(AdamWHP),
 _sig("al_workspace_size", _int, _int, _i64, _i64, _int, C.POINTER(C.c_size_t))
 _sig("al_adafactor_step", _int, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _vp, _int, _int,
      _vp, _vp, _int, C.POINTER(AdafactorHP), _i64, _vp, C.c_size_t, _vp)
+_sig("al_adafactor_step_noalloc", _int, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _vp, _int, _int,
+     _vp, _vp, _int, C.POINTER(AdafactorHP), _i64, _vp)
+_sig("al_adafactor_noalloc_capacity", C.c_size_t)
 _sig("al_came_step", _int, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _vp, _int, _int,
      _vp, _vp, _vp, _vp, _int, _int, _vp, _vp, _int, C.POINTER(CameHP), _i64, _vp,
      C.c_size_t, _vp)
@@ -216,6 +219,23 @@ def al_adafactor_step(p, g, rows, cols, r_codes, r_meta, c_codes, c_meta, fac_bi
         _ptr(c_meta), fac_bits, fac_block, _ptr(m_codes), _ptr(m_absmax), m_block,
         C.byref(h), t, _ptr(workspace), workspace.numel() * workspace.element_size(),
         _stream(stream)))
+
+
+def al_adafactor_step_noalloc(p, g, rows, cols, r_codes, r_meta, c_codes, c_meta, fac_bits,
+                              fac_block, m_codes, m_absmax, m_block, hp: dict, t: int,
+                              stream=None):
+    """al_adafactor_step without a workspace argument: the library supplies
+    the scratch from a fixed array of al_adafactor_noalloc_capacity() bytes
+    (for callers that cannot allocate device memory)."""
+    h = _hp(AdafactorHP, hp)
+    _check("al_adafactor_step_noalloc", lib.al_adafactor_step_noalloc(
+        _ptr(p), _ptr(g), rows, cols, _ptr(r_codes), _ptr(r_meta), _ptr(c_codes),
+        _ptr(c_meta), fac_bits, fac_block, _ptr(m_codes), _ptr(m_absmax), m_block,
+        C.byref(h), t, _stream(stream)))
+
+
+def al_adafactor_noalloc_capacity() -> int:
+    return int(lib.al_adafactor_noalloc_capacity())
 
 
 def al_came_step(p, g, rows, cols, vr_codes, vr_meta, vc_codes, vc_meta, v_bits,
