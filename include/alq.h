@@ -39,9 +39,10 @@
  *  - Alignment: fp32 arrays and code arrays that are streamed element-wise must
  *    be 16-byte aligned; metadata arrays 8-byte aligned. Misalignment returns
  *    ALQ_ERR_ALIGN.
- *  - Floating-point contract: state EMAs and updates are IEEE fp32 with no
- *    fused multiply-add contraction, in the operation order documented per
- *    entry point; log2/exp2 in the codec are evaluated as if in double and
+ *  - Floating-point contract: state EMAs and updates are IEEE fp32 in the
+ *    operation order documented per entry point, with a fused multiply-add
+ *    (one rounding) exactly where the order writes fma(a, b, c) and no other
+ *    contraction; log2/exp2 in the codec are evaluated as if in double and
  *    rounded once to fp32. Within that contract the results are reproducible
  *    run to run (no floating-point atomics).
  *  - Scalar step counters `t` start at 1.
@@ -156,9 +157,10 @@ typedef struct {
  * Scalars computed on the host in double and rounded to fp32 once:
  *   decay = 1 - lr*wd, step = lr / (1 - beta1^t), c2 = 1 / sqrt(1 - beta2^t),
  *   omb1 = 1 - beta1, omb2 = 1 - beta2.
- * Per element, in fp32, in this order:
- *   p1 = p*decay;  m = beta1*m_hat + omb1*g;  v = beta2*v_hat + omb2*(g*g);
- *   den = sqrt(v)*c2 + eps;  p = p1 - step*(m/den);
+ * Per element, in fp32, in this order (fma: one rounding):
+ *   p1 = p*decay;  m = fma(beta1, m_hat, omb1*g);
+ *   v = fma(beta2, v_hat, omb2*(g*g));  den = fma(sqrt(v), c2, eps);
+ *   p = fma(-step, m/den, p1);
  * then m is UF8-encoded (m_block) and v is AL-encoded (v_block, log_floor).
  * The parameter update uses the fresh fp32 m and v, not their re-decoded
  * values.

@@ -192,11 +192,13 @@ void ora_adamw_update_fp32(float* p, const float* g, float* m, float* v,
     const float b1 = hp->beta1, b2 = hp->beta2, eps = hp->eps;
     for (int64_t i = 0; i < n; ++i) {
         float gi = g[i];
+        /* Eq. (1) in fp32; a product that is added is fused with the sum
+         * (one rounding), every other operation rounds on its own */
         float p1 = p[i] * decay;
-        float mi = b1 * m[i] + omb1 * gi;
-        float vi = b2 * v[i] + omb2 * (gi * gi);
-        float den = sqrtf(vi) * c2 + eps;
-        p[i] = p1 - step * (mi / den);
+        float mi = fmaf(b1, m[i], omb1 * gi);
+        float vi = fmaf(b2, v[i], omb2 * (gi * gi));
+        float den = fmaf(sqrtf(vi), c2, eps);
+        p[i] = fmaf(-step, mi / den, p1);
         m[i] = mi;
         v[i] = vi;
     }

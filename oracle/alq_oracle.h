@@ -7,8 +7,9 @@
  *
  * Plain, slow, single-threaded C. Transcendentals (log2, exp2) and all
  * reductions are computed in double and rounded once to fp32; the state EMAs
- * and parameter updates are fp32 in the operation order stated below (the
- * file is compiled with -ffp-contract=off so no multiply-add is fused).
+ * and parameter updates are fp32 in the operation order stated in the source
+ * (the file is compiled with -ffp-contract=off: a multiply-add is fused only
+ * where the source calls fmaf).
  *
  * Codes are stored as uint8_t when bits <= 8 and uint16_t when bits > 8.
  * Metadata is (l_min, Delta) per block, interleaved.
@@ -55,7 +56,9 @@ typedef struct {
     float lr, beta1, beta2, eps, weight_decay, log_floor;
 } ora_adamw_hp;
 
-/* fp32-state AdamW (m, v are fp32 arrays updated in place). */
+/* fp32-state AdamW (m, v are fp32 arrays updated in place):
+ * p1 = p decay; m = fma(b1, m, (1-b1) g); v = fma(b2, v, (1-b2) g^2);
+ * p = fma(-step, m / fma(sqrt(v), c2, eps), p1). */
 void ora_adamw_update_fp32(float* p, const float* g, float* m, float* v,
                            int64_t n, const ora_adamw_hp* hp, int64_t t);
 

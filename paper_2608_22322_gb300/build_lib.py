@@ -4,6 +4,8 @@ Every translation unit under csrc/ is compiled for sm_103a in parallel and
 linked into one shared library that exports the C ABI of include/alq.h.
 -fmad=false is part of the arithmetic contract (no silent multiply-add
 fusion); the codec's fused operations are written explicitly with fmaf().
+The flag is also passed to ptxas: the paired fp32 instructions (f32x2) are
+otherwise fused there even with an explicit rounding modifier.
 """
 from __future__ import annotations
 
@@ -22,7 +24,7 @@ OBJ_DIR = os.path.join(ROOT, "_build", "alq_obj")
 LIB = os.path.join(OUT_DIR, "libalq.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-fmad=false",
+NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-fmad=false", "-Xptxas", "--fmad=false",
                      "-Xcompiler", "-fPIC", "-I", CSRC, "-I", INCLUDE]
 
 

@@ -22,10 +22,41 @@ constexpr int kCH = 2;
 constexpr int kASeg = 128 * kCH;
 constexpr int kATile = 8 * kASeg;
 
+// Step scalars as broadcast pairs: the element arithmetic runs on pairs of
+// elements with the paired fp32 instructions (each component rounded exactly
+// as the scalar operation), and a pair operand held in the kernel's
+// parameter space costs no registers.
+struct AdamWPairs {
+    float2 decay, nstep, c2, omb1, omb2, beta1, beta2, eps;
+    float log_floor;
+};
+
+static AdamWPairs adamw_pairs(const AdamWScalars& s) {
+    AdamWPairs q;
+    q.decay = make_float2(s.decay, s.decay);
+    q.nstep = make_float2(-s.step, -s.step);  // p1 + (-step) q == p1 - step q exactly
+    q.c2 = make_float2(s.c2, s.c2);
+    q.omb1 = make_float2(s.omb1, s.omb1);
+    q.omb2 = make_float2(s.omb2, s.omb2);
+    q.beta1 = make_float2(s.beta1, s.beta1);
+    q.beta2 = make_float2(s.beta2, s.beta2);
+    q.eps = make_float2(s.eps, s.eps);
+    q.log_floor = s.log_floor;
+    return q;
+}
+
+__device__ __forceinline__ PlanEntry plan_entry(const PlanEntry* table, int ntensors,
+                                                const PlanEntry& single, int64_t tile,
+                                                int& cur) {
+    if (!table) return single;
+    while (cur + 1 < ntensors && table[cur + 1].first_tile <= tile) ++cur;
+    return table[cur];
+}
+
 template <int CPBV, int CPBM, int VBITS>
 __global__ void __launch_bounds__(kThreads, 3)
 adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t total_tiles,
-                   PlanEntry single, int v_block, int m_block, AdamWScalars s) {
+                   PlanEntry single, int v_block, int m_block, AdamWPairs s) {
     const int v_shift = __ffs(v_block) - 1, m_shift = __ffs(m_block) - 1;  // powers of two
     constexpr int NBV = kCH / CPBV;
     constexpr int NBM = kCH / CPBM;
@@ -38,42 +69,50 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
     const int wpbv = v_block > kASeg ? v_block / kASeg : 1;
     const int wpbm = m_block > kASeg ? m_block / kASeg : 1;
     const float kf = al8_table_k(lane);
+    const int G = gridDim.x;
     int cur = 0;
-    for (int64_t tile = blockIdx.x; tile < total_tiles; tile += gridDim.x) {
-        PlanEntry d;
-        if (table) {
-            while (cur + 1 < ntensors && table[cur + 1].first_tile <= tile) ++cur;
-            d = table[cur];
-        } else {
-            d = single;
-        }
+    for (int64_t tile = blockIdx.x; tile < total_tiles; tile += G) {
+        const PlanEntry d = plan_entry(table, ntensors, single, tile, cur);
         const int64_t n = d.n;
-        const int64_t seg0 = (tile - d.first_tile) * kATile + (int64_t)warp * kASeg;
-
-        // ---- stream in p, g and the codes of this lane's chunks
+        const int64_t t0 = (tile - d.first_tile) * kATile;
+        const int64_t seg0 = t0 + (int64_t)warp * kASeg;
+        // ---- p, g and the codes of this lane's chunks
         const bool full = seg0 + kASeg <= n;  // warp-uniform: unmasked I/O
+        const int64_t e0 = seg0 + 4 * lane;   // this lane's first element
         float4 g[kCH], p[kCH];
         uint32_t mw[kCH], vw[kCH * VBITS / 8];
+        if (full) {
+            // chunk c starts 128 c elements further: immediate offsets
+            const float4* gp = reinterpret_cast<const float4*>(d.g + e0);
+            const float4* pp = reinterpret_cast<const float4*>(d.p + e0);
+            const unsigned* mp = reinterpret_cast<const unsigned*>(d.m_codes + e0);
 #pragma unroll
-        for (int c = 0; c < kCH; ++c) {
-            const int64_t idx = chunk_index(seg0, c, lane);
-            if (full) {
-                g[c] = __ldcs(reinterpret_cast<const float4*>(d.g + idx));
-                p[c] = __ldcs(reinterpret_cast<const float4*>(d.p + idx));
-                mw[c] = __ldcs(reinterpret_cast<const unsigned int*>(d.m_codes + idx));
-            } else {
+            for (int c = 0; c < kCH; ++c) {
+                g[c] = __ldcs(gp + 32 * c);
+                p[c] = __ldcs(pp + 32 * c);
+                mw[c] = __ldcs(mp + 32 * c);
+                if constexpr (VBITS == 8) {
+                    vw[c] = __ldcs(reinterpret_cast<const unsigned*>((const uint8_t*)d.v_codes + e0) + 32 * c);
+                } else {
+                    const uint2 h = __ldcs(reinterpret_cast<const uint2*>((const uint16_t*)d.v_codes + e0) + 32 * c);
+                    vw[2 * c] = h.x;
+                    vw[2 * c + 1] = h.y;
+                }
+            }
+        } else {
+#pragma unroll
+            for (int c = 0; c < kCH; ++c) {
+                const int64_t idx = e0 + 128 * c;
                 g[c] = load4f(d.g, idx, n);
                 p[c] = load4f(d.p, idx, n);
                 mw[c] = load4b((const uint8_t*)d.m_codes, idx, n);
-            }
-            if constexpr (VBITS == 8) {
-                vw[c] = full ? __ldcs(reinterpret_cast<const unsigned int*>((const uint8_t*)d.v_codes + idx))
-                             : load4b((const uint8_t*)d.v_codes, idx, n);
-            } else {
-                const uint2 h = full ? __ldcs(reinterpret_cast<const uint2*>((const uint16_t*)d.v_codes + idx))
-                                     : load4h((const uint16_t*)d.v_codes, idx, n);
-                vw[2 * c] = h.x;
-                vw[2 * c + 1] = h.y;
+                if constexpr (VBITS == 8) {
+                    vw[c] = load4b((const uint8_t*)d.v_codes, idx, n);
+                } else {
+                    const uint2 h = load4h((const uint16_t*)d.v_codes, idx, n);
+                    vw[2 * c] = h.x;
+                    vw[2 * c + 1] = h.y;
+                }
             }
         }
 
@@ -106,38 +145,54 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
                                     odelta[e / 4 / CPBV]);
         }
 
-        // ---- update, write p; keep the fresh m and v
-        float mf[NE], vf[NE];
+        // ---- update, write p; keep the fresh m and v (element pairs)
+        float2 mf[NE / 2], vf2[NE / 2];
         uint32_t cvmin[kCH], cvmax[kCH], cmabs[kCH];
 #pragma unroll
         for (int c = 0; c < kCH; ++c) {
             const int bm = c / CPBM;
-            float pn[4];
+            const float2 dm2 = make_float2(dm[bm], dm[bm]);
+            // momentum bytes as exact floats: (q + 128) placed in the low
+            // mantissa of 1.5 * 2^23, then shifted back by 1.5 * 2^23 + 128
+            const uint32_t mx = mw[c] ^ 0x80808080u;
+            float2 pn[2];
             cvmin[c] = 0xFFFFFFFFu;
             cvmax[c] = 0u;
             cmabs[c] = 0u;
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const float mh = s8_to_float((mw[c] >> (8 * i)) & 0xFFu) * dm[bm];
-                const float gi = f4get(g[c], i);
-                const float p1 = f4get(p[c], i) * s.decay;
-                const float mm = s.beta1 * mh + s.omb1 * gi;
-                const float vv = s.beta2 * vh[4 * c + i] + s.omb2 * (gi * gi);
-                const float den = sqrtf(vv) * s.c2 + s.eps;
-                pn[i] = p1 - s.step * (mm / den);
-                mf[4 * c + i] = mm;
-                vf[4 * c + i] = vv;
-                const uint32_t vb = f2u(vv);
-                cvmin[c] = umix<false>(cvmin[c], vb - 1u);  // 0 -> max: min positive
-                cvmax[c] = umix<true>(cvmax[c], vb);
-                cmabs[c] = umix<true>(cmabs[c], f2u(mm) & 0x7FFFFFFFu);
+            for (int h = 0; h < 2; ++h) {
+                const float2 qf = make_float2(u2f(__byte_perm(mx, 0x4B400000u, 0x7640u | (2 * h))),
+                                              u2f(__byte_perm(mx, 0x4B400000u, 0x7640u | (2 * h + 1))));
+                const float2 mh = mul2(add2(qf, make_float2(-12583040.0f, -12583040.0f)), dm2);
+                const float2 gi = h == 0 ? make_float2(g[c].x, g[c].y) : make_float2(g[c].z, g[c].w);
+                const float2 pi = h == 0 ? make_float2(p[c].x, p[c].y) : make_float2(p[c].z, p[c].w);
+                // products enter sums only through fma2: a paired product
+                // feeding a paired add could be contracted by the compiler
+                const float2 p1 = mul2(pi, s.decay);
+                const float2 mm = fma2(s.beta1, mh, mul2(s.omb1, gi));
+                const float2 vh2 = make_float2(vh[4 * c + 2 * h], vh[4 * c + 2 * h + 1]);
+                const float2 vv = fma2(s.beta2, vh2, mul2(s.omb2, mul2(gi, gi)));
+                const float2 den = fma2(make_float2(sqrtf(vv.x), sqrtf(vv.y)), s.c2, s.eps);
+                const float2 u = make_float2(mm.x / den.x, mm.y / den.y);
+                pn[h] = fma2(s.nstep, u, p1);
+                mf[2 * c + h] = mm;
+                vf2[2 * c + h] = vv;
+                const uint32_t vbx = f2u(vv.x), vby = f2u(vv.y);
+                cvmin[c] = umix<false>(cvmin[c], umix<false>(vbx - 1u, vby - 1u));  // 0 -> max: min positive
+                cvmax[c] = umix<true>(cvmax[c], umix<true>(vbx, vby));
+                cmabs[c] = umix<true>(cmabs[c], umix<true>(f2u(mm.x) & 0x7FFFFFFFu, f2u(mm.y) & 0x7FFFFFFFu));
             }
-            const int64_t idx = chunk_index(seg0, c, lane);
-            const float4 pv = make_float4(pn[0], pn[1], pn[2], pn[3]);
+            const float4 pv = make_float4(pn[0].x, pn[0].y, pn[1].x, pn[1].y);
             if (full)
-                __stcs(reinterpret_cast<float4*>(d.p + idx), pv);
+                __stcs(reinterpret_cast<float4*>(d.p + e0) + 32 * c, pv);
             else
-                store4f(d.p, idx, n, pv);
+                store4f(d.p, e0 + 128 * c, n, pv);
+        }
+        float vf[NE];
+#pragma unroll
+        for (int j = 0; j < NE / 2; ++j) {
+            vf[2 * j] = vf2[j].x;
+            vf[2 * j + 1] = vf2[j].y;
         }
 
         // ---- new block statistics
@@ -175,20 +230,26 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
 #pragma unroll
         for (int c = 0; c < kCH; ++c) {
             const int bm = c / CPBM;
-            const int64_t idx = chunk_index(seg0, c, lane);
-            uint32_t qm = 0;
-            if (ms[bm] > 0.0f) {
+            const int64_t idx = e0 + 128 * c;
+            // q = rint((m sc) inv) (scalar: the product must round before
+            // the rounding add) as the low byte of 1.5 * 2^23 + q, the two's
+            // complement byte for q < 0; all codes are 0 when the block's
+            // absmax is 0 (inv = 0)
+            uint32_t rb[4];
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    qm |= ((uint32_t)uf8_quantize(mf[4 * c + i], msc[bm], minv[bm]) & 0xFFu) << (8 * i);
+            for (int i = 0; i < 4; ++i) {
+                const float2 m2 = mf[2 * c + i / 2];
+                rb[i] = f2u(((i & 1 ? m2.y : m2.x) * msc[bm]) * minv[bm] + 12582912.0f);
             }
+            const uint32_t qm = __byte_perm(__byte_perm(rb[0], rb[1], 0x0040u),
+                                            __byte_perm(rb[2], rb[3], 0x0040u), 0x5410u);
             if (full) {
-                __stcs(reinterpret_cast<unsigned int*>(d.m_codes + idx), qm);
+                __stcs(reinterpret_cast<unsigned int*>(d.m_codes + e0) + 32 * c, qm);
                 if constexpr (VBITS == 8)
-                    __stcs(reinterpret_cast<unsigned int*>((uint8_t*)d.v_codes + idx),
+                    __stcs(reinterpret_cast<unsigned int*>((uint8_t*)d.v_codes + e0) + 32 * c,
                            qv[4 * c] | (qv[4 * c + 1] << 8) | (qv[4 * c + 2] << 16) | (qv[4 * c + 3] << 24));
                 else
-                    __stcs(reinterpret_cast<uint2*>((uint16_t*)d.v_codes + idx),
+                    __stcs(reinterpret_cast<uint2*>((uint16_t*)d.v_codes + e0) + 32 * c,
                            make_uint2(qv[4 * c] | (qv[4 * c + 1] << 16), qv[4 * c + 2] | (qv[4 * c + 3] << 16)));
             } else {
                 store4b((uint8_t*)d.m_codes, idx, n, qm);
@@ -227,7 +288,8 @@ static int launch_adamw_t(const PlanEntry* table, int ntensors, int64_t total_ti
                           const AdamWScalars& s, cudaStream_t stream) {
     auto k = adamw_fused_kernel<CPBV, CPBM, VBITS>;
     const int grid = persistent_grid((const void*)k, kThreads, 0, total_tiles);
-    k<<<grid, kThreads, 0, stream>>>(table, ntensors, total_tiles, single, v_block, m_block, s);
+    k<<<grid, kThreads, 0, stream>>>(table, ntensors, total_tiles, single, v_block, m_block,
+                                     adamw_pairs(s));
     return check_launch();
 }
 

@@ -60,6 +60,9 @@ int persistent_grid(const void* kernel, int threads, size_t smem, int64_t ntiles
         if (it != cache.end()) occ = it->second;
     }
     if (occ == 0) {
+        // dynamic shared memory beyond the default 48 KB needs an opt-in per
+        // kernel and device; the launch reports a failure if it is refused
+        if (smem > 0) cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kernel, threads, smem) != cudaSuccess ||
             occ < 1)
             occ = 1;

@@ -23,6 +23,7 @@
 
 #include <mutex>
 
+#include "alq_async.cuh"
 #include "alq_kernels.cuh"
 
 namespace alq {
@@ -33,7 +34,6 @@ constexpr int kStages = 4;
 constexpr int kAStage = kGM * kGK * 2;     // 16 KB
 constexpr int kBStage = 256 * kGK * 2;     // 32 KB (rank <= 256)
 constexpr int kGemmSmem = kStages * (kAStage + kBStage) + 1024 + 256;
-constexpr uint32_t kWaitLimit = 1u << 26;  // bounded mbarrier polls
 
 // ------------------------------------------------------------ workspace --
 struct ApWs {
@@ -109,34 +109,6 @@ to_bf16_t_kernel(const float* __restrict__ g, int rows, int cols, uint16_t* __re
 }
 
 // ------------------------------------------------------ PTX primitives --
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-    return (uint32_t)__cvta_generic_to_shared(p);
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-                 : "memory");
-}
-
-// Bounded wait on an mbarrier phase; false after kWaitLimit polls.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
-    for (uint32_t i = 0; i < kWaitLimit; ++i) {
-        uint32_t done;
-        asm volatile(
-            "{\n.reg .pred p;\nmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-            "selp.b32 %0, 1, 0, p;\n}\n"
-            : "=r"(done)
-            : "r"(bar), "r"(parity)
-            : "memory");
-        if (done) return true;
-    }
-    return false;
-}
-
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
                                             uint32_t bar) {
     asm volatile(
@@ -231,7 +203,7 @@ apollo_project_kernel(const __grid_constant__ CUtensorMap tmA,
             mbar_init(empty0 + 8 * s, 1);
         }
         mbar_init(accum, 1);
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        mbar_init_fence();
     }
     if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(

@@ -63,7 +63,9 @@ int record_cuda(cudaError_t e);       // ALQ_OK or ALQ_ERR_CUDA (and records tex
 int check_launch();                   // cudaGetLastError -> status
 int sm_count();                       // multiprocessors of the current device
 // Persistent-grid size: min(ntiles, SMs x resident CTAs of `kernel`), the
-// residency queried once per kernel and device.
+// residency queried once per kernel and device (which also opts the kernel
+// in to `smem` bytes of dynamic shared memory; every launch of a kernel must
+// pass the same `smem`).
 int persistent_grid(const void* kernel, int threads, size_t smem, int64_t ntiles);
 int64_t blocks_of(int64_t n, int block);
 

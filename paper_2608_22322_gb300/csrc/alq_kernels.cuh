@@ -18,6 +18,37 @@
 
 namespace alq {
 
+// ----------------------------------------------- paired fp32 arithmetic --
+// Two independent fp32 operations per instruction (sm_100 and later). The
+// explicit .rn modifier makes each component round exactly like the scalar
+// operation and forbids contraction into a fused multiply-add.
+__device__ __forceinline__ float2 mul2(float2 a, float2 b) {
+    float2 r;
+    asm("{\n.reg .b64 a, b, d;\nmov.b64 a, {%2, %3};\nmov.b64 b, {%4, %5};\n"
+        "mul.rn.f32x2 d, a, b;\nmov.b64 {%0, %1}, d;\n}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return r;
+}
+
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+    float2 r;
+    asm("{\n.reg .b64 a, b, d;\nmov.b64 a, {%2, %3};\nmov.b64 b, {%4, %5};\n"
+        "add.rn.f32x2 d, a, b;\nmov.b64 {%0, %1}, d;\n}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return r;
+}
+
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+    float2 r;
+    asm("{\n.reg .b64 a, b, c, d;\nmov.b64 a, {%2, %3};\nmov.b64 b, {%4, %5};\n"
+        "mov.b64 c, {%6, %7};\nfma.rn.f32x2 d, a, b, c;\nmov.b64 {%0, %1}, d;\n}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return r;
+}
+
 // ------------------------------------------------------------- chunk I/O --
 __device__ __forceinline__ int64_t blocks_of_dev(int64_t n, int block) {
     return (n + block - 1) / block;
@@ -213,7 +244,7 @@ __device__ __forceinline__ void al8_decode_chunks(const uint32_t (&w)[CH], const
             any_fb |= (q != 0u) & (fb | !fast);
         }
     }
-    if (__any_sync(0xFFFFFFFFu, any_fb)) {
+    if (__builtin_expect(__any_sync(0xFFFFFFFFu, any_fb), 0)) {
         // rare: redo the boundary test per element and recompute in FP64
 #pragma unroll
         for (int c = 0; c < CH; ++c) {
@@ -250,7 +281,7 @@ __device__ __forceinline__ void al_encode_chunks(const float (&x)[4 * CH], const
         q[e] = nz ? v : 0u;
         any_fb |= nz & fb;
     }
-    if (__any_sync(0xFFFFFFFFu, any_fb)) {
+    if (__builtin_expect(__any_sync(0xFFFFFFFFu, any_fb), 0)) {
 #pragma unroll
         for (int e = 0; e < 4 * CH; ++e) {
             const int b = e / 4 / CPB;
@@ -289,7 +320,7 @@ __device__ __forceinline__ void al8_build_values(float* vals, float2* tab,
             any_fb |= (q != 0u) & (fb | !fast);
         }
     }
-    if (__any_sync(0xFFFFFFFFu, any_fb)) {
+    if (__builtin_expect(__any_sync(0xFFFFFFFFu, any_fb), 0)) {
 #pragma unroll
         for (int b = 0; b < NB; ++b) {
             const bool fast = al8_fast_ok(lmin[b], delta[b]);
@@ -331,8 +362,7 @@ __device__ __forceinline__ float al_decode_direct(uint32_t q, float lmin, float 
     if (lmin >= -96.0f && delta > 0.0f) {
         float rh, rl;
         al_level_ff(lmin, delta, int_to_float_small((int)q - 1), Lm2, 1.0f / Lm2, rh, rl);
-        const float hu = half_ulp_below(rh);
-        if (fabsf(rl) < hu - hu * 0x1p-16f) return rh;
+        if (!ziv_fails(rh, rl)) return rh;  // rh + rl: relative error below 2^-45
     }
     return al_dequantize_fp64(q, lmin, delta, (double)Lm2);
 }
