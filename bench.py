@@ -15,6 +15,8 @@ region), SM clocks sampled during the timed region, and the kernel launch
 count. With N > 1 (torchrun) every rank runs an independent replica (the
 AdamW step has no cross-rank exchange); value = params of all ranks / max
 rank time. --impl reference times the CPU oracle instead (the reference arm).
+--workload adafactor|came|apollo|codec times the other hot-path rows instead,
+one JSON line each (see run_rows).
 """
 from __future__ import annotations
 
@@ -53,6 +55,10 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--workload", default="adamw",
+                    choices=["adamw", "adafactor", "came", "apollo", "codec"],
+                    help="adamw: the headline TinyLlama AdamW step (default); the others "
+                         "time the remaining hot-path rows, one JSON line each")
     return ap.parse_args()
 
 
@@ -378,9 +384,335 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+# ------------------------------------------------- the other hot-path rows --
+ROW_METRICS = {
+    "adafactor": "optimizer-step params/sec and achieved HBM GB/s, Adafactor (AL16 factors, "
+                 "UF8 momentum)",
+    "came": "optimizer-step params/sec and achieved HBM GB/s, CAME (AL16 factored V and C, "
+            "UF8 momentum)",
+    "apollo": "optimizer-step params/sec and achieved HBM GB/s, APOLLO (rank-256 projection, "
+              "UF8 M^P, AL8 V^P)",
+    "codec": "codec elements/sec and achieved HBM GB/s, AL8 and UF8 encode + decode",
+}
+
+
+def _device_student_t(torch, t, scale, nu, seed):
+    """scale * z / sqrt(chi2_nu / nu), drawn on the device from a seeded
+    generator (nu integer: chi2 as a sum of nu squared normals)."""
+    gen = torch.Generator(device=t.device)
+    gen.manual_seed(seed)
+    t.normal_(0.0, 1.0, generator=gen)
+    chi = torch.zeros_like(t)
+    z = torch.empty_like(t)
+    for _ in range(int(nu)):
+        z.normal_(0.0, 1.0, generator=gen)
+        chi.addcmul_(z, z)
+    t.mul_(scale).div_(torch.sqrt(chi / nu))
+    del chi, z
+
+
+def _row_adafactor(torch, np, wl, B, dev):
+    """Adafactor on one 4096 x 4096 weight: row and column factors AL16 in
+    blocks of 128, momentum UF8 in blocks of 256, gradients N(0, 1e-3) with a
+    lognormal(0, 1) scale per column and 5% exact zeros. Algorithmic bytes:
+    G read once (4), p read and written (8), momentum codes read and written
+    (2), absmax and factor states; the factored sums make the library read G
+    three times (22 B/param), which is not counted."""
+    cfg = wl.CONFIGS["adafactor"]
+    rows, cols = cfg["shape"]
+    n = rows * cols
+    hp = dict(lr=cfg["lr"], eps1=cfg["eps1"], clip_d=cfg["clip_d"], decay_rate=cfg["decay_rate"],
+              beta1=cfg["beta1"], weight_decay=cfg["weight_decay"],
+              log_floor=float(np.float32(np.log2(cfg["eps1"]))))
+    p = torch.empty(n, dtype=torch.float32, device=dev)
+    wl.torch_device_normal_(p, 0.02, 20262)
+    colscale = torch.from_numpy(wl.rng(20263).lognormal(0.0, 1.0, cols).astype(np.float32)).to(dev)
+    gs = []
+    for k in range(2):
+        g = torch.empty(n, dtype=torch.float32, device=dev)
+        wl.torch_device_normal_(g, cfg["grad_std"], 20270 + k)
+        g.view(rows, cols).mul_(colscale)
+        wl.torch_device_zero_(g, cfg["zero_frac"], 20280 + k)
+        gs.append(g)
+    fb, fbits = cfg["fac_block"], cfg["fac_bits"]
+    st = {}
+    for name, m in (("r", rows), ("c", cols)):
+        st[name] = (torch.zeros(m, dtype=torch.int16, device=dev),
+                    torch.zeros(2 * ((m + fb - 1) // fb), dtype=torch.float32, device=dev))
+    mc = torch.zeros(n, dtype=torch.int8, device=dev)
+    ma = torch.zeros((n + 255) // 256, dtype=torch.float32, device=dev)
+    ws = torch.empty(B.al_workspace_size(B.AL_OP_ADAFACTOR, rows, cols), dtype=torch.uint8,
+                     device=dev)
+
+    def step(t):
+        B.al_adafactor_step(p, gs[t % 2], rows, cols, st["r"][0], st["r"][1], st["c"][0],
+                            st["c"][1], fbits, fb, mc, ma, 256, hp, t, ws)
+
+    fac = sum(2 * 2 * m + 16 * ((m + fb - 1) // fb) for m in (rows, cols))
+    nbytes = 14 * n + 8 * ma.numel() + fac
+
+    def oracle_sample(ora, t):
+        import numpy as np_
+        ph, gh = p.cpu().numpy().copy(), gs[0].cpu().numpy()
+        rc, rm = st["r"][0].cpu().numpy().view(np_.uint16).copy(), st["r"][1].cpu().numpy().copy()
+        cc, cm = st["c"][0].cpu().numpy().view(np_.uint16).copy(), st["c"][1].cpu().numpy().copy()
+        mch, mah = mc.cpu().numpy().copy(), ma.cpu().numpy().copy()
+        t0 = time.perf_counter()
+        ora.adafactor_step(ph, gh, rows, cols, rc, rm, cc, cm, fbits, fb, mch, mah, 256, hp, t)
+        dt = time.perf_counter() - t0
+        return n / dt, f"one step of the whole {rows}x{cols} matrix ({dt:.1f} s, single thread)"
+
+    return dict(step=step, n=n, bytes=nbytes, launches=6, oracle=oracle_sample,
+                workload=f"Adafactor {rows}x{cols}, AL16 factors block 128, UF8 momentum block 256",
+                bytes_note="algorithmic minimum 14.03 B/param (G read once)")
+
+
+def _row_came(torch, np, wl, B, dev):
+    """CAME on 22 matrices of 2048 x 5632 (253,755,392 params): factored V
+    and confidence C in AL16 blocks of 128, UF8 momentum in blocks of 256,
+    gradients 1e-3 * Student-t(3) with 5% exact zeros. Algorithmic bytes: G
+    read once (4), p read and written (8), momentum codes read and written
+    (2), absmax and the four factor states; the library's passes read G three
+    times and the momentum codes twice, which is not counted."""
+    cfg = wl.CONFIGS["came"]
+    rows, cols = cfg["shape"]
+    nm = cfg["n_mats"]
+    n1 = rows * cols
+    hp = dict(lr=cfg["lr"], beta1=cfg["beta1"], beta2=cfg["beta2"], beta3=cfg["beta3"],
+              eps1=cfg["eps1"], eps2=cfg["eps2"], clip_d=cfg["clip_d"],
+              weight_decay=cfg["weight_decay"],
+              log_floor_v=float(np.float32(np.log2(cfg["eps1"]))),
+              log_floor_c=float(np.float32(np.log2(cfg["eps2"]))))
+    vb, cb = cfg["v_block"], cfg["c_block"]
+
+    def fac(m, blk):
+        return (torch.zeros(m, dtype=torch.int16, device=dev),
+                torch.zeros(2 * ((m + blk - 1) // blk), dtype=torch.float32, device=dev))
+
+    mats = []
+    for i in range(nm):
+        p = torch.empty(n1, dtype=torch.float32, device=dev)
+        wl.torch_device_normal_(p, 0.02, 20300 + i)
+        gs = []
+        for k in range(2):
+            g = torch.empty(n1, dtype=torch.float32, device=dev)
+            _device_student_t(torch, g, cfg["grad_scale"], cfg["nu"], 20400 + 100 * k + i)
+            wl.torch_device_zero_(g, cfg["zero_frac"], 20600 + 100 * k + i)
+            gs.append(g)
+        mats.append(dict(p=p, gs=gs, vr=fac(rows, vb), vc=fac(cols, vb), cr=fac(rows, cb),
+                         cc=fac(cols, cb), mc=torch.zeros(n1, dtype=torch.int8, device=dev),
+                         ma=torch.zeros((n1 + 255) // 256, dtype=torch.float32, device=dev)))
+    ws = torch.empty(B.al_workspace_size(B.AL_OP_CAME, rows, cols), dtype=torch.uint8, device=dev)
+
+    def step(t):
+        for m in mats:
+            B.al_came_step(m["p"], m["gs"][t % 2], rows, cols, m["vr"][0], m["vr"][1], m["vc"][0],
+                           m["vc"][1], 16, vb, m["cr"][0], m["cr"][1], m["cc"][0], m["cc"][1],
+                           16, cb, m["mc"], m["ma"], 256, hp, t, ws)
+
+    facb = sum(2 * 2 * mm + 16 * ((mm + blk - 1) // blk)
+               for mm, blk in ((rows, vb), (cols, vb), (rows, cb), (cols, cb)))
+    nbytes = nm * (14 * n1 + 8 * ((n1 + 255) // 256) + facb)
+
+    def oracle_sample(ora, t):
+        import numpy as np_
+        m = mats[0]
+        h = lambda x: x.cpu().numpy().copy()
+        u16 = lambda x: x.cpu().numpy().view(np_.uint16).copy()
+        ph, gh = h(m["p"]), m["gs"][0].cpu().numpy()
+        args = [u16(m["vr"][0]), h(m["vr"][1]), u16(m["vc"][0]), h(m["vc"][1]), 16, vb,
+                u16(m["cr"][0]), h(m["cr"][1]), u16(m["cc"][0]), h(m["cc"][1]), 16, cb,
+                h(m["mc"]), h(m["ma"]), 256]
+        t0 = time.perf_counter()
+        ora.came_step(ph, gh, rows, cols, *args, hp, t)
+        dt = time.perf_counter() - t0
+        return n1 / dt, f"one step of one {rows}x{cols} matrix ({dt:.1f} s, single thread)"
+
+    return dict(step=step, n=nm * n1, bytes=nbytes, launches=9 * nm, oracle=oracle_sample,
+                workload=f"CAME {nm} x {rows}x{cols}, AL16 factored V and C block 128, "
+                         f"UF8 momentum block 256",
+                bytes_note="algorithmic minimum 14.03 B/param (G read once)")
+
+
+def _row_apollo(torch, np, wl, B, dev):
+    """APOLLO over the 154 TinyLlama-1.1B attention/MLP matrices
+    (968,884,224 params): one Gaussian rank-256 projection per matrix (bf16),
+    projected moments UF8 / AL8 in blocks of 256, gradients N(0, 1e-3).
+    Algorithmic bytes: G read for the projection and again for the scaled
+    update (8), p read and written (8), projected states and their block
+    constants; the bf16 staging copy of G is not counted. FLOPs: 2 r s L per
+    matrix for the projection."""
+    cfg = wl.CONFIGS["tinyllama_apollo"]
+    r = cfg["rank"]
+    hp = dict(lr=cfg["lr"], beta1=cfg["beta1"], beta2=cfg["beta2"], eps=cfg["eps"],
+              alpha=cfg["alpha"], weight_decay=cfg["weight_decay"], norm_growth_gamma=0.0,
+              log_floor=float(np.float32(np.log2(1e-16))), rank=r)
+    mats, nbytes, flops, n_tot, ws_bytes = [], 0, 0, 0, 0
+    for i, (_, (rows, cols)) in enumerate(wl.tinyllama_matrices()):
+        n1 = rows * cols
+        s_, L = min(rows, cols), max(rows, cols)
+        p = torch.empty(n1, dtype=torch.float32, device=dev)
+        wl.torch_device_normal_(p, 0.02, 21000 + i)
+        gs = []
+        for k in range(2):
+            g = torch.empty(n1, dtype=torch.float32, device=dev)
+            wl.torch_device_normal_(g, cfg["grad_std"], 22000 + 1000 * k + i)
+            gs.append(g)
+        P = torch.empty(r * s_, dtype=torch.float32, device=dev)
+        wl.torch_device_normal_(P, float(np.sqrt(1.0 / r)), 24000 + i)
+        Pb = P.to(torch.bfloat16).view(torch.int16)
+        del P
+        npj = L * r
+        mats.append(dict(p=p, gs=gs, rows=rows, cols=cols, P=Pb,
+                         mc=torch.zeros(npj, dtype=torch.int8, device=dev),
+                         ma=torch.zeros(npj // 256, dtype=torch.float32, device=dev),
+                         vc=torch.zeros(npj, dtype=torch.uint8, device=dev),
+                         vm=torch.zeros(2 * (npj // 256), dtype=torch.float32, device=dev),
+                         prev=torch.zeros(1, dtype=torch.float32, device=dev)))
+        nbytes += 16 * n1 + 4 * npj + 24 * (npj // 256)
+        flops += 2 * r * s_ * L
+        n_tot += n1
+        ws_bytes = max(ws_bytes, B.al_workspace_size(B.AL_OP_APOLLO, rows, cols, r))
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+
+    def step(t):
+        for m in mats:
+            B.al_apollo_step(m["p"], m["gs"][t % 2], m["rows"], m["cols"], m["P"], m["mc"],
+                             m["ma"], 256, m["vc"], m["vm"], 8, 256, m["prev"], hp, t, ws)
+
+    def oracle_sample(ora, t):
+        m = mats[0]
+        rows, cols = m["rows"], m["cols"]
+        h = lambda x: x.cpu().numpy().copy()
+        Ph = m["P"].cpu().numpy().view(np.uint16).copy()
+        t0 = time.perf_counter()
+        ora.apollo_step(h(m["p"]), m["gs"][0].cpu().numpy(), rows, cols, Ph, h(m["mc"]),
+                        h(m["ma"]), 256, h(m["vc"]), h(m["vm"]), 8, 256, np.float32(0.0), hp, t)
+        dt = time.perf_counter() - t0
+        return rows * cols / dt, (f"one step of one {rows}x{cols} matrix incl. the rank-{r} "
+                                  f"projection in double ({dt:.1f} s, single thread)")
+
+    return dict(step=step, n=n_tot, bytes=nbytes, flops=flops, launches=4 * len(mats),
+                oracle=oracle_sample,
+                workload=f"APOLLO TinyLlama-1.1B {len(mats)} matrices, rank {r}, UF8 M^P, "
+                         f"AL8 V^P block 256",
+                bytes_note="G twice, p read+write, projected states; bf16 staging not counted")
+
+
+def _row_codec(torch, np, wl, B, dev):
+    """AL8 encode + AL8 decode + UF8 encode + UF8 decode of 2^28 elements
+    (blocks of 256): second-moment-like values 1e-6 * chi2_1 with 1% exact
+    zeros for AL8, N(0, 1e-3) for UF8. Bytes: encode reads 4 and writes 1 per
+    element, decode the reverse, plus block constants."""
+    n = 1 << 28
+    x = torch.empty(n, dtype=torch.float32, device=dev)
+    wl.torch_device_normal_(x, 1.0, 25000)
+    x.mul_(x).mul_(1e-6)
+    wl.torch_device_zero_(x, 0.01, 25001)
+    m = torch.empty(n, dtype=torch.float32, device=dev)
+    wl.torch_device_normal_(m, 1e-3, 25002)
+    vc = torch.empty(n, dtype=torch.uint8, device=dev)
+    vm = torch.empty(2 * (n // 256), dtype=torch.float32, device=dev)
+    mc = torch.empty(n, dtype=torch.int8, device=dev)
+    ma = torch.empty(n // 256, dtype=torch.float32, device=dev)
+    out = torch.empty(n, dtype=torch.float32, device=dev)
+    floor = float(np.float32(np.log2(1e-16)))
+
+    def step(t):
+        B.al_encode(x, 256, 8, floor, vc, vm)
+        B.al_decode(vc, vm, 256, 8, out)
+        B.uf8_encode(m, 256, mc, ma)
+        B.uf8_decode(mc, ma, 256, out)
+
+    nbytes = 20 * n + 2 * (8 * (n // 256)) + 2 * (4 * (n // 256))
+
+    def oracle_sample(ora, t):
+        k = 1 << 24
+        xh = x[:k].cpu().numpy()
+        t0 = time.perf_counter()
+        codes, meta = ora.al_encode(xh, 256, 8, floor)
+        ora.al_decode(codes, meta, 256, 8)
+        dt = time.perf_counter() - t0
+        return k / dt, f"AL8 encode + decode of {k} elements ({dt:.1f} s, single thread)"
+
+    return dict(step=step, n=n, bytes=nbytes, launches=4, oracle=oracle_sample,
+                workload="codec 2^28 elements, AL8 encode+decode and UF8 encode+decode, block 256",
+                bytes_note="20 B/element + block constants")
+
+
+def run_rows(args):
+    """One JSON line for a non-headline hot-path row: device time of whole
+    steps (all of the row's launches) with CUDA events, bytes/time against the
+    measured HBM copy peak, the oracle on a bounded sample, SM clocks."""
+    import numpy as np
+    import torch
+
+    from paper_2608_22322_gb300 import build_lib
+    build_lib.build()
+    from paper_2608_22322_gb300 import binding as B
+    from paper_2608_22322_gb300 import workloads as wl
+
+    if int(os.environ.get("RANK", "0")) != 0:
+        return  # the rows are single-GPU measurements
+    dev = torch.device("cuda", 0)
+    build = {"adafactor": _row_adafactor, "came": _row_came, "apollo": _row_apollo,
+             "codec": _row_codec}[args.workload]
+    w = build(torch, np, wl, B, dev)
+    t = 0
+    for _ in range(args.warmup):
+        t += 1
+        w["step"](t)
+    torch.cuda.synchronize(dev)
+    props = torch.cuda.get_device_properties(dev)
+    sampler = ClockSampler(str(getattr(props, "uuid", "") or "").replace("GPU-", ""))
+    sampler.start()
+    time.sleep(0.3)
+    stream = torch.cuda.current_stream(dev)
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize(dev)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        t += 1
+        w["step"](t)
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    ms_step = ev0.elapsed_time(ev1) / args.steps
+    clocks = sampler.stop()
+    peaks, peak_src = measured_peaks()
+    peak = float(peaks.get("hbm_gbs", 6800.0))
+    achieved = w["bytes"] / (ms_step * 1e-3) / 1e9
+    cpu = None
+    if not args.no_cpu:
+        import oracle as ora
+        v, sample = w["oracle"](ora, t + 1)
+        cpu = {"value": v, "unit": "params/s" if args.workload != "codec" else "elements/s",
+               "cores": 1, "kind": "oracle", "sample": sample}
+    line = {
+        "metric": ROW_METRICS[args.workload], "value": w["n"] / (ms_step * 1e-3),
+        "unit": "params/s" if args.workload != "codec" else "elements/s", "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": w["workload"], "params_per_gpu": w["n"], "bytes_per_step": w["bytes"],
+                   "bytes": w["bytes_note"], "parallelism": "single GPU"},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": None,
+                     "peak_source": f"{peak_src} hbm_gbs",
+                     "kernel": "whole step (all launches; per-kernel shares in profiles/)"},
+        "cpu_baseline": cpu, "e2e": None, "clocks": clocks,
+        "gpu_launches": w["launches"] * args.steps,
+    }
+    if "flops" in w:
+        line["projection_tflops"] = w["flops"] / (ms_step * 1e-3) / 1e12
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse_args()
-    if args.impl == "reference":
+    if args.workload != "adamw":
+        run_rows(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)
