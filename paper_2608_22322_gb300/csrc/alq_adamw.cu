@@ -53,8 +53,11 @@ __device__ __forceinline__ PlanEntry plan_entry(const PlanEntry* table, int nten
     return table[cur];
 }
 
+// Four CTAs per SM (64 registers): the step is bound by the latency of each
+// warp's dependent chains more than by issue slots, and 32 resident warps
+// hide more of it than 24 do, despite a few spilled registers.
 template <int CPBV, int CPBM, int VBITS>
-__global__ void __launch_bounds__(kThreads, 3)
+__global__ void __launch_bounds__(kThreads, 4)
 adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t total_tiles,
                    PlanEntry single, int v_block, int m_block, AdamWPairs s) {
     const int v_shift = __ffs(v_block) - 1, m_shift = __ffs(m_block) - 1;  // powers of two

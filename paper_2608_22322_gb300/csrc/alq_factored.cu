@@ -41,6 +41,8 @@ struct FacWs {
     float* a2;        // [rows]
     float* b2;        // [cols]
     float* scal;      // [4]: icf
+    double* rsum;     // [rows / 128 + 1]: per-block sums of the fresh row factor (V)
+    double* rsum2;    // same for the confidence row factor (C)
     size_t bytes;
 };
 
@@ -68,6 +70,8 @@ static FacWs fac_layout(void* base, int64_t rows, int64_t cols) {
     w.a2 = (float*)take(sizeof(float) * rows);
     w.b2 = (float*)take(sizeof(float) * cols);
     w.scal = (float*)take(sizeof(float) * 4);
+    w.rsum = (double*)take(sizeof(double) * (rows / 128 + 1));
+    w.rsum2 = (double*)take(sizeof(double) * (rows / 128 + 1));
     w.bytes = off;
     return w;
 }
@@ -98,51 +102,76 @@ sumsq_kernel(const float* __restrict__ g, int rows, int cols, ResidualArgs ra,
 #pragma unroll
     for (int k = 0; k < 16; ++k) ch[k] = cl[k] = 0.0f;
     float icf = 0.0f;
-    if (MODE == 1) icf = __ldg(ra.scal);
-    for (int rr = 0; rr < kFR / 8; ++rr) {
-        const int row = r0 + warp + 8 * rr;
-        float rh = 0.0f, rl = 0.0f;
-        if (row < rows) {
-            float ai = 0.0f;
-            if (MODE == 1) ai = __ldg(ra.a + row);
+    float4 bv[4];  // column scales of this lane's columns (CAME residual)
+    if (MODE == 1) {
+        icf = __ldg(ra.scal);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int col = c0 + 128 * k + 4 * lane;
+            bv[k] = col < cols ? __ldg(reinterpret_cast<const float4*>(ra.b + col))
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+    }
+    // two rows per pass: all loads first (zero past the matrix), then the
+    // terms in row order, so the sums keep the order of a row-by-row walk
+    for (int rr = 0; rr < kFR / 8; rr += 2) {
+        float4 gv[2][4];
+        uint32_t mw[2][4];
+        float dm[2][4], ai[2];
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const int row = r0 + warp + 8 * (rr + q);
+            ai[q] = (MODE == 1 && row < rows) ? __ldg(ra.a + row) : 0.0f;
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
                 const int col = c0 + 128 * k + 4 * lane;
-                if (col < cols) {
+                gv[q][k] = make_float4(0.f, 0.f, 0.f, 0.f);
+                mw[q][k] = 0u;
+                dm[q][k] = 0.0f;
+                if (row < rows && col < cols) {
                     const int64_t idx = (int64_t)row * cols + col;
-                    const float4 gv = __ldcs(reinterpret_cast<const float4*>(g + idx));
-                    float4 bv;
-                    uint32_t mw = 0;
-                    float dm = 0.0f;
+                    gv[q][k] = __ldcs(reinterpret_cast<const float4*>(g + idx));
                     if (MODE == 1) {
-                        bv = __ldg(reinterpret_cast<const float4*>(ra.b + col));
-                        mw = __ldcs(reinterpret_cast<const unsigned int*>(ra.m_codes + idx));
-                        dm = __ldg(ra.m_absmax + (idx >> ra.m_shift)) / 127.0f;
-                    }
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const float x = f4get(gv, j);
-                        float h, l;
-                        if (MODE == 0) {
-                            two_prod(x, x, h, l);
-                        } else {
-                            const float u = (x * ai) * f4get(bv, j);
-                            const float uh = u * icf;
-                            const float mh = s8_to_float((mw >> (8 * j)) & 0xFFu) * dm;
-                            const float mk = ra.beta1 * mh + ra.omb1 * uh;
-                            const float d = uh - mk;
-                            h = d * d + ra.eps2;
-                            l = 0.0f;
-                        }
-                        ff_acc(ch[4 * k + j], cl[4 * k + j], h, l);
-                        ff_acc(rh, rl, h, l);
+                        mw[q][k] = __ldcs(reinterpret_cast<const unsigned int*>(ra.m_codes + idx));
+                        dm[q][k] = __ldg(ra.m_absmax + (idx >> ra.m_shift)) / 127.0f;
                     }
                 }
             }
         }
-        ff_warp_sum(rh, rl);
-        if (lane == 0 && row < rows)
-            rowpart[(int64_t)blockIdx.x * rows + row] = (double)rh + (double)rl;
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const int row = r0 + warp + 8 * (rr + q);
+            float rh = 0.0f, rl = 0.0f;
+            if (row < rows) {
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const int col = c0 + 128 * k + 4 * lane;
+                    if (col < cols) {
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            const float x = f4get(gv[q][k], j);
+                            float h, l;
+                            if (MODE == 0) {
+                                two_prod(x, x, h, l);
+                            } else {
+                                const float u = (x * ai[q]) * f4get(bv[k], j);
+                                const float uh = u * icf;
+                                const float mh = s8_to_float((mw[q][k] >> (8 * j)) & 0xFFu) * dm[q][k];
+                                const float mk = ra.beta1 * mh + ra.omb1 * uh;
+                                const float d = uh - mk;
+                                h = d * d + ra.eps2;
+                                l = 0.0f;
+                            }
+                            ff_acc(ch[4 * k + j], cl[4 * k + j], h, l);
+                            ff_acc(rh, rl, h, l);
+                        }
+                    }
+                }
+            }
+            ff_warp_sum(rh, rl);
+            if (lane == 0 && row < rows)
+                rowpart[(int64_t)blockIdx.x * rows + row] = (double)rh + (double)rl;
+        }
     }
 #pragma unroll
     for (int k = 0; k < 4; ++k)
@@ -182,9 +211,14 @@ __device__ __forceinline__ uint32_t fac_code(const FactorDesc& f, int64_t i) {
     return f.bits == 8 ? (uint32_t)((const uint8_t*)f.codes)[i] : (uint32_t)((const uint16_t*)f.codes)[i];
 }
 
+// KPT = elements per thread (block / 256, at least 1). rsum (nullable)
+// receives, for the blocks of f0, the fp64 sum of the block's fresh values in
+// a fixed order (the scale pass builds mean(R) from them).
+template <int KPT>
 __global__ void __launch_bounds__(kThreads)
-factor_kernel(FactorDesc f0, FactorDesc f1, int nb0) {
+factor_kernel(FactorDesc f0, FactorDesc f1, int nb0, double* __restrict__ rsum) {
     __shared__ uint32_t s_part[2][kThreads / 32];
+    __shared__ double s_sum[kThreads / 32];
     const bool first = (int)blockIdx.x < nb0;
     const FactorDesc& f = first ? f0 : f1;
     const int64_t b = first ? blockIdx.x : blockIdx.x - nb0;
@@ -192,10 +226,10 @@ factor_kernel(FactorDesc f0, FactorDesc f1, int nb0) {
     const int64_t hi = lo + f.block < f.len ? lo + f.block : f.len;
     const float2 om = __ldg(reinterpret_cast<const float2*>(f.meta) + b);
     const float Lm2 = f.bits == 8 ? 254.0f : 65534.0f;
-    float v[16];
+    float v[KPT];
     uint32_t vmin = 0xFFFFFFFFu, vmax = 0u;
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
+    for (int k = 0; k < KPT; ++k) {
         const int64_t i = lo + threadIdx.x + (int64_t)kThreads * k;
         v[k] = 0.0f;
         if (i < hi) {
@@ -210,15 +244,29 @@ factor_kernel(FactorDesc f0, FactorDesc f1, int nb0) {
             vmax = umix<true>(vmax, vb);
         }
     }
+    if (first && rsum) {
+        // fixed order: per thread, then shuffle tree, then warps in order
+        double t = 0.0;
+#pragma unroll
+        for (int k = 0; k < KPT; ++k) t += (double)v[k];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xFFFFFFFFu, t, o);
+        if ((threadIdx.x & 31) == 0) s_sum[threadIdx.x >> 5] = t;
+    }
     vmin = __reduce_min_sync(0xFFFFFFFFu, vmin);
     vmax = __reduce_max_sync(0xFFFFFFFFu, vmax);
     vmin = cta_group_reduce<false>(vmin, s_part[0], kThreads / 32);
     vmax = cta_group_reduce<true>(vmax, s_part[1], kThreads / 32);
+    if (first && rsum && threadIdx.x == 0) {
+        double t = 0.0;
+        for (int w = 0; w < kThreads / 32; ++w) t += s_sum[w];
+        rsum[b] = t;
+    }
     float lmin, delta, K, E;
     al_block_params(u2f(vmin + 1u), u2f(vmax), f.log_floor, lmin, delta);
     al_encode_consts(delta, Lm2, K, E);
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
+    for (int k = 0; k < KPT; ++k) {
         const int64_t i = lo + threadIdx.x + (int64_t)kThreads * k;
         if (i < hi) {
             uint32_t q = 0;
@@ -237,23 +285,26 @@ factor_kernel(FactorDesc f0, FactorDesc f1, int nb0) {
 }
 
 // ----------------------------------------------------------------- scale --
-// a_i = 1/sqrt(R_i / mean(R)), b_j = 1/sqrt(C_j); mean(R) in fp64 with a fixed
-// tree order, rounded once.
-__global__ void __launch_bounds__(1024)
+// a_i = 1/sqrt(R_i / mean(R)), b_j = 1/sqrt(C_j). mean(R) in fp64 from the
+// factor pass's per-block sums, added in block order by every CTA (the same
+// value everywhere), rounded once. One element per thread over rows + cols.
+__global__ void __launch_bounds__(kThreads)
 scale_kernel(const float* __restrict__ R, int rows, const float* __restrict__ C, int cols,
-             float* __restrict__ a, float* __restrict__ b) {
-    __shared__ double s[1024];
-    double acc = 0.0;
-    for (int i = threadIdx.x; i < rows; i += 1024) acc += (double)R[i];
-    s[threadIdx.x] = acc;
-    __syncthreads();
-    for (int st = 512; st > 0; st >>= 1) {
-        if ((int)threadIdx.x < st) s[threadIdx.x] += s[threadIdx.x + st];
-        __syncthreads();
+             const double* __restrict__ rsum, int nrb, float* __restrict__ a,
+             float* __restrict__ b) {
+    __shared__ float s_mean;
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int k = 0; k < nrb; ++k) t += rsum[k];
+        s_mean = (float)(t / (double)rows);
     }
-    const float meanR = (float)(s[0] / (double)rows);
-    for (int i = threadIdx.x; i < rows; i += 1024) a[i] = 1.0f / sqrtf(R[i] / meanR);
-    for (int j = threadIdx.x; j < cols; j += 1024) b[j] = 1.0f / sqrtf(C[j]);
+    __syncthreads();
+    const float meanR = s_mean;
+    const int i = blockIdx.x * kThreads + threadIdx.x;
+    if (i < rows)
+        a[i] = 1.0f / sqrtf(R[i] / meanR);
+    else if (i < rows + cols)
+        b[i - rows] = 1.0f / sqrtf(C[i - rows]);
 }
 
 // ------------------------------------------------------------------- usq --
@@ -483,6 +534,21 @@ static FactorDesc factor_desc(const double* part, int nparts, int64_t len, int64
     return f;
 }
 
+// One launch of the factor pass for a row and a column factor (same block).
+static void launch_factor(const FactorDesc& fr, const FactorDesc& fc, double* rsum,
+                          cudaStream_t st) {
+    const int nb0 = (int)blocks_of(fr.len, fr.block), nb1 = (int)blocks_of(fc.len, fc.block);
+    const int kpt = fr.block <= kThreads ? 1 : fr.block / kThreads;
+    const unsigned grid = (unsigned)(nb0 + nb1);
+    switch (kpt) {
+        case 1: factor_kernel<1><<<grid, kThreads, 0, st>>>(fr, fc, nb0, rsum); break;
+        case 2: factor_kernel<2><<<grid, kThreads, 0, st>>>(fr, fc, nb0, rsum); break;
+        case 4: factor_kernel<4><<<grid, kThreads, 0, st>>>(fr, fc, nb0, rsum); break;
+        case 8: factor_kernel<8><<<grid, kThreads, 0, st>>>(fr, fc, nb0, rsum); break;
+        default: factor_kernel<16><<<grid, kThreads, 0, st>>>(fr, fc, nb0, rsum); break;
+    }
+}
+
 // G pass 1 (g^2 sums), factor update, scales, G pass 2 (RMS) -> a, b, icf.
 static int second_moment_passes(const float* g, int64_t rows, int64_t cols, const FacWs& w,
                                 FactorDesc fr, FactorDesc fc, float clip_d, cudaStream_t st,
@@ -491,9 +557,10 @@ static int second_moment_passes(const float* g, int64_t rows, int64_t cols, cons
     ResidualArgs none{};
     sumsq_kernel<0><<<dim3(ncb, nrb), kThreads, 0, st>>>(g, (int)rows, (int)cols, none,
                                                         w.rowpart, w.colpart);
-    const int nb0 = (int)blocks_of(rows, fr.block), nb1 = (int)blocks_of(cols, fc.block);
-    factor_kernel<<<nb0 + nb1, kThreads, 0, st>>>(fr, fc, nb0);
-    scale_kernel<<<1, 1024, 0, st>>>(fr.fresh, (int)rows, fc.fresh, (int)cols, a, b);
+    const int nb0 = (int)blocks_of(rows, fr.block);
+    launch_factor(fr, fc, w.rsum, st);
+    scale_kernel<<<(unsigned)blocks_of(rows + cols, kThreads), kThreads, 0, st>>>(
+        fr.fresh, (int)rows, fc.fresh, (int)cols, w.rsum, nb0, a, b);
     const int64_t n = rows * cols;
     const int64_t ntiles = blocks_of(n, kTile);
     int grid = persistent_grid((const void*)usq_kernel, kThreads, 0, ntiles);
@@ -609,8 +676,9 @@ int al_came_step(float* p, const float* g, int64_t rows, int64_t cols, void* vr_
     FactorDesc cc = factor_desc(w.colpart, nrb, cols, rows, 0.0, hp->beta3, omb3, cc_codes,
                                 cc_meta, c_bits, c_block, hp->log_floor_c, w.fc2);
     const int nb0 = (int)blocks_of(rows, c_block), nb1 = (int)blocks_of(cols, c_block);
-    factor_kernel<<<nb0 + nb1, kThreads, 0, s>>>(cr, cc, nb0);
-    scale_kernel<<<1, 1024, 0, s>>>(w.fr2, (int)rows, w.fc2, (int)cols, w.a2, w.b2);
+    launch_factor(cr, cc, w.rsum2, s);
+    scale_kernel<<<(unsigned)blocks_of(rows + cols, kThreads), kThreads, 0, s>>>(
+        w.fr2, (int)rows, w.fc2, (int)cols, w.rsum2, (int)blocks_of(rows, cr.block), w.a2, w.b2);
     st = check_launch();
     if (st) return st;
 
