@@ -541,13 +541,14 @@ def _row_apollo(torch, np, wl, B, dev):
     Algorithmic bytes: G read for the projection and again for the scaled
     update (8), p read and written (8), projected states and their block
     constants; the bf16 staging copy of G is not counted. FLOPs: 2 r s L per
-    matrix for the projection."""
+    matrix for the projection. One grouped step (al_apollo_step_multi: four
+    launches for all matrices)."""
     cfg = wl.CONFIGS["tinyllama_apollo"]
     r = cfg["rank"]
     hp = dict(lr=cfg["lr"], beta1=cfg["beta1"], beta2=cfg["beta2"], eps=cfg["eps"],
               alpha=cfg["alpha"], weight_decay=cfg["weight_decay"], norm_growth_gamma=0.0,
               log_floor=float(np.float32(np.log2(1e-16))), rank=r)
-    mats, nbytes, flops, n_tot, ws_bytes = [], 0, 0, 0, 0
+    mats, nbytes, flops, n_tot = [], 0, 0, 0
     for i, (_, (rows, cols)) in enumerate(wl.tinyllama_matrices()):
         n1 = rows * cols
         s_, L = min(rows, cols), max(rows, cols)
@@ -572,13 +573,14 @@ def _row_apollo(torch, np, wl, B, dev):
         nbytes += 16 * n1 + 4 * npj + 24 * (npj // 256)
         flops += 2 * r * s_ * L
         n_tot += n1
-        ws_bytes = max(ws_bytes, B.al_workspace_size(B.AL_OP_APOLLO, rows, cols, r))
-    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    # one grouped plan per gradient buffer (a plan binds its gradients)
+    plans = [B.ApolloPlan([dict(p=m["p"], g=m["gs"][k], rows=m["rows"], cols=m["cols"],
+                                proj=m["P"], m_codes=m["mc"], m_absmax=m["ma"],
+                                v_codes=m["vc"], v_meta=m["vm"]) for m in mats], r, 8)
+             for k in range(2)]
 
     def step(t):
-        for m in mats:
-            B.al_apollo_step(m["p"], m["gs"][t % 2], m["rows"], m["cols"], m["P"], m["mc"],
-                             m["ma"], 256, m["vc"], m["vm"], 8, 256, m["prev"], hp, t, ws)
+        plans[t % 2].step(hp, t)
 
     def oracle_sample(ora, t):
         m = mats[0]
@@ -592,10 +594,10 @@ def _row_apollo(torch, np, wl, B, dev):
         return rows * cols / dt, (f"one step of one {rows}x{cols} matrix incl. the rank-{r} "
                                   f"projection in double ({dt:.1f} s, single thread)")
 
-    return dict(step=step, n=n_tot, bytes=nbytes, flops=flops, launches=4 * len(mats),
+    return dict(step=step, n=n_tot, bytes=nbytes, flops=flops, launches=4,
                 oracle=oracle_sample,
-                workload=f"APOLLO TinyLlama-1.1B {len(mats)} matrices, rank {r}, UF8 M^P, "
-                         f"AL8 V^P block 256",
+                workload=f"APOLLO TinyLlama-1.1B {len(mats)} matrices (one grouped step), "
+                         f"rank {r}, UF8 M^P, AL8 V^P block 256",
                 bytes_note="G twice, p read+write, projected states; bf16 staging not counted")
 
 

@@ -362,6 +362,69 @@ int al_apollo_step(float* p, const float* g, int64_t rows, int64_t cols,
                    int v_block, float* prev_norm, const al_apollo_hp* hp,
                    int64_t t, void* workspace, size_t ws_bytes, void* stream);
 
+/* ---------------------------------------------------- grouped APOLLO step -- */
+/*
+ * One APOLLO step over many matrices in four launches (bf16 staging of every
+ * G, one projection launch whose grid covers every matrix's 128-channel
+ * tiles, one moments launch, one update launch) instead of four launches per
+ * matrix. Each matrix gets exactly the arithmetic of al_apollo_step (the
+ * results are bit-identical). This grouping is the library's; the paper
+ * applies the method matrix by matrix.
+ *
+ * Usage: al_apollo_workspace_multi -> allocate the workspace (256-byte
+ * aligned); al_apollo_plan_bytes -> allocate a host buffer and a device
+ * buffer (64-byte aligned) of that size; al_apollo_plan fills the host
+ * buffer; copy it to the device buffer once; then call al_apollo_step_multi
+ * every step. The plan records the matrices' pointers, the workspace and the
+ * TMA descriptors of the projection operands: rebuild it if any of them
+ * changes (a refreshed projection written into the same proj buffer needs no
+ * rebuild). The norm-growth limiter is not available here
+ * (hp->norm_growth_gamma > 0 returns ALQ_ERR_UNSUPPORTED).
+ */
+typedef struct {
+    float* p;              /* [rows x cols] fp32, as in al_apollo_step      */
+    const float* g;
+    int64_t rows, cols;
+    const uint16_t* proj;  /* bf16 bits [rank x min(rows, cols)]            */
+    int8_t* m_codes;       /* [max(rows, cols) x rank] UF8, block = rank    */
+    float* m_absmax;
+    void* v_codes;         /* [max(rows, cols) x rank] AL8 or AL16          */
+    float* v_meta;
+} al_apollo_matrix;
+
+/* Summary of a grouped plan (host struct, filled by al_apollo_plan). */
+typedef struct {
+    int32_t nmat, rank, v_bits, reserved;
+    int64_t total_params;   /* sum of rows * cols                            */
+    int64_t total_channels; /* sum of max(rows, cols)                        */
+    int64_t conv_tiles;     /* tiles of the bf16 staging pass                */
+    int64_t gemm_tiles;     /* 128-channel tiles of the grouped projection   */
+    int64_t mom_tiles;      /* 4096-value tiles of the moments pass          */
+    int64_t upd_tiles;      /* 4096-parameter tiles of the update pass       */
+    void* workspace;        /* the workspace the plan is bound to            */
+} al_apollo_info;
+
+/* Bytes of a plan over these matrices (host and device copies alike). */
+int al_apollo_plan_bytes(const al_apollo_matrix* mats, int nmat, size_t* bytes);
+
+/* Scratch bytes of a grouped step: every matrix's bf16 operand, projection
+ * and channel scales side by side. */
+int al_apollo_workspace_multi(const al_apollo_matrix* mats, int nmat, int rank,
+                              size_t* bytes);
+
+/* Validates every matrix as al_apollo_step does (rank 128 or 256, v_bits 8
+ * or 16) and writes the plan into plan_host. Returns ALQ_ERR_WORKSPACE when
+ * the workspace is missing, misaligned or too small, ALQ_ERR_CUDA when a TMA
+ * descriptor cannot be encoded. */
+int al_apollo_plan(const al_apollo_matrix* mats, int nmat, int rank,
+                   int v_bits, void* workspace, size_t ws_bytes,
+                   void* plan_host, size_t plan_bytes, al_apollo_info* info);
+
+/* One grouped step. plan_dev is the device copy of the plan; info and hp
+ * are host pointers; hp->rank must equal the plan's rank. */
+int al_apollo_step_multi(const void* plan_dev, const al_apollo_info* info,
+                         const al_apollo_hp* hp, int64_t t, void* stream);
+
 #ifdef __cplusplus
 } /* extern "C" */
 #endif

@@ -64,6 +64,20 @@ class AdamWTensor(C.Structure):
                 ("v_meta", C.c_void_p), ("n", C.c_int64)]
 
 
+class ApolloMatrix(C.Structure):
+    _fields_ = [("p", C.c_void_p), ("g", C.c_void_p), ("rows", C.c_int64),
+                ("cols", C.c_int64), ("proj", C.c_void_p), ("m_codes", C.c_void_p),
+                ("m_absmax", C.c_void_p), ("v_codes", C.c_void_p), ("v_meta", C.c_void_p)]
+
+
+class ApolloInfo(C.Structure):
+    _fields_ = [("nmat", C.c_int32), ("rank", C.c_int32), ("v_bits", C.c_int32),
+                ("reserved", C.c_int32), ("total_params", C.c_int64),
+                ("total_channels", C.c_int64), ("conv_tiles", C.c_int64),
+                ("gemm_tiles", C.c_int64), ("mom_tiles", C.c_int64),
+                ("upd_tiles", C.c_int64), ("workspace", C.c_void_p)]
+
+
 class MultiInfo(C.Structure):
     _fields_ = [("ntensors", C.c_int32), ("m_block", C.c_int32),
                 ("v_block", C.c_int32), ("v_bits", C.c_int32),
@@ -103,6 +117,12 @@ _sig("al_adafactor_noalloc_capacity", C.c_size_t)
 _sig("al_came_step", _int, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _vp, _int, _int,
      _vp, _vp, _vp, _vp, _int, _int, _vp, _vp, _int, C.POINTER(CameHP), _i64, _vp,
      C.c_size_t, _vp)
+_sig("al_apollo_plan_bytes", _int, C.POINTER(ApolloMatrix), _int, C.POINTER(C.c_size_t))
+_sig("al_apollo_workspace_multi", _int, C.POINTER(ApolloMatrix), _int, _int,
+     C.POINTER(C.c_size_t))
+_sig("al_apollo_plan", _int, C.POINTER(ApolloMatrix), _int, _int, _int, _vp, C.c_size_t, _vp,
+     C.c_size_t, C.POINTER(ApolloInfo))
+_sig("al_apollo_step_multi", _int, _vp, C.POINTER(ApolloInfo), C.POINTER(ApolloHP), _i64, _vp)
 _sig("al_apollo_step", _int, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _int, _vp, _vp,
      _int, _int, _vp, C.POINTER(ApolloHP), _i64, _vp, C.c_size_t, _vp)
 
@@ -257,3 +277,37 @@ def al_apollo_step(p, g, rows, cols, proj, m_codes, m_absmax, m_block, v_codes, 
         _ptr(p), _ptr(g), rows, cols, _ptr(proj), _ptr(m_codes), _ptr(m_absmax), m_block,
         _ptr(v_codes), _ptr(v_meta), v_bits, v_block, _ptr(prev_norm), C.byref(h), t,
         _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+class ApolloPlan:
+    """A grouped APOLLO step over many matrices (al_apollo_plan /
+    al_apollo_step_multi): owns the workspace and the device copy of the
+    plan. `mats` is a list of dicts with keys p, g, rows, cols, proj, m_codes,
+    m_absmax, v_codes, v_meta (torch CUDA tensors; proj holds bf16 bits)."""
+
+    def __init__(self, mats, rank, v_bits, device=None):
+        nm = len(mats)
+        arr = (ApolloMatrix * nm)()
+        for i, m in enumerate(mats):
+            arr[i] = ApolloMatrix(_ptr(m["p"]), _ptr(m["g"]), m["rows"], m["cols"],
+                                  _ptr(m["proj"]), _ptr(m["m_codes"]), _ptr(m["m_absmax"]),
+                                  _ptr(m["v_codes"]), _ptr(m["v_meta"]))
+        dev = device if device is not None else mats[0]["p"].device
+        ws = C.c_size_t(0)
+        _check("al_apollo_workspace_multi",
+               lib.al_apollo_workspace_multi(arr, nm, rank, C.byref(ws)))
+        self.workspace = torch.zeros(ws.value, dtype=torch.uint8, device=dev)
+        nbytes = C.c_size_t(0)
+        _check("al_apollo_plan_bytes", lib.al_apollo_plan_bytes(arr, nm, C.byref(nbytes)))
+        host = torch.zeros(nbytes.value, dtype=torch.uint8)
+        self.info = ApolloInfo()
+        _check("al_apollo_plan", lib.al_apollo_plan(
+            arr, nm, rank, v_bits, _ptr(self.workspace), ws.value, host.data_ptr(),
+            nbytes.value, C.byref(self.info)))
+        self.dev = host.to(dev)
+        self.mats = mats  # keep the arrays alive while the plan is used
+
+    def step(self, hp: dict, t: int, stream=None):
+        h = _hp(ApolloHP, hp)
+        _check("al_apollo_step_multi", lib.al_apollo_step_multi(
+            _ptr(self.dev), C.byref(self.info), C.byref(h), t, _stream(stream)))

@@ -75,26 +75,33 @@ int al_apollo_workspace(int64_t rows, int64_t cols, int rank, size_t* bytes) {
 }
 
 // --------------------------------------------------------------- convert --
-// rows > cols: A[j][i] = bf16(G[j][i]) (channels are rows, K = cols).
-__global__ void __launch_bounds__(kThreads)
-to_bf16_kernel(const float* __restrict__ g, int64_t n, uint16_t* __restrict__ A) {
-    for (int64_t i = 4 * ((int64_t)blockIdx.x * kThreads + threadIdx.x); i < n;
-         i += 4 * (int64_t)gridDim.x * kThreads) {
-        const float4 v = __ldcs(reinterpret_cast<const float4*>(g + i));
-        const uint32_t lo = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.x)) |
-                            ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.y)) << 16);
-        const uint32_t hi = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.z)) |
-                            ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.w)) << 16);
-        *reinterpret_cast<uint2*>(A + i) = make_uint2(lo, hi);
+// rows > cols: A[j][i] = bf16(G[j][i]) (channels are rows, K = cols). One
+// tile = kTile elements, four float4 per thread (n is a multiple of 4).
+__device__ __forceinline__ void convert_rows_tile(const float* __restrict__ g, int64_t n,
+                                                  uint16_t* __restrict__ A, int64_t tile) {
+    const int64_t base = tile * kTile + 4 * (int64_t)threadIdx.x;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int64_t i = base + (int64_t)k * 4 * kThreads;
+        if (i < n) {
+            const float4 v = __ldcs(reinterpret_cast<const float4*>(g + i));
+            const uint32_t lo = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.x)) |
+                                ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.y)) << 16);
+            const uint32_t hi = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.z)) |
+                                ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.w)) << 16);
+            *reinterpret_cast<uint2*>(A + i) = make_uint2(lo, hi);
+        }
     }
 }
 
 // rows <= cols: A[j][i] = bf16(G[i][j]) (channels are columns, K = rows),
-// through 32 x 32 shared-memory tiles.
-__global__ void __launch_bounds__(256)
-to_bf16_t_kernel(const float* __restrict__ g, int rows, int cols, uint16_t* __restrict__ A) {
-    __shared__ float t[32][33];
-    const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+// one 32 x 32 tile (tile row tr, tile column tc) through shared memory.
+// Every thread of the CTA must call it; it ends with a barrier so that the
+// shared tile can be reused.
+__device__ __forceinline__ void convert_cols_tile(const float* __restrict__ g, int rows, int cols,
+                                                  uint16_t* __restrict__ A, int64_t tr,
+                                                  int64_t tc, float (*t)[33]) {
+    const int c0 = (int)tc * 32, r0 = (int)tr * 32;
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;  // 32 x 8
     for (int k = ty; k < 32; k += 8) {
         const int r = r0 + k, c = c0 + tx;
@@ -106,6 +113,18 @@ to_bf16_t_kernel(const float* __restrict__ g, int rows, int cols, uint16_t* __re
         if (j < cols && i < rows)
             A[(int64_t)j * rows + i] = __bfloat16_as_ushort(__float2bfloat16_rn(t[tx][k]));
     }
+    __syncthreads();
+}
+
+__global__ void __launch_bounds__(kThreads)
+to_bf16_kernel(const float* __restrict__ g, int64_t n, uint16_t* __restrict__ A, int64_t ntiles) {
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) convert_rows_tile(g, n, A, tile);
+}
+
+__global__ void __launch_bounds__(kThreads)
+to_bf16_t_kernel(const float* __restrict__ g, int rows, int cols, uint16_t* __restrict__ A) {
+    __shared__ float t[32][33];
+    convert_cols_tile(g, rows, cols, A, blockIdx.y, blockIdx.x, t);
 }
 
 // ------------------------------------------------------ PTX primitives --
@@ -182,17 +201,17 @@ struct GemmArgs {
     int* err;
 };
 
-__global__ void __launch_bounds__(128, 1)
-apollo_project_kernel(const __grid_constant__ CUtensorMap tmA,
-                      const __grid_constant__ CUtensorMap tmB, GemmArgs a) {
-    extern __shared__ uint8_t smem_raw[];
+// One 128-channel tile of R = A * P^T: rows m0 .. m0 + 127 of A against
+// the whole projection, K in a.kblocks steps of 64. The tensor maps may live
+// in the kernel's parameters or in global memory.
+__device__ __forceinline__ void project_tile(const CUtensorMap* tmA, const CUtensorMap* tmB,
+                                             const GemmArgs& a, int m0, uint8_t* smem_raw) {
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t* sA = smem;
     uint8_t* sB = smem + kStages * kAStage;
     uint64_t* bars = (uint64_t*)(sB + kStages * kBStage);  // full[4], empty[4], accum
     uint32_t* tmem_slot = (uint32_t*)(bars + 2 * kStages + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.x * kGM;
     const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + kStages);
     const uint32_t accum = smem_u32(bars + 2 * kStages);
     const uint32_t ncols = a.rank <= 128 ? 128u : 256u;
@@ -226,8 +245,8 @@ apollo_project_kernel(const __grid_constant__ CUtensorMap tmA,
             if (kb >= kStages) ok = mbar_wait(empty0 + 8 * s, ((kb / kStages) - 1) & 1);
             if (!ok) break;
             mbar_expect_tx(full0 + 8 * s, kAStage + b_bytes);
-            tma_load_2d(smem_u32(sA + s * kAStage), &tmA, kb * kGK, m0, full0 + 8 * s);
-            tma_load_2d(smem_u32(sB + s * kBStage), &tmB, kb * kGK, 0, full0 + 8 * s);
+            tma_load_2d(smem_u32(sA + s * kAStage), tmA, kb * kGK, m0, full0 + 8 * s);
+            tma_load_2d(smem_u32(sB + s * kBStage), tmB, kb * kGK, 0, full0 + 8 * s);
         }
     } else if (warp == 1 && lane == 0) {
         // MMA issuer: four K = 16 steps per stage, 32 bytes apart in the row
@@ -278,6 +297,13 @@ apollo_project_kernel(const __grid_constant__ CUtensorMap tmA,
                      : "memory");
 }
 
+__global__ void __launch_bounds__(128, 1)
+apollo_project_kernel(const __grid_constant__ CUtensorMap tmA,
+                      const __grid_constant__ CUtensorMap tmB, GemmArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    project_tile(&tmA, &tmB, a, blockIdx.x * kGM, smem_raw);
+}
+
 // ------------------------------------------------------------- moments --
 // Projected Adam moments, one quantization block per channel (block = rank).
 struct MomentArgs {
@@ -292,17 +318,17 @@ struct MomentArgs {
     float beta1, beta2, omb1, omb2, ic1, c2, eps, log_floor;
 };
 
+// One tile (kTile projected values) of the moments pass; tab is this warp's
+// decode-table slot (NB * 32 entries).
 template <int CPB, int VBITS>
-__global__ void __launch_bounds__(kThreads)
-apollo_moments_kernel(MomentArgs m, int64_t ntiles) {
+__device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, float2* tab) {
     constexpr int NB = 4 / CPB;
     constexpr float Lm2 = VBITS == 8 ? 254.0f : 65534.0f;
-    __shared__ float2 s_tab[kThreads / 32][NB * 32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const float kf = al8_table_k(lane);
     const int64_t nblk = blocks_of_dev(m.n, m.block);
     const int bshift = __ffs(m.block) - 1;
-    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+    {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
         const int64_t b0 = seg0 >> bshift;
         float4 r[4];
@@ -333,7 +359,7 @@ apollo_moments_kernel(MomentArgs m, int64_t ntiles) {
             odelta[b] = mt.y;
             dm[b] = sa / 127.0f;
         }
-        if (VBITS == 8) al8_build_tables<NB>(s_tab[warp], olmin, odelta, kf);
+        if (VBITS == 8) al8_build_tables<NB>(tab, olmin, odelta, kf);
         float mf[16], vf[16];
         uint32_t cvmin[4], cvmax[4], cmabs[4];
         float nrh[NB], nrl[NB], ngh[NB], ngl[NB];
@@ -350,7 +376,7 @@ apollo_moments_kernel(MomentArgs m, int64_t ntiles) {
             for (int i = 0; i < 4; ++i) {
                 const uint32_t qv = code_of<VBITS>(vw, c, i);
                 const float vh = VBITS == 8
-                                     ? al8_decode(qv, s_tab[warp] + 32 * b, fast, olmin[b], odelta[b])
+                                     ? al8_decode(qv, tab + 32 * b, fast, olmin[b], odelta[b])
                                      : al16_decode(qv, olmin[b], odelta[b]);
                 const float mh = s8_to_float((mw[c] >> (8 * i)) & 0xFFu) * dm[b];
                 const float rv = f4get(r[c], i);
@@ -425,6 +451,14 @@ apollo_moments_kernel(MomentArgs m, int64_t ntiles) {
     }
 }
 
+template <int CPB, int VBITS>
+__global__ void __launch_bounds__(kThreads)
+apollo_moments_kernel(MomentArgs m, int64_t ntiles) {
+    __shared__ float2 s_tab[kThreads / 32][(4 / CPB) * 32];
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x)
+        moments_tile<CPB, VBITS>(m, tile, s_tab[threadIdx.x >> 5]);
+}
+
 // ------------------------------------------------------ limiter, update --
 struct ApUpdateArgs {
     float* p;
@@ -494,11 +528,10 @@ __global__ void apollo_limit_kernel(const double* __restrict__ part, int nparts,
     }
 }
 
-__global__ void __launch_bounds__(kThreads)
-apollo_update_kernel(ApUpdateArgs u, int64_t ntiles) {
+// One tile (kTile parameters) of p = p (1 - lr wd) - (lr alpha) lim (g s_j).
+__device__ __forceinline__ void update_tile(const ApUpdateArgs& u, int64_t tile, float lim) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const float lim = u.lim ? __ldg(u.lim) : 1.0f;
-    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+    {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
@@ -524,6 +557,127 @@ apollo_update_kernel(ApUpdateArgs u, int64_t ntiles) {
             }
             __stcs(reinterpret_cast<float4*>(u.p + idx), make_float4(pn[0], pn[1], pn[2], pn[3]));
         }
+    }
+}
+
+__global__ void __launch_bounds__(kThreads)
+apollo_update_kernel(ApUpdateArgs u, int64_t ntiles) {
+    const float lim = u.lim ? __ldg(u.lim) : 1.0f;
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) update_tile(u, tile, lim);
+}
+
+// ------------------------------------------------------- grouped step --
+// Plan of a grouped step: a header, then one 64-byte-aligned entry per
+// matrix (its TMA descriptors first), then the projection tile -> matrix map.
+constexpr uint32_t kApPlanMagic = 0x41504C31u;  // "APL1"
+
+struct ApPlanHeader {
+    uint32_t magic;
+    int32_t nmat, rank, v_bits;
+    int64_t conv_tiles, gemm_tiles, mom_tiles, upd_tiles;
+    int64_t total_params, total_channels;
+    int64_t reserved[2];
+};
+static_assert(sizeof(ApPlanHeader) == 80, "plan header layout");
+
+struct ApEntry {  // aligned as CUtensorMap (at least 64 bytes)
+    CUtensorMap tmA;  // bf16 A [L][s] in the workspace, box [128][64]
+    CUtensorMap tmB;  // bf16 P [rank][s], box [rank][64]
+    float* p;
+    const float* g;
+    int8_t* m_codes;
+    float* m_absmax;
+    void* v_codes;
+    float* v_meta;
+    uint16_t* A;
+    float* R;
+    float* scale;
+    int64_t rows, cols, n, L, s, npj;
+    Divider dv;
+    int32_t rows_short, kblocks;
+    int64_t conv_t0, gemm_t0, mom_t0, upd_t0;  // first tile of each pass
+};
+
+constexpr size_t kApEntryOffset = 128;  // header rounded up to the entry alignment
+static_assert(kApEntryOffset % alignof(ApEntry) == 0 && sizeof(ApEntry) % 64 == 0,
+              "plan entries keep their tensor maps 64-byte aligned");
+
+__device__ __forceinline__ int entry_for(const ApEntry* __restrict__ tab, int nmat, int64_t tile,
+                                         int cur, int64_t ApEntry::*t0) {
+    while (cur + 1 < nmat && tab[cur + 1].*t0 <= tile) ++cur;
+    return cur;
+}
+
+__global__ void __launch_bounds__(kThreads)
+apollo_convert_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t ntiles) {
+    __shared__ float t[32][33];
+    int cur = 0;
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        cur = entry_for(tab, nmat, tile, cur, &ApEntry::conv_t0);
+        const ApEntry& e = tab[cur];
+        const int64_t lt = tile - e.conv_t0;
+        if (e.rows_short) {
+            const int64_t ntc = (e.cols + 31) / 32;
+            convert_cols_tile(e.g, (int)e.rows, (int)e.cols, e.A, lt / ntc, lt % ntc, t);
+        } else {
+            convert_rows_tile(e.g, e.n, e.A, lt);
+        }
+    }
+}
+
+__global__ void __launch_bounds__(128, 1)
+apollo_project_multi_kernel(const ApEntry* __restrict__ tab, const uint16_t* __restrict__ tile_mat,
+                            int rank, int* err) {
+    extern __shared__ uint8_t smem_raw[];
+    const ApEntry* e = tab + tile_mat[blockIdx.x];
+    if (threadIdx.x == 0) {
+        // the descriptors were written through the generic proxy (a copy to
+        // device memory): make them visible to the tensor-map proxy
+        asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(&e->tmA)
+                     : "memory");
+        asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(&e->tmB)
+                     : "memory");
+    }
+    const GemmArgs a{e->R, (int)e->L, rank, e->kblocks, err};
+    project_tile(&e->tmA, &e->tmB, a, (int)(blockIdx.x - e->gemm_t0) * kGM, smem_raw);
+}
+
+template <int CPB, int VBITS>
+__global__ void __launch_bounds__(kThreads)
+apollo_moments_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t ntiles,
+                            MomentArgs base) {
+    __shared__ float2 s_tab[kThreads / 32][(4 / CPB) * 32];
+    int cur = 0;
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        cur = entry_for(tab, nmat, tile, cur, &ApEntry::mom_t0);
+        const ApEntry& e = tab[cur];
+        MomentArgs m = base;
+        m.R = e.R;
+        m.n = e.npj;
+        m.m_codes = e.m_codes;
+        m.m_absmax = e.m_absmax;
+        m.v_codes = e.v_codes;
+        m.v_meta = e.v_meta;
+        m.scale = e.scale;
+        moments_tile<CPB, VBITS>(m, tile - e.mom_t0, s_tab[threadIdx.x >> 5]);
+    }
+}
+
+__global__ void __launch_bounds__(kThreads)
+apollo_update_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t ntiles,
+                           ApUpdateArgs base) {
+    int cur = 0;
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        cur = entry_for(tab, nmat, tile, cur, &ApEntry::upd_t0);
+        const ApEntry& e = tab[cur];
+        ApUpdateArgs u = base;
+        u.p = e.p;
+        u.g = e.g;
+        u.n = e.n;
+        u.dv = e.dv;
+        u.rows_short = e.rows_short;
+        u.scale = e.scale;
+        update_tile(u, tile - e.upd_t0, 1.0f);
     }
 }
 
@@ -576,6 +730,39 @@ static int launch_project(const uint16_t* A, const uint16_t* P, int64_t L, int64
     return check_launch();
 }
 
+// The checks al_apollo_step applies to one matrix.
+static int check_apollo_matrix(const al_apollo_matrix& m, int rank, int v_bits) {
+    if (!m.p || !m.g || !m.proj || !m.m_codes || !m.m_absmax || !m.v_codes || !m.v_meta ||
+        m.rows < 1 || m.cols < 1)
+        return ALQ_ERR_INVALID_ARG;
+    const int64_t s = m.rows <= m.cols ? m.rows : m.cols, L = m.rows <= m.cols ? m.cols : m.rows;
+    if ((rank != 128 && rank != 256) || (v_bits != 8 && v_bits != 16) || m.cols % 4 != 0 ||
+        s % 8 != 0 || m.rows * m.cols >= (int64_t)1 << 31 || L > (1 << 30))
+        return ALQ_ERR_UNSUPPORTED;
+    if (!aligned(m.p, 16) || !aligned(m.g, 16) || !aligned(m.proj, 16) ||
+        !aligned(m.m_codes, 16) || !aligned(m.v_codes, 16) || !aligned(m.v_meta, 8) ||
+        !aligned(m.m_absmax, 4))
+        return ALQ_ERR_ALIGN;
+    return ALQ_OK;
+}
+
+// Moment-pass scalars of step t (bias corrections in double, rounded once).
+static MomentArgs moment_scalars(const al_apollo_hp* hp, int64_t t, int rank) {
+    const double bc1 = 1.0 - pow((double)hp->beta1, (double)t);
+    const double bc2 = 1.0 - pow((double)hp->beta2, (double)t);
+    MomentArgs m{};
+    m.block = rank;
+    m.beta1 = hp->beta1;
+    m.beta2 = hp->beta2;
+    m.omb1 = (float)(1.0 - (double)hp->beta1);
+    m.omb2 = (float)(1.0 - (double)hp->beta2);
+    m.ic1 = (float)(1.0 / bc1);
+    m.c2 = (float)(1.0 / sqrt(bc2));
+    m.eps = hp->eps;
+    m.log_floor = hp->log_floor;
+    return m;
+}
+
 template <int CPB, int VBITS>
 static void launch_moments_t(const MomentArgs& m, cudaStream_t st) {
     const int64_t ntiles = blocks_of(m.n, kTile);
@@ -592,19 +779,14 @@ extern "C" int al_apollo_step(float* p, const float* g, int64_t rows, int64_t co
                               void* v_codes, float* v_meta, int v_bits, int v_block,
                               float* prev_norm, const al_apollo_hp* hp, int64_t t,
                               void* workspace, size_t ws_bytes, void* stream) {
-    if (!p || !g || !proj || !m_codes || !m_absmax || !v_codes || !v_meta || !hp || t < 1 ||
-        rows < 1 || cols < 1)
-        return ALQ_ERR_INVALID_ARG;
+    if (!hp || t < 1) return ALQ_ERR_INVALID_ARG;
     const int rank = hp->rank;
+    if (m_block != rank || v_block != rank) return ALQ_ERR_UNSUPPORTED;
+    const al_apollo_matrix mat{p, g, rows, cols, proj, m_codes, m_absmax, v_codes, v_meta};
+    int rc0 = check_apollo_matrix(mat, rank, v_bits);
+    if (rc0) return rc0;
     const int64_t s = rows <= cols ? rows : cols, L = rows <= cols ? cols : rows;
-    if ((rank != 128 && rank != 256) || m_block != rank || v_block != rank ||
-        (v_bits != 8 && v_bits != 16) || cols % 4 != 0 || s % 8 != 0 ||
-        rows * cols >= (int64_t)1 << 31 || L > (1 << 30))
-        return ALQ_ERR_UNSUPPORTED;
     if (hp->norm_growth_gamma > 0.0f && !prev_norm) return ALQ_ERR_INVALID_ARG;
-    if (!aligned(p, 16) || !aligned(g, 16) || !aligned(proj, 16) || !aligned(m_codes, 16) ||
-        !aligned(v_codes, 16) || !aligned(v_meta, 8) || !aligned(m_absmax, 4))
-        return ALQ_ERR_ALIGN;
     const ApWs w = ap_layout(workspace, rows, cols, rank);
     if (!workspace || ws_bytes < w.bytes || !aligned(workspace, 256)) return ALQ_ERR_WORKSPACE;
     cudaStream_t st = (cudaStream_t)stream;
@@ -615,35 +797,23 @@ extern "C" int al_apollo_step(float* p, const float* g, int64_t rows, int64_t co
         dim3 grid((unsigned)blocks_of(cols, 32), (unsigned)blocks_of(rows, 32));
         to_bf16_t_kernel<<<grid, 256, 0, st>>>(g, (int)rows, (int)cols, w.A);
     } else {
-        const int64_t n = rows * cols;
-        int grid = (int)blocks_of(n / 4, kThreads);
-        if (grid > 8 * sm_count()) grid = 8 * sm_count();
-        to_bf16_kernel<<<grid, kThreads, 0, st>>>(g, n, w.A);
+        const int64_t n = rows * cols, ntiles = blocks_of(n, kTile);
+        to_bf16_kernel<<<persistent_grid((const void*)to_bf16_kernel, kThreads, 0, ntiles),
+                         kThreads, 0, st>>>(g, n, w.A, ntiles);
     }
     int rc = check_launch();
     if (rc) return rc;
     rc = launch_project(w.A, proj, L, s, rank, w.R, w.err, st);
     if (rc) return rc;
 
-    const double bc1 = 1.0 - pow((double)hp->beta1, (double)t);
-    const double bc2 = 1.0 - pow((double)hp->beta2, (double)t);
-    MomentArgs m;
+    MomentArgs m = moment_scalars(hp, t, rank);
     m.R = w.R;
     m.n = L * rank;
     m.m_codes = m_codes;
     m.m_absmax = m_absmax;
     m.v_codes = v_codes;
     m.v_meta = v_meta;
-    m.block = rank;
     m.scale = w.scale;
-    m.beta1 = hp->beta1;
-    m.beta2 = hp->beta2;
-    m.omb1 = (float)(1.0 - (double)hp->beta1);
-    m.omb2 = (float)(1.0 - (double)hp->beta2);
-    m.ic1 = (float)(1.0 / bc1);
-    m.c2 = (float)(1.0 / sqrt(bc2));
-    m.eps = hp->eps;
-    m.log_floor = hp->log_floor;
     if (rank == 128) {
         if (v_bits == 8) launch_moments_t<1, 8>(m, st); else launch_moments_t<1, 16>(m, st);
     } else {
@@ -673,5 +843,208 @@ extern "C" int al_apollo_step(float* p, const float* g, int64_t rows, int64_t co
     }
     apollo_update_kernel<<<persistent_grid((const void*)apollo_update_kernel, kThreads, 0, ntiles),
                            kThreads, 0, st>>>(u, ntiles);
+    return check_launch();
+}
+
+// ------------------------------------------------------- grouped step --
+namespace alq {
+
+struct ApShape {
+    int64_t s, L, n;
+    int rows_short;
+};
+
+static ApShape ap_shape(const al_apollo_matrix& m) {
+    ApShape a;
+    a.rows_short = m.rows <= m.cols;
+    a.s = a.rows_short ? m.rows : m.cols;
+    a.L = a.rows_short ? m.cols : m.rows;
+    a.n = m.rows * m.cols;
+    return a;
+}
+
+static int64_t conv_tiles_of(const al_apollo_matrix& m) {
+    const ApShape a = ap_shape(m);
+    return a.rows_short ? blocks_of(m.cols, 32) * blocks_of(m.rows, 32) : blocks_of(a.n, kTile);
+}
+
+// Per-matrix scratch of a grouped step: A, R, scale, each 256-byte aligned.
+static size_t multi_ws_bytes(const al_apollo_matrix& m, int rank) {
+    const ApShape a = ap_shape(m);
+    return r256(2 * (size_t)a.L * a.s) + r256(4 * (size_t)a.L * rank) + r256(4 * (size_t)a.L);
+}
+
+static int check_matrices(const al_apollo_matrix* mats, int nmat) {
+    if (!mats || nmat < 1 || nmat > 65535) return ALQ_ERR_INVALID_ARG;
+    return ALQ_OK;
+}
+
+static size_t plan_size(const al_apollo_matrix* mats, int nmat) {
+    int64_t gemm = 0;
+    for (int i = 0; i < nmat; ++i) gemm += blocks_of(ap_shape(mats[i]).L, kGM);
+    return kApEntryOffset + (size_t)nmat * sizeof(ApEntry) + r256(2 * (size_t)gemm);
+}
+
+}  // namespace alq
+
+extern "C" int al_apollo_plan_bytes(const al_apollo_matrix* mats, int nmat, size_t* bytes) {
+    if (!bytes) return ALQ_ERR_INVALID_ARG;
+    const int rc = check_matrices(mats, nmat);
+    if (rc) return rc;
+    for (int i = 0; i < nmat; ++i)
+        if (mats[i].rows < 1 || mats[i].cols < 1) return ALQ_ERR_INVALID_ARG;
+    *bytes = plan_size(mats, nmat);
+    return ALQ_OK;
+}
+
+extern "C" int al_apollo_workspace_multi(const al_apollo_matrix* mats, int nmat, int rank,
+                                         size_t* bytes) {
+    if (!bytes) return ALQ_ERR_INVALID_ARG;
+    int rc = check_matrices(mats, nmat);
+    if (rc) return rc;
+    if (rank != 128 && rank != 256) return ALQ_ERR_UNSUPPORTED;
+    size_t tot = 256;  // the projection's timeout flag
+    for (int i = 0; i < nmat; ++i) {
+        if (mats[i].rows < 1 || mats[i].cols < 1) return ALQ_ERR_INVALID_ARG;
+        tot += multi_ws_bytes(mats[i], rank);
+    }
+    *bytes = tot;
+    return ALQ_OK;
+}
+
+extern "C" int al_apollo_plan(const al_apollo_matrix* mats, int nmat, int rank, int v_bits,
+                              void* workspace, size_t ws_bytes, void* plan_host,
+                              size_t plan_bytes, al_apollo_info* info) {
+    int rc = check_matrices(mats, nmat);
+    if (rc) return rc;
+    if (!plan_host || !info) return ALQ_ERR_INVALID_ARG;
+    for (int i = 0; i < nmat; ++i) {
+        rc = check_apollo_matrix(mats[i], rank, v_bits);
+        if (rc) return rc;
+    }
+    size_t need = 0;
+    al_apollo_workspace_multi(mats, nmat, rank, &need);
+    if (!workspace || ws_bytes < need || !aligned(workspace, 256)) return ALQ_ERR_WORKSPACE;
+    if (plan_bytes < plan_size(mats, nmat)) return ALQ_ERR_INVALID_ARG;
+
+    char* base = (char*)plan_host;
+    memset(base, 0, plan_size(mats, nmat));
+    uint16_t* tile_mat =
+        (uint16_t*)(base + kApEntryOffset + (size_t)nmat * sizeof(ApEntry));
+    char* ws = (char*)workspace + 256;  // first 256 bytes: timeout flag
+    ApPlanHeader h{};
+    h.magic = kApPlanMagic;
+    h.nmat = nmat;
+    h.rank = rank;
+    h.v_bits = v_bits;
+    for (int i = 0; i < nmat; ++i) {
+        const al_apollo_matrix& m = mats[i];
+        const ApShape a = ap_shape(m);
+        ApEntry e;
+        memset(&e, 0, sizeof(e));
+        e.p = m.p;
+        e.g = m.g;
+        e.m_codes = m.m_codes;
+        e.m_absmax = m.m_absmax;
+        e.v_codes = m.v_codes;
+        e.v_meta = m.v_meta;
+        e.A = (uint16_t*)ws;
+        e.R = (float*)(ws + r256(2 * (size_t)a.L * a.s));
+        e.scale = (float*)(ws + r256(2 * (size_t)a.L * a.s) + r256(4 * (size_t)a.L * rank));
+        ws += multi_ws_bytes(m, rank);
+        e.rows = m.rows;
+        e.cols = m.cols;
+        e.n = a.n;
+        e.L = a.L;
+        e.s = a.s;
+        e.npj = a.L * rank;
+        e.dv = make_divider((uint32_t)m.cols);
+        e.rows_short = a.rows_short;
+        e.kblocks = (int32_t)blocks_of(a.s, kGK);
+        e.conv_t0 = h.conv_tiles;
+        e.gemm_t0 = h.gemm_tiles;
+        e.mom_t0 = h.mom_tiles;
+        e.upd_t0 = h.upd_tiles;
+        if (!make_map(&e.tmA, e.A, (uint64_t)a.s, (uint64_t)a.L, kGM) ||
+            !make_map(&e.tmB, m.proj, (uint64_t)a.s, (uint64_t)rank, (uint32_t)rank))
+            return record_cuda(cudaErrorInvalidValue);
+        const int64_t gt = blocks_of(a.L, kGM);
+        for (int64_t k = 0; k < gt; ++k) tile_mat[h.gemm_tiles + k] = (uint16_t)i;
+        h.conv_tiles += conv_tiles_of(m);
+        h.gemm_tiles += gt;
+        h.mom_tiles += blocks_of(e.npj, kTile);
+        h.upd_tiles += blocks_of(a.n, kTile);
+        h.total_params += a.n;
+        h.total_channels += a.L;
+        memcpy(base + kApEntryOffset + (size_t)i * sizeof(ApEntry), &e, sizeof(e));
+    }
+    memcpy(base, &h, sizeof(h));
+    info->nmat = nmat;
+    info->rank = rank;
+    info->v_bits = v_bits;
+    info->reserved = 0;
+    info->total_params = h.total_params;
+    info->total_channels = h.total_channels;
+    info->conv_tiles = h.conv_tiles;
+    info->gemm_tiles = h.gemm_tiles;
+    info->mom_tiles = h.mom_tiles;
+    info->upd_tiles = h.upd_tiles;
+    info->workspace = workspace;
+    return ALQ_OK;
+}
+
+extern "C" int al_apollo_step_multi(const void* plan_dev, const al_apollo_info* info,
+                                    const al_apollo_hp* hp, int64_t t, void* stream) {
+    if (!plan_dev || !info || !hp || t < 1 || info->nmat < 1 || !info->workspace)
+        return ALQ_ERR_INVALID_ARG;
+    if (!aligned(plan_dev, 64)) return ALQ_ERR_ALIGN;
+    if (hp->rank != info->rank) return ALQ_ERR_INVALID_ARG;
+    if (hp->norm_growth_gamma > 0.0f) return ALQ_ERR_UNSUPPORTED;
+    cudaStream_t st = (cudaStream_t)stream;
+    const ApEntry* tab = (const ApEntry*)((const char*)plan_dev + kApEntryOffset);
+    const uint16_t* tile_mat = (const uint16_t*)((const char*)plan_dev + kApEntryOffset +
+                                                 (size_t)info->nmat * sizeof(ApEntry));
+    int* err = (int*)info->workspace;
+
+    apollo_convert_multi_kernel<<<persistent_grid((const void*)apollo_convert_multi_kernel,
+                                                  kThreads, 0, info->conv_tiles),
+                                  kThreads, 0, st>>>(tab, info->nmat, info->conv_tiles);
+    int rc = check_launch();
+    if (rc) return rc;
+
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [] {
+        attr_err = cudaFuncSetAttribute(apollo_project_multi_kernel,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);
+    });
+    if (attr_err != cudaSuccess) return record_cuda(attr_err);
+    apollo_project_multi_kernel<<<(unsigned)info->gemm_tiles, 128, kGemmSmem, st>>>(
+        tab, tile_mat, info->rank, err);
+    rc = check_launch();
+    if (rc) return rc;
+
+    const MomentArgs m = moment_scalars(hp, t, info->rank);
+    const int64_t nt = info->mom_tiles;
+#define ALQ_MOM(CPB, VB)                                                                     \
+    apollo_moments_multi_kernel<CPB, VB><<<                                                  \
+        persistent_grid((const void*)apollo_moments_multi_kernel<CPB, VB>, kThreads, 0, nt), \
+        kThreads, 0, st>>>(tab, info->nmat, nt, m)
+    if (info->rank == 128) {
+        if (info->v_bits == 8) ALQ_MOM(1, 8); else ALQ_MOM(1, 16);
+    } else {
+        if (info->v_bits == 8) ALQ_MOM(2, 8); else ALQ_MOM(2, 16);
+    }
+#undef ALQ_MOM
+    rc = check_launch();
+    if (rc) return rc;
+
+    ApUpdateArgs u{};
+    u.lim = nullptr;
+    u.decay = (float)(1.0 - (double)hp->lr * (double)hp->weight_decay);
+    u.lr_a = (float)((double)hp->lr * (double)hp->alpha);
+    apollo_update_multi_kernel<<<persistent_grid((const void*)apollo_update_multi_kernel,
+                                                 kThreads, 0, info->upd_tiles),
+                                 kThreads, 0, st>>>(tab, info->nmat, info->upd_tiles, u);
     return check_launch();
 }

@@ -155,3 +155,72 @@ def test_apollo_norm_growth_limiter(B):
         torch.cuda.synchronize()
         assert abs(float(a.dprev.item()) - float(a.prev)) <= 1e-5 * float(a.prev)
         assert _rel(a.d["p"].cpu().numpy(), a.h["p"]) < 1e-5
+
+
+# ------------------------------------------------------------ grouped step --
+def _mat_state(rows, cols, rank, v_bits, seed):
+    s_, L = min(rows, cols), max(rows, cols)
+    P = wl.bf16_bits(wl.gaussian_projection(rank, s_, seed))
+    n_p = L * rank
+    vdt = np.uint8 if v_bits == 8 else np.uint16
+    return dict(p=wl.param_init((rows, cols), seed + 1).ravel(), proj=P,
+                m_codes=np.zeros(n_p, np.int8), m_absmax=np.zeros(n_p // rank, np.float32),
+                v_codes=np.zeros(n_p, vdt), v_meta=np.zeros(2 * (n_p // rank), np.float32))
+
+
+@pytest.mark.parametrize("rank,v_bits", [(128, 8), (256, 8), (256, 16)])
+def test_apollo_grouped_step_matches_single(B, rank, v_bits):
+    """One grouped launch sequence over matrices of mixed shape (channels
+    along columns and along rows, short side below, equal to and above the
+    rank, ragged 128-channel tiles) gives, matrix by matrix, bit-for-bit the
+    results of al_apollo_step: parameters, projected-moment codes and block
+    metadata, over three steps."""
+    import torch
+    shapes = [(64, 256), (384, 128), (256, 256), (136, 1000), (1000, 136), (512, 2048)]
+    hp = dict(HP, rank=rank)
+    single, grouped = [], []
+    for i, (rows, cols) in enumerate(shapes):
+        st = _mat_state(rows, cols, rank, v_bits, 300 + 7 * i)
+        single.append({k: _t(v) for k, v in st.items()})
+        grouped.append({k: _t(v) for k, v in st.items()})
+        single[-1]["prev"] = torch.zeros(1, dtype=torch.float32, device="cuda")
+    grads = {}
+    for t in range(1, 4):
+        for i, (rows, cols) in enumerate(shapes):
+            grads[(i, t)] = _t(wl.gaussian_grad((rows, cols), 1e-3, 9000 + 13 * i + t).ravel())
+    plans = {}
+    for t in range(1, 4):
+        for i, (rows, cols) in enumerate(shapes):
+            d = single[i]
+            ws = torch.zeros(B.al_workspace_size(B.AL_OP_APOLLO, rows, cols, rank),
+                             dtype=torch.uint8, device="cuda")
+            B.al_apollo_step(d["p"], grads[(i, t)], rows, cols, d["proj"], d["m_codes"],
+                             d["m_absmax"], rank, d["v_codes"], d["v_meta"], v_bits, rank,
+                             d["prev"], hp, t, ws)
+        # the plan binds the gradient buffers, so step t gets its own plan
+        mats = [dict(grouped[i], g=grads[(i, t)], rows=rows, cols=cols)
+                for i, (rows, cols) in enumerate(shapes)]
+        plans[t] = B.ApolloPlan(mats, rank, v_bits)
+        plans[t].step(hp, t)
+        torch.cuda.synchronize()
+        for i in range(len(shapes)):
+            for k in ("p", "m_codes", "m_absmax", "v_codes", "v_meta"):
+                a = single[i][k].cpu().numpy().view(np.uint8)
+                b = grouped[i][k].cpu().numpy().view(np.uint8)
+                assert np.array_equal(a, b), (shapes[i], k, t)
+    info = plans[3].info
+    assert info.nmat == len(shapes)
+    assert info.gemm_tiles == sum((max(r, c) + 127) // 128 for r, c in shapes)
+
+
+def test_apollo_grouped_rejects_limiter_and_bad_arguments(B):
+    import torch
+    st = {k: _t(v) for k, v in _mat_state(64, 256, 128, 8, 5).items()}
+    g = torch.zeros(64 * 256, dtype=torch.float32, device="cuda")
+    plan = B.ApolloPlan([dict(st, g=g, rows=64, cols=256)], 128, 8)
+    with pytest.raises(B.AlqError):
+        plan.step(dict(HP, rank=128, norm_growth_gamma=1.01), 1)
+    with pytest.raises(B.AlqError):
+        plan.step(dict(HP, rank=256), 1)  # rank differs from the plan's
+    with pytest.raises(B.AlqError):
+        B.ApolloPlan([dict(st, g=g, rows=64, cols=254)], 128, 8)  # cols % 4 != 0
