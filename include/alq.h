@@ -399,7 +399,7 @@ typedef struct {
     int64_t total_channels; /* sum of max(rows, cols)                        */
     int64_t conv_tiles;     /* tiles of the bf16 staging pass                */
     int64_t gemm_tiles;     /* 128-channel tiles of the grouped projection   */
-    int64_t mom_tiles;      /* 4096-value tiles of the moments pass          */
+    int64_t mom_tiles;      /* 2048-value tiles of the moments pass          */
     int64_t upd_tiles;      /* 4096-parameter tiles of the update pass       */
     void* workspace;        /* the workspace the plan is bound to            */
 } al_apollo_info;

@@ -95,23 +95,38 @@ __device__ __forceinline__ void convert_rows_tile(const float* __restrict__ g, i
 }
 
 // rows <= cols: A[j][i] = bf16(G[i][j]) (channels are columns, K = rows),
-// one 32 x 32 tile (tile row tr, tile column tc) through shared memory.
-// Every thread of the CTA must call it; it ends with a barrier so that the
-// shared tile can be reused.
+// one 64 x 64 tile (tile row tr over i, tile column tc over j) through
+// shared memory: 16-byte loads along G's rows, 8-byte stores (four bf16)
+// along A's rows. Every thread of the CTA must call it; it ends with a
+// barrier so that the shared tile can be reused. rows and cols are multiples
+// of 4 (the entry points require cols % 4 == 0 and rows % 8 == 0 here).
+constexpr int kTT = 64;
 __device__ __forceinline__ void convert_cols_tile(const float* __restrict__ g, int rows, int cols,
                                                   uint16_t* __restrict__ A, int64_t tr,
-                                                  int64_t tc, float (*t)[33]) {
-    const int c0 = (int)tc * 32, r0 = (int)tr * 32;
-    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;  // 32 x 8
-    for (int k = ty; k < 32; k += 8) {
-        const int r = r0 + k, c = c0 + tx;
-        t[k][tx] = (r < rows && c < cols) ? g[(int64_t)r * cols + c] : 0.0f;
+                                                  int64_t tc, float (*t)[kTT + 1]) {
+    const int i0 = (int)tr * kTT, j0 = (int)tc * kTT;
+    const int x4 = 4 * (threadIdx.x & 15), y = threadIdx.x >> 4;  // 16 x 16 threads
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int i = i0 + y + 16 * q, j = j0 + x4;
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (i < rows && j < cols) v = __ldcs(reinterpret_cast<const float4*>(g + (int64_t)i * cols + j));
+        t[y + 16 * q][x4] = v.x;
+        t[y + 16 * q][x4 + 1] = v.y;
+        t[y + 16 * q][x4 + 2] = v.z;
+        t[y + 16 * q][x4 + 3] = v.w;
     }
     __syncthreads();
-    for (int k = ty; k < 32; k += 8) {
-        const int j = c0 + k, i = r0 + tx;  // A row j (channel), column i
-        if (j < cols && i < rows)
-            A[(int64_t)j * rows + i] = __bfloat16_as_ushort(__float2bfloat16_rn(t[tx][k]));
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int jl = y + 16 * q, j = j0 + jl, i = i0 + x4;  // A row j, columns i .. i + 3
+        if (j < cols && i < rows) {
+            const uint32_t lo = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t[x4][jl])) |
+                                ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t[x4 + 1][jl])) << 16);
+            const uint32_t hi = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t[x4 + 2][jl])) |
+                                ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t[x4 + 3][jl])) << 16);
+            *reinterpret_cast<uint2*>(A + (int64_t)j * rows + i) = make_uint2(lo, hi);
+        }
     }
     __syncthreads();
 }
@@ -123,7 +138,7 @@ to_bf16_kernel(const float* __restrict__ g, int64_t n, uint16_t* __restrict__ A,
 
 __global__ void __launch_bounds__(kThreads)
 to_bf16_t_kernel(const float* __restrict__ g, int rows, int cols, uint16_t* __restrict__ A) {
-    __shared__ float t[32][33];
+    __shared__ float t[kTT][kTT + 1];
     convert_cols_tile(g, rows, cols, A, blockIdx.y, blockIdx.x, t);
 }
 
@@ -318,145 +333,163 @@ struct MomentArgs {
     float beta1, beta2, omb1, omb2, ic1, c2, eps, log_floor;
 };
 
-// One tile (kTile projected values) of the moments pass; tab is this warp's
-// decode-table slot (NB * 32 entries).
+// Geometry of the moments pass: a warp owns a 256-element segment (two
+// 4-element chunks per lane, 128 elements apart), so one rank-256 channel
+// (or two rank-128 channels); a CTA owns a 2048-element tile.
+constexpr int kMCH = 2;
+constexpr int kMSeg = 128 * kMCH;
+constexpr int kMTile = 8 * kMSeg;
+
+// One tile of the moments pass. tab and vals are this warp's shared slots
+// for the AL8 decode tables (NB * 32 pairs) and the blocks' 256 decoded
+// values (NB * 256).
 template <int CPB, int VBITS>
-__device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, float2* tab) {
-    constexpr int NB = 4 / CPB;
+__device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, float2* tab,
+                                             float* vals) {
+    constexpr int NB = kMCH / CPB;
+    constexpr int NE = 4 * kMCH;
     constexpr float Lm2 = VBITS == 8 ? 254.0f : 65534.0f;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const float kf = al8_table_k(lane);
     const int64_t nblk = blocks_of_dev(m.n, m.block);
     const int bshift = __ffs(m.block) - 1;
-    {
-        const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
-        const int64_t b0 = seg0 >> bshift;
-        float4 r[4];
-        uint32_t mw[4], vw[4 * VBITS / 8];
+    const int64_t seg0 = tile * kMTile + (int64_t)warp * kMSeg;
+    const int64_t b0 = seg0 >> bshift;
+    float4 r[kMCH];
+    uint32_t mw[kMCH], vw[kMCH * VBITS / 8];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            const int64_t idx = chunk_index(seg0, c, lane);
-            r[c] = load4f(m.R, idx, m.n);
-            mw[c] = load4b((const uint8_t*)m.m_codes, idx, m.n);
-            if (VBITS == 8) {
-                vw[c] = load4b((const uint8_t*)m.v_codes, idx, m.n);
-            } else {
-                const uint2 h = load4h((const uint16_t*)m.v_codes, idx, m.n);
-                vw[2 * c] = h.x;
-                vw[2 * c + 1] = h.y;
-            }
+    for (int c = 0; c < kMCH; ++c) {
+        const int64_t idx = chunk_index(seg0, c, lane);
+        r[c] = load4f(m.R, idx, m.n);
+        mw[c] = load4b((const uint8_t*)m.m_codes, idx, m.n);
+        if constexpr (VBITS == 8) {
+            vw[c] = load4b((const uint8_t*)m.v_codes, idx, m.n);
+        } else {
+            const uint2 h = load4h((const uint16_t*)m.v_codes, idx, m.n);
+            vw[2 * c] = h.x;
+            vw[2 * c + 1] = h.y;
         }
-        float olmin[NB], odelta[NB], dm[NB];
-#pragma unroll
-        for (int b = 0; b < NB; ++b) {
-            float2 mt = make_float2(0.f, 0.f);
-            float sa = 0.0f;
-            if (b0 + b < nblk) {
-                mt = __ldg(reinterpret_cast<const float2*>(m.v_meta) + b0 + b);
-                sa = __ldg(m.m_absmax + b0 + b);
-            }
-            olmin[b] = mt.x;
-            odelta[b] = mt.y;
-            dm[b] = sa / 127.0f;
-        }
-        if (VBITS == 8) al8_build_tables<NB>(tab, olmin, odelta, kf);
-        float mf[16], vf[16];
-        uint32_t cvmin[4], cvmax[4], cmabs[4];
-        float nrh[NB], nrl[NB], ngh[NB], ngl[NB];
-#pragma unroll
-        for (int b = 0; b < NB; ++b) nrh[b] = nrl[b] = ngh[b] = ngl[b] = 0.0f;
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            const int b = c / CPB;
-            const bool fast = al8_fast_ok(olmin[b], odelta[b]);
-            cvmin[c] = 0xFFFFFFFFu;
-            cvmax[c] = 0u;
-            cmabs[c] = 0u;
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const uint32_t qv = code_of<VBITS>(vw, c, i);
-                const float vh = VBITS == 8
-                                     ? al8_decode(qv, tab + 32 * b, fast, olmin[b], odelta[b])
-                                     : al16_decode(qv, olmin[b], odelta[b]);
-                const float mh = s8_to_float((mw[c] >> (8 * i)) & 0xFFu) * dm[b];
-                const float rv = f4get(r[c], i);
-                const float mq = m.beta1 * mh + m.omb1 * rv;
-                const float vq = m.beta2 * vh + m.omb2 * (rv * rv);
-                const float rt = (mq * m.ic1) / (sqrtf(vq) * m.c2 + m.eps);
-                mf[4 * c + i] = mq;
-                vf[4 * c + i] = vq;
-                float h, l;
-                two_prod(rt, rt, h, l);
-                ff_acc(nrh[b], nrl[b], h, l);
-                two_prod(rv, rv, h, l);
-                ff_acc(ngh[b], ngl[b], h, l);
-                const uint32_t vb = f2u(vq);
-                cvmin[c] = umix<false>(cvmin[c], vb - 1u);
-                cvmax[c] = umix<true>(cvmax[c], vb);
-                cmabs[c] = umix<true>(cmabs[c], f2u(mq) & 0x7FFFFFFFu);
-            }
-        }
-        uint32_t bvmin[NB], bvmax[NB], bmabs[NB];
-        warp_blocks_reduce<CPB, false>(cvmin, bvmin);
-        warp_blocks_reduce<CPB, true>(cvmax, bvmax);
-        warp_blocks_reduce<CPB, true>(cmabs, bmabs);
-#pragma unroll
-        for (int b = 0; b < NB; ++b) {
-            ff_warp_sum(nrh[b], nrl[b]);
-            ff_warp_sum(ngh[b], ngl[b]);
-        }
-        float vmn[NB], vmx[NB], nlmin[NB], ndelta[NB], K[NB], E[NB], ms[NB], sc[NB], inv[NB];
-#pragma unroll
-        for (int b = 0; b < NB; ++b) {
-            vmn[b] = u2f(bvmin[b] + 1u);
-            vmx[b] = u2f(bvmax[b]);
-            ms[b] = u2f(bmabs[b]);
-            sc[b] = 1.0f;
-            inv[b] = 0.0f;
-            if (ms[b] > 0.0f) uf8_encode_consts(ms[b], sc[b], inv[b]);
-        }
-        al_blocks_params<NB>(vmn, vmx, m.log_floor, nlmin, ndelta);
-#pragma unroll
-        for (int b = 0; b < NB; ++b) al_encode_consts(ndelta[b], Lm2, K[b], E[b]);
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            const int b = c / CPB;
-            const int64_t idx = chunk_index(seg0, c, lane);
-            uint32_t qm = 0, qv[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                if (ms[b] > 0.0f)
-                    qm |= ((uint32_t)uf8_quantize(mf[4 * c + i], sc[b], inv[b]) & 0xFFu) << (8 * i);
-                qv[i] = al_encode_elem<VBITS>(vf[4 * c + i], nlmin[b], ndelta[b], K[b], E[b]);
-            }
-            store4b((uint8_t*)m.m_codes, idx, m.n, qm);
-            if (VBITS == 8)
-                store4b((uint8_t*)m.v_codes, idx, m.n, qv[0] | (qv[1] << 8) | (qv[2] << 16) | (qv[3] << 24));
-            else
-                store4h((uint16_t*)m.v_codes, idx, m.n,
-                        make_uint2(qv[0] | (qv[1] << 16), qv[2] | (qv[3] << 16)));
-        }
-        if (lane == 0) {
-#pragma unroll
-            for (int b = 0; b < NB; ++b) {
-                if (b0 + b >= nblk) continue;
-                reinterpret_cast<float2*>(m.v_meta)[b0 + b] = make_float2(nlmin[b], ndelta[b]);
-                m.m_absmax[b0 + b] = ms[b];
-                const double nr = (double)nrh[b] + (double)nrl[b];
-                const double ng = (double)ngh[b] + (double)ngl[b];
-                m.scale[b0 + b] = (float)(sqrt(nr) / (sqrt(ng) + 1e-8));
-            }
-        }
-        __syncwarp();
     }
+    float olmin[NB], odelta[NB], dm[NB];
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+        float2 mt = make_float2(0.f, 0.f);
+        float sa = 0.0f;
+        if (b0 + b < nblk) {
+            mt = __ldg(reinterpret_cast<const float2*>(m.v_meta) + b0 + b);
+            sa = __ldg(m.m_absmax + b0 + b);
+        }
+        olmin[b] = mt.x;
+        odelta[b] = mt.y;
+        dm[b] = sa / 127.0f;
+    }
+    // previous V: AL8 through the blocks' tables of exactly rounded values
+    float vh[NE];
+    if constexpr (VBITS == 8) {
+        al8_build_values<NB>(vals, tab, olmin, odelta, kf);
+#pragma unroll
+        for (int e = 0; e < NE; ++e)
+            vh[e] = vals[256 * (e / 4 / CPB) + ((vw[e / 4] >> (8 * (e % 4))) & 0xFFu)];
+    } else {
+#pragma unroll
+        for (int e = 0; e < NE; ++e)
+            vh[e] = al16_decode(code_of<VBITS>(vw, e / 4, e % 4), olmin[e / 4 / CPB],
+                                odelta[e / 4 / CPB]);
+    }
+    float mf[NE], vf[NE];
+    uint32_t cvmin[kMCH], cvmax[kMCH], cmabs[kMCH];
+    float nrh[NB], nrl[NB], ngh[NB], ngl[NB];
+#pragma unroll
+    for (int b = 0; b < NB; ++b) nrh[b] = nrl[b] = ngh[b] = ngl[b] = 0.0f;
+#pragma unroll
+    for (int c = 0; c < kMCH; ++c) {
+        const int b = c / CPB;
+        cvmin[c] = 0xFFFFFFFFu;
+        cvmax[c] = 0u;
+        cmabs[c] = 0u;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float mh = s8_to_float((mw[c] >> (8 * i)) & 0xFFu) * dm[b];
+            const float rv = f4get(r[c], i);
+            const float mq = m.beta1 * mh + m.omb1 * rv;
+            const float vq = m.beta2 * vh[4 * c + i] + m.omb2 * (rv * rv);
+            const float rt = (mq * m.ic1) / (sqrtf(vq) * m.c2 + m.eps);
+            mf[4 * c + i] = mq;
+            vf[4 * c + i] = vq;
+            float h, l;
+            two_prod(rt, rt, h, l);
+            ff_acc(nrh[b], nrl[b], h, l);
+            two_prod(rv, rv, h, l);
+            ff_acc(ngh[b], ngl[b], h, l);
+            const uint32_t vb = f2u(vq);
+            cvmin[c] = umix<false>(cvmin[c], vb - 1u);
+            cvmax[c] = umix<true>(cvmax[c], vb);
+            cmabs[c] = umix<true>(cmabs[c], f2u(mq) & 0x7FFFFFFFu);
+        }
+    }
+    uint32_t bvmin[NB], bvmax[NB], bmabs[NB];
+    warp_blocks_reduce<CPB, false>(cvmin, bvmin);
+    warp_blocks_reduce<CPB, true>(cvmax, bvmax);
+    warp_blocks_reduce<CPB, true>(cmabs, bmabs);
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+        ff_warp_sum(nrh[b], nrl[b]);
+        ff_warp_sum(ngh[b], ngl[b]);
+    }
+    float vmn[NB], vmx[NB], nlmin[NB], ndelta[NB], K[NB], E[NB], ms[NB], sc[NB], inv[NB];
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+        vmn[b] = u2f(bvmin[b] + 1u);
+        vmx[b] = u2f(bvmax[b]);
+        ms[b] = u2f(bmabs[b]);
+        sc[b] = 1.0f;
+        inv[b] = 0.0f;
+        if (ms[b] > 0.0f) uf8_encode_consts(ms[b], sc[b], inv[b]);
+    }
+    al_blocks_params<NB>(vmn, vmx, m.log_floor, nlmin, ndelta);
+#pragma unroll
+    for (int b = 0; b < NB; ++b) al_encode_consts(ndelta[b], Lm2, K[b], E[b]);
+    uint32_t qv[NE];
+    al_encode_chunks<VBITS, CPB, NB, kMCH>(vf, nlmin, ndelta, K, E, qv);
+#pragma unroll
+    for (int c = 0; c < kMCH; ++c) {
+        const int b = c / CPB;
+        const int64_t idx = chunk_index(seg0, c, lane);
+        uint32_t qm = 0;
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            qm |= ((uint32_t)uf8_quantize(mf[4 * c + i], sc[b], inv[b]) & 0xFFu) << (8 * i);
+        store4b((uint8_t*)m.m_codes, idx, m.n, qm);
+        if constexpr (VBITS == 8)
+            store4b((uint8_t*)m.v_codes, idx, m.n,
+                    qv[4 * c] | (qv[4 * c + 1] << 8) | (qv[4 * c + 2] << 16) | (qv[4 * c + 3] << 24));
+        else
+            store4h((uint16_t*)m.v_codes, idx, m.n,
+                    make_uint2(qv[4 * c] | (qv[4 * c + 1] << 16), qv[4 * c + 2] | (qv[4 * c + 3] << 16)));
+    }
+    if (lane == 0) {
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            if (b0 + b >= nblk) continue;
+            reinterpret_cast<float2*>(m.v_meta)[b0 + b] = make_float2(nlmin[b], ndelta[b]);
+            m.m_absmax[b0 + b] = ms[b];
+            const double nr = (double)nrh[b] + (double)nrl[b];
+            const double ng = (double)ngh[b] + (double)ngl[b];
+            m.scale[b0 + b] = (float)(sqrt(nr) / (sqrt(ng) + 1e-8));
+        }
+    }
+    __syncwarp();
 }
 
 template <int CPB, int VBITS>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 3)
 apollo_moments_kernel(MomentArgs m, int64_t ntiles) {
-    __shared__ float2 s_tab[kThreads / 32][(4 / CPB) * 32];
+    constexpr int NB = kMCH / CPB;
+    __shared__ float2 s_tab[kThreads / 32][NB * 32];
+    __shared__ float s_val[kThreads / 32][VBITS == 8 ? NB * 256 : 1];
+    const int warp = threadIdx.x >> 5;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x)
-        moments_tile<CPB, VBITS>(m, tile, s_tab[threadIdx.x >> 5]);
+        moments_tile<CPB, VBITS>(m, tile, s_tab[warp], s_val[warp]);
 }
 
 // ------------------------------------------------------ limiter, update --
@@ -610,14 +643,14 @@ __device__ __forceinline__ int entry_for(const ApEntry* __restrict__ tab, int nm
 
 __global__ void __launch_bounds__(kThreads)
 apollo_convert_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t ntiles) {
-    __shared__ float t[32][33];
+    __shared__ float t[kTT][kTT + 1];
     int cur = 0;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         cur = entry_for(tab, nmat, tile, cur, &ApEntry::conv_t0);
         const ApEntry& e = tab[cur];
         const int64_t lt = tile - e.conv_t0;
         if (e.rows_short) {
-            const int64_t ntc = (e.cols + 31) / 32;
+            const int64_t ntc = (e.cols + kTT - 1) / kTT;
             convert_cols_tile(e.g, (int)e.rows, (int)e.cols, e.A, lt / ntc, lt % ntc, t);
         } else {
             convert_rows_tile(e.g, e.n, e.A, lt);
@@ -643,10 +676,13 @@ apollo_project_multi_kernel(const ApEntry* __restrict__ tab, const uint16_t* __r
 }
 
 template <int CPB, int VBITS>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 3)
 apollo_moments_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t ntiles,
                             MomentArgs base) {
-    __shared__ float2 s_tab[kThreads / 32][(4 / CPB) * 32];
+    constexpr int NB = kMCH / CPB;
+    __shared__ float2 s_tab[kThreads / 32][NB * 32];
+    __shared__ float s_val[kThreads / 32][VBITS == 8 ? NB * 256 : 1];
+    const int warp = threadIdx.x >> 5;
     int cur = 0;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         cur = entry_for(tab, nmat, tile, cur, &ApEntry::mom_t0);
@@ -659,7 +695,7 @@ apollo_moments_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t n
         m.v_codes = e.v_codes;
         m.v_meta = e.v_meta;
         m.scale = e.scale;
-        moments_tile<CPB, VBITS>(m, tile - e.mom_t0, s_tab[threadIdx.x >> 5]);
+        moments_tile<CPB, VBITS>(m, tile - e.mom_t0, s_tab[warp], s_val[warp]);
     }
 }
 
@@ -765,7 +801,7 @@ static MomentArgs moment_scalars(const al_apollo_hp* hp, int64_t t, int rank) {
 
 template <int CPB, int VBITS>
 static void launch_moments_t(const MomentArgs& m, cudaStream_t st) {
-    const int64_t ntiles = blocks_of(m.n, kTile);
+    const int64_t ntiles = blocks_of(m.n, kMTile);
     auto k = apollo_moments_kernel<CPB, VBITS>;
     k<<<persistent_grid((const void*)k, kThreads, 0, ntiles), kThreads, 0, st>>>(m, ntiles);
 }
@@ -794,8 +830,8 @@ extern "C" int al_apollo_step(float* p, const float* g, int64_t rows, int64_t co
 
     // bf16 operand with the short side contiguous
     if (rows_short) {
-        dim3 grid((unsigned)blocks_of(cols, 32), (unsigned)blocks_of(rows, 32));
-        to_bf16_t_kernel<<<grid, 256, 0, st>>>(g, (int)rows, (int)cols, w.A);
+        dim3 grid((unsigned)blocks_of(cols, kTT), (unsigned)blocks_of(rows, kTT));
+        to_bf16_t_kernel<<<grid, kThreads, 0, st>>>(g, (int)rows, (int)cols, w.A);
     } else {
         const int64_t n = rows * cols, ntiles = blocks_of(n, kTile);
         to_bf16_kernel<<<persistent_grid((const void*)to_bf16_kernel, kThreads, 0, ntiles),
@@ -865,7 +901,7 @@ static ApShape ap_shape(const al_apollo_matrix& m) {
 
 static int64_t conv_tiles_of(const al_apollo_matrix& m) {
     const ApShape a = ap_shape(m);
-    return a.rows_short ? blocks_of(m.cols, 32) * blocks_of(m.rows, 32) : blocks_of(a.n, kTile);
+    return a.rows_short ? blocks_of(m.cols, kTT) * blocks_of(m.rows, kTT) : blocks_of(a.n, kTile);
 }
 
 // Per-matrix scratch of a grouped step: A, R, scale, each 256-byte aligned.
@@ -972,7 +1008,7 @@ extern "C" int al_apollo_plan(const al_apollo_matrix* mats, int nmat, int rank, 
         for (int64_t k = 0; k < gt; ++k) tile_mat[h.gemm_tiles + k] = (uint16_t)i;
         h.conv_tiles += conv_tiles_of(m);
         h.gemm_tiles += gt;
-        h.mom_tiles += blocks_of(e.npj, kTile);
+        h.mom_tiles += blocks_of(e.npj, kMTile);
         h.upd_tiles += blocks_of(a.n, kTile);
         h.total_params += a.n;
         h.total_channels += a.L;
