@@ -11,7 +11,8 @@
 //   scale      a_i = 1/sqrt(R_i / mean(R)), b_j = 1/sqrt(C_j).
 //   usq        G read again: u = (g a_i) b_j, exact float-float sum of u^2,
 //              one fp64 partial per CTA of a persistent grid (fixed order).
-//   clip       1 / max(1, RMS(u) / d).
+//              The last CTA of usq adds the partials and writes the clip
+//              factor 1 / max(1, RMS(u) / d).
 //   update     G read a third time: u_hat, optional UF8 momentum, p update.
 // CAME inserts, before its update, a second sumsq pass over the residual
 // (u_hat - m)^2 + eps2 (recomputing m from the old momentum codes), a second
@@ -43,6 +44,7 @@ struct FacWs {
     float* scal;      // [4]: icf
     double* rsum;     // [rows / 128 + 1]: per-block sums of the fresh row factor (V)
     double* rsum2;    // same for the confidence row factor (C)
+    unsigned int* ticket;  // CTAs of the RMS pass that have finished
     size_t bytes;
 };
 
@@ -72,6 +74,7 @@ static FacWs fac_layout(void* base, int64_t rows, int64_t cols) {
     w.scal = (float*)take(sizeof(float) * 4);
     w.rsum = (double*)take(sizeof(double) * (rows / 128 + 1));
     w.rsum2 = (double*)take(sizeof(double) * (rows / 128 + 1));
+    w.ticket = (unsigned int*)take(sizeof(unsigned int));
     w.bytes = off;
     return w;
 }
@@ -233,8 +236,18 @@ factor_kernel(FactorDesc f0, FactorDesc f1, int nb0, double* __restrict__ rsum) 
         const int64_t i = lo + threadIdx.x + (int64_t)kThreads * k;
         v[k] = 0.0f;
         if (i < hi) {
+            // partials in index order; loads issued eight at a time
             double s = 0.0;
-            for (int p = 0; p < f.nparts; ++p) s += f.part[(int64_t)p * f.len + i];
+            const double* pp = f.part + i;
+            int p = 0;
+            for (; p + 8 <= f.nparts; p += 8) {
+                double t8[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) t8[q] = pp[(int64_t)(p + q) * f.len];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) s += t8[q];
+            }
+            for (; p < f.nparts; ++p) s += pp[(int64_t)p * f.len];
             const float stat = (float)(s / f.mean_len + f.add_eps);
             const float old = al_decode_direct(fac_code(f, i), om.x, om.y, Lm2);
             v[k] = f.beta * old + f.omb * stat;
@@ -291,8 +304,9 @@ factor_kernel(FactorDesc f0, FactorDesc f1, int nb0, double* __restrict__ rsum) 
 __global__ void __launch_bounds__(kThreads)
 scale_kernel(const float* __restrict__ R, int rows, const float* __restrict__ C, int cols,
              const double* __restrict__ rsum, int nrb, float* __restrict__ a,
-             float* __restrict__ b) {
+             float* __restrict__ b, unsigned int* __restrict__ ticket) {
     __shared__ float s_mean;
+    if (ticket && blockIdx.x == 0 && threadIdx.x == 0) *ticket = 0u;  // for the RMS pass
     if (threadIdx.x == 0) {
         double t = 0.0;
         for (int k = 0; k < nrb; ++k) t += rsum[k];
@@ -309,11 +323,17 @@ scale_kernel(const float* __restrict__ R, int rows, const float* __restrict__ C,
 
 // ------------------------------------------------------------------- usq --
 // Sum of u^2, u = (g a_i) b_j, over the whole matrix: exact squares in
-// two-float per thread, fixed warp/CTA order, one fp64 partial per CTA.
+// two-float per thread, fixed warp/CTA order, one fp64 partial per CTA. The
+// last CTA to finish (an atomic ticket, zeroed by the scale pass) adds the
+// partials in CTA order and writes the clip factor
+// scal[0] = 1 / max(1, sqrt(sum / count) / clip_d).
 __global__ void __launch_bounds__(kThreads)
 usq_kernel(const float* __restrict__ g, int64_t n, Divider dv, const float* __restrict__ a,
-           const float* __restrict__ b, int64_t ntiles, double* __restrict__ upart) {
-    __shared__ double s_w[kThreads / 32];
+           const float* __restrict__ b, int64_t ntiles, double* __restrict__ upart,
+           unsigned int* __restrict__ ticket, double count, float clip_d,
+           float* __restrict__ scal) {
+    __shared__ double s_w[kThreads];
+    __shared__ bool s_last;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     float hi = 0.0f, lo = 0.0f;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
@@ -344,29 +364,29 @@ usq_kernel(const float* __restrict__ g, int64_t n, Divider dv, const float* __re
         double s = 0.0;
         for (int w = 0; w < kThreads / 32; ++w) s += s_w[w];
         upart[blockIdx.x] = s;
+        __threadfence();
+        s_last = atomicAdd(ticket, 1u) == gridDim.x - 1;
     }
-}
-
-// ------------------------------------------------------------------ clip --
-__global__ void __launch_bounds__(1024)
-clip_kernel(const double* __restrict__ upart, int nparts, double count, float clip_d,
-            float* __restrict__ scal) {
-    __shared__ double s[1024];
-    double acc = 0.0;
-    for (int i = threadIdx.x; i < nparts; i += 1024) acc += upart[i];
-    s[threadIdx.x] = acc;
     __syncthreads();
-    for (int st = 512; st > 0; st >>= 1) {
-        if ((int)threadIdx.x < st) s[threadIdx.x] += s[threadIdx.x + st];
+    if (!s_last) return;
+    __threadfence();
+    // fixed order: per thread over a stride of kThreads, then a tree
+    double acc = 0.0;
+    for (int i = threadIdx.x; i < (int)gridDim.x; i += kThreads) acc += ((volatile double*)upart)[i];
+    s_w[threadIdx.x] = acc;
+    __syncthreads();
+    for (int st = kThreads / 2; st > 0; st >>= 1) {
+        if ((int)threadIdx.x < st) s_w[threadIdx.x] += s_w[threadIdx.x + st];
         __syncthreads();
     }
     if (threadIdx.x == 0) {
-        const double rms = sqrt(s[0] / count);
+        const double rms = sqrt(s_w[0] / count);
         double cf = rms / (double)clip_d;
         if (cf < 1.0) cf = 1.0;
         scal[0] = (float)(1.0 / cf);
     }
 }
+
 
 // ---------------------------------------------------------------- update --
 // MODE 0: Adafactor without momentum; 1: Adafactor with UF8 momentum;
@@ -560,14 +580,13 @@ static int second_moment_passes(const float* g, int64_t rows, int64_t cols, cons
     const int nb0 = (int)blocks_of(rows, fr.block);
     launch_factor(fr, fc, w.rsum, st);
     scale_kernel<<<(unsigned)blocks_of(rows + cols, kThreads), kThreads, 0, st>>>(
-        fr.fresh, (int)rows, fc.fresh, (int)cols, w.rsum, nb0, a, b);
+        fr.fresh, (int)rows, fc.fresh, (int)cols, w.rsum, nb0, a, b, w.ticket);
     const int64_t n = rows * cols;
     const int64_t ntiles = blocks_of(n, kTile);
     int grid = persistent_grid((const void*)usq_kernel, kThreads, 0, ntiles);
     if (grid > kMaxParts) grid = kMaxParts;
     usq_kernel<<<grid, kThreads, 0, st>>>(g, n, make_divider((uint32_t)cols), a, b, ntiles,
-                                          w.upart);
-    clip_kernel<<<1, 1024, 0, st>>>(w.upart, grid, (double)n, clip_d, w.scal);
+                                          w.upart, w.ticket, (double)n, clip_d, w.scal);
     return check_launch();
 }
 
@@ -678,7 +697,8 @@ int al_came_step(float* p, const float* g, int64_t rows, int64_t cols, void* vr_
     const int nb0 = (int)blocks_of(rows, c_block), nb1 = (int)blocks_of(cols, c_block);
     launch_factor(cr, cc, w.rsum2, s);
     scale_kernel<<<(unsigned)blocks_of(rows + cols, kThreads), kThreads, 0, s>>>(
-        w.fr2, (int)rows, w.fc2, (int)cols, w.rsum2, (int)blocks_of(rows, cr.block), w.a2, w.b2);
+        w.fr2, (int)rows, w.fc2, (int)cols, w.rsum2, (int)blocks_of(rows, cr.block), w.a2, w.b2,
+        nullptr);
     st = check_launch();
     if (st) return st;
 
