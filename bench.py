@@ -502,13 +502,25 @@ def _row_came(torch, np, wl, B, dev):
         mats.append(dict(p=p, gs=gs, vr=fac(rows, vb), vc=fac(cols, vb), cr=fac(rows, cb),
                          cc=fac(cols, cb), mc=torch.zeros(n1, dtype=torch.int8, device=dev),
                          ma=torch.zeros((n1 + 255) // 256, dtype=torch.float32, device=dev)))
-    ws = torch.empty(B.al_workspace_size(B.AL_OP_CAME, rows, cols), dtype=torch.uint8, device=dev)
+    # the matrices' steps are independent: spread them over a few streams
+    # (one workspace each) so that one matrix's short passes overlap with
+    # another's streaming passes
+    nstreams = int(os.environ.get("ALQ_BENCH_STREAMS", "8"))
+    streams = [torch.cuda.Stream(device=dev) for _ in range(nstreams)]
+    wss = [torch.empty(B.al_workspace_size(B.AL_OP_CAME, rows, cols), dtype=torch.uint8,
+                       device=dev) for _ in range(nstreams)]
 
     def step(t):
-        for m in mats:
+        main = torch.cuda.current_stream(dev)
+        for st in streams:
+            st.wait_stream(main)
+        for i, m in enumerate(mats):
+            k = i % nstreams
             B.al_came_step(m["p"], m["gs"][t % 2], rows, cols, m["vr"][0], m["vr"][1], m["vc"][0],
                            m["vc"][1], 16, vb, m["cr"][0], m["cr"][1], m["cc"][0], m["cc"][1],
-                           16, cb, m["mc"], m["ma"], 256, hp, t, ws)
+                           16, cb, m["mc"], m["ma"], 256, hp, t, wss[k], stream=streams[k])
+        for st in streams:
+            main.wait_stream(st)
 
     facb = sum(2 * 2 * mm + 16 * ((mm + blk - 1) // blk)
                for mm, blk in ((rows, vb), (cols, vb), (rows, cb), (cols, cb)))
@@ -530,7 +542,7 @@ def _row_came(torch, np, wl, B, dev):
 
     return dict(step=step, n=nm * n1, bytes=nbytes, launches=9 * nm, oracle=oracle_sample,
                 workload=f"CAME {nm} x {rows}x{cols}, AL16 factored V and C block 128, "
-                         f"UF8 momentum block 256",
+                         f"UF8 momentum block 256, matrices spread over {nstreams} streams",
                 bytes_note="algorithmic minimum 14.03 B/param (G read once)")
 
 

@@ -217,7 +217,11 @@ int al_adamw_step_multi(const void* plan_dev, const al_multi_info* info,
 #define AL_OP_CAME 2
 #define AL_OP_APOLLO 3
 
-/* Scratch bytes that al_adafactor_step / al_came_step / al_apollo_step need
+/* Steps of independent matrices may run concurrently on different streams,
+ * each call with its own workspace; for many small matrices this overlaps
+ * one matrix's short passes with another's streaming passes.
+ *
+ * Scratch bytes that al_adafactor_step / al_came_step / al_apollo_step need
  * for a rows x cols matrix (rank is used by APOLLO only). Host-only. */
 int al_workspace_size(int op, int64_t rows, int64_t cols, int rank,
                       size_t* bytes);
