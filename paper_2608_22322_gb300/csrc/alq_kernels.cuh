@@ -264,6 +264,30 @@ __device__ __forceinline__ void al8_decode_chunks(const uint32_t (&w)[CH], const
     }
 }
 
+// Fixed-size arrays passed by value to the out-of-line rare paths (so that
+// the hot path's register arrays never need an address).
+template <typename T, int N>
+struct Arr {
+    T v[N];
+};
+
+// Rare path of al_encode_chunks, out of line: redo the boundary tests and
+// recompute the flagged codes in FP64.
+template <int BITS, int CPB, int NB, int CH>
+static __device__ __noinline__ Arr<uint32_t, 4 * CH> al_encode_fixup(
+    Arr<float, 4 * CH> x, Arr<float, NB> lmin, Arr<float, NB> delta, Arr<float, NB> K,
+    Arr<float, NB> E, Arr<uint32_t, 4 * CH> q) {
+    constexpr float Lm2 = BITS == 8 ? 254.0f : 65534.0f;
+#pragma unroll
+    for (int e = 0; e < 4 * CH; ++e) {
+        const int b = e / 4 / CPB;
+        bool fb;
+        al_quantize_fast(x.v[e], lmin.v[b], K.v[b], E.v[b], Lm2, fb);
+        if (x.v[e] != 0.0f && fb) q.v[e] = al_quantize_fp64(x.v[e], lmin.v[b], delta.v[b], (double)Lm2);
+    }
+    return q;
+}
+
 // Eq. (4) for the 4 CH values of a lane's chunks, branch-free with the same
 // bit-mask fixup in FP64 for values near a half-integer of t.
 template <int BITS, int CPB, int NB, int CH>
@@ -282,13 +306,41 @@ __device__ __forceinline__ void al_encode_chunks(const float (&x)[4 * CH], const
         any_fb |= nz & fb;
     }
     if (__builtin_expect(__any_sync(0xFFFFFFFFu, any_fb), 0)) {
+        Arr<float, 4 * CH> xa;
+        Arr<uint32_t, 4 * CH> qa;
+        Arr<float, NB> la, da, ka, ea;
 #pragma unroll
         for (int e = 0; e < 4 * CH; ++e) {
-            const int b = e / 4 / CPB;
-            bool fb;
-            al_quantize_fast(x[e], lmin[b], K[b], E[b], Lm2, fb);
-            if (x[e] != 0.0f && fb) q[e] = al_quantize_fp64(x[e], lmin[b], delta[b], (double)Lm2);
+            xa.v[e] = x[e];
+            qa.v[e] = q[e];
         }
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            la.v[b] = lmin[b];
+            da.v[b] = delta[b];
+            ka.v[b] = K[b];
+            ea.v[b] = E[b];
+        }
+        qa = al_encode_fixup<BITS, CPB, NB, CH>(xa, la, da, ka, ea, qa);
+#pragma unroll
+        for (int e = 0; e < 4 * CH; ++e) q[e] = qa.v[e];
+    }
+}
+
+// Rare path of al8_build_values, out of line so that the hot loop stays
+// compact: redo this lane's eight boundary tests of one block and recompute
+// the flagged values in FP64.
+static __device__ __noinline__ void al8_values_fixup(float* vals, const float2* tab, float lmin,
+                                                     float delta) {
+    const int lane = threadIdx.x & 31;
+    const bool fast = al8_fast_ok(lmin, delta);
+    for (int k = 0; k < 8; ++k) {
+        const uint32_t q = (uint32_t)(lane + 32 * k);
+        const float2 A = tab[16 + (q >> 4)];
+        const float2 Bt = tab[q & 15u];
+        bool fb;
+        al8_decode_pair(A.x, A.y, Bt.x, Bt.y, fb);
+        if ((q != 0u) && (fb || !fast)) vals[q] = al_dequantize_fp64(q, lmin, delta, 254.0);
     }
 }
 
@@ -322,19 +374,7 @@ __device__ __forceinline__ void al8_build_values(float* vals, float2* tab,
     }
     if (__builtin_expect(__any_sync(0xFFFFFFFFu, any_fb), 0)) {
 #pragma unroll
-        for (int b = 0; b < NB; ++b) {
-            const bool fast = al8_fast_ok(lmin[b], delta[b]);
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                const uint32_t q = (uint32_t)(lane + 32 * k);
-                const float2 A = tab[32 * b + 16 + (q >> 4)];
-                const float2 Bt = tab[32 * b + (q & 15u)];
-                bool fb;
-                al8_decode_pair(A.x, A.y, Bt.x, Bt.y, fb);
-                if ((q != 0u) && (fb || !fast))
-                    vals[256 * b + q] = al_dequantize_fp64(q, lmin[b], delta[b], 254.0);
-            }
-        }
+        for (int b = 0; b < NB; ++b) al8_values_fixup(vals + 256 * b, tab + 32 * b, lmin[b], delta[b]);
     }
     __syncwarp();
 }
