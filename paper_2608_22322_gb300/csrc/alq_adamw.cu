@@ -22,6 +22,52 @@ constexpr int kCH = 2;
 constexpr int kASeg = 128 * kCH;
 constexpr int kATile = 8 * kASeg;
 
+// ------------------------------------------------ ragged-segment I/O --
+// Masked loads and stores of a segment that crosses the end of its tensor
+// (one per tensor), out of line so that the fused loop body stays compact.
+template <int VBITS>
+struct SegIn {
+    float4 g[kCH], p[kCH];
+    uint32_t mw[kCH], vw[kCH * VBITS / 8];
+};
+
+template <int VBITS>
+static __device__ __noinline__ SegIn<VBITS> load_seg_masked(const float* g, const float* p,
+                                                            const int8_t* m_codes,
+                                                            const void* v_codes, int64_t e0,
+                                                            int64_t n) {
+    SegIn<VBITS> r;
+#pragma unroll
+    for (int c = 0; c < kCH; ++c) {
+        const int64_t idx = e0 + 128 * c;
+        r.g[c] = load4f(g, idx, n);
+        r.p[c] = load4f(p, idx, n);
+        r.mw[c] = load4b((const uint8_t*)m_codes, idx, n);
+        if constexpr (VBITS == 8) {
+            r.vw[c] = load4b((const uint8_t*)v_codes, idx, n);
+        } else {
+            const uint2 h = load4h((const uint16_t*)v_codes, idx, n);
+            r.vw[2 * c] = h.x;
+            r.vw[2 * c + 1] = h.y;
+        }
+    }
+    return r;
+}
+
+static __device__ __noinline__ void store_p_masked(float* p, int64_t idx, int64_t n, float4 v) {
+    store4f(p, idx, n, v);
+}
+
+template <int VBITS>
+static __device__ __noinline__ void store_codes_masked(int8_t* m_codes, void* v_codes, int64_t idx,
+                                                       int64_t n, uint32_t qm, uint2 qv) {
+    store4b((uint8_t*)m_codes, idx, n, qm);
+    if constexpr (VBITS == 8)
+        store4b((uint8_t*)v_codes, idx, n, qv.x);
+    else
+        store4h((uint16_t*)v_codes, idx, n, qv);
+}
+
 // Step scalars as broadcast pairs: the element arithmetic runs on pairs of
 // elements with the paired fp32 instructions (each component rounded exactly
 // as the scalar operation), and a pair operand held in the kernel's
@@ -103,20 +149,15 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
                 }
             }
         } else {
+            const SegIn<VBITS> r = load_seg_masked<VBITS>(d.g, d.p, d.m_codes, d.v_codes, e0, n);
 #pragma unroll
             for (int c = 0; c < kCH; ++c) {
-                const int64_t idx = e0 + 128 * c;
-                g[c] = load4f(d.g, idx, n);
-                p[c] = load4f(d.p, idx, n);
-                mw[c] = load4b((const uint8_t*)d.m_codes, idx, n);
-                if constexpr (VBITS == 8) {
-                    vw[c] = load4b((const uint8_t*)d.v_codes, idx, n);
-                } else {
-                    const uint2 h = load4h((const uint16_t*)d.v_codes, idx, n);
-                    vw[2 * c] = h.x;
-                    vw[2 * c + 1] = h.y;
-                }
+                g[c] = r.g[c];
+                p[c] = r.p[c];
+                mw[c] = r.mw[c];
             }
+#pragma unroll
+            for (int k = 0; k < kCH * VBITS / 8; ++k) vw[k] = r.vw[k];
         }
 
         // ---- previous block constants
@@ -189,7 +230,7 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
             if (full)
                 __stcs(reinterpret_cast<float4*>(d.p + e0) + 32 * c, pv);
             else
-                store4f(d.p, e0 + 128 * c, n, pv);
+                store_p_masked(d.p, e0 + 128 * c, n, pv);
         }
         float vf[NE];
 #pragma unroll
@@ -255,13 +296,10 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
                     __stcs(reinterpret_cast<uint2*>((uint16_t*)d.v_codes + e0) + 32 * c,
                            make_uint2(qv[4 * c] | (qv[4 * c + 1] << 16), qv[4 * c + 2] | (qv[4 * c + 3] << 16)));
             } else {
-                store4b((uint8_t*)d.m_codes, idx, n, qm);
-                if constexpr (VBITS == 8)
-                    store4b((uint8_t*)d.v_codes, idx, n,
-                            qv[4 * c] | (qv[4 * c + 1] << 8) | (qv[4 * c + 2] << 16) | (qv[4 * c + 3] << 24));
-                else
-                    store4h((uint16_t*)d.v_codes, idx, n,
-                            make_uint2(qv[4 * c] | (qv[4 * c + 1] << 16), qv[4 * c + 2] | (qv[4 * c + 3] << 16)));
+                const uint2 w = VBITS == 8
+                    ? make_uint2(qv[4 * c] | (qv[4 * c + 1] << 8) | (qv[4 * c + 2] << 16) | (qv[4 * c + 3] << 24), 0u)
+                    : make_uint2(qv[4 * c] | (qv[4 * c + 1] << 16), qv[4 * c + 2] | (qv[4 * c + 3] << 16));
+                store_codes_masked<VBITS>(d.m_codes, d.v_codes, idx, n, qm, w);
             }
         }
         if (lane == 0) {
