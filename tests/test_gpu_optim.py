@@ -1,0 +1,215 @@
+"""The torch.optim wrappers (paper_2608_22322_gb300/optim.py) against direct
+C-ABI calls: the wrappers only group parameters and keep state, so every
+step must equal the direct calls bit for bit. Also covered: torch.optim
+conventions (closures, learning-rate schedulers, state_dict round trips with
+integer code tensors), AL8 <-> AL16 migration of trained states (Sec. 6.2
+per-role precision), and APOLLO's routing of non-matrix parameters to the
+quantized AdamW step."""
+import math
+
+import numpy as np
+import pytest
+
+from gpu_util import ADAMW_HP, gpu_available
+from paper_2608_22322_gb300 import workloads as wl
+
+pytestmark = [pytest.mark.gpu,
+              pytest.mark.skipif(not gpu_available(), reason="needs a CUDA GPU")]
+
+
+@pytest.fixture(scope="module")
+def mods():
+    from paper_2608_22322_gb300 import binding, optim
+    return binding, optim
+
+
+def _params(shapes, seed):
+    import torch
+    return [torch.nn.Parameter(torch.from_numpy(wl.param_init(s, seed + i)).cuda())
+            for i, s in enumerate(shapes)]
+
+
+def _grads(params, t, seed):
+    import torch
+    for i, p in enumerate(params):
+        p.grad = torch.from_numpy(
+            wl.gaussian_grad(tuple(p.shape), 1e-3, seed + 100 * t + i,
+                             wl.zero_mask(tuple(p.shape), 0.05, seed + i))).cuda()
+
+
+def _same(a, b):
+    return np.array_equal(a.detach().cpu().numpy().view(np.uint8),
+                          b.detach().cpu().numpy().view(np.uint8))
+
+
+def test_adamw_wrapper_matches_fused_plan(mods):
+    """Three parameters, three steps, a scheduler halving lr after step 1:
+    the wrapper's parameters and codes equal al_adamw_step_multi's."""
+    import torch
+    B, optim = mods
+    shapes = [(64, 300), (2048,), (37, 111)]
+    pw, pd = _params(shapes, 10), _params(shapes, 10)
+    opt = optim.AdamW(pw, lr=1e-3, weight_decay=0.01)
+    sched = torch.optim.lr_scheduler.StepLR(opt, step_size=1, gamma=0.5)
+    st = [dict(m_codes=torch.zeros(p.numel(), dtype=torch.int8, device="cuda"),
+               m_absmax=torch.zeros((p.numel() + 255) // 256, dtype=torch.float32, device="cuda"),
+               v_codes=torch.zeros(p.numel(), dtype=torch.uint8, device="cuda"),
+               v_meta=torch.zeros(2 * ((p.numel() + 255) // 256), dtype=torch.float32,
+                                  device="cuda")) for p in pd]
+    lr = 1e-3
+    for t in (1, 2, 3):
+        _grads(pw, t, 500)
+        _grads(pd, t, 500)
+        opt.step()
+        sched.step()
+        plan = B.AdamWPlan([dict(p=p.data, g=p.grad, **s) for p, s in zip(pd, st)], 256, 256, 8)
+        plan.step(dict(ADAMW_HP, lr=lr), t)
+        lr *= 0.5
+        torch.cuda.synchronize()
+        for a, b, s in zip(pw, pd, st):
+            assert _same(a, b)
+            assert _same(opt.state[a]["v_codes"], s["v_codes"])
+            assert _same(opt.state[a]["m_codes"], s["m_codes"])
+
+
+def test_adamw_state_dict_round_trip_and_closure(mods):
+    import torch
+    _, optim = mods
+    shapes = [(128, 256), (512,)]
+    pa, pb = _params(shapes, 20), _params(shapes, 20)
+    oa = optim.AdamW(pa, v_bits=16, v_block=128)
+    for t in (1, 2):
+        _grads(pa, t, 900)
+        oa.step()
+    import io
+    buf = io.BytesIO()
+    torch.save(oa.state_dict(), buf)  # a checkpoint: state_dict() holds live references
+    buf.seek(0)
+    sd = torch.load(buf, weights_only=False)
+    for p, q in zip(pa, pb):
+        q.data.copy_(p.data)
+    ob = optim.AdamW(pb, v_bits=16, v_block=128)
+    ob.load_state_dict(sd)
+    for p in pb:
+        assert ob.state[p]["v_codes"].dtype == torch.int16
+        assert ob.state[p]["m_codes"].dtype == torch.int8
+    _grads(pa, 3, 900)
+    _grads(pb, 3, 900)
+    calls = []
+    oa.step(lambda: calls.append(1) or torch.tensor(0.0))
+    ob.step()
+    torch.cuda.synchronize()
+    assert calls == [1]
+    for p, q in zip(pa, pb):
+        assert _same(p, q)
+
+
+def test_migrate_al8_to_al16_keeps_decoded_state(mods):
+    """Sec. 6.2 per-role precision: re-coding a trained V from AL8 to AL16
+    keeps every decoded value within AL16's half log-step of the AL8 value."""
+    import torch
+    B, optim = mods
+    p = _params([(256, 512)], 30)
+    opt = optim.AdamW(p)
+    for t in (1, 2, 3):
+        _grads(p, t, 700)
+        opt.step()
+    st = opt.state[p[0]]
+    before = torch.empty(p[0].numel(), dtype=torch.float32, device="cuda")
+    B.al_decode(st["v_codes"], st["v_meta"], 256, 8, before)
+    opt.migrate_bits("v_bits", 16)
+    assert opt.param_groups[0]["v_bits"] == 16 and st["v_codes"].dtype == torch.int16
+    after = torch.empty_like(before)
+    B.al_decode(st["v_codes"], st["v_meta"], 256, 16, after)
+    b, a = before.cpu().numpy().astype(np.float64), after.cpu().numpy().astype(np.float64)
+    assert np.array_equal(b == 0, a == 0)
+    meta = st["v_meta"].cpu().numpy().reshape(-1, 2)
+    step = np.repeat(meta[:, 1], 256)[: b.size] / 65534.0  # log2 step of AL16 per block
+    nz = b > 0
+    assert np.all(np.abs(np.log2(a[nz]) - np.log2(b[nz])) <= 0.5 * step[nz] * (1 + 1e-6) + 1e-7)
+    _grads(p, 4, 700)
+    opt.step()  # keeps stepping with AL16 states
+
+
+def test_adafactor_and_came_wrappers_match_direct_calls(mods):
+    import torch
+    B, optim = mods
+    shapes = [(256, 384), (384,)]
+    for kind in ("adafactor", "came"):
+        pw, pd = _params(shapes, 40), _params(shapes, 40)
+        opt = optim.Adafactor(pw) if kind == "adafactor" else optim.CAME(pw)
+        for t in (1, 2):
+            _grads(pw, t, 300)
+            _grads(pd, t, 300)
+            opt.step()
+            for i, p in enumerate(pd):
+                rows, cols = (p.shape[0], p.shape[1]) if p.dim() == 2 else (1, p.numel())
+                st = opt.state[pw[i]]
+                if t == 1:
+                    ref = {k: torch.zeros_like(v) for k, v in st.items() if torch.is_tensor(v)}
+                    pd[i]._ref = ref
+                ref = pd[i]._ref
+                if kind == "adafactor":
+                    ws = torch.empty(B.al_workspace_size(B.AL_OP_ADAFACTOR, rows, cols),
+                                     dtype=torch.uint8, device="cuda")
+                    hp = {k: opt.param_groups[0][k] for k in ("lr", "eps1", "clip_d", "decay_rate",
+                                                              "beta1", "weight_decay", "log_floor")}
+                    B.al_adafactor_step(p.data, p.grad, rows, cols, ref["r_codes"], ref["r_meta"],
+                                        ref["c_codes"], ref["c_meta"], 16, 128, ref["m_codes"],
+                                        ref["m_absmax"], 256, hp, t, ws)
+                else:
+                    ws = torch.empty(B.al_workspace_size(B.AL_OP_CAME, rows, cols),
+                                     dtype=torch.uint8, device="cuda")
+                    g = opt.param_groups[0]
+                    hp = dict(lr=g["lr"], beta1=g["betas"][0], beta2=g["betas"][1],
+                              beta3=g["betas"][2], eps1=g["eps"][0], eps2=g["eps"][1],
+                              clip_d=g["clip_d"], weight_decay=g["weight_decay"],
+                              log_floor_v=g["log_floor_v"], log_floor_c=g["log_floor_c"])
+                    B.al_came_step(p.data, p.grad, rows, cols, ref["vr_codes"], ref["vr_meta"],
+                                   ref["vc_codes"], ref["vc_meta"], 16, 128, ref["cr_codes"],
+                                   ref["cr_meta"], ref["cc_codes"], ref["cc_meta"], 16, 128,
+                                   ref["m_codes"], ref["m_absmax"], 256, hp, t, ws)
+            torch.cuda.synchronize()
+            for a, b in zip(pw, pd):
+                assert _same(a, b), (kind, t)
+
+
+def test_apollo_wrapper_grouped_step_and_routing(mods):
+    """Matrices go through the grouped APOLLO step with the wrapper's own
+    projections (checked against a direct plan fed the same projections);
+    a vector parameter is routed to the quantized AdamW step."""
+    import torch
+    B, optim = mods
+    shapes = [(256, 512), (512, 256), (256,)]
+    pw, pd = _params(shapes, 60), _params(shapes, 60)
+    opt = optim.Apollo(pw, lr=1e-4, rank=128, proj_gap=2)
+    vec_before = pw[2].detach().clone()
+    ref = None
+    for t in (1, 2, 3):
+        _grads(pw, t, 800)
+        _grads(pd, t, 800)
+        opt.step()
+        if ref is None:
+            ref = [{k: torch.zeros_like(v) for k, v in opt.state[p].items()
+                    if torch.is_tensor(v) and k != "proj"} for p in pw[:2]]
+        mats = [dict(p=pd[i].data, g=pd[i].grad, rows=pd[i].shape[0], cols=pd[i].shape[1],
+                     proj=opt.state[pw[i]]["proj"], **ref[i]) for i in range(2)]
+        hp = dict(lr=1e-4, beta1=0.9, beta2=0.999, eps=1e-8, alpha=1.0, weight_decay=0.0,
+                  norm_growth_gamma=0.0, log_floor=opt.param_groups[0]["log_floor"], rank=128)
+        B.ApolloPlan(mats, 128, 8).step(hp, t)
+        torch.cuda.synchronize()
+        for i in range(2):
+            assert _same(pw[i], pd[i]), (i, t)
+    assert not _same(pw[2], vec_before)  # the vector was stepped (by AdamW)
+    assert "proj" not in opt.state[pw[2]]
+    sd = opt.state_dict()
+    assert "adamw" in sd
+
+
+def test_wrappers_reject_cpu_parameters(mods):
+    import torch
+    _, optim = mods
+    p = torch.nn.Parameter(torch.zeros(16))
+    p.grad = torch.zeros(16)
+    with pytest.raises(ValueError):
+        optim.AdamW([p]).step()
