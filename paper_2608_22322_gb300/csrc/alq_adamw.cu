@@ -113,13 +113,14 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
     constexpr float Lm2 = VBITS == 8 ? 254.0f : 65534.0f;
     __shared__ float2 s_tab[kThreads / 32][NBV * 32];
     __shared__ float s_val[kThreads / 32][VBITS == 8 ? NBV * 256 : 1];
-    __shared__ uint32_t s_part[3][kThreads / 32];
+    __shared__ uint32_t s_part[2][3][kThreads / 32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int wpbv = v_block > kASeg ? v_block / kASeg : 1;
     const int wpbm = m_block > kASeg ? m_block / kASeg : 1;
     const float kf = al8_table_k(lane);
     const int G = gridDim.x;
     int cur = 0;
+    int parity = 0;  // slot of the next cross-warp block reduction
     for (int64_t tile = blockIdx.x; tile < total_tiles; tile += G) {
         const PlanEntry d = plan_entry(table, ntensors, single, tile, cur);
         const int64_t n = d.n;
@@ -244,11 +245,36 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
         warp_blocks_reduce<CPBV, false>(cvmin, bvmin);
         warp_blocks_reduce<CPBV, true>(cvmax, bvmax);
         warp_blocks_reduce<CPBM, true>(cmabs, bmabs);
-        if (wpbv > 1) {
-            bvmin[0] = cta_group_reduce<false>(bvmin[0], s_part[0], wpbv);
-            bvmax[0] = cta_group_reduce<true>(bvmax[0], s_part[1], wpbv);
+        if (wpbv > 1 || wpbm > 1) {
+            // blocks wider than a segment (then one block per warp): one
+            // shared round for all three statistics, one barrier; the slots
+            // alternate between iterations, so a warp one iteration ahead
+            // never overwrites values another warp has yet to read
+            uint32_t(*sp)[kThreads / 32] = s_part[parity];
+            parity ^= 1;
+            if (lane == 0) {
+                sp[0][warp] = bvmin[0];
+                sp[1][warp] = bvmax[0];
+                sp[2][warp] = bmabs[0];
+            }
+            __syncthreads();
+            if (wpbv > 1) {
+                const int g0 = (warp / wpbv) * wpbv;
+                uint32_t a = sp[0][g0], b = sp[1][g0];
+                for (int k = 1; k < wpbv; ++k) {
+                    a = umix<false>(a, sp[0][g0 + k]);
+                    b = umix<true>(b, sp[1][g0 + k]);
+                }
+                bvmin[0] = a;
+                bvmax[0] = b;
+            }
+            if (wpbm > 1) {
+                const int g0 = (warp / wpbm) * wpbm;
+                uint32_t a = sp[2][g0];
+                for (int k = 1; k < wpbm; ++k) a = umix<true>(a, sp[2][g0 + k]);
+                bmabs[0] = a;
+            }
         }
-        if (wpbm > 1) bmabs[0] = cta_group_reduce<true>(bmabs[0], s_part[2], wpbm);
 
         float vmn[NBV], vmx[NBV], nlmin[NBV], ndelta[NBV], K[NBV], E[NBV];
 #pragma unroll
