@@ -56,18 +56,20 @@ al_encode_kernel(const float* __restrict__ x, int64_t n, int block, float log_fl
         al_blocks_params<NB>(mn, mx, log_floor, lmin, delta);
 #pragma unroll
         for (int b = 0; b < NB; ++b) al_encode_consts(delta[b], Lm2, K[b], E[b]);
+        float xv[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) xv[e] = f4get(v[e / 4], e % 4);
+        uint32_t q[16];
+        al_encode_chunks<BITS, CPB, NB, 4>(xv, lmin, delta, K, E, q);
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
-            const int b = c / CPB;
-            uint32_t q[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-                q[i] = al_encode_elem<BITS>(f4get(v[c], i), lmin[b], delta[b], K[b], E[b]);
             const int64_t idx = chunk_index(seg0, c, lane);
             if (BITS == 8)
-                store4b((uint8_t*)codes, idx, n, q[0] | (q[1] << 8) | (q[2] << 16) | (q[3] << 24));
+                store4b((uint8_t*)codes, idx, n,
+                        q[4 * c] | (q[4 * c + 1] << 8) | (q[4 * c + 2] << 16) | (q[4 * c + 3] << 24));
             else
-                store4h((uint16_t*)codes, idx, n, make_uint2(q[0] | (q[1] << 16), q[2] | (q[3] << 16)));
+                store4h((uint16_t*)codes, idx, n,
+                        make_uint2(q[4 * c] | (q[4 * c + 1] << 16), q[4 * c + 2] | (q[4 * c + 3] << 16)));
         }
         if (lane == 0 && (warp % wpb) == 0) {
             const int64_t gb0 = seg0 >> bshift;
@@ -86,6 +88,7 @@ al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta,
                  int block, float* __restrict__ out, int64_t ntiles) {
     constexpr int NB = 4 / CPB;
     __shared__ float2 s_tab[kThreads / 32][NB * 32];
+    __shared__ float s_val[kThreads / 32][BITS == 8 ? NB * 256 : 1];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const float kf = al8_table_k(lane);
     const int64_t nblk = blocks_of_dev(n, block);
@@ -113,17 +116,20 @@ al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta,
             lmin[b] = mt.x;
             delta[b] = mt.y;
         }
-        if (BITS == 8) al8_build_tables<NB>(s_tab[warp], lmin, delta, kf);
+        // AL8: the blocks' 256 exactly rounded values in shared memory, then
+        // one lookup per element; AL16: each level directly
+        if constexpr (BITS == 8) al8_build_values<NB>(s_val[warp], s_tab[warp], lmin, delta, kf);
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
             const int b = c / CPB;
-            const bool fast = al8_fast_ok(lmin[b], delta[b]);
             float r[4];
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const uint32_t q = code_of<BITS>(w, c, i);
-                r[i] = BITS == 8 ? al8_decode(q, s_tab[warp] + 32 * b, fast, lmin[b], delta[b])
-                                 : al16_decode(q, lmin[b], delta[b]);
+                if constexpr (BITS == 8)
+                    r[i] = s_val[warp][256 * b + q];
+                else
+                    r[i] = al16_decode(q, lmin[b], delta[b]);
             }
             store4f(out, chunk_index(seg0, c, lane), n, make_float4(r[0], r[1], r[2], r[3]));
         }
