@@ -101,13 +101,16 @@ def test_adafactor_matches_oracle(B, rows, cols, bits, fblock, mom, steps):
     print(f"adafactor {rows}x{cols}: code flips over {steps} steps = {flips}")
 
 
-@pytest.mark.parametrize("rows,cols,steps", [(256, 1408, 10), (130, 516, 5), (2048, 5632, 3)])
-def test_came_matches_oracle(B, rows, cols, steps):
+@pytest.mark.parametrize("rows,cols,steps,bits,fblock", [
+    (256, 1408, 10, 16, 128), (130, 516, 5, 16, 128), (2048, 5632, 3, 16, 128),
+    (512, 4096, 6, 8, 2048),  # the paper's all-AL8 CAME variant (Sec. 6.2 table, B = 2048)
+])
+def test_came_matches_oracle(B, rows, cols, steps, bits, fblock):
     import torch
     n = rows * cols
     p = wl.param_init((rows, cols), 8).ravel()
-    st = [_state(rows, 16, 128), _state(cols, 16, 128), _state(rows, 16, 128),
-          _state(cols, 16, 128)]
+    st = [_state(rows, bits, fblock), _state(cols, bits, fblock), _state(rows, bits, fblock),
+          _state(cols, bits, fblock)]
     mc = np.zeros(n, np.int8)
     ma = np.zeros((n + 255) // 256, np.float32)
     dp = _t(p)
@@ -118,15 +121,15 @@ def test_came_matches_oracle(B, rows, cols, steps):
     flips = 0
     for t in range(1, steps + 1):
         g = wl.student_t_grad((rows, cols), 1e-3, 3.0, 0.05, 8000 + t).ravel()
-        ora.came_step(p, g, rows, cols, st[0][0], st[0][1], st[1][0], st[1][1], 16, 128,
-                      st[2][0], st[2][1], st[3][0], st[3][1], 16, 128, mc, ma, 256, CAME_HP, t)
-        B.al_came_step(dp, _t(g), rows, cols, dst[0][0], dst[0][1], dst[1][0], dst[1][1], 16,
-                       128, dst[2][0], dst[2][1], dst[3][0], dst[3][1], 16, 128, dmc, dma, 256,
-                       CAME_HP, t, ws)
+        ora.came_step(p, g, rows, cols, st[0][0], st[0][1], st[1][0], st[1][1], bits, fblock,
+                      st[2][0], st[2][1], st[3][0], st[3][1], bits, fblock, mc, ma, 256, CAME_HP, t)
+        B.al_came_step(dp, _t(g), rows, cols, dst[0][0], dst[0][1], dst[1][0], dst[1][1], bits,
+                       fblock, dst[2][0], dst[2][1], dst[3][0], dst[3][1], bits, fblock, dmc, dma,
+                       256, CAME_HP, t, ws)
         torch.cuda.synchronize()
         _cmp_p(p, dp, f"step {t}")
         for (c, _), (dc, _) in zip(st, dst):
-            flips += _cmp_codes("factor codes", c, dc, 16)
+            flips += _cmp_codes("factor codes", c, dc, bits)
         flips += _cmp_codes("M codes", mc, dmc, 8)
     print(f"came {rows}x{cols}: code flips over {steps} steps = {flips}")
 
