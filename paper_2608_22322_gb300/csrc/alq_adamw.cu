@@ -111,7 +111,7 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
     constexpr int NBM = kCH / CPBM;
     constexpr int NE = 4 * kCH;
     constexpr float Lm2 = VBITS == 8 ? 254.0f : 65534.0f;
-    __shared__ float2 s_tab[kThreads / 32][NBV * 32];
+    __shared__ __align__(16) float2 s_tab[kThreads / 32][NBV * 32];
     __shared__ float s_val[kThreads / 32][VBITS == 8 ? NBV * 256 : 1];
     __shared__ uint32_t s_part[2][3][kThreads / 32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;

@@ -485,7 +485,7 @@ template <int CPB, int VBITS>
 __global__ void __launch_bounds__(kThreads, 3)
 apollo_moments_kernel(MomentArgs m, int64_t ntiles) {
     constexpr int NB = kMCH / CPB;
-    __shared__ float2 s_tab[kThreads / 32][NB * 32];
+    __shared__ __align__(16) float2 s_tab[kThreads / 32][NB * 32];
     __shared__ float s_val[kThreads / 32][VBITS == 8 ? NB * 256 : 1];
     const int warp = threadIdx.x >> 5;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x)
@@ -680,7 +680,7 @@ __global__ void __launch_bounds__(kThreads, 3)
 apollo_moments_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t ntiles,
                             MomentArgs base) {
     constexpr int NB = kMCH / CPB;
-    __shared__ float2 s_tab[kThreads / 32][NB * 32];
+    __shared__ __align__(16) float2 s_tab[kThreads / 32][NB * 32];
     __shared__ float s_val[kThreads / 32][VBITS == 8 ? NB * 256 : 1];
     const int warp = threadIdx.x >> 5;
     int cur = 0;

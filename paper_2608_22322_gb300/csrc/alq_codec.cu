@@ -87,7 +87,7 @@ __global__ void __launch_bounds__(kThreads)
 al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta, int64_t n,
                  int block, float* __restrict__ out, int64_t ntiles) {
     constexpr int NB = 4 / CPB;
-    __shared__ float2 s_tab[kThreads / 32][NB * 32];
+    __shared__ __align__(16) float2 s_tab[kThreads / 32][NB * 32];
     __shared__ float s_val[kThreads / 32][BITS == 8 ? NB * 256 : 1];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const float kf = al8_table_k(lane);

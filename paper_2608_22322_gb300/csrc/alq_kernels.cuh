@@ -40,6 +40,15 @@ __device__ __forceinline__ float2 add2(float2 a, float2 b) {
     return r;
 }
 
+__device__ __forceinline__ float2 sub2(float2 a, float2 b) {
+    float2 r;
+    asm("{\n.reg .b64 a, b, d;\nmov.b64 a, {%2, %3};\nmov.b64 b, {%4, %5};\n"
+        "sub.rn.f32x2 d, a, b;\nmov.b64 {%0, %1}, d;\n}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return r;
+}
+
 __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
     float2 r;
     asm("{\n.reg .b64 a, b, c, d;\nmov.b64 a, {%2, %3};\nmov.b64 b, {%4, %5};\n"
@@ -190,14 +199,21 @@ __device__ __forceinline__ void al_blocks_params(const float (&mn)[NB], const fl
 
 // ------------------------------------------------------ AL8 decode tables --
 // The two 16-entry level tables of each of the NB blocks of a segment
-// (Eq. (5)): entry b < 16 holds 2^((b-1) d), entry 16 + a holds
-// 2^(l_min + 16 a d), d = Delta / 254, as two-float pairs; code q decodes to
-// entry[16 + (q >> 4)] * entry[q & 15]. One entry per lane per block.
-// Blocks whose l_min is below -96 (or that are empty) take the FP64 path.
+// (Eq. (5)): entry b < 16 holds T_lo[b] = 2^((b-1) d), entries 16..31 hold
+// T_hi[a] = 2^(l_min + 16 a d), d = Delta / 254, as two-float pairs; code
+// q = 16 a + b decodes to T_hi[a] * T_lo[b]. T_hi is stored even a first
+// (slots 16..23), then odd a (24..31): lane l decodes the codes l + 32 k,
+// whose factors T_hi[2 k + (l >> 4)] are then contiguous. One entry per lane
+// per block. Blocks whose l_min is below -96 (or that are empty) take the
+// FP64 path.
 // Level index of this lane's table entry: k = b - 1 for lanes b < 16,
 // k = 16 (lane - 16) for the others (as a float).
 __device__ __forceinline__ float al8_table_k(int lane) {
     return int_to_float_small(lane >= 16 ? 16 * (lane - 16) : lane - 1);
+}
+
+__device__ __forceinline__ int al8_hi_slot(uint32_t a) {
+    return 16 + (int)((a & 1u) << 3) + (int)(a >> 1);
 }
 
 template <int NB>
@@ -205,12 +221,13 @@ __device__ __forceinline__ void al8_build_tables(float2* tab, const float (&lmin
                                                  const float (&delta)[NB], float kf) {
     const int lane = threadIdx.x & 31;
     const bool hi = lane >= 16;
+    const int slot = hi ? al8_hi_slot((uint32_t)(lane - 16)) : lane;
 #pragma unroll
     for (int b = 0; b < NB; ++b) {
         float rh = 0.0f, rl = 0.0f;
         if (delta[b] > 0.0f && lmin[b] >= -96.0f)
             al_level_ff(hi ? lmin[b] : 0.0f, delta[b], kf, 254.0f, 1.0f / 254.0f, rh, rl);
-        tab[32 * b + lane] = make_float2(rh, rl);
+        tab[32 * b + slot] = make_float2(rh, rl);
     }
     __syncwarp();
 }
@@ -219,49 +236,19 @@ __device__ __forceinline__ bool al8_fast_ok(float lmin, float delta) {
     return delta > 0.0f && lmin >= -96.0f;
 }
 
-// AL8 decode of the 16 codes of a lane's four chunks through their blocks'
-// tables, branch-free: the fast results are selected per element and the
-// rare elements whose two-float product lies too close to an fp32 rounding
-// boundary (or whose block is outside the fast range) are marked in a bit
-// mask and recomputed in FP64 under one warp-uniform, rarely taken branch.
-template <int CPB, int NB, int CH>
-__device__ __forceinline__ void al8_decode_chunks(const uint32_t (&w)[CH], const float2* tab,
-                                                  const float (&lmin)[NB], const float (&delta)[NB],
-                                                  float (&out)[4 * CH]) {
-    bool any_fb = false;
-#pragma unroll
-    for (int c = 0; c < CH; ++c) {
-        const int b = c / CPB;
-        const bool fast = al8_fast_ok(lmin[b], delta[b]);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const uint32_t q = (w[c] >> (8 * i)) & 0xFFu;
-            const float2 A = tab[32 * b + 16 + (q >> 4)];
-            const float2 Bt = tab[32 * b + (q & 15u)];
-            bool fb;
-            const float r = al8_decode_pair(A.x, A.y, Bt.x, Bt.y, fb);
-            out[4 * c + i] = q == 0u ? 0.0f : r;
-            any_fb |= (q != 0u) & (fb | !fast);
-        }
-    }
-    if (__builtin_expect(__any_sync(0xFFFFFFFFu, any_fb), 0)) {
-        // rare: redo the boundary test per element and recompute in FP64
-#pragma unroll
-        for (int c = 0; c < CH; ++c) {
-            const int b = c / CPB;
-            const bool fast = al8_fast_ok(lmin[b], delta[b]);
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const uint32_t q = (w[c] >> (8 * i)) & 0xFFu;
-                const float2 A = tab[32 * b + 16 + (q >> 4)];
-                const float2 Bt = tab[32 * b + (q & 15u)];
-                bool fb;
-                al8_decode_pair(A.x, A.y, Bt.x, Bt.y, fb);
-                if ((q != 0u) && (fb || !fast))
-                    out[4 * c + i] = al_dequantize_fp64(q, lmin[b], delta[b], 254.0);
-            }
-        }
-    }
+// al8_decode_pair (alq_numerics.h) on two values with the same low factor
+// (bh, bl), step for step in paired instructions (each component rounds as
+// the scalar operation does).
+__device__ __forceinline__ float2 al8_decode_pair2(float2 ah, float2 al, float2 bh, float2 bl,
+                                                   float2 nbh, bool& fb0, bool& fb1) {
+    const float2 c = fma2(ah, bl, mul2(al, bh));
+    const float2 r = fma2(ah, bh, c);
+    const float2 t = fma2(ah, nbh, r);
+    const float2 res = sub2(c, t);
+    const float2 z = fma2(res, make_float2(1.0f + 0x1p-15f, 1.0f + 0x1p-15f), r);
+    fb0 = z.x != r.x;
+    fb1 = z.y != r.y;
+    return r;
 }
 
 // Fixed-size arrays passed by value to the out-of-line rare paths (so that
@@ -336,7 +323,7 @@ static __device__ __noinline__ void al8_values_fixup(float* vals, const float2* 
     const bool fast = al8_fast_ok(lmin, delta);
     for (int k = 0; k < 8; ++k) {
         const uint32_t q = (uint32_t)(lane + 32 * k);
-        const float2 A = tab[16 + (q >> 4)];
+        const float2 A = tab[al8_hi_slot(q >> 4)];
         const float2 Bt = tab[q & 15u];
         bool fb;
         al8_decode_pair(A.x, A.y, Bt.x, Bt.y, fb);
@@ -347,10 +334,12 @@ static __device__ __noinline__ void al8_values_fixup(float* vals, const float2* 
 // The 256 decoded values of each of the NB blocks of a segment (Eq. (5), code
 // 0 -> 0), exactly as the double expression rounds them, in shared memory:
 // lane l computes codes l, l + 32, ..., l + 224 from the block's two-float
-// level tables (T_hi[q >> 4] * T_lo[q & 15]); entries whose two-float product
-// lies too close to an fp32 rounding boundary, and blocks outside the fast
-// range, are recomputed in FP64 under one warp-uniform branch. An element
-// decode is then a single shared-memory load.
+// level tables (T_hi[q >> 4] * T_lo[q & 15], two codes per paired step:
+// T_lo[l & 15] is the same for all eight, the T_hi factors are read four at
+// a time); entries whose two-float product lies too close to an fp32
+// rounding boundary, and blocks outside the fast range, are recomputed in
+// FP64 under one warp-uniform branch. An element decode is then a single
+// shared-memory load. tab must be 16-byte aligned.
 template <int NB>
 __device__ __forceinline__ void al8_build_values(float* vals, float2* tab,
                                                  const float (&lmin)[NB],
@@ -361,15 +350,22 @@ __device__ __forceinline__ void al8_build_values(float* vals, float2* tab,
 #pragma unroll
     for (int b = 0; b < NB; ++b) {
         const bool fast = al8_fast_ok(lmin[b], delta[b]);
+        const float2 Bt = tab[32 * b + (lane & 15)];
+        const float2 bh = make_float2(Bt.x, Bt.x), bl = make_float2(Bt.y, Bt.y);
+        const float2 nbh = make_float2(-Bt.x, -Bt.x);
+        const float4* A4 = reinterpret_cast<const float4*>(tab + 32 * b + 16 + 8 * (lane >> 4));
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const uint32_t q = (uint32_t)(lane + 32 * k);
-            const float2 A = tab[32 * b + 16 + (q >> 4)];
-            const float2 Bt = tab[32 * b + (q & 15u)];
-            bool fb;
-            const float r = al8_decode_pair(A.x, A.y, Bt.x, Bt.y, fb);
-            vals[256 * b + q] = q == 0u ? 0.0f : r;
-            any_fb |= (q != 0u) & (fb | !fast);
+        for (int j = 0; j < 4; ++j) {
+            // codes q0 = l + 64 j and q0 + 32: factors T_hi[4 j + (l >> 4)]
+            // and T_hi[4 j + 2 + (l >> 4)]
+            const float4 a = A4[j];
+            bool f0, f1;
+            const float2 r = al8_decode_pair2(make_float2(a.x, a.z), make_float2(a.y, a.w), bh,
+                                              bl, nbh, f0, f1);
+            const uint32_t q0 = (uint32_t)(lane + 64 * j);
+            vals[256 * b + q0] = q0 == 0u ? 0.0f : r.x;
+            vals[256 * b + q0 + 32] = r.y;
+            any_fb |= ((q0 != 0u) & f0) | f1 | !fast;
         }
     }
     if (__builtin_expect(__any_sync(0xFFFFFFFFu, any_fb), 0)) {
@@ -377,21 +373,6 @@ __device__ __forceinline__ void al8_build_values(float* vals, float2* tab,
         for (int b = 0; b < NB; ++b) al8_values_fixup(vals + 256 * b, tab + 32 * b, lmin[b], delta[b]);
     }
     __syncwarp();
-}
-
-// AL8 element decode through a block's tables; FP64 when the two-float
-// product may round differently, or the block is outside the fast range.
-__device__ __forceinline__ float al8_decode(uint32_t q, const float2* tab, bool fast,
-                                            float lmin, float delta) {
-    if (q == 0u) return 0.0f;
-    if (fast) {
-        const float2 a = tab[16 + (q >> 4)];
-        const float2 b = tab[q & 15u];
-        bool fb;
-        const float r = al8_decode_pair(a.x, a.y, b.x, b.y, fb);
-        if (!fb) return r;
-    }
-    return al_dequantize_fp64(q, lmin, delta, 254.0);
 }
 
 // Element decode with the level computed directly in two-float form (any
