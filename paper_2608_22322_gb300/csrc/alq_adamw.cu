@@ -296,7 +296,7 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
 
         // ---- encode and write the codes and block constants
         uint32_t qv[NE];
-        al_encode_chunks<VBITS, CPBV, NBV, kCH>(vf, nlmin, ndelta, K, E, qv);
+        al_encode_chunks<VBITS, CPBV, NBV, kCH>(vf, vmn, nlmin, ndelta, K, E, qv);
 #pragma unroll
         for (int c = 0; c < kCH; ++c) {
             const int bm = c / CPBM;

@@ -450,7 +450,7 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
 #pragma unroll
     for (int b = 0; b < NB; ++b) al_encode_consts(ndelta[b], Lm2, K[b], E[b]);
     uint32_t qv[NE];
-    al_encode_chunks<VBITS, CPB, NB, kMCH>(vf, nlmin, ndelta, K, E, qv);
+    al_encode_chunks<VBITS, CPB, NB, kMCH>(vf, vmn, nlmin, ndelta, K, E, qv);
 #pragma unroll
     for (int c = 0; c < kMCH; ++c) {
         const int b = c / CPB;

@@ -60,7 +60,7 @@ al_encode_kernel(const float* __restrict__ x, int64_t n, int block, float log_fl
 #pragma unroll
         for (int e = 0; e < 16; ++e) xv[e] = f4get(v[e / 4], e % 4);
         uint32_t q[16];
-        al_encode_chunks<BITS, CPB, NB, 4>(xv, lmin, delta, K, E, q);
+        al_encode_chunks<BITS, CPB, NB, 4>(xv, mn, lmin, delta, K, E, q);
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
             const int64_t idx = chunk_index(seg0, c, lane);

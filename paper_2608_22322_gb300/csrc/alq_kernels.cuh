@@ -258,8 +258,9 @@ struct Arr {
     T v[N];
 };
 
-// Rare path of al_encode_chunks, out of line: redo the boundary tests and
-// recompute the flagged codes in FP64.
+// Rare path of al_encode_chunks, out of line: zero codes for zeros, redo the
+// boundary tests (with the subnormal test) and recompute the flagged codes
+// in FP64.
 template <int BITS, int CPB, int NB, int CH>
 static __device__ __noinline__ Arr<uint32_t, 4 * CH> al_encode_fixup(
     Arr<float, 4 * CH> x, Arr<float, NB> lmin, Arr<float, NB> delta, Arr<float, NB> K,
@@ -270,27 +271,50 @@ static __device__ __noinline__ Arr<uint32_t, 4 * CH> al_encode_fixup(
         const int b = e / 4 / CPB;
         bool fb;
         al_quantize_fast(x.v[e], lmin.v[b], K.v[b], E.v[b], Lm2, fb);
-        if (x.v[e] != 0.0f && fb) q.v[e] = al_quantize_fp64(x.v[e], lmin.v[b], delta.v[b], (double)Lm2);
+        if (x.v[e] == 0.0f)
+            q.v[e] = 0u;
+        else if (fb)
+            q.v[e] = al_quantize_fp64(x.v[e], lmin.v[b], delta.v[b], (double)Lm2);
     }
     return q;
 }
 
-// Eq. (4) for the 4 CH values of a lane's chunks, branch-free with the same
-// bit-mask fixup in FP64 for values near a half-integer of t.
+// Eq. (4) for the 4 CH values of a lane's chunks: al_quantize_fast on pairs
+// of values in paired instructions, branch-free, with the same fixup in
+// FP64 for values near a half-integer of t. mn is each block's minimum
+// positive value (0 for a block without one); a block with a subnormal
+// minimum sends the whole segment through the fixup, so that the fast path
+// needs no per-value subnormal test. Zero (and -0) codes as 0: its biased
+// exponent 0 gives t <= -K < 0 (l_min >= -126 without subnormals), so
+// q = rint(clip(t)) + [x != 0] = 0.
 template <int BITS, int CPB, int NB, int CH>
-__device__ __forceinline__ void al_encode_chunks(const float (&x)[4 * CH], const float (&lmin)[NB],
+__device__ __forceinline__ void al_encode_chunks(const float (&x)[4 * CH], const float (&mn)[NB],
+                                                 const float (&lmin)[NB],
                                                  const float (&delta)[NB], const float (&K)[NB],
                                                  const float (&E)[NB], uint32_t (&q)[4 * CH]) {
     constexpr float Lm2 = BITS == 8 ? 254.0f : 65534.0f;
     bool any_fb = false;
 #pragma unroll
-    for (int e = 0; e < 4 * CH; ++e) {
+    for (int b = 0; b < NB; ++b) any_fb |= (mn[b] > 0.0f) & (mn[b] < 0x1p-126f);
+    const float2 e0 = make_float2(8388735.0f, 8388735.0f);  // 2^23 + 127
+    const float2 rc = make_float2(12582912.0f, 12582912.0f);  // 1.5 * 2^23
+#pragma unroll
+    for (int e = 0; e < 4 * CH; e += 2) {
         const int b = e / 4 / CPB;
-        bool fb;
-        const uint32_t v = al_quantize_fast(x[e], lmin[b], K[b], E[b], Lm2, fb);
-        const bool nz = x[e] != 0.0f;
-        q[e] = nz ? v : 0u;
-        any_fb |= nz & fb;
+        const uint32_t x0 = f2u(x[e]), x1 = f2u(x[e + 1]);
+        const float2 eb = make_float2(u2f(0x4B000000u | ((x0 >> 23) & 0xFFu)),
+                                      u2f(0x4B000000u | ((x1 >> 23) & 0xFFu)));
+        const float2 lg = make_float2(lg2_mant(u2f((x0 & 0x007FFFFFu) | 0x3F800000u)),
+                                      lg2_mant(u2f((x1 & 0x007FFFFFu) | 0x3F800000u)));
+        const float2 d = add2(sub2(sub2(eb, e0), make_float2(lmin[b], lmin[b])), lg);
+        const float2 t = mul2(d, make_float2(K[b], K[b]));
+        const float2 tc = make_float2(fminf(fmaxf(t.x, 0.0f), Lm2), fminf(fmaxf(t.y, 0.0f), Lm2));
+        const float2 rr = add2(tc, rc);
+        const float2 df = sub2(tc, sub2(rr, rc));
+        const float h = 0.5f - E[b];
+        any_fb |= (fabsf(df.x) > h) | (fabsf(df.y) > h);
+        q[e] = (f2u(rr.x) - 0x4B400000u) + min(x0 << 1, 1u);
+        q[e + 1] = (f2u(rr.y) - 0x4B400000u) + min(x1 << 1, 1u);
     }
     if (__builtin_expect(__any_sync(0xFFFFFFFFu, any_fb), 0)) {
         Arr<float, 4 * CH> xa;

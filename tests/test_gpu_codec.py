@@ -44,6 +44,49 @@ def test_al_encode_bit_exact(B, bits, block):
     assert int(np.sum(got != codes)) == 0
 
 
+def _subnormal_mix(n, block, seed):
+    """Blocks whose minimum positive value is subnormal (the encoder's
+    exact path for a whole segment), mixed with zeros, -0.0 and normal
+    values reaching up to 2^20, next to blocks of normal values only."""
+    r = wl.rng(seed)
+    x = np.exp2(r.uniform(-40, 20, n)).astype(np.float32)
+    nb = (n + block - 1) // block
+    for b in range(0, nb, 3):
+        lo, hi = b * block, min(n, (b + 1) * block)
+        k = hi - lo
+        sub = (r.integers(1, 1 << 23, k, dtype=np.uint32)).view(np.float32)
+        pick = r.random(k)
+        seg = x[lo:hi].copy()
+        seg[pick < 0.3] = sub[pick < 0.3]
+        seg[(pick >= 0.3) & (pick < 0.4)] = 0.0
+        seg[(pick >= 0.4) & (pick < 0.45)] = -0.0
+        if b % 2 == 0:
+            seg[:] = np.where(pick < 0.5, sub, seg)  # mostly tiny values
+        x[lo:hi] = seg
+    return x
+
+
+@pytest.mark.parametrize("bits", [8, 16])
+@pytest.mark.parametrize("block", [128, 256, 2048])
+@pytest.mark.parametrize("floor", [FLOOR, -160.0])
+def test_al_encode_subnormal_blocks(B, bits, block, floor):
+    """Subnormal minima put l_min below -126 with a low floor: zeros must
+    still code as 0 and every value must match Eq. (4) in double."""
+    import torch
+    n = 12 * block + 37
+    x = _subnormal_mix(n, block, seed=block + bits)
+    codes, meta = ora.al_encode(x, block, bits, floor)
+    tc = torch.zeros(n, dtype=torch.uint8 if bits == 8 else torch.int16, device="cuda")
+    tm = torch.zeros(2 * B.al_num_blocks(n, block), dtype=torch.float32, device="cuda")
+    B.al_encode(_dev(x), block, bits, floor, tc, tm)
+    torch.cuda.synchronize()
+    assert bytes_equal(meta, tm.cpu().numpy()) == 0
+    got = tc.cpu().numpy().view(ora.code_dtype(bits))
+    assert int(np.sum(got != codes)) == 0
+    assert np.all(got[x == 0] == 0)
+    assert float(meta[0::2].min()) < -126.0 or floor > -126.0
+
+
 @pytest.mark.parametrize("bits", [8, 16])
 @pytest.mark.parametrize("block", [128, 256, 2048])
 def test_al_decode_bit_exact(B, bits, block):
