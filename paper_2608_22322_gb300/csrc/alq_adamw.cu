@@ -74,6 +74,7 @@ static __device__ __noinline__ void store_codes_masked(int8_t* m_codes, void* v_
 // parameter space costs no registers.
 struct AdamWPairs {
     float2 decay, nstep, c2, omb1, omb2, beta1, beta2, eps;
+    float2 one;  // (1, 1), opaque to the compiler: f * one + c rounds as f + c
     float log_floor;
 };
 
@@ -87,6 +88,7 @@ static AdamWPairs adamw_pairs(const AdamWScalars& s) {
     q.beta1 = make_float2(s.beta1, s.beta1);
     q.beta2 = make_float2(s.beta2, s.beta2);
     q.eps = make_float2(s.eps, s.eps);
+    q.one = make_float2(1.0f, 1.0f);
     q.log_floor = s.log_floor;
     return q;
 }
@@ -192,7 +194,8 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
 
         // ---- update, write p; keep the fresh m and v (element pairs)
         float2 mf[NE / 2], vf2[NE / 2];
-        uint32_t cvmin[kCH], cvmax[kCH], cmabs[kCH];
+        uint32_t cvmin[kCH], cvmax[kCH];
+        float cmabs[kCH];  // |m| >= 0: float and unsigned order agree
 #pragma unroll
         for (int c = 0; c < kCH; ++c) {
             const int bm = c / CPBM;
@@ -203,7 +206,7 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
             float2 pn[2];
             cvmin[c] = 0xFFFFFFFFu;
             cvmax[c] = 0u;
-            cmabs[c] = 0u;
+            cmabs[c] = 0.0f;
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
                 const float2 qf = make_float2(u2f(__byte_perm(mx, 0x4B400000u, 0x7640u | (2 * h))),
@@ -225,7 +228,7 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
                 const uint32_t vbx = f2u(vv.x), vby = f2u(vv.y);
                 cvmin[c] = umix<false>(cvmin[c], umix<false>(vbx - 1u, vby - 1u));  // 0 -> max: min positive
                 cvmax[c] = umix<true>(cvmax[c], umix<true>(vbx, vby));
-                cmabs[c] = umix<true>(cmabs[c], umix<true>(f2u(mm.x) & 0x7FFFFFFFu, f2u(mm.y) & 0x7FFFFFFFu));
+                cmabs[c] = fmaxf(cmabs[c], fmaxf(fabsf(mm.x), fabsf(mm.y)));
             }
             const float4 pv = make_float4(pn[0].x, pn[0].y, pn[1].x, pn[1].y);
             if (full)
@@ -244,7 +247,10 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
         uint32_t bvmin[NBV], bvmax[NBV], bmabs[NBM];
         warp_blocks_reduce<CPBV, false>(cvmin, bvmin);
         warp_blocks_reduce<CPBV, true>(cvmax, bvmax);
-        warp_blocks_reduce<CPBM, true>(cmabs, bmabs);
+        uint32_t cmabs_u[kCH];
+#pragma unroll
+        for (int c = 0; c < kCH; ++c) cmabs_u[c] = f2u(cmabs[c]);
+        warp_blocks_reduce<CPBM, true>(cmabs_u, bmabs);
         if (wpbv > 1 || wpbm > 1) {
             // blocks wider than a segment (then one block per warp): one
             // shared round for all three statistics, one barrier; the slots
@@ -301,15 +307,18 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
         for (int c = 0; c < kCH; ++c) {
             const int bm = c / CPBM;
             const int64_t idx = e0 + 128 * c;
-            // q = rint((m sc) inv) (scalar: the product must round before
-            // the rounding add) as the low byte of 1.5 * 2^23 + q, the two's
-            // complement byte for q < 0; all codes are 0 when the block's
-            // absmax is 0 (inv = 0)
+            // q = rint((m sc) inv) as the low byte of 1.5 * 2^23 + q, the
+            // two's complement byte for q < 0; all codes are 0 when the
+            // block's absmax is 0 (inv = 0). The rounding add is a fused
+            // multiply-add by the opaque one, so the product rounds first.
+            const float2 sc2 = make_float2(msc[bm], msc[bm]), inv2 = make_float2(minv[bm], minv[bm]);
             uint32_t rb[4];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const float2 m2 = mf[2 * c + i / 2];
-                rb[i] = f2u(((i & 1 ? m2.y : m2.x) * msc[bm]) * minv[bm] + 12582912.0f);
+            for (int i = 0; i < 2; ++i) {
+                const float2 f = mul2(mul2(mf[2 * c + i], sc2), inv2);
+                const float2 r = fma2(f, s.one, make_float2(12582912.0f, 12582912.0f));
+                rb[2 * i] = f2u(r.x);
+                rb[2 * i + 1] = f2u(r.y);
             }
             const uint32_t qm = __byte_perm(__byte_perm(rb[0], rb[1], 0x0040u),
                                             __byte_perm(rb[2], rb[3], 0x0040u), 0x5410u);

@@ -88,15 +88,17 @@ def test_adamw_redrawn_mask(B):
 
 
 @pytest.mark.parametrize("m_block,v_block", [(256, 2048), (128, 128), (512, 1024),
-                                             (2048, 256), (128, 2048)])
+                                             (2048, 256), (128, 2048), (128, 256),
+                                             (256, 128), (2048, 128), (512, 512)])
 def test_adamw_block_sizes(B, m_block, v_block):
     w = wl.AdamWSingle(shape=(37, 1111))  # 41107 elements: ragged tiles and blocks
     _run_single(B, w, m_block, v_block, 8, 4)
 
 
-def test_adamw_al16(B):
+@pytest.mark.parametrize("m_block,v_block", [(256, 256), (256, 128), (128, 1024)])
+def test_adamw_al16(B, m_block, v_block):
     w = wl.AdamWSingle(shape=(64, 777))
-    _run_single(B, w, 256, 256, 16, 4)
+    _run_single(B, w, m_block, v_block, 16, 4)
 
 
 def test_adamw_plan_many_tensors(B):
