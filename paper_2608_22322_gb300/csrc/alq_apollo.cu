@@ -340,12 +340,49 @@ constexpr int kMCH = 2;
 constexpr int kMSeg = 128 * kMCH;
 constexpr int kMTile = 8 * kMSeg;
 
+// Channel scales waiting for their FP64 evaluation: lane k of a warp holds
+// the two-float norm sums of the warp's k-th pending channel (FP64 runs at a
+// small fraction of the fp32 rate on this part, so the warp evaluates 32
+// channels in one pass instead of one per segment).
+struct PendingScales {
+    float nrh = 0.0f, nrl = 0.0f, ngh = 0.0f, ngl = 0.0f;
+    float* dst = nullptr;
+    int count = 0;
+
+    // s_j = ||Rt_j|| / (||R_j|| + 1e-8) from the sums in double, rounded once
+    __device__ __forceinline__ void flush() {
+        if (dst) {
+            const double nr = (double)nrh + (double)nrl;
+            const double ng = (double)ngh + (double)ngl;
+            *dst = (float)(sqrt(nr) / (sqrt(ng) + 1e-8));
+        }
+        dst = nullptr;
+        count = 0;
+    }
+    // a channel's sums as lane 0 holds them (the butterfly leaves the low
+    // parts of other lanes rounded in another order) go to lane count
+    __device__ __forceinline__ void add(float rh, float rl, float gh, float gl, float* d) {
+        rh = __shfl_sync(0xFFFFFFFFu, rh, 0);
+        rl = __shfl_sync(0xFFFFFFFFu, rl, 0);
+        gh = __shfl_sync(0xFFFFFFFFu, gh, 0);
+        gl = __shfl_sync(0xFFFFFFFFu, gl, 0);
+        if ((int)(threadIdx.x & 31) == count) {
+            nrh = rh;
+            nrl = rl;
+            ngh = gh;
+            ngl = gl;
+            dst = d;
+        }
+        if (++count == 32) flush();
+    }
+};
+
 // One tile of the moments pass. tab and vals are this warp's shared slots
 // for the AL8 decode tables (NB * 32 pairs) and the blocks' 256 decoded
-// values (NB * 256).
+// values (NB * 256); the channels' norm sums join ps.
 template <int CPB, int VBITS>
 __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, float2* tab,
-                                             float* vals) {
+                                             float* vals, PendingScales& ps) {
     constexpr int NB = kMCH / CPB;
     constexpr int NE = 4 * kMCH;
     constexpr float Lm2 = VBITS == 8 ? 254.0f : 65534.0f;
@@ -473,11 +510,11 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
             if (b0 + b >= nblk) continue;
             reinterpret_cast<float2*>(m.v_meta)[b0 + b] = make_float2(nlmin[b], ndelta[b]);
             m.m_absmax[b0 + b] = ms[b];
-            const double nr = (double)nrh[b] + (double)nrl[b];
-            const double ng = (double)ngh[b] + (double)ngl[b];
-            m.scale[b0 + b] = (float)(sqrt(nr) / (sqrt(ng) + 1e-8));
         }
     }
+#pragma unroll
+    for (int b = 0; b < NB; ++b)
+        if (b0 + b < nblk) ps.add(nrh[b], nrl[b], ngh[b], ngl[b], m.scale + b0 + b);
     __syncwarp();
 }
 
@@ -488,8 +525,10 @@ apollo_moments_kernel(MomentArgs m, int64_t ntiles) {
     __shared__ __align__(16) float2 s_tab[kThreads / 32][NB * 32];
     __shared__ float s_val[kThreads / 32][VBITS == 8 ? NB * 256 : 1];
     const int warp = threadIdx.x >> 5;
+    PendingScales ps;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x)
-        moments_tile<CPB, VBITS>(m, tile, s_tab[warp], s_val[warp]);
+        moments_tile<CPB, VBITS>(m, tile, s_tab[warp], s_val[warp], ps);
+    ps.flush();
 }
 
 // ------------------------------------------------------ limiter, update --
@@ -683,6 +722,7 @@ apollo_moments_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t n
     __shared__ __align__(16) float2 s_tab[kThreads / 32][NB * 32];
     __shared__ float s_val[kThreads / 32][VBITS == 8 ? NB * 256 : 1];
     const int warp = threadIdx.x >> 5;
+    PendingScales ps;
     int cur = 0;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         cur = entry_for(tab, nmat, tile, cur, &ApEntry::mom_t0);
@@ -695,8 +735,9 @@ apollo_moments_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t n
         m.v_codes = e.v_codes;
         m.v_meta = e.v_meta;
         m.scale = e.scale;
-        moments_tile<CPB, VBITS>(m, tile - e.mom_t0, s_tab[warp], s_val[warp]);
+        moments_tile<CPB, VBITS>(m, tile - e.mom_t0, s_tab[warp], s_val[warp], ps);
     }
+    ps.flush();
 }
 
 __global__ void __launch_bounds__(kThreads)
