@@ -368,10 +368,9 @@ int al_apollo_step(float* p, const float* g, int64_t rows, int64_t cols,
 
 /* ---------------------------------------------------- grouped APOLLO step -- */
 /*
- * One APOLLO step over many matrices in four launches (bf16 staging of every
- * G, one projection launch whose grid covers every matrix's 128-channel
- * tiles, one moments launch, one update launch) instead of four launches per
- * matrix. Each matrix gets exactly the arithmetic of al_apollo_step (the
+ * One APOLLO step over many matrices in three launches (one projection
+ * launch whose grid covers every matrix's 128-channel tiles, one moments
+ * launch, one update launch) instead of three launches per matrix. Each matrix gets exactly the arithmetic of al_apollo_step (the
  * results are bit-identical). This grouping is the library's; the paper
  * applies the method matrix by matrix.
  *
@@ -380,7 +379,7 @@ int al_apollo_step(float* p, const float* g, int64_t rows, int64_t cols,
  * buffer (64-byte aligned) of that size; al_apollo_plan fills the host
  * buffer; copy it to the device buffer once; then call al_apollo_step_multi
  * every step. The plan records the matrices' pointers, the workspace and the
- * TMA descriptors of the projection operands: rebuild it if any of them
+ * TMA descriptors of the projections: rebuild it if any of them
  * changes (a refreshed projection written into the same proj buffer needs no
  * rebuild). The norm-growth limiter is not available here
  * (hp->norm_growth_gamma > 0 returns ALQ_ERR_UNSUPPORTED).
@@ -401,7 +400,6 @@ typedef struct {
     int32_t nmat, rank, v_bits, reserved;
     int64_t total_params;   /* sum of rows * cols                            */
     int64_t total_channels; /* sum of max(rows, cols)                        */
-    int64_t conv_tiles;     /* tiles of the bf16 staging pass                */
     int64_t gemm_tiles;     /* 128-channel tiles of the grouped projection   */
     int64_t mom_tiles;      /* 2048-value tiles of the moments pass          */
     int64_t upd_tiles;      /* 4096-parameter tiles of the update pass       */
@@ -411,8 +409,8 @@ typedef struct {
 /* Bytes of a plan over these matrices (host and device copies alike). */
 int al_apollo_plan_bytes(const al_apollo_matrix* mats, int nmat, size_t* bytes);
 
-/* Scratch bytes of a grouped step: every matrix's bf16 operand, projection
- * and channel scales side by side. */
+/* Scratch bytes of a grouped step: every matrix's projection R and channel
+ * scales side by side. */
 int al_apollo_workspace_multi(const al_apollo_matrix* mats, int nmat, int rank,
                               size_t* bytes);
 

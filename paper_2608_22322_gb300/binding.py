@@ -73,8 +73,7 @@ class ApolloMatrix(C.Structure):
 class ApolloInfo(C.Structure):
     _fields_ = [("nmat", C.c_int32), ("rank", C.c_int32), ("v_bits", C.c_int32),
                 ("reserved", C.c_int32), ("total_params", C.c_int64),
-                ("total_channels", C.c_int64), ("conv_tiles", C.c_int64),
-                ("gemm_tiles", C.c_int64), ("mom_tiles", C.c_int64),
+                ("total_channels", C.c_int64), ("gemm_tiles", C.c_int64), ("mom_tiles", C.c_int64),
                 ("upd_tiles", C.c_int64), ("workspace", C.c_void_p)]
 
 

@@ -3,15 +3,14 @@
 // the original gradient; rank 256, channel-wise scaling in Sec. 6.1).
 //
 // Launch sequence of one step:
-//   convert   G (fp32) -> A (bf16, round to nearest even), laid out
-//             [channels][short side] so that the projection's reduction
-//             dimension is contiguous (a tiled transpose when the rows are
-//             the short side, a plain conversion otherwise).
-//   project   R = A * P^T on the tensor cores: TMA loads 128-row tiles of A
-//             and the whole P tile (128-byte swizzle) into a 4-stage shared
-//             memory ring; one thread issues tcgen05.mma (bf16 x bf16 -> fp32)
-//             into a 128 x rank accumulator in tensor memory; the epilogue
-//             reads it back with tcgen05.ld and writes R [channels][rank].
+//   project   R = bf16(G) * P^T on the tensor cores: four converter warps
+//             read 128-channel tiles of G (fp32) and write them as bf16
+//             (round to nearest even) into a 4-stage shared-memory ring in
+//             the 128-byte-swizzled K-major layout, transposing when the
+//             channels are G's columns; TMA loads the matching P tiles; one
+//             thread issues tcgen05.mma (bf16 x bf16 -> fp32) into a
+//             128 x rank accumulator in tensor memory; the epilogue reads it
+//             back with tcgen05.ld and writes R [channels][rank].
 //   moments   per channel (one quantization block = rank values): decode
 //             UF8 M^P and AL8 V^P, Adam EMAs with bias correction, channel
 //             norms of Rt and R (exact two-float sums) -> s_j, re-encode.
@@ -37,7 +36,6 @@ constexpr int kGemmSmem = kStages * (kAStage + kBStage) + 1024 + 256;
 
 // ------------------------------------------------------------ workspace --
 struct ApWs {
-    uint16_t* A;     // [L][s] bf16
     float* R;        // [L][rank]
     float* scale;    // [L]
     double* npart;   // [kMaxNormParts] limiter partials
@@ -59,7 +57,7 @@ static ApWs ap_layout(void* base, int64_t rows, int64_t cols, int rank) {
         off += r256(b);
         return r;
     };
-    w.A = (uint16_t*)take(2 * (size_t)L * s);
+    (void)s;
     w.R = (float*)take(4 * (size_t)L * rank);
     w.scale = (float*)take(4 * (size_t)L);
     w.npart = (double*)take(8 * (size_t)kMaxNormParts);
@@ -72,74 +70,6 @@ static ApWs ap_layout(void* base, int64_t rows, int64_t cols, int rank) {
 int al_apollo_workspace(int64_t rows, int64_t cols, int rank, size_t* bytes) {
     *bytes = ap_layout(nullptr, rows, cols, rank).bytes;
     return ALQ_OK;
-}
-
-// --------------------------------------------------------------- convert --
-// rows > cols: A[j][i] = bf16(G[j][i]) (channels are rows, K = cols). One
-// tile = kTile elements, four float4 per thread (n is a multiple of 4).
-__device__ __forceinline__ void convert_rows_tile(const float* __restrict__ g, int64_t n,
-                                                  uint16_t* __restrict__ A, int64_t tile) {
-    const int64_t base = tile * kTile + 4 * (int64_t)threadIdx.x;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const int64_t i = base + (int64_t)k * 4 * kThreads;
-        if (i < n) {
-            const float4 v = __ldcs(reinterpret_cast<const float4*>(g + i));
-            const uint32_t lo = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.x)) |
-                                ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.y)) << 16);
-            const uint32_t hi = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.z)) |
-                                ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.w)) << 16);
-            *reinterpret_cast<uint2*>(A + i) = make_uint2(lo, hi);
-        }
-    }
-}
-
-// rows <= cols: A[j][i] = bf16(G[i][j]) (channels are columns, K = rows),
-// one 64 x 64 tile (tile row tr over i, tile column tc over j) through
-// shared memory: 16-byte loads along G's rows, 8-byte stores (four bf16)
-// along A's rows. Every thread of the CTA must call it; it ends with a
-// barrier so that the shared tile can be reused. rows and cols are multiples
-// of 4 (the entry points require cols % 4 == 0 and rows % 8 == 0 here).
-constexpr int kTT = 64;
-__device__ __forceinline__ void convert_cols_tile(const float* __restrict__ g, int rows, int cols,
-                                                  uint16_t* __restrict__ A, int64_t tr,
-                                                  int64_t tc, float (*t)[kTT + 1]) {
-    const int i0 = (int)tr * kTT, j0 = (int)tc * kTT;
-    const int x4 = 4 * (threadIdx.x & 15), y = threadIdx.x >> 4;  // 16 x 16 threads
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        const int i = i0 + y + 16 * q, j = j0 + x4;
-        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (i < rows && j < cols) v = __ldcs(reinterpret_cast<const float4*>(g + (int64_t)i * cols + j));
-        t[y + 16 * q][x4] = v.x;
-        t[y + 16 * q][x4 + 1] = v.y;
-        t[y + 16 * q][x4 + 2] = v.z;
-        t[y + 16 * q][x4 + 3] = v.w;
-    }
-    __syncthreads();
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        const int jl = y + 16 * q, j = j0 + jl, i = i0 + x4;  // A row j, columns i .. i + 3
-        if (j < cols && i < rows) {
-            const uint32_t lo = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t[x4][jl])) |
-                                ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t[x4 + 1][jl])) << 16);
-            const uint32_t hi = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t[x4 + 2][jl])) |
-                                ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t[x4 + 3][jl])) << 16);
-            *reinterpret_cast<uint2*>(A + (int64_t)j * rows + i) = make_uint2(lo, hi);
-        }
-    }
-    __syncthreads();
-}
-
-__global__ void __launch_bounds__(kThreads)
-to_bf16_kernel(const float* __restrict__ g, int64_t n, uint16_t* __restrict__ A, int64_t ntiles) {
-    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) convert_rows_tile(g, n, A, tile);
-}
-
-__global__ void __launch_bounds__(kThreads)
-to_bf16_t_kernel(const float* __restrict__ g, int rows, int cols, uint16_t* __restrict__ A) {
-    __shared__ float t[kTT][kTT + 1];
-    convert_cols_tile(g, rows, cols, A, blockIdx.y, blockIdx.x, t);
 }
 
 // ------------------------------------------------------ PTX primitives --
@@ -209,31 +139,146 @@ __host__ __device__ constexpr uint32_t umma_idesc_bf16(int M, int N) {
 
 // ---------------------------------------------------------- projection --
 struct GemmArgs {
-    float* R;
-    int L;
+    const float* g;  // G [rows][cols] fp32
+    int64_t cols;    // row pitch of G
+    int64_t K;       // short side s: the reduction length
+    float* R;        // [L][rank]
+    int L;           // channels (the long side)
     int rank;
     int kblocks;
+    int rows_short;  // channels are G's columns (rows <= cols)
     int* err;
 };
 
-// One 128-channel tile of R = A * P^T: rows m0 .. m0 + 127 of A against
-// the whole projection, K in a.kblocks steps of 64. The tensor maps may live
-// in the kernel's parameters or in global memory.
-__device__ __forceinline__ void project_tile(const CUtensorMap* tmA, const CUtensorMap* tmB,
-                                             const GemmArgs& a, int m0, uint8_t* smem_raw) {
+// CTA of the projection: warp 0 issues the TMA loads of P, warp 1 the
+// tensor-core MMAs, warps 2..5 convert G to bf16 into the operand stages and
+// then read the accumulator back.
+constexpr int kConvWarps = 4;
+constexpr int kProjThreads = 64 + 32 * kConvWarps;
+
+// bf16 (round to nearest even) of two values, lo in the low half.
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    const __nv_bfloat162 b = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t*>(&b);
+}
+
+// One converter warp's share (64 values per lane) of K block kb of the
+// 128-channel tile at m0. Channels are G's rows (RS false: K contiguous;
+// warp c takes tile rows 32c .. 32c + 31, two rows per load, 16 lanes x 16
+// bytes along K) or G's columns (RS true: K strided; warp c takes K rows
+// 16c .. 16c + 15, lane l the channels l + 32 q, each load a 128-byte row
+// slice). Outside G the values are 0.
+template <bool RS>
+__device__ __forceinline__ void conv_load(const GemmArgs& a, int m0, int kb, int c, int lane,
+                                          float (&v)[64]) {
+    if constexpr (!RS) {
+        const int64_t k = (int64_t)kb * kGK + 4 * (lane & 15);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const int64_t j = m0 + 32 * c + 2 * i + (lane >> 4);
+            float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (j < a.L && k < a.K) x = __ldcs(reinterpret_cast<const float4*>(a.g + j * a.cols + k));
+            v[4 * i] = x.x;
+            v[4 * i + 1] = x.y;
+            v[4 * i + 2] = x.z;
+            v[4 * i + 3] = x.w;
+        }
+    } else {
+#pragma unroll
+        for (int kk = 0; kk < 16; ++kk) {
+            const int64_t k = (int64_t)kb * kGK + 16 * c + kk;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int64_t j = m0 + lane + 32 * q;
+                v[16 * q + kk] = (k < a.K && j < a.L) ? __ldcs(a.g + k * a.cols + j) : 0.0f;
+            }
+        }
+    }
+}
+
+// The same share as bf16 into an operand stage in the layout a 128-byte
+// swizzled TMA load writes (row r of 128 bytes, 16-byte chunk x stored at
+// chunk x ^ (r & 7)): K-major, as the MMA's shared-memory descriptor reads.
+// Each store of a warp covers all 32 banks once per 128 bytes.
+template <bool RS>
+__device__ __forceinline__ void conv_store(uint8_t* sa, int c, int lane, const float (&v)[64]) {
+    if constexpr (!RS) {
+        const int kq = lane & 15;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const int r = 32 * c + 2 * i + (lane >> 4);
+            const uint2 w = make_uint2(pack_bf16x2(v[4 * i], v[4 * i + 1]),
+                                       pack_bf16x2(v[4 * i + 2], v[4 * i + 3]));
+            *reinterpret_cast<uint2*>(sa + r * 128 + (((kq >> 1) ^ (r & 7)) << 4) + ((kq & 1) << 3)) = w;
+        }
+    } else {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int r = lane + 32 * q;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const float* x = v + 16 * q + 8 * h;
+                const uint4 w = make_uint4(pack_bf16x2(x[0], x[1]), pack_bf16x2(x[2], x[3]),
+                                           pack_bf16x2(x[4], x[5]), pack_bf16x2(x[6], x[7]));
+                *reinterpret_cast<uint4*>(sa + r * 128 + (((2 * c + h) ^ (r & 7)) << 4)) = w;
+            }
+        }
+    }
+}
+
+// Stage kb of a converter warp: wait until the MMAs that read the stage's
+// previous contents retired, write it, make the writes visible to the tensor
+// cores and arrive (one arrival per converter warp).
+template <bool RS>
+__device__ __forceinline__ bool conv_stage(const float (&v)[64], int kb, uint8_t* sA,
+                                           uint32_t afull0, uint32_t empty0, int c, int lane) {
+    const int s = kb % kStages;
+    if (kb >= kStages && !mbar_wait(empty0 + 8 * s, ((kb / kStages) - 1) & 1)) return false;
+    conv_store<RS>(sA + s * kAStage, c, lane, v);
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(afull0 + 8 * s);
+    return true;
+}
+
+// All K blocks of a converter warp, the loads of block kb + 1 in flight
+// while block kb is converted and stored.
+template <bool RS>
+__device__ __forceinline__ bool conv_all(const GemmArgs& a, int m0, uint8_t* sA, uint32_t afull0,
+                                         uint32_t empty0, int c, int lane) {
+    float va[64], vb[64];
+    conv_load<RS>(a, m0, 0, c, lane, va);
+    for (int kb = 0; kb < a.kblocks; kb += 2) {
+        if (kb + 1 < a.kblocks) conv_load<RS>(a, m0, kb + 1, c, lane, vb);
+        if (!conv_stage<RS>(va, kb, sA, afull0, empty0, c, lane)) return false;
+        if (kb + 1 >= a.kblocks) break;
+        if (kb + 2 < a.kblocks) conv_load<RS>(a, m0, kb + 2, c, lane, va);
+        if (!conv_stage<RS>(vb, kb + 1, sA, afull0, empty0, c, lane)) return false;
+    }
+    return true;
+}
+
+// One 128-channel tile of R = bf16(G) * P^T: channels m0 .. m0 + 127
+// against the whole projection, K in a.kblocks steps of 64. G is read once,
+// as fp32, and converted on its way into the operand stages (no bf16 copy
+// in memory). The tensor map of P may live in the kernel's parameters or in
+// global memory.
+__device__ __forceinline__ void project_tile(const CUtensorMap* tmB, const GemmArgs& a, int m0,
+                                             uint8_t* smem_raw) {
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t* sA = smem;
     uint8_t* sB = smem + kStages * kAStage;
-    uint64_t* bars = (uint64_t*)(sB + kStages * kBStage);  // full[4], empty[4], accum
-    uint32_t* tmem_slot = (uint32_t*)(bars + 2 * kStages + 1);
+    uint64_t* bars = (uint64_t*)(sB + kStages * kBStage);  // bfull[4], afull[4], empty[4], accum
+    uint32_t* tmem_slot = (uint32_t*)(bars + 3 * kStages + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + kStages);
-    const uint32_t accum = smem_u32(bars + 2 * kStages);
+    const uint32_t bfull0 = smem_u32(bars), afull0 = smem_u32(bars + kStages);
+    const uint32_t empty0 = smem_u32(bars + 2 * kStages), accum = smem_u32(bars + 3 * kStages);
     const uint32_t ncols = a.rank <= 128 ? 128u : 256u;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
-            mbar_init(full0 + 8 * s, 1);
+            mbar_init(bfull0 + 8 * s, 1);
+            mbar_init(afull0 + 8 * s, kConvWarps);
             mbar_init(empty0 + 8 * s, 1);
         }
         mbar_init(accum, 1);
@@ -253,55 +298,66 @@ __device__ __forceinline__ void project_tile(const CUtensorMap* tmA, const CUten
     const uint32_t b_bytes = (uint32_t)a.rank * kGK * 2;
 
     bool ok = true;
-    if (warp == 0 && lane == 0) {
-        // TMA producer: stage s is refilled once the MMAs that read it retire
-        for (int kb = 0; kb < a.kblocks && ok; ++kb) {
-            const int s = kb % kStages;
-            if (kb >= kStages) ok = mbar_wait(empty0 + 8 * s, ((kb / kStages) - 1) & 1);
-            if (!ok) break;
-            mbar_expect_tx(full0 + 8 * s, kAStage + b_bytes);
-            tma_load_2d(smem_u32(sA + s * kAStage), tmA, kb * kGK, m0, full0 + 8 * s);
-            tma_load_2d(smem_u32(sB + s * kBStage), tmB, kb * kGK, 0, full0 + 8 * s);
+    if (warp == 0) {
+        if (lane == 0) {
+            // TMA producer of P: stage s is refilled once the MMAs that read
+            // it retire
+            for (int kb = 0; kb < a.kblocks && ok; ++kb) {
+                const int s = kb % kStages;
+                if (kb >= kStages) ok = mbar_wait(empty0 + 8 * s, ((kb / kStages) - 1) & 1);
+                if (!ok) break;
+                mbar_expect_tx(bfull0 + 8 * s, b_bytes);
+                tma_load_2d(smem_u32(sB + s * kBStage), tmB, kb * kGK, 0, bfull0 + 8 * s);
+            }
         }
-    } else if (warp == 1 && lane == 0) {
-        // MMA issuer: four K = 16 steps per stage, 32 bytes apart in the row
-        const uint32_t idesc = umma_idesc_bf16(kGM, a.rank);
-        for (int kb = 0; kb < a.kblocks && ok; ++kb) {
-            const int s = kb % kStages;
-            ok = mbar_wait(full0 + 8 * s, (kb / kStages) & 1);
-            if (!ok) break;
-            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            const uint32_t a0 = smem_u32(sA + s * kAStage), b0 = smem_u32(sB + s * kBStage);
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // MMA issuer: four K = 16 steps per stage, 32 bytes apart in the row
+            const uint32_t idesc = umma_idesc_bf16(kGM, a.rank);
+            for (int kb = 0; kb < a.kblocks && ok; ++kb) {
+                const int s = kb % kStages;
+                const uint32_t par = (kb / kStages) & 1;
+                ok = mbar_wait(afull0 + 8 * s, par) && mbar_wait(bfull0 + 8 * s, par);
+                if (!ok) break;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t a0 = smem_u32(sA + s * kAStage), b0 = smem_u32(sB + s * kBStage);
 #pragma unroll
-            for (int k = 0; k < kGK / 16; ++k)
-                umma_bf16(tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc,
-                          (kb | k) != 0);
-            umma_commit(empty0 + 8 * s);
+                for (int k = 0; k < kGK / 16; ++k)
+                    umma_bf16(tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc,
+                              (kb | k) != 0);
+                umma_commit(empty0 + 8 * s);
+            }
+            if (ok) umma_commit(accum);
         }
-        if (ok) umma_commit(accum);
+    } else {
+        const int c = warp - 2;
+        ok = a.rows_short ? conv_all<true>(a, m0, sA, afull0, empty0, c, lane)
+                          : conv_all<false>(a, m0, sA, afull0, empty0, c, lane);
     }
     if (!ok) atomicExch(a.err, 1);
-    __syncwarp();
 
-    // epilogue: warp w reads TMEM lanes 32w..32w+31 (tile rows), 32 columns
-    // at a time
-    const bool have = mbar_wait(accum, 0);
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    const int row = m0 + warp * 32 + lane;
-    if (!have && lane == 0) atomicExch(a.err, 1);
-    for (int c0 = 0; c0 < a.rank; c0 += 32) {
-        float v[32];
-        if (have) {
-            tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
-        } else {
+    if (warp >= 2) {
+        // epilogue: a warp may read TMEM lanes 32 (warp % 4) .. + 31 (tile
+        // rows), 32 columns at a time
+        const int q = warp & 3;
+        const bool have = mbar_wait(accum, 0);
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const int row = m0 + q * 32 + lane;
+        if (!have && lane == 0) atomicExch(a.err, 1);
+        for (int c0 = 0; c0 < a.rank; c0 += 32) {
+            float v[32];
+            if (have) {
+                tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, v);
+            } else {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = __int_as_float(0x7FC00000);  // NaN marks a failure
-        }
-        if (row < a.L) {
-            float4* dst = reinterpret_cast<float4*>(a.R + (int64_t)row * a.rank + c0);
+                for (int i = 0; i < 32; ++i) v[i] = __int_as_float(0x7FC00000);  // NaN marks a failure
+            }
+            if (row < a.L) {
+                float4* dst = reinterpret_cast<float4*>(a.R + (int64_t)row * a.rank + c0);
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
-                dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+                for (int i = 0; i < 8; ++i)
+                    dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+            }
         }
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -312,11 +368,10 @@ __device__ __forceinline__ void project_tile(const CUtensorMap* tmA, const CUten
                      : "memory");
 }
 
-__global__ void __launch_bounds__(128, 1)
-apollo_project_kernel(const __grid_constant__ CUtensorMap tmA,
-                      const __grid_constant__ CUtensorMap tmB, GemmArgs a) {
+__global__ void __launch_bounds__(kProjThreads, 1)
+apollo_project_kernel(const __grid_constant__ CUtensorMap tmB, GemmArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    project_tile(&tmA, &tmB, a, blockIdx.x * kGM, smem_raw);
+    project_tile(&tmB, a, blockIdx.x * kGM, smem_raw);
 }
 
 // ------------------------------------------------------------- moments --
@@ -331,6 +386,8 @@ struct MomentArgs {
     int block;
     float* scale;
     float beta1, beta2, omb1, omb2, ic1, c2, eps, log_floor;
+    float one;   // 1 and 0, opaque to the compiler: f * one + c rounds as
+    float zero;  // f + c, fma(x, y, zero) as x y
 };
 
 // Geometry of the moments pass: a warp owns a 256-element segment (two
@@ -433,45 +490,79 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
             vh[e] = al16_decode(code_of<VBITS>(vw, e / 4, e % 4), olmin[e / 4 / CPB],
                                 odelta[e / 4 / CPB]);
     }
-    float mf[NE], vf[NE];
-    uint32_t cvmin[kMCH], cvmax[kMCH], cmabs[kMCH];
-    float nrh[NB], nrl[NB], ngh[NB], ngl[NB];
+    // Moments and channel norms on pairs of elements (paired fp32
+    // instructions, each component rounded as the scalar operation; a sum
+    // of two rounded products is a fused multiply-add by the opaque one, so
+    // that no product is contracted into it). The norms accumulate the
+    // exact squares (two-float products) in two-float sums, even and odd
+    // elements apart, merged before the warp sum.
+    const float2 one = make_float2(m.one, m.one);
+    const float2 b1 = make_float2(m.beta1, m.beta1), o1 = make_float2(m.omb1, m.omb1);
+    const float2 b2 = make_float2(m.beta2, m.beta2), o2 = make_float2(m.omb2, m.omb2);
+    const float2 ic1 = make_float2(m.ic1, m.ic1), c2 = make_float2(m.c2, m.c2);
+    const float2 eps = make_float2(m.eps, m.eps), neg = make_float2(-1.0f, -1.0f);
+    const float2 zero = make_float2(m.zero, m.zero);
+    float vf[NE];
+    float2 mf2[NE / 2];
+    uint32_t cvmin[kMCH], cvmax[kMCH];
+    float cmabs[kMCH];
+    float2 nrh[NB], nrl[NB], ngh[NB], ngl[NB];
 #pragma unroll
-    for (int b = 0; b < NB; ++b) nrh[b] = nrl[b] = ngh[b] = ngl[b] = 0.0f;
+    for (int b = 0; b < NB; ++b)
+        nrh[b] = nrl[b] = ngh[b] = ngl[b] = make_float2(0.0f, 0.0f);
 #pragma unroll
     for (int c = 0; c < kMCH; ++c) {
         const int b = c / CPB;
+        const float2 dm2 = make_float2(dm[b], dm[b]);
+        const uint32_t mx = mw[c] ^ 0x80808080u;
         cvmin[c] = 0xFFFFFFFFu;
         cvmax[c] = 0u;
-        cmabs[c] = 0u;
+        cmabs[c] = 0.0f;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const float mh = s8_to_float((mw[c] >> (8 * i)) & 0xFFu) * dm[b];
-            const float rv = f4get(r[c], i);
-            const float mq = m.beta1 * mh + m.omb1 * rv;
-            const float vq = m.beta2 * vh[4 * c + i] + m.omb2 * (rv * rv);
-            const float rt = (mq * m.ic1) / (sqrtf(vq) * m.c2 + m.eps);
-            mf[4 * c + i] = mq;
-            vf[4 * c + i] = vq;
-            float h, l;
-            two_prod(rt, rt, h, l);
-            ff_acc(nrh[b], nrl[b], h, l);
-            two_prod(rv, rv, h, l);
-            ff_acc(ngh[b], ngl[b], h, l);
-            const uint32_t vb = f2u(vq);
-            cvmin[c] = umix<false>(cvmin[c], vb - 1u);
-            cvmax[c] = umix<true>(cvmax[c], vb);
-            cmabs[c] = umix<true>(cmabs[c], f2u(mq) & 0x7FFFFFFFu);
+        for (int i = 0; i < 2; ++i) {
+            // momentum bytes as exact floats (see s8_to_float)
+            const float2 qf = make_float2(u2f(__byte_perm(mx, 0x4B400000u, 0x7640u | (2 * i))),
+                                          u2f(__byte_perm(mx, 0x4B400000u, 0x7640u | (2 * i + 1))));
+            const float2 mh = mul2(add2(qf, make_float2(-12583040.0f, -12583040.0f)), dm2);
+            const float2 rv = i == 0 ? make_float2(r[c].x, r[c].y) : make_float2(r[c].z, r[c].w);
+            const float2 vh2 = make_float2(vh[4 * c + 2 * i], vh[4 * c + 2 * i + 1]);
+            const float2 mq = fma2(mul2(b1, mh), one, mul2(o1, rv));
+            const float2 vq = fma2(mul2(b2, vh2), one, mul2(o2, mul2(rv, rv)));
+            const float2 den = fma2(mul2(make_float2(sqrtf(vq.x), sqrtf(vq.y)), c2), one, eps);
+            const float2 num = mul2(mq, ic1);
+            const float2 rt = make_float2(num.x / den.x, num.y / den.y);
+            mf2[2 * c + i] = mq;
+            vf[4 * c + 2 * i] = vq.x;
+            vf[4 * c + 2 * i + 1] = vq.y;
+            ff_acc_sq2(nrh[b], nrl[b], rt, neg, zero);
+            ff_acc_sq2(ngh[b], ngl[b], rv, neg, zero);
+            const uint32_t vbx = f2u(vq.x), vby = f2u(vq.y);
+            cvmin[c] = umix<false>(cvmin[c], umix<false>(vbx - 1u, vby - 1u));
+            cvmax[c] = umix<true>(cvmax[c], umix<true>(vbx, vby));
+            cmabs[c] = fmaxf(cmabs[c], fmaxf(fabsf(mq.x), fabsf(mq.y)));
         }
     }
+    float nrhs[NB], nrls[NB], nghs[NB], ngls[NB];
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+        nrhs[b] = nrh[b].x;
+        nrls[b] = nrl[b].x;
+        ff_acc(nrhs[b], nrls[b], nrh[b].y, nrl[b].y);
+        nghs[b] = ngh[b].x;
+        ngls[b] = ngl[b].x;
+        ff_acc(nghs[b], ngls[b], ngh[b].y, ngl[b].y);
+    }
+    uint32_t cmabs_u[kMCH];
+#pragma unroll
+    for (int c = 0; c < kMCH; ++c) cmabs_u[c] = f2u(cmabs[c]);
     uint32_t bvmin[NB], bvmax[NB], bmabs[NB];
     warp_blocks_reduce<CPB, false>(cvmin, bvmin);
     warp_blocks_reduce<CPB, true>(cvmax, bvmax);
-    warp_blocks_reduce<CPB, true>(cmabs, bmabs);
+    warp_blocks_reduce<CPB, true>(cmabs_u, bmabs);
 #pragma unroll
     for (int b = 0; b < NB; ++b) {
-        ff_warp_sum(nrh[b], nrl[b]);
-        ff_warp_sum(ngh[b], ngl[b]);
+        ff_warp_sum(nrhs[b], nrls[b]);
+        ff_warp_sum(nghs[b], ngls[b]);
     }
     float vmn[NB], vmx[NB], nlmin[NB], ndelta[NB], K[NB], E[NB], ms[NB], sc[NB], inv[NB];
 #pragma unroll
@@ -492,10 +583,19 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
     for (int c = 0; c < kMCH; ++c) {
         const int b = c / CPB;
         const int64_t idx = chunk_index(seg0, c, lane);
-        uint32_t qm = 0;
+        // q = rint((m sc) inv) as the low byte of 1.5 * 2^23 + q (two's
+        // complement for q < 0); the rounding add by the opaque one
+        const float2 sc2 = make_float2(sc[b], sc[b]), inv2 = make_float2(inv[b], inv[b]);
+        uint32_t rb[4];
 #pragma unroll
-        for (int i = 0; i < 4; ++i)
-            qm |= ((uint32_t)uf8_quantize(mf[4 * c + i], sc[b], inv[b]) & 0xFFu) << (8 * i);
+        for (int i = 0; i < 2; ++i) {
+            const float2 f = mul2(mul2(mf2[2 * c + i], sc2), inv2);
+            const float2 rr = fma2(f, one, make_float2(12582912.0f, 12582912.0f));
+            rb[2 * i] = f2u(rr.x);
+            rb[2 * i + 1] = f2u(rr.y);
+        }
+        const uint32_t qm = __byte_perm(__byte_perm(rb[0], rb[1], 0x0040u),
+                                        __byte_perm(rb[2], rb[3], 0x0040u), 0x5410u);
         store4b((uint8_t*)m.m_codes, idx, m.n, qm);
         if constexpr (VBITS == 8)
             store4b((uint8_t*)m.v_codes, idx, m.n,
@@ -514,7 +614,7 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
     }
 #pragma unroll
     for (int b = 0; b < NB; ++b)
-        if (b0 + b < nblk) ps.add(nrh[b], nrl[b], ngh[b], ngl[b], m.scale + b0 + b);
+        if (b0 + b < nblk) ps.add(nrhs[b], nrls[b], nghs[b], ngls[b], m.scale + b0 + b);
     __syncwarp();
 }
 
@@ -646,14 +746,13 @@ constexpr uint32_t kApPlanMagic = 0x41504C31u;  // "APL1"
 struct ApPlanHeader {
     uint32_t magic;
     int32_t nmat, rank, v_bits;
-    int64_t conv_tiles, gemm_tiles, mom_tiles, upd_tiles;
+    int64_t gemm_tiles, mom_tiles, upd_tiles;
     int64_t total_params, total_channels;
-    int64_t reserved[2];
+    int64_t reserved[3];
 };
 static_assert(sizeof(ApPlanHeader) == 80, "plan header layout");
 
 struct ApEntry {  // aligned as CUtensorMap (at least 64 bytes)
-    CUtensorMap tmA;  // bf16 A [L][s] in the workspace, box [128][64]
     CUtensorMap tmB;  // bf16 P [rank][s], box [rank][64]
     float* p;
     const float* g;
@@ -661,13 +760,12 @@ struct ApEntry {  // aligned as CUtensorMap (at least 64 bytes)
     float* m_absmax;
     void* v_codes;
     float* v_meta;
-    uint16_t* A;
     float* R;
     float* scale;
     int64_t rows, cols, n, L, s, npj;
     Divider dv;
     int32_t rows_short, kblocks;
-    int64_t conv_t0, gemm_t0, mom_t0, upd_t0;  // first tile of each pass
+    int64_t gemm_t0, mom_t0, upd_t0;  // first tile of each pass
 };
 
 constexpr size_t kApEntryOffset = 128;  // header rounded up to the entry alignment
@@ -680,38 +778,19 @@ __device__ __forceinline__ int entry_for(const ApEntry* __restrict__ tab, int nm
     return cur;
 }
 
-__global__ void __launch_bounds__(kThreads)
-apollo_convert_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t ntiles) {
-    __shared__ float t[kTT][kTT + 1];
-    int cur = 0;
-    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-        cur = entry_for(tab, nmat, tile, cur, &ApEntry::conv_t0);
-        const ApEntry& e = tab[cur];
-        const int64_t lt = tile - e.conv_t0;
-        if (e.rows_short) {
-            const int64_t ntc = (e.cols + kTT - 1) / kTT;
-            convert_cols_tile(e.g, (int)e.rows, (int)e.cols, e.A, lt / ntc, lt % ntc, t);
-        } else {
-            convert_rows_tile(e.g, e.n, e.A, lt);
-        }
-    }
-}
-
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(kProjThreads, 1)
 apollo_project_multi_kernel(const ApEntry* __restrict__ tab, const uint16_t* __restrict__ tile_mat,
                             int rank, int* err) {
     extern __shared__ uint8_t smem_raw[];
     const ApEntry* e = tab + tile_mat[blockIdx.x];
     if (threadIdx.x == 0) {
-        // the descriptors were written through the generic proxy (a copy to
-        // device memory): make them visible to the tensor-map proxy
-        asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(&e->tmA)
-                     : "memory");
+        // the descriptor was written through the generic proxy (a copy to
+        // device memory): make it visible to the tensor-map proxy
         asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(&e->tmB)
                      : "memory");
     }
-    const GemmArgs a{e->R, (int)e->L, rank, e->kblocks, err};
-    project_tile(&e->tmA, &e->tmB, a, (int)(blockIdx.x - e->gemm_t0) * kGM, smem_raw);
+    const GemmArgs a{e->g, e->cols, e->s, e->R, (int)e->L, rank, e->kblocks, e->rows_short, err};
+    project_tile(&e->tmB, a, (int)(blockIdx.x - e->gemm_t0) * kGM, smem_raw);
 }
 
 template <int CPB, int VBITS>
@@ -789,11 +868,12 @@ static bool make_map(CUtensorMap* map, const void* base, uint64_t k, uint64_t ro
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-static int launch_project(const uint16_t* A, const uint16_t* P, int64_t L, int64_t s, int rank,
-                          float* R, int* err, cudaStream_t st) {
-    CUtensorMap ma, mb;
-    if (!make_map(&ma, A, (uint64_t)s, (uint64_t)L, kGM) ||
-        !make_map(&mb, P, (uint64_t)s, (uint64_t)rank, (uint32_t)rank))
+static int launch_project(const float* g, int64_t rows, int64_t cols, const uint16_t* P,
+                          int rank, float* R, int* err, cudaStream_t st) {
+    const int rows_short = rows <= cols;
+    const int64_t s = rows_short ? rows : cols, L = rows_short ? cols : rows;
+    CUtensorMap mb;
+    if (!make_map(&mb, P, (uint64_t)s, (uint64_t)rank, (uint32_t)rank))
         return record_cuda(cudaErrorInvalidValue);
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
@@ -802,8 +882,8 @@ static int launch_project(const uint16_t* A, const uint16_t* P, int64_t L, int64
                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);
     });
     if (attr_err != cudaSuccess) return record_cuda(attr_err);
-    GemmArgs a{R, (int)L, rank, (int)blocks_of(s, kGK), err};
-    apollo_project_kernel<<<(unsigned)blocks_of(L, kGM), 128, kGemmSmem, st>>>(ma, mb, a);
+    GemmArgs a{g, cols, s, R, (int)L, rank, (int)blocks_of(s, kGK), rows_short, err};
+    apollo_project_kernel<<<(unsigned)blocks_of(L, kGM), kProjThreads, kGemmSmem, st>>>(mb, a);
     return check_launch();
 }
 
@@ -837,6 +917,8 @@ static MomentArgs moment_scalars(const al_apollo_hp* hp, int64_t t, int rank) {
     m.c2 = (float)(1.0 / sqrt(bc2));
     m.eps = hp->eps;
     m.log_floor = hp->log_floor;
+    m.one = 1.0f;
+    m.zero = 0.0f;
     return m;
 }
 
@@ -862,25 +944,14 @@ extern "C" int al_apollo_step(float* p, const float* g, int64_t rows, int64_t co
     const al_apollo_matrix mat{p, g, rows, cols, proj, m_codes, m_absmax, v_codes, v_meta};
     int rc0 = check_apollo_matrix(mat, rank, v_bits);
     if (rc0) return rc0;
-    const int64_t s = rows <= cols ? rows : cols, L = rows <= cols ? cols : rows;
+    const int64_t L = rows <= cols ? cols : rows;
     if (hp->norm_growth_gamma > 0.0f && !prev_norm) return ALQ_ERR_INVALID_ARG;
     const ApWs w = ap_layout(workspace, rows, cols, rank);
     if (!workspace || ws_bytes < w.bytes || !aligned(workspace, 256)) return ALQ_ERR_WORKSPACE;
     cudaStream_t st = (cudaStream_t)stream;
     const int rows_short = rows <= cols;
 
-    // bf16 operand with the short side contiguous
-    if (rows_short) {
-        dim3 grid((unsigned)blocks_of(cols, kTT), (unsigned)blocks_of(rows, kTT));
-        to_bf16_t_kernel<<<grid, kThreads, 0, st>>>(g, (int)rows, (int)cols, w.A);
-    } else {
-        const int64_t n = rows * cols, ntiles = blocks_of(n, kTile);
-        to_bf16_kernel<<<persistent_grid((const void*)to_bf16_kernel, kThreads, 0, ntiles),
-                         kThreads, 0, st>>>(g, n, w.A, ntiles);
-    }
-    int rc = check_launch();
-    if (rc) return rc;
-    rc = launch_project(w.A, proj, L, s, rank, w.R, w.err, st);
+    int rc = launch_project(g, rows, cols, proj, rank, w.R, w.err, st);
     if (rc) return rc;
 
     MomentArgs m = moment_scalars(hp, t, rank);
@@ -940,15 +1011,10 @@ static ApShape ap_shape(const al_apollo_matrix& m) {
     return a;
 }
 
-static int64_t conv_tiles_of(const al_apollo_matrix& m) {
-    const ApShape a = ap_shape(m);
-    return a.rows_short ? blocks_of(m.cols, kTT) * blocks_of(m.rows, kTT) : blocks_of(a.n, kTile);
-}
-
-// Per-matrix scratch of a grouped step: A, R, scale, each 256-byte aligned.
+// Per-matrix scratch of a grouped step: R, scale, each 256-byte aligned.
 static size_t multi_ws_bytes(const al_apollo_matrix& m, int rank) {
     const ApShape a = ap_shape(m);
-    return r256(2 * (size_t)a.L * a.s) + r256(4 * (size_t)a.L * rank) + r256(4 * (size_t)a.L);
+    return r256(4 * (size_t)a.L * rank) + r256(4 * (size_t)a.L);
 }
 
 static int check_matrices(const al_apollo_matrix* mats, int nmat) {
@@ -1025,9 +1091,8 @@ extern "C" int al_apollo_plan(const al_apollo_matrix* mats, int nmat, int rank, 
         e.m_absmax = m.m_absmax;
         e.v_codes = m.v_codes;
         e.v_meta = m.v_meta;
-        e.A = (uint16_t*)ws;
-        e.R = (float*)(ws + r256(2 * (size_t)a.L * a.s));
-        e.scale = (float*)(ws + r256(2 * (size_t)a.L * a.s) + r256(4 * (size_t)a.L * rank));
+        e.R = (float*)ws;
+        e.scale = (float*)(ws + r256(4 * (size_t)a.L * rank));
         ws += multi_ws_bytes(m, rank);
         e.rows = m.rows;
         e.cols = m.cols;
@@ -1038,16 +1103,13 @@ extern "C" int al_apollo_plan(const al_apollo_matrix* mats, int nmat, int rank, 
         e.dv = make_divider((uint32_t)m.cols);
         e.rows_short = a.rows_short;
         e.kblocks = (int32_t)blocks_of(a.s, kGK);
-        e.conv_t0 = h.conv_tiles;
         e.gemm_t0 = h.gemm_tiles;
         e.mom_t0 = h.mom_tiles;
         e.upd_t0 = h.upd_tiles;
-        if (!make_map(&e.tmA, e.A, (uint64_t)a.s, (uint64_t)a.L, kGM) ||
-            !make_map(&e.tmB, m.proj, (uint64_t)a.s, (uint64_t)rank, (uint32_t)rank))
+        if (!make_map(&e.tmB, m.proj, (uint64_t)a.s, (uint64_t)rank, (uint32_t)rank))
             return record_cuda(cudaErrorInvalidValue);
         const int64_t gt = blocks_of(a.L, kGM);
         for (int64_t k = 0; k < gt; ++k) tile_mat[h.gemm_tiles + k] = (uint16_t)i;
-        h.conv_tiles += conv_tiles_of(m);
         h.gemm_tiles += gt;
         h.mom_tiles += blocks_of(e.npj, kMTile);
         h.upd_tiles += blocks_of(a.n, kTile);
@@ -1062,7 +1124,6 @@ extern "C" int al_apollo_plan(const al_apollo_matrix* mats, int nmat, int rank, 
     info->reserved = 0;
     info->total_params = h.total_params;
     info->total_channels = h.total_channels;
-    info->conv_tiles = h.conv_tiles;
     info->gemm_tiles = h.gemm_tiles;
     info->mom_tiles = h.mom_tiles;
     info->upd_tiles = h.upd_tiles;
@@ -1083,12 +1144,7 @@ extern "C" int al_apollo_step_multi(const void* plan_dev, const al_apollo_info* 
                                                  (size_t)info->nmat * sizeof(ApEntry));
     int* err = (int*)info->workspace;
 
-    apollo_convert_multi_kernel<<<persistent_grid((const void*)apollo_convert_multi_kernel,
-                                                  kThreads, 0, info->conv_tiles),
-                                  kThreads, 0, st>>>(tab, info->nmat, info->conv_tiles);
-    int rc = check_launch();
-    if (rc) return rc;
-
+    int rc;
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [] {
@@ -1096,7 +1152,7 @@ extern "C" int al_apollo_step_multi(const void* plan_dev, const al_apollo_info* 
                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);
     });
     if (attr_err != cudaSuccess) return record_cuda(attr_err);
-    apollo_project_multi_kernel<<<(unsigned)info->gemm_tiles, 128, kGemmSmem, st>>>(
+    apollo_project_multi_kernel<<<(unsigned)info->gemm_tiles, kProjThreads, kGemmSmem, st>>>(
         tab, tile_mat, info->rank, err);
     rc = check_launch();
     if (rc) return rc;

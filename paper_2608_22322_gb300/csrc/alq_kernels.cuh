@@ -467,6 +467,23 @@ __device__ __forceinline__ void ff_acc(float& hi, float& lo, float h, float l) {
     lo = lo + (e + l);
 }
 
+// Two-float accumulation of the exact squares of a pair of values (two
+// independent sums): x^2 = h + l with h = RN(x x) and -l = RN(h - x x)
+// (exact), then Knuth's TwoSum of hi and h; neg = (-1, -1). h is a fused
+// multiply-add with zero, a value the compiler cannot see (from the
+// kernel's parameters): a paired product feeding the sums could otherwise
+// be contracted into them.
+__device__ __forceinline__ void ff_acc_sq2(float2& hi, float2& lo, float2 x, float2 neg,
+                                           float2 zero) {
+    const float2 h = fma2(x, x, zero);
+    const float2 nl = fma2(mul2(x, neg), x, h);
+    const float2 s = add2(hi, h);
+    const float2 bb = sub2(s, hi);
+    const float2 e = add2(sub2(hi, sub2(s, bb)), sub2(h, bb));
+    hi = s;
+    lo = add2(lo, sub2(e, nl));
+}
+
 __device__ __forceinline__ void ff_warp_sum(float& hi, float& lo) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
