@@ -556,9 +556,9 @@ def _row_apollo(torch, np, wl, B, dev):
     projected moments UF8 / AL8 in blocks of 256, gradients N(0, 1e-3).
     Algorithmic bytes: G read for the projection and again for the scaled
     update (8), p read and written (8), projected states and their block
-    constants; the bf16 staging copy of G is not counted. FLOPs: 2 r s L per
-    matrix for the projection. One grouped step (al_apollo_step_multi: four
-    launches for all matrices)."""
+    constants (the projection converts G to bf16 in shared memory: no
+    staging copy). FLOPs: 2 r s L per matrix for the projection. One grouped
+    step (al_apollo_step_multi: three launches for all matrices)."""
     cfg = wl.CONFIGS["tinyllama_apollo"]
     r = cfg["rank"]
     hp = dict(lr=cfg["lr"], beta1=cfg["beta1"], beta2=cfg["beta2"], eps=cfg["eps"],
@@ -610,11 +610,11 @@ def _row_apollo(torch, np, wl, B, dev):
         return rows * cols / dt, (f"one step of one {rows}x{cols} matrix incl. the rank-{r} "
                                   f"projection in double ({dt:.1f} s, single thread)")
 
-    return dict(step=step, n=n_tot, bytes=nbytes, flops=flops, launches=4,
+    return dict(step=step, n=n_tot, bytes=nbytes, flops=flops, launches=3,
                 oracle=oracle_sample,
                 workload=f"APOLLO TinyLlama-1.1B {len(mats)} matrices (one grouped step), "
                          f"rank {r}, UF8 M^P, AL8 V^P block 256",
-                bytes_note="G twice, p read+write, projected states; bf16 staging not counted")
+                bytes_note="G twice, p read+write, projected states")
 
 
 def _row_codec(torch, np, wl, B, dev):
