@@ -327,6 +327,81 @@ int al_came_step(float* p, const float* g, int64_t rows, int64_t cols,
                  const al_came_hp* hp, int64_t t, void* workspace,
                  size_t ws_bytes, void* stream);
 
+/* --------------------------------------------- grouped Adafactor / CAME -- */
+/*
+ * One Adafactor or CAME step over many matrices with one launch per pass
+ * (Adafactor: g^2 sums, factors, scales, RMS, update = 5 launches; CAME adds
+ * the residual sums, the confidence factors and their scales = 8 launches)
+ * instead of those launches per matrix. Every pass works in tiles that never
+ * cross a matrix, with the per-tile code of al_adafactor_step / al_came_step,
+ * so each matrix's results are bit-identical to the per-matrix call. The
+ * grouping is the library's; the paper steps matrix by matrix.
+ *
+ * Usage: al_factored_workspace_multi -> allocate the workspace (256-byte
+ * aligned); al_factored_plan_bytes -> allocate a host buffer and a device
+ * buffer (64-byte aligned) of that size; al_factored_plan fills the host
+ * buffer; copy it to the device buffer once; then call
+ * al_adafactor_step_multi or al_came_step_multi every step. The plan records
+ * the matrices' pointers and the workspace: rebuild it if any of them
+ * changes.
+ */
+typedef struct {
+    float* p;             /* [rows x cols] fp32, row-major                   */
+    const float* g;
+    int64_t rows, cols;   /* cols % 4 == 0, rows * cols < 2^31               */
+    void* vr_codes;       /* second-moment row factor [rows] (Adafactor R)   */
+    float* vr_meta;
+    void* vc_codes;       /* second-moment column factor [cols] (C)          */
+    float* vc_meta;
+    void* cr_codes;       /* CAME confidence row factor [rows]; NULL for      */
+    float* cr_meta;       /* Adafactor                                       */
+    void* cc_codes;       /* CAME confidence column factor [cols]            */
+    float* cc_meta;
+    int8_t* m_codes;      /* UF8 momentum [rows x cols]; NULL for Adafactor  */
+    float* m_absmax;      /* without momentum (then for every matrix)        */
+} al_factored_matrix;
+
+/* Summary of a grouped factored plan (host struct, filled by
+ * al_factored_plan). */
+typedef struct {
+    int32_t nmat;
+    int32_t op;           /* AL_OP_ADAFACTOR or AL_OP_CAME                   */
+    int32_t v_bits, v_block, c_bits, c_block, m_block;
+    int32_t has_momentum;
+    int64_t total_params;
+    int64_t sumsq_tiles;  /* 64 x 512 tiles of the sums passes               */
+    int64_t factor_tiles; /* factor blocks (rows and columns) of V           */
+    int64_t factor2_tiles;/* factor blocks of CAME's confidence (else 0)     */
+    int64_t scale_tiles;  /* 256-entry tiles of the scale passes             */
+    int64_t tiles;        /* 4096-parameter tiles of the RMS and update      */
+    void* workspace;      /* the workspace the plan is bound to              */
+} al_factored_info;
+
+/* Bytes of a plan over these matrices (host and device copies alike). */
+int al_factored_plan_bytes(const al_factored_matrix* mats, int nmat, size_t* bytes);
+
+/* Scratch bytes of a grouped step: every matrix's al_workspace_size
+ * scratch side by side. */
+int al_factored_workspace_multi(const al_factored_matrix* mats, int nmat, size_t* bytes);
+
+/* Validates every matrix as al_adafactor_step (op AL_OP_ADAFACTOR: v_bits
+ * and v_block are fac_bits and fac_block, c_* ignored) or al_came_step (op
+ * AL_OP_CAME) does, with one set of bit widths and block sizes for all, and
+ * writes the plan into plan_host. Momentum must be present in every matrix
+ * or in none (CAME: in every matrix). Returns ALQ_ERR_WORKSPACE when the
+ * workspace is missing, misaligned or too small. */
+int al_factored_plan(int op, const al_factored_matrix* mats, int nmat, int v_bits,
+                     int v_block, int c_bits, int c_block, int m_block, void* workspace,
+                     size_t ws_bytes, void* plan_host, size_t plan_bytes,
+                     al_factored_info* info);
+
+/* One grouped step. plan_dev is the device copy of the plan; info and hp are
+ * host pointers; the plan's op must match the call. */
+int al_adafactor_step_multi(const void* plan_dev, const al_factored_info* info,
+                            const al_adafactor_hp* hp, int64_t t, void* stream);
+int al_came_step_multi(const void* plan_dev, const al_factored_info* info,
+                       const al_came_hp* hp, int64_t t, void* stream);
+
 /* ---------------------------------------------------------------- APOLLO -- */
 typedef struct {
     float lr;

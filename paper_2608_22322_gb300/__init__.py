@@ -14,7 +14,7 @@ _BINDING_NAMES = {
     "al_encode", "al_decode", "uf8_encode", "uf8_decode", "al_adamw_step",
     "AdamWPlan", "al_adafactor_step", "al_came_step", "al_apollo_step",
     "al_num_blocks", "al_state_bytes", "al_workspace_size", "version", "AlqError",
-    "AL_OP_ADAFACTOR", "AL_OP_CAME", "AL_OP_APOLLO", "ApolloPlan",
+    "AL_OP_ADAFACTOR", "AL_OP_CAME", "AL_OP_APOLLO", "ApolloPlan", "FactoredPlan",
 }
 
 

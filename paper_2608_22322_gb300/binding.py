@@ -77,6 +77,23 @@ class ApolloInfo(C.Structure):
                 ("upd_tiles", C.c_int64), ("workspace", C.c_void_p)]
 
 
+class FactoredMatrix(C.Structure):
+    _fields_ = [("p", C.c_void_p), ("g", C.c_void_p), ("rows", C.c_int64),
+                ("cols", C.c_int64), ("vr_codes", C.c_void_p), ("vr_meta", C.c_void_p),
+                ("vc_codes", C.c_void_p), ("vc_meta", C.c_void_p), ("cr_codes", C.c_void_p),
+                ("cr_meta", C.c_void_p), ("cc_codes", C.c_void_p), ("cc_meta", C.c_void_p),
+                ("m_codes", C.c_void_p), ("m_absmax", C.c_void_p)]
+
+
+class FactoredInfo(C.Structure):
+    _fields_ = [("nmat", C.c_int32), ("op", C.c_int32), ("v_bits", C.c_int32),
+                ("v_block", C.c_int32), ("c_bits", C.c_int32), ("c_block", C.c_int32),
+                ("m_block", C.c_int32), ("has_momentum", C.c_int32),
+                ("total_params", C.c_int64), ("sumsq_tiles", C.c_int64),
+                ("factor_tiles", C.c_int64), ("factor2_tiles", C.c_int64),
+                ("scale_tiles", C.c_int64), ("tiles", C.c_int64), ("workspace", C.c_void_p)]
+
+
 class MultiInfo(C.Structure):
     _fields_ = [("ntensors", C.c_int32), ("m_block", C.c_int32),
                 ("v_block", C.c_int32), ("v_bits", C.c_int32),
@@ -116,6 +133,14 @@ _sig("al_adafactor_noalloc_capacity", C.c_size_t)
 _sig("al_came_step", _int, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _vp, _int, _int,
      _vp, _vp, _vp, _vp, _int, _int, _vp, _vp, _int, C.POINTER(CameHP), _i64, _vp,
      C.c_size_t, _vp)
+_sig("al_factored_plan_bytes", _int, C.POINTER(FactoredMatrix), _int, C.POINTER(C.c_size_t))
+_sig("al_factored_workspace_multi", _int, C.POINTER(FactoredMatrix), _int,
+     C.POINTER(C.c_size_t))
+_sig("al_factored_plan", _int, _int, C.POINTER(FactoredMatrix), _int, _int, _int, _int, _int,
+     _int, _vp, C.c_size_t, _vp, C.c_size_t, C.POINTER(FactoredInfo))
+_sig("al_adafactor_step_multi", _int, _vp, C.POINTER(FactoredInfo), C.POINTER(AdafactorHP),
+     _i64, _vp)
+_sig("al_came_step_multi", _int, _vp, C.POINTER(FactoredInfo), C.POINTER(CameHP), _i64, _vp)
 _sig("al_apollo_plan_bytes", _int, C.POINTER(ApolloMatrix), _int, C.POINTER(C.c_size_t))
 _sig("al_apollo_workspace_multi", _int, C.POINTER(ApolloMatrix), _int, _int,
      C.POINTER(C.c_size_t))
@@ -276,6 +301,52 @@ def al_apollo_step(p, g, rows, cols, proj, m_codes, m_absmax, m_block, v_codes, 
         _ptr(p), _ptr(g), rows, cols, _ptr(proj), _ptr(m_codes), _ptr(m_absmax), m_block,
         _ptr(v_codes), _ptr(v_meta), v_bits, v_block, _ptr(prev_norm), C.byref(h), t,
         _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+class FactoredPlan:
+    """A grouped Adafactor or CAME step over many matrices (al_factored_plan
+    / al_adafactor_step_multi / al_came_step_multi): owns the workspace and
+    the device copy of the plan. `op` is AL_OP_ADAFACTOR or AL_OP_CAME;
+    `mats` is a list of dicts with keys p, g, rows, cols, vr_codes, vr_meta,
+    vc_codes, vc_meta, and for CAME cr_codes, cr_meta, cc_codes, cc_meta,
+    and optionally (always for CAME) m_codes, m_absmax (torch CUDA
+    tensors)."""
+
+    _KEYS = ("vr_codes", "vr_meta", "vc_codes", "vc_meta", "cr_codes", "cr_meta", "cc_codes",
+             "cc_meta", "m_codes", "m_absmax")
+
+    def __init__(self, op, mats, v_bits, v_block, c_bits=16, c_block=128, m_block=256,
+                 device=None):
+        nm = len(mats)
+        arr = (FactoredMatrix * nm)()
+        for i, m in enumerate(mats):
+            arr[i] = FactoredMatrix(_ptr(m["p"]), _ptr(m["g"]), m["rows"], m["cols"],
+                                    *[_ptr(m.get(k)) for k in self._KEYS])
+        dev = device if device is not None else mats[0]["p"].device
+        ws = C.c_size_t(0)
+        _check("al_factored_workspace_multi",
+               lib.al_factored_workspace_multi(arr, nm, C.byref(ws)))
+        self.workspace = torch.zeros(ws.value, dtype=torch.uint8, device=dev)
+        nbytes = C.c_size_t(0)
+        _check("al_factored_plan_bytes", lib.al_factored_plan_bytes(arr, nm, C.byref(nbytes)))
+        host = torch.zeros(nbytes.value, dtype=torch.uint8)
+        self.info = FactoredInfo()
+        _check("al_factored_plan", lib.al_factored_plan(
+            op, arr, nm, v_bits, v_block, c_bits, c_block, m_block, _ptr(self.workspace),
+            ws.value, host.data_ptr(), nbytes.value, C.byref(self.info)))
+        self.op = op
+        self.dev = host.to(dev)
+        self.mats = mats  # keep the arrays alive while the plan is used
+
+    def step(self, hp: dict, t: int, stream=None):
+        if self.op == AL_OP_ADAFACTOR:
+            h = _hp(AdafactorHP, hp)
+            _check("al_adafactor_step_multi", lib.al_adafactor_step_multi(
+                _ptr(self.dev), C.byref(self.info), C.byref(h), t, _stream(stream)))
+        else:
+            h = _hp(CameHP, hp)
+            _check("al_came_step_multi", lib.al_came_step_multi(
+                _ptr(self.dev), C.byref(self.info), C.byref(h), t, _stream(stream)))
 
 
 class ApolloPlan:

@@ -10,9 +10,9 @@
 //              decode the old factor, EMA, AL-encode the fresh factor.
 //   scale      a_i = 1/sqrt(R_i / mean(R)), b_j = 1/sqrt(C_j).
 //   usq        G read again: u = (g a_i) b_j, exact float-float sum of u^2,
-//              one fp64 partial per CTA of a persistent grid (fixed order).
-//              The last CTA of usq adds the partials and writes the clip
-//              factor 1 / max(1, RMS(u) / d).
+//              one fp64 partial per 4096-element tile (fixed order). The CTA
+//              that finishes a matrix's last tile adds its partials and
+//              writes the clip factor 1 / max(1, RMS(u) / d).
 //   update     G read a third time: u_hat, optional UF8 momentum, p update.
 // CAME inserts, before its update, a second sumsq pass over the residual
 // (u_hat - m)^2 + eps2 (recomputing m from the old momentum codes), a second
@@ -20,19 +20,23 @@
 // m / sqrt(S) with S from the confidence factors.
 // Every reduction is deterministic: error-free fp32 transforms inside a
 // thread, fixed shuffle and tree orders, fp64 merges; no float atomics.
+//
+// Each pass is a per-tile device function; the single-matrix kernels and
+// the grouped ones (one launch per pass over many matrices, tiles never
+// crossing a matrix) call the same functions, so a matrix's results do not
+// depend on which path stepped it.
 #include "alq_kernels.cuh"
 
 namespace alq {
 
 constexpr int kFR = 64;   // rows per sumsq tile
 constexpr int kFC = 512;  // columns per sumsq tile
-constexpr int kMaxParts = 4096;
 
 // ------------------------------------------------------------ workspace --
 struct FacWs {
     double* rowpart;  // [ncb][rows]
     double* colpart;  // [nrb][cols]
-    double* upart;    // [kMaxParts]
+    double* upart;    // [tiles of kTile elements]: RMS partials
     float* fr;        // fresh row factor (V)
     float* fc;        // fresh column factor (V)
     float* fr2;       // fresh row factor (C)
@@ -62,7 +66,7 @@ static FacWs fac_layout(void* base, int64_t rows, int64_t cols) {
     };
     w.rowpart = (double*)take(sizeof(double) * ncb * rows);
     w.colpart = (double*)take(sizeof(double) * nrb * cols);
-    w.upart = (double*)take(sizeof(double) * kMaxParts);
+    w.upart = (double*)take(sizeof(double) * blocks_of(rows * cols, kTile));
     w.fr = (float*)take(sizeof(float) * rows);
     w.fc = (float*)take(sizeof(float) * cols);
     w.fr2 = (float*)take(sizeof(float) * rows);
@@ -94,13 +98,15 @@ struct ResidualArgs {
 // ----------------------------------------------------------------- sumsq --
 // MODE 0: terms g^2 (exact two-float squares). MODE 1: terms CAME's
 // residual (u_hat - m)^2 + eps2 rounded to fp32 as the update defines it.
+// One 64-row x 512-column tile (bx over columns, by over rows); every
+// thread of the CTA calls it, with the CTA's shared scratch s_col.
 template <int MODE>
-__global__ void __launch_bounds__(kThreads)
-sumsq_kernel(const float* __restrict__ g, int rows, int cols, ResidualArgs ra,
-             double* __restrict__ rowpart, double* __restrict__ colpart) {
-    __shared__ double s_col[kThreads / 32][kFC];
+__device__ __forceinline__ void sumsq_tile(const float* __restrict__ g, int rows, int cols,
+                                           const ResidualArgs& ra, double* __restrict__ rowpart,
+                                           double* __restrict__ colpart, int bx, int by,
+                                           double (*s_col)[kFC]) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int c0 = blockIdx.x * kFC, r0 = blockIdx.y * kFR;
+    const int c0 = bx * kFC, r0 = by * kFR;
     float ch[16], cl[16];
 #pragma unroll
     for (int k = 0; k < 16; ++k) ch[k] = cl[k] = 0.0f;
@@ -173,7 +179,7 @@ sumsq_kernel(const float* __restrict__ g, int rows, int cols, ResidualArgs ra,
             }
             ff_warp_sum(rh, rl);
             if (lane == 0 && row < rows)
-                rowpart[(int64_t)blockIdx.x * rows + row] = (double)rh + (double)rl;
+                rowpart[(int64_t)bx * rows + row] = (double)rh + (double)rl;
         }
     }
 #pragma unroll
@@ -187,8 +193,16 @@ sumsq_kernel(const float* __restrict__ g, int rows, int cols, ResidualArgs ra,
         double s = 0.0;
 #pragma unroll
         for (int w = 0; w < kThreads / 32; ++w) s += s_col[w][t];
-        colpart[(int64_t)blockIdx.y * cols + c0 + t] = s;
+        colpart[(int64_t)by * cols + c0 + t] = s;
     }
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kThreads)
+sumsq_kernel(const float* __restrict__ g, int rows, int cols, ResidualArgs ra,
+             double* __restrict__ rowpart, double* __restrict__ colpart) {
+    __shared__ double s_col[kThreads / 32][kFC];
+    sumsq_tile<MODE>(g, rows, cols, ra, rowpart, colpart, blockIdx.x, blockIdx.y, s_col);
 }
 
 // ---------------------------------------------------------------- factor --
@@ -217,14 +231,13 @@ __device__ __forceinline__ uint32_t fac_code(const FactorDesc& f, int64_t i) {
 // KPT = elements per thread (block / 256, at least 1). rsum (nullable)
 // receives, for the blocks of f0, the fp64 sum of the block's fresh values in
 // a fixed order (the scale pass builds mean(R) from them).
+// Block b of factor f, by one CTA; rsum (nullable) as above.
 template <int KPT>
-__global__ void __launch_bounds__(kThreads)
-factor_kernel(FactorDesc f0, FactorDesc f1, int nb0, double* __restrict__ rsum) {
+__device__ __forceinline__ void factor_block(const FactorDesc& f, int64_t b,
+                                             double* __restrict__ rsum) {
     __shared__ uint32_t s_part[2][kThreads / 32];
     __shared__ double s_sum[kThreads / 32];
-    const bool first = (int)blockIdx.x < nb0;
-    const FactorDesc& f = first ? f0 : f1;
-    const int64_t b = first ? blockIdx.x : blockIdx.x - nb0;
+    const bool first = rsum != nullptr;
     const int64_t lo = b * f.block;
     const int64_t hi = lo + f.block < f.len ? lo + f.block : f.len;
     const float2 om = __ldg(reinterpret_cast<const float2*>(f.meta) + b);
@@ -257,7 +270,7 @@ factor_kernel(FactorDesc f0, FactorDesc f1, int nb0, double* __restrict__ rsum) 
             vmax = umix<true>(vmax, vb);
         }
     }
-    if (first && rsum) {
+    if (first) {
         // fixed order: per thread, then shuffle tree, then warps in order
         double t = 0.0;
 #pragma unroll
@@ -270,7 +283,7 @@ factor_kernel(FactorDesc f0, FactorDesc f1, int nb0, double* __restrict__ rsum) 
     vmax = __reduce_max_sync(0xFFFFFFFFu, vmax);
     vmin = cta_group_reduce<false>(vmin, s_part[0], kThreads / 32);
     vmax = cta_group_reduce<true>(vmax, s_part[1], kThreads / 32);
-    if (first && rsum && threadIdx.x == 0) {
+    if (first && threadIdx.x == 0) {
         double t = 0.0;
         for (int w = 0; w < kThreads / 32; ++w) t += s_sum[w];
         rsum[b] = t;
@@ -297,16 +310,26 @@ factor_kernel(FactorDesc f0, FactorDesc f1, int nb0, double* __restrict__ rsum) 
     if (threadIdx.x == 0) reinterpret_cast<float2*>(f.meta)[b] = make_float2(lmin, delta);
 }
 
+// Blocks 0 .. nb0 - 1 of f0 (with the block sums into rsum), then f1's.
+template <int KPT>
+__global__ void __launch_bounds__(kThreads)
+factor_kernel(FactorDesc f0, FactorDesc f1, int nb0, double* __restrict__ rsum) {
+    const bool first = (int)blockIdx.x < nb0;
+    factor_block<KPT>(first ? f0 : f1, first ? blockIdx.x : blockIdx.x - nb0,
+                      first ? rsum : nullptr);
+}
+
 // ----------------------------------------------------------------- scale --
 // a_i = 1/sqrt(R_i / mean(R)), b_j = 1/sqrt(C_j). mean(R) in fp64 from the
 // factor pass's per-block sums, added in block order by every CTA (the same
 // value everywhere), rounded once. One element per thread over rows + cols.
-__global__ void __launch_bounds__(kThreads)
-scale_kernel(const float* __restrict__ R, int rows, const float* __restrict__ C, int cols,
-             const double* __restrict__ rsum, int nrb, float* __restrict__ a,
-             float* __restrict__ b, unsigned int* __restrict__ ticket) {
+__device__ __forceinline__ void scale_tile(const float* __restrict__ R, int rows,
+                                           const float* __restrict__ C, int cols,
+                                           const double* __restrict__ rsum, int nrb,
+                                           float* __restrict__ a, float* __restrict__ b,
+                                           unsigned int* __restrict__ ticket, int tile) {
     __shared__ float s_mean;
-    if (ticket && blockIdx.x == 0 && threadIdx.x == 0) *ticket = 0u;  // for the RMS pass
+    if (ticket && tile == 0 && threadIdx.x == 0) *ticket = 0u;  // for the RMS pass
     if (threadIdx.x == 0) {
         double t = 0.0;
         for (int k = 0; k < nrb; ++k) t += rsum[k];
@@ -314,65 +337,86 @@ scale_kernel(const float* __restrict__ R, int rows, const float* __restrict__ C,
     }
     __syncthreads();
     const float meanR = s_mean;
-    const int i = blockIdx.x * kThreads + threadIdx.x;
+    const int i = tile * kThreads + threadIdx.x;
     if (i < rows)
         a[i] = 1.0f / sqrtf(R[i] / meanR);
     else if (i < rows + cols)
         b[i - rows] = 1.0f / sqrtf(C[i - rows]);
 }
 
+__global__ void __launch_bounds__(kThreads)
+scale_kernel(const float* __restrict__ R, int rows, const float* __restrict__ C, int cols,
+             const double* __restrict__ rsum, int nrb, float* __restrict__ a,
+             float* __restrict__ b, unsigned int* __restrict__ ticket) {
+    scale_tile(R, rows, C, cols, rsum, nrb, a, b, ticket, blockIdx.x);
+}
+
 // ------------------------------------------------------------------- usq --
 // Sum of u^2, u = (g a_i) b_j, over the whole matrix: exact squares in
-// two-float per thread, fixed warp/CTA order, one fp64 partial per CTA. The
-// last CTA to finish (an atomic ticket, zeroed by the scale pass) adds the
-// partials in CTA order and writes the clip factor
+// two-float per thread, fixed warp/CTA order, one fp64 partial per tile.
+// The CTA that finishes a matrix's last tile (an atomic ticket, zeroed by
+// the scale pass) adds the partials in tile order and writes the clip factor
 // scal[0] = 1 / max(1, sqrt(sum / count) / clip_d).
-__global__ void __launch_bounds__(kThreads)
-usq_kernel(const float* __restrict__ g, int64_t n, Divider dv, const float* __restrict__ a,
-           const float* __restrict__ b, int64_t ntiles, double* __restrict__ upart,
-           unsigned int* __restrict__ ticket, double count, float clip_d,
-           float* __restrict__ scal) {
-    __shared__ double s_w[kThreads];
-    __shared__ bool s_last;
+struct UsqArgs {
+    const float* g;
+    int64_t n;
+    Divider dv;
+    const float* a;
+    const float* b;
+    double* upart;
+    unsigned int* ticket;
+    float* scal;
+};
+
+// The tile's partial (every thread of the CTA calls it; thread 0 returns it).
+__device__ __forceinline__ double usq_tile_sum(const UsqArgs& q, int64_t tile, double* s_w) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     float hi = 0.0f, lo = 0.0f;
-    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-        const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
+    const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            const int64_t idx = chunk_index(seg0, c, lane);
-            if (idx < n) {
-                const uint32_t row = divide((uint32_t)idx, dv);
-                const uint32_t col = (uint32_t)idx - row * dv.d;
-                const float4 gv = __ldcs(reinterpret_cast<const float4*>(g + idx));
-                const float4 bv = __ldg(reinterpret_cast<const float4*>(b + col));
-                const float ai = __ldg(a + row);
+    for (int c = 0; c < 4; ++c) {
+        const int64_t idx = chunk_index(seg0, c, lane);
+        if (idx < q.n) {
+            const uint32_t row = divide((uint32_t)idx, q.dv);
+            const uint32_t col = (uint32_t)idx - row * q.dv.d;
+            const float4 gv = __ldcs(reinterpret_cast<const float4*>(q.g + idx));
+            const float4 bv = __ldg(reinterpret_cast<const float4*>(q.b + col));
+            const float ai = __ldg(q.a + row);
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const float u = (f4get(gv, j) * ai) * f4get(bv, j);
-                    float h, l;
-                    two_prod(u, u, h, l);
-                    ff_acc(hi, lo, h, l);
-                }
+            for (int j = 0; j < 4; ++j) {
+                const float u = (f4get(gv, j) * ai) * f4get(bv, j);
+                float h, l;
+                two_prod(u, u, h, l);
+                ff_acc(hi, lo, h, l);
             }
         }
     }
     ff_warp_sum(hi, lo);
+    __syncthreads();  // s_w may still be read by the previous tile's finish
     if (lane == 0) s_w[warp] = (double)hi + (double)lo;
     __syncthreads();
+    double t = 0.0;
+    if (threadIdx.x == 0)
+        for (int w = 0; w < kThreads / 32; ++w) t += s_w[w];
+    return t;
+}
+
+// One tile of the RMS pass: its partial, and the clip factor if this CTA
+// completes the matrix (ntiles tiles).
+__device__ __forceinline__ void usq_tile(const UsqArgs& q, int64_t tile, int64_t ntiles,
+                                         float clip_d, double* s_w, bool* s_last) {
+    const double t = usq_tile_sum(q, tile, s_w);
     if (threadIdx.x == 0) {
-        double s = 0.0;
-        for (int w = 0; w < kThreads / 32; ++w) s += s_w[w];
-        upart[blockIdx.x] = s;
+        q.upart[tile] = t;
         __threadfence();
-        s_last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+        *s_last = atomicAdd(q.ticket, 1u) == (unsigned int)(ntiles - 1);
     }
     __syncthreads();
-    if (!s_last) return;
+    if (!*s_last) return;
     __threadfence();
     // fixed order: per thread over a stride of kThreads, then a tree
     double acc = 0.0;
-    for (int i = threadIdx.x; i < (int)gridDim.x; i += kThreads) acc += ((volatile double*)upart)[i];
+    for (int64_t i = threadIdx.x; i < ntiles; i += kThreads) acc += ((volatile double*)q.upart)[i];
     s_w[threadIdx.x] = acc;
     __syncthreads();
     for (int st = kThreads / 2; st > 0; st >>= 1) {
@@ -380,11 +424,19 @@ usq_kernel(const float* __restrict__ g, int64_t n, Divider dv, const float* __re
         __syncthreads();
     }
     if (threadIdx.x == 0) {
-        const double rms = sqrt(s_w[0] / count);
+        const double rms = sqrt(s_w[0] / (double)q.n);
         double cf = rms / (double)clip_d;
         if (cf < 1.0) cf = 1.0;
-        scal[0] = (float)(1.0 / cf);
+        q.scal[0] = (float)(1.0 / cf);
     }
+}
+
+__global__ void __launch_bounds__(kThreads)
+usq_kernel(UsqArgs q, int64_t ntiles, float clip_d) {
+    __shared__ double s_w[kThreads];
+    __shared__ bool s_last;
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x)
+        usq_tile(q, tile, ntiles, clip_d, s_w, &s_last);
 }
 
 
@@ -407,17 +459,17 @@ struct UpdateArgs {
     float beta1, omb1, decay, lr;
 };
 
+// One tile of the update; every thread of the CTA calls it (momentum blocks
+// wider than a warp's segment meet in s_part).
 template <int MODE, int CPBM>
-__global__ void __launch_bounds__(kThreads)
-update_kernel(UpdateArgs u, int64_t ntiles) {
+__device__ __forceinline__ void update_tile(const UpdateArgs& u, int64_t tile, uint32_t* s_part) {
     constexpr int NBM = 4 / CPBM;
-    __shared__ uint32_t s_part[kThreads / 32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int wpbm = u.m_block > kSeg ? u.m_block / kSeg : 1;
     const float icf = __ldg(u.scal);
     const int64_t nmb = blocks_of_dev(u.n, u.m_block);
     const int mshift = __ffs(u.m_block) - 1;
-    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+    {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
         const int64_t mb0 = seg0 >> mshift;
         float dm[NBM];
@@ -464,7 +516,7 @@ update_kernel(UpdateArgs u, int64_t ntiles) {
             }
             __stcs(reinterpret_cast<float4*>(u.p + idx), make_float4(pn[0], pn[1], pn[2], pn[3]));
         }
-        if (MODE == 0) continue;
+        if (MODE == 0) return;
         uint32_t babs[NBM];
         warp_blocks_reduce<CPBM, true>(cabs, babs);
         if (wpbm > 1) babs[0] = cta_group_reduce<true>(babs[0], s_part, wpbm);
@@ -494,6 +546,14 @@ update_kernel(UpdateArgs u, int64_t ntiles) {
                 if (mb0 + b < nmb) u.m_absmax[mb0 + b] = ms[b];
         }
     }
+}
+
+template <int MODE, int CPBM>
+__global__ void __launch_bounds__(kThreads)
+update_kernel(UpdateArgs u, int64_t ntiles) {
+    __shared__ uint32_t s_part[kThreads / 32];
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x)
+        update_tile<MODE, CPBM>(u, tile, s_part);
 }
 
 // ------------------------------------------------------------- host side --
@@ -583,10 +643,9 @@ static int second_moment_passes(const float* g, int64_t rows, int64_t cols, cons
         fr.fresh, (int)rows, fc.fresh, (int)cols, w.rsum, nb0, a, b, w.ticket);
     const int64_t n = rows * cols;
     const int64_t ntiles = blocks_of(n, kTile);
-    int grid = persistent_grid((const void*)usq_kernel, kThreads, 0, ntiles);
-    if (grid > kMaxParts) grid = kMaxParts;
-    usq_kernel<<<grid, kThreads, 0, st>>>(g, n, make_divider((uint32_t)cols), a, b, ntiles,
-                                          w.upart, w.ticket, (double)n, clip_d, w.scal);
+    const UsqArgs q{g, n, make_divider((uint32_t)cols), a, b, w.upart, w.ticket, w.scal};
+    usq_kernel<<<persistent_grid((const void*)usq_kernel, kThreads, 0, ntiles), kThreads, 0, st>>>(
+        q, ntiles, clip_d);
     return check_launch();
 }
 
@@ -720,6 +779,405 @@ int al_came_step(float* p, const float* g, int64_t rows, int64_t cols, void* vr_
     u.decay = (float)(1.0 - (double)hp->lr * (double)hp->weight_decay);
     u.lr = hp->lr;
     return launch_update<2>(u, s);
+}
+
+}  // extern "C"
+
+// ------------------------------------------------------- grouped step --
+namespace alq {
+
+constexpr uint32_t kFacPlanMagic = 0x46504C31u;  // "FPL1"
+
+struct FacPlanHeader {
+    uint32_t magic;
+    int32_t nmat, op, reserved;
+};
+constexpr size_t kFacEntryOffset = 64;
+
+// One matrix of a grouped plan: its arguments, its scratch, and the first
+// tile of each pass in the launch that covers all matrices.
+struct FacEntry {
+    float* p;
+    const float* g;
+    int64_t rows, cols, n, ntiles;
+    Divider dv;
+    void* vr_codes;
+    float* vr_meta;
+    void* vc_codes;
+    float* vc_meta;
+    void* cr_codes;
+    float* cr_meta;
+    void* cc_codes;
+    float* cc_meta;
+    int8_t* m_codes;
+    float* m_absmax;
+    FacWs w;
+    int32_t ncb, nrb;  // the sums passes' tile grid (columns, rows)
+    int64_t sq_t0, fac_t0, fac2_t0, sc_t0, usq_t0, upd_t0;
+};
+
+// Per-step scalars of the grouped passes.
+struct FacStep {
+    int op;
+    int v_bits, v_block, c_bits, c_block, m_block, m_shift;
+    float rho_v, omb_v;   // second-moment factor EMA (Adafactor: rho_t)
+    float rho_c, omb_c;   // confidence factor EMA (CAME: beta3)
+    double eps1;
+    float log_floor_v, log_floor_c;
+    float clip_d;
+    float beta1, omb1, eps2, decay, lr;
+};
+
+// The entry whose pass (first tile t0) holds a launch-wide tile: entries are
+// in increasing t0 and every matrix has at least one tile in every pass.
+__device__ __forceinline__ const FacEntry& fac_entry(const FacEntry* __restrict__ tab, int nmat,
+                                                     int64_t tile, int64_t FacEntry::*t0) {
+    int lo = 0, hi = nmat - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (tab[mid].*t0 <= tile) lo = mid; else hi = mid - 1;
+    }
+    return tab[lo];
+}
+
+// Forward cursor for persistent loops (a CTA's tiles only increase).
+__device__ __forceinline__ int fac_advance(const FacEntry* __restrict__ tab, int nmat, int64_t tile,
+                                           int cur, int64_t FacEntry::*t0) {
+    while (cur + 1 < nmat && tab[cur + 1].*t0 <= tile) ++cur;
+    return cur;
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kThreads)
+sumsq_multi_kernel(const FacEntry* __restrict__ tab, int nmat, FacStep fs) {
+    __shared__ double s_col[kThreads / 32][kFC];
+    const FacEntry& e = fac_entry(tab, nmat, blockIdx.x, &FacEntry::sq_t0);
+    const int64_t lt = blockIdx.x - e.sq_t0;
+    ResidualArgs ra{};
+    if (MODE == 1)
+        ra = ResidualArgs{e.m_codes, e.m_absmax, fs.m_shift, e.w.a, e.w.b, e.w.scal,
+                          fs.beta1, fs.omb1, fs.eps2};
+    sumsq_tile<MODE>(e.g, (int)e.rows, (int)e.cols, ra, e.w.rowpart, e.w.colpart,
+                     (int)(lt % e.ncb), (int)(lt / e.ncb), s_col);
+}
+
+// which = 0: the second-moment factors; 1: CAME's confidence factors.
+template <int KPT>
+__global__ void __launch_bounds__(kThreads)
+factor_multi_kernel(const FacEntry* __restrict__ tab, int nmat, FacStep fs, int which) {
+    const FacEntry& e = fac_entry(tab, nmat, blockIdx.x, which ? &FacEntry::fac2_t0 : &FacEntry::fac_t0);
+    const int64_t lt = blockIdx.x - (which ? e.fac2_t0 : e.fac_t0);
+    const int block = which ? fs.c_block : fs.v_block;
+    const int64_t nbr = blocks_of_dev(e.rows, block);
+    const bool row = lt < nbr;
+    FactorDesc f;
+    f.part = row ? e.w.rowpart : e.w.colpart;
+    f.nparts = row ? e.ncb : e.nrb;
+    f.len = row ? e.rows : e.cols;
+    f.mean_len = (double)(row ? e.cols : e.rows);
+    f.add_eps = which ? 0.0 : fs.eps1;
+    f.beta = which ? fs.rho_c : fs.rho_v;
+    f.omb = which ? fs.omb_c : fs.omb_v;
+    f.codes = which ? (row ? e.cr_codes : e.cc_codes) : (row ? e.vr_codes : e.vc_codes);
+    f.meta = which ? (row ? e.cr_meta : e.cc_meta) : (row ? e.vr_meta : e.vc_meta);
+    f.bits = which ? fs.c_bits : fs.v_bits;
+    f.block = block;
+    f.log_floor = which ? fs.log_floor_c : fs.log_floor_v;
+    f.fresh = which ? (row ? e.w.fr2 : e.w.fc2) : (row ? e.w.fr : e.w.fc);
+    double* rsum = row ? (which ? e.w.rsum2 : e.w.rsum) : nullptr;
+    factor_block<KPT>(f, row ? lt : lt - nbr, rsum);
+}
+
+__global__ void __launch_bounds__(kThreads)
+scale_multi_kernel(const FacEntry* __restrict__ tab, int nmat, FacStep fs, int which) {
+    const FacEntry& e = fac_entry(tab, nmat, blockIdx.x, &FacEntry::sc_t0);
+    const int lt = (int)(blockIdx.x - e.sc_t0);
+    if (which == 0)
+        scale_tile(e.w.fr, (int)e.rows, e.w.fc, (int)e.cols, e.w.rsum,
+                   (int)blocks_of_dev(e.rows, fs.v_block), e.w.a, e.w.b, e.w.ticket, lt);
+    else
+        scale_tile(e.w.fr2, (int)e.rows, e.w.fc2, (int)e.cols, e.w.rsum2,
+                   (int)blocks_of_dev(e.rows, fs.c_block), e.w.a2, e.w.b2, nullptr, lt);
+}
+
+__global__ void __launch_bounds__(kThreads)
+usq_multi_kernel(const FacEntry* __restrict__ tab, int nmat, int64_t ntiles, float clip_d) {
+    __shared__ double s_w[kThreads];
+    __shared__ bool s_last;
+    int cur = 0;
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        cur = fac_advance(tab, nmat, tile, cur, &FacEntry::usq_t0);
+        const FacEntry& e = tab[cur];
+        const UsqArgs q{e.g, e.n, e.dv, e.w.a, e.w.b, e.w.upart, e.w.ticket, e.w.scal};
+        usq_tile(q, tile - e.usq_t0, e.ntiles, clip_d, &s_w[0], &s_last);
+    }
+}
+
+template <int MODE, int CPBM>
+__global__ void __launch_bounds__(kThreads)
+update_multi_kernel(const FacEntry* __restrict__ tab, int nmat, int64_t ntiles, FacStep fs) {
+    __shared__ uint32_t s_part[kThreads / 32];
+    int cur = 0;
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        cur = fac_advance(tab, nmat, tile, cur, &FacEntry::upd_t0);
+        const FacEntry& e = tab[cur];
+        UpdateArgs u{};
+        u.p = e.p;
+        u.g = e.g;
+        u.n = e.n;
+        u.dv = e.dv;
+        u.a = e.w.a;
+        u.b = e.w.b;
+        u.a2 = e.w.a2;
+        u.b2 = e.w.b2;
+        u.scal = e.w.scal;
+        u.m_codes = e.m_codes;
+        u.m_absmax = e.m_absmax;
+        u.m_block = MODE > 0 ? fs.m_block : 4096;
+        u.beta1 = fs.beta1;
+        u.omb1 = fs.omb1;
+        u.decay = fs.decay;
+        u.lr = fs.lr;
+        update_tile<MODE, CPBM>(u, tile - e.upd_t0, s_part);
+    }
+}
+
+static size_t fac_plan_size(int nmat) {
+    return kFacEntryOffset + (size_t)nmat * sizeof(FacEntry);
+}
+
+static int check_factored_matrices(const al_factored_matrix* mats, int nmat) {
+    if (!mats || nmat < 1) return ALQ_ERR_INVALID_ARG;
+    for (int i = 0; i < nmat; ++i)
+        if (mats[i].rows < 1 || mats[i].cols < 1) return ALQ_ERR_INVALID_ARG;
+    return ALQ_OK;
+}
+
+template <int KPT>
+static void launch_factor_multi(const FacEntry* tab, int nmat, const FacStep& fs, int which,
+                                int64_t tiles, cudaStream_t st) {
+    factor_multi_kernel<KPT><<<(unsigned)tiles, kThreads, 0, st>>>(tab, nmat, fs, which);
+}
+
+static void factor_multi(const FacEntry* tab, int nmat, const FacStep& fs, int which,
+                         int64_t tiles, cudaStream_t st) {
+    const int block = which ? fs.c_block : fs.v_block;
+    const int kpt = block <= kThreads ? 1 : block / kThreads;
+    switch (kpt) {
+        case 1: launch_factor_multi<1>(tab, nmat, fs, which, tiles, st); break;
+        case 2: launch_factor_multi<2>(tab, nmat, fs, which, tiles, st); break;
+        case 4: launch_factor_multi<4>(tab, nmat, fs, which, tiles, st); break;
+        case 8: launch_factor_multi<8>(tab, nmat, fs, which, tiles, st); break;
+        default: launch_factor_multi<16>(tab, nmat, fs, which, tiles, st); break;
+    }
+}
+
+template <int MODE>
+static void update_multi(const FacEntry* tab, int nmat, int64_t tiles, const FacStep& fs,
+                         cudaStream_t st) {
+    const int cpb = MODE == 0 ? 4 : cpb_of(fs.m_block);
+    const void* k = cpb == 1 ? (const void*)update_multi_kernel<MODE, 1>
+                  : cpb == 2 ? (const void*)update_multi_kernel<MODE, 2>
+                             : (const void*)update_multi_kernel<MODE, 4>;
+    const int grid = persistent_grid(k, kThreads, 0, tiles);
+    if (cpb == 1) update_multi_kernel<MODE, 1><<<grid, kThreads, 0, st>>>(tab, nmat, tiles, fs);
+    else if (cpb == 2) update_multi_kernel<MODE, 2><<<grid, kThreads, 0, st>>>(tab, nmat, tiles, fs);
+    else update_multi_kernel<MODE, 4><<<grid, kThreads, 0, st>>>(tab, nmat, tiles, fs);
+}
+
+// The passes both optimizers share: g^2 sums, second-moment factors, their
+// scales (which also zero the RMS tickets), the RMS pass.
+static void second_moment_multi(const FacEntry* tab, const al_factored_info* info,
+                                const FacStep& fs, cudaStream_t st) {
+    sumsq_multi_kernel<0><<<(unsigned)info->sumsq_tiles, kThreads, 0, st>>>(tab, info->nmat, fs);
+    factor_multi(tab, info->nmat, fs, 0, info->factor_tiles, st);
+    scale_multi_kernel<<<(unsigned)info->scale_tiles, kThreads, 0, st>>>(tab, info->nmat, fs, 0);
+    usq_multi_kernel<<<persistent_grid((const void*)usq_multi_kernel, kThreads, 0, info->tiles),
+                       kThreads, 0, st>>>(tab, info->nmat, info->tiles, fs.clip_d);
+}
+
+static int check_multi_call(const void* plan_dev, const al_factored_info* info, int op) {
+    if (!plan_dev || !info || info->nmat < 1 || !info->workspace) return ALQ_ERR_INVALID_ARG;
+    if (!aligned(plan_dev, 64)) return ALQ_ERR_ALIGN;
+    if (info->op != op) return ALQ_ERR_INVALID_ARG;
+    return ALQ_OK;
+}
+
+}  // namespace alq
+
+extern "C" {
+
+int al_factored_plan_bytes(const al_factored_matrix* mats, int nmat, size_t* bytes) {
+    if (!bytes) return ALQ_ERR_INVALID_ARG;
+    const int rc = check_factored_matrices(mats, nmat);
+    if (rc) return rc;
+    *bytes = fac_plan_size(nmat);
+    return ALQ_OK;
+}
+
+int al_factored_workspace_multi(const al_factored_matrix* mats, int nmat, size_t* bytes) {
+    if (!bytes) return ALQ_ERR_INVALID_ARG;
+    const int rc = check_factored_matrices(mats, nmat);
+    if (rc) return rc;
+    size_t tot = 0;
+    for (int i = 0; i < nmat; ++i) tot += fac_layout(nullptr, mats[i].rows, mats[i].cols).bytes;
+    *bytes = tot;
+    return ALQ_OK;
+}
+
+int al_factored_plan(int op, const al_factored_matrix* mats, int nmat, int v_bits, int v_block,
+                     int c_bits, int c_block, int m_block, void* workspace, size_t ws_bytes,
+                     void* plan_host, size_t plan_bytes, al_factored_info* info) {
+    int rc = check_factored_matrices(mats, nmat);
+    if (rc) return rc;
+    if (!plan_host || !info || (op != AL_OP_ADAFACTOR && op != AL_OP_CAME))
+        return ALQ_ERR_INVALID_ARG;
+    const bool came = op == AL_OP_CAME;
+    const bool has_m = mats[0].m_codes != nullptr;
+    for (int i = 0; i < nmat; ++i) {
+        const al_factored_matrix& m = mats[i];
+        rc = check_matrix(m.p, m.g, m.rows, m.cols);
+        if (!rc) rc = check_factor(m.vr_codes, m.vr_meta, v_bits, v_block);
+        if (!rc) rc = check_factor(m.vc_codes, m.vc_meta, v_bits, v_block);
+        if (!rc && came) rc = check_factor(m.cr_codes, m.cr_meta, c_bits, c_block);
+        if (!rc && came) rc = check_factor(m.cc_codes, m.cc_meta, c_bits, c_block);
+        if (!rc && (m.m_codes != nullptr) != has_m) rc = ALQ_ERR_INVALID_ARG;
+        if (!rc && came && !has_m) rc = ALQ_ERR_INVALID_ARG;
+        if (!rc && has_m) rc = check_momentum(m.m_codes, m.m_absmax, m_block);
+        if (rc) return rc;
+    }
+    size_t need = 0;
+    al_factored_workspace_multi(mats, nmat, &need);
+    if (!workspace || ws_bytes < need || !aligned(workspace, 256)) return ALQ_ERR_WORKSPACE;
+    if (plan_bytes < fac_plan_size(nmat)) return ALQ_ERR_INVALID_ARG;
+
+    char* base = (char*)plan_host;
+    memset(base, 0, fac_plan_size(nmat));
+    FacPlanHeader h{kFacPlanMagic, nmat, op, 0};
+    memcpy(base, &h, sizeof(h));
+    char* ws = (char*)workspace;
+    memset(info, 0, sizeof(*info));
+    for (int i = 0; i < nmat; ++i) {
+        const al_factored_matrix& m = mats[i];
+        FacEntry e;
+        memset(&e, 0, sizeof(e));
+        e.p = m.p;
+        e.g = m.g;
+        e.rows = m.rows;
+        e.cols = m.cols;
+        e.n = m.rows * m.cols;
+        e.ntiles = blocks_of(e.n, kTile);
+        e.dv = make_divider((uint32_t)m.cols);
+        e.vr_codes = m.vr_codes;
+        e.vr_meta = m.vr_meta;
+        e.vc_codes = m.vc_codes;
+        e.vc_meta = m.vc_meta;
+        e.cr_codes = came ? m.cr_codes : nullptr;
+        e.cr_meta = came ? m.cr_meta : nullptr;
+        e.cc_codes = came ? m.cc_codes : nullptr;
+        e.cc_meta = came ? m.cc_meta : nullptr;
+        e.m_codes = has_m ? m.m_codes : nullptr;
+        e.m_absmax = has_m ? m.m_absmax : nullptr;
+        e.w = fac_layout(ws, m.rows, m.cols);
+        ws += e.w.bytes;
+        e.ncb = (int32_t)blocks_of(m.cols, kFC);
+        e.nrb = (int32_t)blocks_of(m.rows, kFR);
+        e.sq_t0 = info->sumsq_tiles;
+        e.fac_t0 = info->factor_tiles;
+        e.fac2_t0 = info->factor2_tiles;
+        e.sc_t0 = info->scale_tiles;
+        e.usq_t0 = info->tiles;
+        e.upd_t0 = info->tiles;
+        info->sumsq_tiles += (int64_t)e.ncb * e.nrb;
+        info->factor_tiles += blocks_of(m.rows, v_block) + blocks_of(m.cols, v_block);
+        if (came) info->factor2_tiles += blocks_of(m.rows, c_block) + blocks_of(m.cols, c_block);
+        info->scale_tiles += blocks_of(m.rows + m.cols, kThreads);
+        info->tiles += e.ntiles;
+        info->total_params += e.n;
+        memcpy(base + kFacEntryOffset + (size_t)i * sizeof(FacEntry), &e, sizeof(e));
+    }
+    // one launch per pass: its grid must fit a launch
+    if (info->sumsq_tiles > INT32_MAX || info->factor_tiles > INT32_MAX ||
+        info->factor2_tiles > INT32_MAX || info->scale_tiles > INT32_MAX)
+        return ALQ_ERR_UNSUPPORTED;
+    info->nmat = nmat;
+    info->op = op;
+    info->v_bits = v_bits;
+    info->v_block = v_block;
+    info->c_bits = came ? c_bits : 0;
+    info->c_block = came ? c_block : 0;
+    info->m_block = has_m ? m_block : 0;
+    info->has_momentum = has_m ? 1 : 0;
+    info->workspace = workspace;
+    return ALQ_OK;
+}
+
+int al_adafactor_step_multi(const void* plan_dev, const al_factored_info* info,
+                            const al_adafactor_hp* hp, int64_t t, void* stream) {
+    int rc = check_multi_call(plan_dev, info, AL_OP_ADAFACTOR);
+    if (rc) return rc;
+    if (!hp || t < 1 || !(hp->eps1 > 0.0f) || !(hp->clip_d > 0.0f)) return ALQ_ERR_INVALID_ARG;
+    cudaStream_t st = (cudaStream_t)stream;
+    const FacEntry* tab = (const FacEntry*)((const char*)plan_dev + kFacEntryOffset);
+    const double omr_d = pow((double)t, (double)hp->decay_rate);
+    FacStep fs{};
+    fs.op = AL_OP_ADAFACTOR;
+    fs.v_bits = info->v_bits;
+    fs.v_block = info->v_block;
+    fs.m_block = info->has_momentum ? info->m_block : 4096;
+    fs.rho_v = (float)(1.0 - omr_d);
+    fs.omb_v = (float)omr_d;
+    fs.eps1 = hp->eps1;
+    fs.log_floor_v = hp->log_floor;
+    fs.clip_d = hp->clip_d;
+    fs.beta1 = hp->beta1;
+    fs.omb1 = (float)(1.0 - (double)hp->beta1);
+    fs.decay = (float)(1.0 - (double)hp->lr * (double)hp->weight_decay);
+    fs.lr = hp->lr;
+    second_moment_multi(tab, info, fs, st);
+    if (info->has_momentum)
+        update_multi<1>(tab, info->nmat, info->tiles, fs, st);
+    else
+        update_multi<0>(tab, info->nmat, info->tiles, fs, st);
+    return check_launch();
+}
+
+int al_came_step_multi(const void* plan_dev, const al_factored_info* info, const al_came_hp* hp,
+                       int64_t t, void* stream) {
+    int rc = check_multi_call(plan_dev, info, AL_OP_CAME);
+    if (rc) return rc;
+    if (!hp || t < 1 || !(hp->eps1 > 0.0f) || !(hp->eps2 > 0.0f) || !(hp->clip_d > 0.0f))
+        return ALQ_ERR_INVALID_ARG;
+    cudaStream_t st = (cudaStream_t)stream;
+    const FacEntry* tab = (const FacEntry*)((const char*)plan_dev + kFacEntryOffset);
+    FacStep fs{};
+    fs.op = AL_OP_CAME;
+    fs.v_bits = info->v_bits;
+    fs.v_block = info->v_block;
+    fs.c_bits = info->c_bits;
+    fs.c_block = info->c_block;
+    fs.m_block = info->m_block;
+    while ((1 << fs.m_shift) < fs.m_block) ++fs.m_shift;
+    fs.rho_v = hp->beta2;
+    fs.omb_v = (float)(1.0 - (double)hp->beta2);
+    fs.rho_c = hp->beta3;
+    fs.omb_c = (float)(1.0 - (double)hp->beta3);
+    fs.eps1 = hp->eps1;
+    fs.eps2 = hp->eps2;
+    fs.log_floor_v = hp->log_floor_v;
+    fs.log_floor_c = hp->log_floor_c;
+    fs.clip_d = hp->clip_d;
+    fs.beta1 = hp->beta1;
+    fs.omb1 = (float)(1.0 - (double)hp->beta1);
+    fs.decay = (float)(1.0 - (double)hp->lr * (double)hp->weight_decay);
+    fs.lr = hp->lr;
+    second_moment_multi(tab, info, fs, st);
+    // residual sums, confidence factors and their scales, update
+    sumsq_multi_kernel<1><<<(unsigned)info->sumsq_tiles, kThreads, 0, st>>>(tab, info->nmat, fs);
+    factor_multi(tab, info->nmat, fs, 1, info->factor2_tiles, st);
+    scale_multi_kernel<<<(unsigned)info->scale_tiles, kThreads, 0, st>>>(tab, info->nmat, fs, 1);
+    update_multi<2>(tab, info->nmat, info->tiles, fs, st);
+    return check_launch();
 }
 
 }  // extern "C"

@@ -64,3 +64,56 @@ def test_validation_rejects_before_launch(lib):
     assert f(None, 1000, 256, 8, -53.0, A, A, None) == -1     # null
     assert f(None, 0, 256, 8, -53.0, None, None, None) == 0   # n == 0: no-op
     assert f(A, -5, 256, 8, -53.0, A, A, None) == -1          # negative size
+
+
+def test_grouped_factored_plan_host_logic(lib):
+    """al_factored_plan on the host: per-pass tile counts, workspace sizes
+    and the argument checks (the plan only records fake pointers)."""
+    from paper_2608_22322_gb300 import binding as Bn
+    lib = Bn.lib  # the binding's handle carries the argument types
+    A = 0x100000
+
+    def mat(rows, cols, came, mom):
+        ptrs = [A] * 8 if came else [A] * 4 + [None] * 4
+        return Bn.FactoredMatrix(A, A, rows, cols, *ptrs, A if mom else None, A if mom else None)
+
+    shapes = [(300, 772), (64, 512), (4096, 4096)]
+    arr = (Bn.FactoredMatrix * 3)(*[mat(r, c, True, True) for r, c in shapes])
+    ws = C.c_size_t(0)
+    assert lib.al_factored_workspace_multi(arr, 3, C.byref(ws)) == 0
+    per = []
+    for r, c in shapes:
+        b = C.c_size_t(0)
+        assert lib.al_workspace_size(2, r, c, 0, C.byref(b)) == 0
+        per.append(b.value)
+    assert ws.value == sum(per)
+    nb = C.c_size_t(0)
+    assert lib.al_factored_plan_bytes(arr, 3, C.byref(nb)) == 0
+    host = (C.c_uint8 * nb.value)()
+    info = Bn.FactoredInfo()
+    args = lambda op, a, w: (op, a, 3, 16, 128, 16, 128, 256, C.c_void_p(A), w, host,
+                             nb.value, C.byref(info))
+    assert lib.al_factored_plan(*args(2, arr, ws.value)) == 0
+    tiles = lambda n, t: -(-n // t)
+    assert info.nmat == 3 and info.op == 2 and info.has_momentum == 1
+    assert info.total_params == sum(r * c for r, c in shapes)
+    assert info.sumsq_tiles == sum(tiles(c, 512) * tiles(r, 64) for r, c in shapes)
+    assert info.factor_tiles == sum(tiles(r, 128) + tiles(c, 128) for r, c in shapes)
+    assert info.factor2_tiles == info.factor_tiles
+    assert info.scale_tiles == sum(tiles(r + c, 256) for r, c in shapes)
+    assert info.tiles == sum(tiles(r * c, 4096) for r, c in shapes)
+    assert lib.al_factored_plan(*args(2, arr, ws.value - 1)) == -4   # workspace too small
+    assert lib.al_factored_plan(*args(3, arr, ws.value)) == -1       # not a factored op
+    # momentum in some matrices only; CAME without momentum; no confidence
+    mixed = (Bn.FactoredMatrix * 3)(mat(300, 772, True, True), mat(64, 512, True, False),
+                                   mat(8, 8, True, True))
+    assert lib.al_factored_plan(*args(2, mixed, ws.value)) == -1
+    nom = (Bn.FactoredMatrix * 3)(*[mat(r, c, True, False) for r, c in shapes])
+    assert lib.al_factored_plan(*args(2, nom, ws.value)) == -1
+    ada = (Bn.FactoredMatrix * 3)(*[mat(r, c, False, False) for r, c in shapes])
+    assert lib.al_factored_plan(*args(1, ada, ws.value)) == 0
+    assert info.has_momentum == 0 and info.factor2_tiles == 0
+    assert lib.al_factored_plan(*args(2, ada, ws.value)) == -1       # CAME needs confidence
+    bad = (Bn.FactoredMatrix * 3)(mat(300, 770, True, True), *[mat(r, c, True, True)
+                                                               for r, c in shapes[1:]])
+    assert lib.al_factored_plan(*args(2, bad, ws.value)) == -2       # cols % 4

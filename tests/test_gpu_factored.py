@@ -146,3 +146,74 @@ def test_factored_rejects_bad_arguments(B):
     with pytest.raises(B.AlqError, match="WORKSPACE"):
         B.al_adafactor_step(x, x, 64, 64, c, m, c, m, 16, 128, None, None, 256, ADA_HP, 1,
                             ws[:16])
+
+
+def _fac_states(rows, cols, bits, block, came, seed):
+    """Zero factored states of one matrix (numpy), with its parameters."""
+    n = rows * cols
+    st = dict(p=wl.param_init((rows, cols), seed).ravel())
+    for k, ln in (("vr", rows), ("vc", cols)) + ((("cr", rows), ("cc", cols)) if came else ()):
+        c, m = _state(ln, bits, block)
+        st[k + "_codes"], st[k + "_meta"] = c, m
+    st["m_codes"] = np.zeros(n, np.int8)
+    st["m_absmax"] = np.zeros((n + 255) // 256, np.float32)
+    return st
+
+
+@pytest.mark.parametrize("op,mom,bits,block", [("adafactor", True, 16, 128),
+                                               ("adafactor", False, 8, 256),
+                                               ("came", True, 16, 128),
+                                               ("came", True, 8, 2048)])
+def test_grouped_factored_step_matches_single(B, op, mom, bits, block):
+    """The grouped step (one launch per pass over all matrices) gives every
+    matrix exactly the per-matrix step's parameters, codes and metadata."""
+    import torch
+    came = op == "came"
+    shapes = [(300, 772), (64, 512), (512, 1024), (130, 516), (257, 2048)]
+    single = [_fac_states(r, c, bits, block, came, 40 + i) for i, (r, c) in enumerate(shapes)]
+    dg = [{k: _t(v) for k, v in s_.items()} for s_ in single]
+    ds = [{k: _t(v) for k, v in s_.items()} for s_ in single]
+    grads = [torch.zeros(r * c, dtype=torch.float32, device="cuda") for r, c in shapes]
+    mats = []
+    for (r, c), d, g in zip(shapes, dg, grads):
+        m = dict(p=d["p"], g=g, rows=r, cols=c, vr_codes=d["vr_codes"], vr_meta=d["vr_meta"],
+                 vc_codes=d["vc_codes"], vc_meta=d["vc_meta"])
+        if came:
+            m.update(cr_codes=d["cr_codes"], cr_meta=d["cr_meta"], cc_codes=d["cc_codes"],
+                     cc_meta=d["cc_meta"])
+        if mom:
+            m.update(m_codes=d["m_codes"], m_absmax=d["m_absmax"])
+        mats.append(m)
+    plan = B.FactoredPlan(B.AL_OP_CAME if came else B.AL_OP_ADAFACTOR, mats, bits, block, bits,
+                          block, 256)
+    assert plan.info.nmat == len(shapes) and plan.info.has_momentum == int(mom)
+    wss = [torch.empty(B.al_workspace_size(B.AL_OP_CAME if came else B.AL_OP_ADAFACTOR, r, c),
+                       dtype=torch.uint8, device="cuda") for r, c in shapes]
+    for t in range(1, 4):
+        for i, (r, c) in enumerate(shapes):
+            grads[i].copy_(torch.from_numpy(
+                wl.student_t_grad((r, c), 1e-3, 3.0, 0.05, 900 + 10 * t + i).ravel()))
+        if came:
+            plan.step(CAME_HP, t)
+        else:
+            plan.step(ADA_HP, t)
+        for i, (r, c) in enumerate(shapes):
+            d = ds[i]
+            if came:
+                B.al_came_step(d["p"], grads[i], r, c, d["vr_codes"], d["vr_meta"], d["vc_codes"],
+                               d["vc_meta"], bits, block, d["cr_codes"], d["cr_meta"],
+                               d["cc_codes"], d["cc_meta"], bits, block, d["m_codes"],
+                               d["m_absmax"], 256, CAME_HP, t, wss[i])
+            else:
+                B.al_adafactor_step(d["p"], grads[i], r, c, d["vr_codes"], d["vr_meta"],
+                                    d["vc_codes"], d["vc_meta"], bits, block,
+                                    d["m_codes"] if mom else None,
+                                    d["m_absmax"] if mom else None, 256, ADA_HP, t, wss[i])
+        torch.cuda.synchronize()
+        for i in range(len(shapes)):
+            for k in dg[i]:
+                if not mom and k.startswith("m_"):
+                    continue
+                a = dg[i][k].cpu().numpy()
+                b = ds[i][k].cpu().numpy()
+                assert bytes_equal(a, b) == 0, (op, t, i, k)
