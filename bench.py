@@ -476,8 +476,9 @@ def _row_came(torch, np, wl, B, dev):
     and confidence C in AL16 blocks of 128, UF8 momentum in blocks of 256,
     gradients 1e-3 * Student-t(3) with 5% exact zeros. Algorithmic bytes: G
     read once (4), p read and written (8), momentum codes read and written
-    (2), absmax and the four factor states; the library's passes read G three
-    times and the momentum codes twice, which is not counted."""
+    (2), absmax and the four factor states; the library's passes read G four
+    times and the momentum codes twice, which is not counted. One grouped step
+    over the 22 matrices (al_came_step_multi: eight launches)."""
     cfg = wl.CONFIGS["came"]
     rows, cols = cfg["shape"]
     nm = cfg["n_mats"]
@@ -506,23 +507,25 @@ def _row_came(torch, np, wl, B, dev):
         mats.append(dict(p=p, gs=gs, vr=fac(rows, vb), vc=fac(cols, vb), cr=fac(rows, cb),
                          cc=fac(cols, cb), mc=torch.zeros(n1, dtype=torch.int8, device=dev),
                          ma=torch.zeros((n1 + 255) // 256, dtype=torch.float32, device=dev)))
-    # the matrices' steps are independent: spread them over a few streams
-    # (one workspace each) so that one matrix's short passes overlap with
-    # another's streaming passes
-    nstreams = int(os.environ.get("ALQ_BENCH_STREAMS", "8"))
-    streams = [torch.cuda.Stream(device=dev) for _ in range(nstreams)]
-    wss = [torch.empty(B.al_workspace_size(B.AL_OP_CAME, rows, cols), dtype=torch.uint8,
-                       device=dev) for _ in range(nstreams)]
+    # grouped steps (one launch per pass over a group of matrices), the
+    # groups on their own streams so that one group's latency-bound passes
+    # overlap another's streaming ones; one plan per group and gradient
+    # buffer (a plan binds its gradients)
+    ngroups = int(os.environ.get("ALQ_BENCH_GROUPS", "4"))
+    groups = [mats[i::ngroups] for i in range(ngroups)]
+    plans = [[B.FactoredPlan(B.AL_OP_CAME, [
+        dict(p=m["p"], g=m["gs"][k], rows=rows, cols=cols, vr_codes=m["vr"][0],
+             vr_meta=m["vr"][1], vc_codes=m["vc"][0], vc_meta=m["vc"][1], cr_codes=m["cr"][0],
+             cr_meta=m["cr"][1], cc_codes=m["cc"][0], cc_meta=m["cc"][1], m_codes=m["mc"],
+             m_absmax=m["ma"]) for m in grp], 16, vb, 16, cb, 256) for grp in groups]
+        for k in range(2)]
+    streams = [torch.cuda.Stream(device=dev) for _ in range(ngroups)]
 
     def step(t):
         main = torch.cuda.current_stream(dev)
-        for st in streams:
+        for st, plan in zip(streams, plans[t % 2]):
             st.wait_stream(main)
-        for i, m in enumerate(mats):
-            k = i % nstreams
-            B.al_came_step(m["p"], m["gs"][t % 2], rows, cols, m["vr"][0], m["vr"][1], m["vc"][0],
-                           m["vc"][1], 16, vb, m["cr"][0], m["cr"][1], m["cc"][0], m["cc"][1],
-                           16, cb, m["mc"], m["ma"], 256, hp, t, wss[k], stream=streams[k])
+            plan.step(hp, t, stream=st)
         for st in streams:
             main.wait_stream(st)
 
@@ -544,9 +547,10 @@ def _row_came(torch, np, wl, B, dev):
         dt = time.perf_counter() - t0
         return n1 / dt, f"one step of one {rows}x{cols} matrix ({dt:.1f} s, single thread)"
 
-    return dict(step=step, n=nm * n1, bytes=nbytes, launches=9 * nm, oracle=oracle_sample,
+    return dict(step=step, n=nm * n1, bytes=nbytes, launches=8 * ngroups, oracle=oracle_sample,
                 workload=f"CAME {nm} x {rows}x{cols}, AL16 factored V and C block 128, "
-                         f"UF8 momentum block 256, matrices spread over {nstreams} streams",
+                         f"UF8 momentum block 256, grouped steps (al_came_step_multi) over "
+                         f"{ngroups} groups of matrices on {ngroups} streams",
                 bytes_note="algorithmic minimum 14.03 B/param (G read once)")
 
 

@@ -373,7 +373,8 @@ typedef struct {
     int64_t factor_tiles; /* factor blocks (rows and columns) of V           */
     int64_t factor2_tiles;/* factor blocks of CAME's confidence (else 0)     */
     int64_t scale_tiles;  /* 256-entry tiles of the scale passes             */
-    int64_t tiles;        /* 4096-parameter tiles of the RMS and update      */
+    int64_t tiles;        /* 4096-parameter tiles of the update              */
+    int64_t rms_chunks;   /* 8-tile chunks of the RMS pass (one partial each) */
     void* workspace;      /* the workspace the plan is bound to              */
 } al_factored_info;
 

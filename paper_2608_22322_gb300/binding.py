@@ -91,7 +91,8 @@ class FactoredInfo(C.Structure):
                 ("m_block", C.c_int32), ("has_momentum", C.c_int32),
                 ("total_params", C.c_int64), ("sumsq_tiles", C.c_int64),
                 ("factor_tiles", C.c_int64), ("factor2_tiles", C.c_int64),
-                ("scale_tiles", C.c_int64), ("tiles", C.c_int64), ("workspace", C.c_void_p)]
+                ("scale_tiles", C.c_int64), ("tiles", C.c_int64), ("rms_chunks", C.c_int64),
+                ("workspace", C.c_void_p)]
 
 
 class MultiInfo(C.Structure):

@@ -31,12 +31,13 @@ namespace alq {
 
 constexpr int kFR = 64;   // rows per sumsq tile
 constexpr int kFC = 512;  // columns per sumsq tile
+constexpr int kUsqChunk = 8;  // tiles of kTile elements per RMS partial
 
 // ------------------------------------------------------------ workspace --
 struct FacWs {
     double* rowpart;  // [ncb][rows]
     double* colpart;  // [nrb][cols]
-    double* upart;    // [tiles of kTile elements]: RMS partials
+    double* upart;    // [chunks of kUsqChunk tiles]: RMS partials
     float* fr;        // fresh row factor (V)
     float* fc;        // fresh column factor (V)
     float* fr2;       // fresh row factor (C)
@@ -66,7 +67,7 @@ static FacWs fac_layout(void* base, int64_t rows, int64_t cols) {
     };
     w.rowpart = (double*)take(sizeof(double) * ncb * rows);
     w.colpart = (double*)take(sizeof(double) * nrb * cols);
-    w.upart = (double*)take(sizeof(double) * blocks_of(rows * cols, kTile));
+    w.upart = (double*)take(sizeof(double) * blocks_of(blocks_of(rows * cols, kTile), kUsqChunk));
     w.fr = (float*)take(sizeof(float) * rows);
     w.fc = (float*)take(sizeof(float) * cols);
     w.fr2 = (float*)take(sizeof(float) * rows);
@@ -93,6 +94,7 @@ struct ResidualArgs {
     const float* b;
     const float* scal;  // scal[0] = 1 / max(1, RMS(u)/d)
     float beta1, omb1, eps2;
+    float one, zero;    // 1 and 0 from the kernel's parameters (see ff_sq2)
 };
 
 // ----------------------------------------------------------------- sumsq --
@@ -104,12 +106,16 @@ template <int MODE>
 __device__ __forceinline__ void sumsq_tile(const float* __restrict__ g, int rows, int cols,
                                            const ResidualArgs& ra, double* __restrict__ rowpart,
                                            double* __restrict__ colpart, int bx, int by,
-                                           double (*s_col)[kFC]) {
+                                           float2 (*s_col)[kFC]) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int c0 = bx * kFC, r0 = by * kFR;
-    float ch[16], cl[16];
+    // column sums of this lane's 16 columns as 8 pairs; each row's sum as
+    // two (even and odd elements) merged before the warp sum
+    float2 ch[8], cl[8];
 #pragma unroll
-    for (int k = 0; k < 16; ++k) ch[k] = cl[k] = 0.0f;
+    for (int k = 0; k < 8; ++k) ch[k] = cl[k] = make_float2(0.0f, 0.0f);
+    const float2 one = make_float2(ra.one, ra.one), zero = make_float2(ra.zero, ra.zero);
+    const float2 neg = make_float2(-1.0f, -1.0f);
     float icf = 0.0f;
     float4 bv[4];  // column scales of this lane's columns (CAME residual)
     if (MODE == 1) {
@@ -121,8 +127,11 @@ __device__ __forceinline__ void sumsq_tile(const float* __restrict__ g, int rows
                                : make_float4(0.f, 0.f, 0.f, 0.f);
         }
     }
+    // this warp's eight row sums, row k's in lane k, converted to fp64 in
+    // one instruction at the end (FP64 is slow on this part)
+    float keep_h = 0.0f, keep_l = 0.0f;
     // two rows per pass: all loads first (zero past the matrix), then the
-    // terms in row order, so the sums keep the order of a row-by-row walk
+    // terms in row order
     for (int rr = 0; rr < kFR / 8; rr += 2) {
         float4 gv[2][4];
         uint32_t mw[2][4];
@@ -150,50 +159,75 @@ __device__ __forceinline__ void sumsq_tile(const float* __restrict__ g, int rows
 #pragma unroll
         for (int q = 0; q < 2; ++q) {
             const int row = r0 + warp + 8 * (rr + q);
-            float rh = 0.0f, rl = 0.0f;
+            float2 rh2 = make_float2(0.0f, 0.0f), rl2 = make_float2(0.0f, 0.0f);
             if (row < rows) {
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
                     const int col = c0 + 128 * k + 4 * lane;
                     if (col < cols) {
+                        const uint32_t mx = mw[q][k] ^ 0x80808080u;
 #pragma unroll
-                        for (int j = 0; j < 4; ++j) {
-                            const float x = f4get(gv[q][k], j);
-                            float h, l;
+                        for (int jp = 0; jp < 2; ++jp) {
+                            const float2 x = jp == 0 ? make_float2(gv[q][k].x, gv[q][k].y)
+                                                     : make_float2(gv[q][k].z, gv[q][k].w);
+                            float2 h, nl;
                             if (MODE == 0) {
-                                two_prod(x, x, h, l);
+                                ff_sq2(x, neg, zero, h, nl);
                             } else {
-                                const float u = (x * ai[q]) * f4get(bv[k], j);
-                                const float uh = u * icf;
-                                const float mh = s8_to_float((mw[q][k] >> (8 * j)) & 0xFFu) * dm[q][k];
-                                const float mk = ra.beta1 * mh + ra.omb1 * uh;
-                                const float d = uh - mk;
-                                h = d * d + ra.eps2;
-                                l = 0.0f;
+                                // the update's residual, each product rounded
+                                // before it enters a sum (opaque one)
+                                const float2 bj = jp == 0 ? make_float2(bv[k].x, bv[k].y)
+                                                          : make_float2(bv[k].z, bv[k].w);
+                                const float2 u = mul2(mul2(x, make_float2(ai[q], ai[q])), bj);
+                                const float2 uh = mul2(u, make_float2(icf, icf));
+                                const float2 qf = make_float2(
+                                    u2f(__byte_perm(mx, 0x4B400000u, 0x7640u | (2 * jp))),
+                                    u2f(__byte_perm(mx, 0x4B400000u, 0x7640u | (2 * jp + 1))));
+                                const float2 mh = mul2(add2(qf, make_float2(-12583040.0f, -12583040.0f)),
+                                                       make_float2(dm[q][k], dm[q][k]));
+                                const float2 nmk = fma2(mul2(make_float2(-ra.beta1, -ra.beta1), mh), one,
+                                                        mul2(make_float2(-ra.omb1, -ra.omb1), uh));
+                                const float2 d = fma2(uh, one, nmk);  // uh - mk
+                                h = fma2(mul2(d, d), one, make_float2(ra.eps2, ra.eps2));
+                                nl = make_float2(0.0f, 0.0f);
                             }
-                            ff_acc(ch[4 * k + j], cl[4 * k + j], h, l);
-                            ff_acc(rh, rl, h, l);
+                            ff_acc2(ch[2 * k + jp], cl[2 * k + jp], h, nl);
+                            ff_acc2(rh2, rl2, h, nl);
                         }
                     }
                 }
             }
+            float rh, rl;
+            ff_merge2(rh2, rl2, rh, rl);
             ff_warp_sum(rh, rl);
-            if (lane == 0 && row < rows)
-                rowpart[(int64_t)bx * rows + row] = (double)rh + (double)rl;
+            if (lane == rr + q) {
+                keep_h = rh;
+                keep_l = rl;
+            }
         }
     }
+    {
+        const int row = r0 + warp + 8 * lane;  // lane k holds row warp + 8 k
+        if (lane < kFR / 8 && row < rows)
+            rowpart[(int64_t)bx * rows + row] = (double)keep_h + (double)keep_l;
+    }
+    // column sums: the warps' two-float sums merged in warp order, one fp64
+    // conversion per column
 #pragma unroll
     for (int k = 0; k < 4; ++k)
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
-            s_col[warp][128 * k + 4 * lane + j] = (double)ch[4 * k + j] + (double)cl[4 * k + j];
+        for (int jp = 0; jp < 2; ++jp) {
+            const float2 h = ch[2 * k + jp], l = cl[2 * k + jp];
+            s_col[warp][128 * k + 4 * lane + 2 * jp] = make_float2(h.x, l.x);
+            s_col[warp][128 * k + 4 * lane + 2 * jp + 1] = make_float2(h.y, l.y);
+        }
     __syncthreads();
     for (int t = threadIdx.x; t < kFC; t += kThreads) {
         if (c0 + t >= cols) continue;
-        double s = 0.0;
+        float hi = s_col[0][t].x, lo = s_col[0][t].y;
 #pragma unroll
-        for (int w = 0; w < kThreads / 32; ++w) s += s_col[w][t];
-        colpart[(int64_t)by * cols + c0 + t] = s;
+        for (int w = 1; w < kThreads / 32; ++w) ff_acc(hi, lo, s_col[w][t].x, s_col[w][t].y);
+        colpart[(int64_t)by * cols + c0 + t] = (double)hi + (double)lo;
     }
 }
 
@@ -201,7 +235,7 @@ template <int MODE>
 __global__ void __launch_bounds__(kThreads)
 sumsq_kernel(const float* __restrict__ g, int rows, int cols, ResidualArgs ra,
              double* __restrict__ rowpart, double* __restrict__ colpart) {
-    __shared__ double s_col[kThreads / 32][kFC];
+    __shared__ float2 s_col[kThreads / 32][kFC];
     sumsq_tile<MODE>(g, rows, cols, ra, rowpart, colpart, blockIdx.x, blockIdx.y, s_col);
 }
 
@@ -353,10 +387,11 @@ scale_kernel(const float* __restrict__ R, int rows, const float* __restrict__ C,
 
 // ------------------------------------------------------------------- usq --
 // Sum of u^2, u = (g a_i) b_j, over the whole matrix: exact squares in
-// two-float per thread, fixed warp/CTA order, one fp64 partial per tile.
-// The CTA that finishes a matrix's last tile (an atomic ticket, zeroed by
-// the scale pass) adds the partials in tile order and writes the clip factor
-// scal[0] = 1 / max(1, sqrt(sum / count) / clip_d).
+// two-float per thread, fixed warp/CTA order, one fp64 partial per chunk of
+// kUsqChunk tiles (4096 elements each, a partition of the matrix that does
+// not depend on the grid). The CTA that finishes a matrix's last chunk (an
+// atomic ticket, zeroed by the scale pass) adds the partials in chunk order
+// and writes the clip factor scal[0] = 1 / max(1, sqrt(sum / count) / clip_d).
 struct UsqArgs {
     const float* g;
     int64_t n;
@@ -366,65 +401,79 @@ struct UsqArgs {
     double* upart;
     unsigned int* ticket;
     float* scal;
+    float zero;  // 0 from the kernel's parameters (see ff_sq2)
 };
 
-// The tile's partial (every thread of the CTA calls it; thread 0 returns it).
-__device__ __forceinline__ double usq_tile_sum(const UsqArgs& q, int64_t tile, double* s_w) {
+__device__ __forceinline__ int64_t usq_chunks(int64_t n) {
+    return blocks_of_dev(blocks_of_dev(n, kTile), kUsqChunk);
+}
+
+// The chunk's partial (every thread of the CTA calls it; thread 0 gets it).
+__device__ __forceinline__ double usq_chunk_sum(const UsqArgs& q, int64_t chunk, float2* s_w) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    float hi = 0.0f, lo = 0.0f;
-    const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
+    const float2 zero = make_float2(q.zero, q.zero), neg = make_float2(-1.0f, -1.0f);
+    float2 hi2 = make_float2(0.0f, 0.0f), lo2 = make_float2(0.0f, 0.0f);
+    for (int k = 0; k < kUsqChunk; ++k) {
+        const int64_t seg0 = (chunk * kUsqChunk + k) * kTile + (int64_t)warp * kSeg;
+        if (seg0 >= q.n) break;
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-        const int64_t idx = chunk_index(seg0, c, lane);
-        if (idx < q.n) {
-            const uint32_t row = divide((uint32_t)idx, q.dv);
-            const uint32_t col = (uint32_t)idx - row * q.dv.d;
-            const float4 gv = __ldcs(reinterpret_cast<const float4*>(q.g + idx));
-            const float4 bv = __ldg(reinterpret_cast<const float4*>(q.b + col));
-            const float ai = __ldg(q.a + row);
+        for (int c = 0; c < 4; ++c) {
+            const int64_t idx = chunk_index(seg0, c, lane);
+            if (idx < q.n) {
+                const uint32_t row = divide((uint32_t)idx, q.dv);
+                const uint32_t col = (uint32_t)idx - row * q.dv.d;
+                const float4 gv = __ldcs(reinterpret_cast<const float4*>(q.g + idx));
+                const float4 bv = __ldg(reinterpret_cast<const float4*>(q.b + col));
+                const float2 ai = make_float2(__ldg(q.a + row), __ldg(q.a + row));
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const float u = (f4get(gv, j) * ai) * f4get(bv, j);
-                float h, l;
-                two_prod(u, u, h, l);
-                ff_acc(hi, lo, h, l);
+                for (int jp = 0; jp < 2; ++jp) {
+                    const float2 x = jp == 0 ? make_float2(gv.x, gv.y) : make_float2(gv.z, gv.w);
+                    const float2 bj = jp == 0 ? make_float2(bv.x, bv.y) : make_float2(bv.z, bv.w);
+                    ff_acc_sq2(hi2, lo2, mul2(mul2(x, ai), bj), neg, zero);  // u = (g a_i) b_j
+                }
             }
         }
     }
+    float hi, lo;
+    ff_merge2(hi2, lo2, hi, lo);
     ff_warp_sum(hi, lo);
-    __syncthreads();  // s_w may still be read by the previous tile's finish
-    if (lane == 0) s_w[warp] = (double)hi + (double)lo;
+    __syncthreads();  // s_w may still be read by the previous chunk's finish
+    if (lane == 0) s_w[warp] = make_float2(hi, lo);
     __syncthreads();
     double t = 0.0;
-    if (threadIdx.x == 0)
-        for (int w = 0; w < kThreads / 32; ++w) t += s_w[w];
+    if (threadIdx.x == 0) {
+        float h = s_w[0].x, l = s_w[0].y;
+        for (int w = 1; w < kThreads / 32; ++w) ff_acc(h, l, s_w[w].x, s_w[w].y);
+        t = (double)h + (double)l;
+    }
     return t;
 }
 
-// One tile of the RMS pass: its partial, and the clip factor if this CTA
-// completes the matrix (ntiles tiles).
-__device__ __forceinline__ void usq_tile(const UsqArgs& q, int64_t tile, int64_t ntiles,
-                                         float clip_d, double* s_w, bool* s_last) {
-    const double t = usq_tile_sum(q, tile, s_w);
+// One chunk of the RMS pass: its partial, and the clip factor if this CTA
+// completes the matrix.
+__device__ __forceinline__ void usq_chunk(const UsqArgs& q, int64_t chunk, float clip_d,
+                                          float2* s_w, double* s_d, bool* s_last) {
+    const int64_t nchunks = usq_chunks(q.n);
+    const double t = usq_chunk_sum(q, chunk, s_w);
     if (threadIdx.x == 0) {
-        q.upart[tile] = t;
+        q.upart[chunk] = t;
         __threadfence();
-        *s_last = atomicAdd(q.ticket, 1u) == (unsigned int)(ntiles - 1);
+        *s_last = atomicAdd(q.ticket, 1u) == (unsigned int)(nchunks - 1);
     }
     __syncthreads();
     if (!*s_last) return;
     __threadfence();
     // fixed order: per thread over a stride of kThreads, then a tree
     double acc = 0.0;
-    for (int64_t i = threadIdx.x; i < ntiles; i += kThreads) acc += ((volatile double*)q.upart)[i];
-    s_w[threadIdx.x] = acc;
+    for (int64_t i = threadIdx.x; i < nchunks; i += kThreads) acc += ((volatile double*)q.upart)[i];
+    s_d[threadIdx.x] = acc;
     __syncthreads();
     for (int st = kThreads / 2; st > 0; st >>= 1) {
-        if ((int)threadIdx.x < st) s_w[threadIdx.x] += s_w[threadIdx.x + st];
+        if ((int)threadIdx.x < st) s_d[threadIdx.x] += s_d[threadIdx.x + st];
         __syncthreads();
     }
     if (threadIdx.x == 0) {
-        const double rms = sqrt(s_w[0] / (double)q.n);
+        const double rms = sqrt(s_d[0] / (double)q.n);
         double cf = rms / (double)clip_d;
         if (cf < 1.0) cf = 1.0;
         q.scal[0] = (float)(1.0 / cf);
@@ -432,11 +481,13 @@ __device__ __forceinline__ void usq_tile(const UsqArgs& q, int64_t tile, int64_t
 }
 
 __global__ void __launch_bounds__(kThreads)
-usq_kernel(UsqArgs q, int64_t ntiles, float clip_d) {
-    __shared__ double s_w[kThreads];
+usq_kernel(UsqArgs q, float clip_d) {
+    __shared__ float2 s_w[kThreads / 32];
+    __shared__ double s_d[kThreads];
     __shared__ bool s_last;
-    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x)
-        usq_tile(q, tile, ntiles, clip_d, s_w, &s_last);
+    const int64_t nchunks = usq_chunks(q.n);
+    for (int64_t chunk = blockIdx.x; chunk < nchunks; chunk += gridDim.x)
+        usq_chunk(q, chunk, clip_d, s_w, s_d, &s_last);
 }
 
 
@@ -635,6 +686,7 @@ static int second_moment_passes(const float* g, int64_t rows, int64_t cols, cons
                                 float* a, float* b) {
     const int ncb = (int)blocks_of(cols, kFC), nrb = (int)blocks_of(rows, kFR);
     ResidualArgs none{};
+    none.one = 1.0f;
     sumsq_kernel<0><<<dim3(ncb, nrb), kThreads, 0, st>>>(g, (int)rows, (int)cols, none,
                                                         w.rowpart, w.colpart);
     const int nb0 = (int)blocks_of(rows, fr.block);
@@ -643,9 +695,10 @@ static int second_moment_passes(const float* g, int64_t rows, int64_t cols, cons
         fr.fresh, (int)rows, fc.fresh, (int)cols, w.rsum, nb0, a, b, w.ticket);
     const int64_t n = rows * cols;
     const int64_t ntiles = blocks_of(n, kTile);
-    const UsqArgs q{g, n, make_divider((uint32_t)cols), a, b, w.upart, w.ticket, w.scal};
-    usq_kernel<<<persistent_grid((const void*)usq_kernel, kThreads, 0, ntiles), kThreads, 0, st>>>(
-        q, ntiles, clip_d);
+    const UsqArgs q{g, n, make_divider((uint32_t)cols), a, b, w.upart, w.ticket, w.scal, 0.0f};
+    const int64_t nchunks = blocks_of(ntiles, kUsqChunk);
+    usq_kernel<<<persistent_grid((const void*)usq_kernel, kThreads, 0, nchunks), kThreads, 0, st>>>(
+        q, clip_d);
     return check_launch();
 }
 
@@ -745,7 +798,7 @@ int al_came_step(float* p, const float* g, int64_t rows, int64_t cols, void* vr_
 
     // residual (u_hat - m)^2 + eps2 from the old momentum codes, its factored
     // confidence (beta3) and the confidence scales
-    ResidualArgs ra{m_codes, m_absmax, 0, w.a, w.b, w.scal, hp->beta1, omb1, hp->eps2};
+    ResidualArgs ra{m_codes, m_absmax, 0, w.a, w.b, w.scal, hp->beta1, omb1, hp->eps2, 1.0f, 0.0f};
     while ((1 << ra.m_shift) < m_block) ++ra.m_shift;
     sumsq_kernel<1><<<dim3(ncb, nrb), kThreads, 0, s>>>(g, (int)rows, (int)cols, ra, w.rowpart,
                                                        w.colpart);
@@ -813,7 +866,7 @@ struct FacEntry {
     float* m_absmax;
     FacWs w;
     int32_t ncb, nrb;  // the sums passes' tile grid (columns, rows)
-    int64_t sq_t0, fac_t0, fac2_t0, sc_t0, usq_t0, upd_t0;
+    int64_t sq_t0, fac_t0, fac2_t0, sc_t0, usq_t0, upd_t0;  // usq_t0 in RMS chunks
 };
 
 // Per-step scalars of the grouped passes.
@@ -826,6 +879,7 @@ struct FacStep {
     float log_floor_v, log_floor_c;
     float clip_d;
     float beta1, omb1, eps2, decay, lr;
+    float one, zero;  // opaque 1 and 0 for the paired sums (see ff_sq2)
 };
 
 // The entry whose pass (first tile t0) holds a launch-wide tile: entries are
@@ -850,13 +904,15 @@ __device__ __forceinline__ int fac_advance(const FacEntry* __restrict__ tab, int
 template <int MODE>
 __global__ void __launch_bounds__(kThreads)
 sumsq_multi_kernel(const FacEntry* __restrict__ tab, int nmat, FacStep fs) {
-    __shared__ double s_col[kThreads / 32][kFC];
+    __shared__ float2 s_col[kThreads / 32][kFC];
     const FacEntry& e = fac_entry(tab, nmat, blockIdx.x, &FacEntry::sq_t0);
     const int64_t lt = blockIdx.x - e.sq_t0;
     ResidualArgs ra{};
     if (MODE == 1)
         ra = ResidualArgs{e.m_codes, e.m_absmax, fs.m_shift, e.w.a, e.w.b, e.w.scal,
-                          fs.beta1, fs.omb1, fs.eps2};
+                          fs.beta1, fs.omb1, fs.eps2, fs.one, fs.zero};
+    ra.one = fs.one;
+    ra.zero = fs.zero;
     sumsq_tile<MODE>(e.g, (int)e.rows, (int)e.cols, ra, e.w.rowpart, e.w.colpart,
                      (int)(lt % e.ncb), (int)(lt / e.ncb), s_col);
 }
@@ -901,15 +957,17 @@ scale_multi_kernel(const FacEntry* __restrict__ tab, int nmat, FacStep fs, int w
 }
 
 __global__ void __launch_bounds__(kThreads)
-usq_multi_kernel(const FacEntry* __restrict__ tab, int nmat, int64_t ntiles, float clip_d) {
-    __shared__ double s_w[kThreads];
+usq_multi_kernel(const FacEntry* __restrict__ tab, int nmat, int64_t nchunks, float clip_d,
+                 float zero) {
+    __shared__ float2 s_w[kThreads / 32];
+    __shared__ double s_d[kThreads];
     __shared__ bool s_last;
     int cur = 0;
-    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-        cur = fac_advance(tab, nmat, tile, cur, &FacEntry::usq_t0);
+    for (int64_t chunk = blockIdx.x; chunk < nchunks; chunk += gridDim.x) {
+        cur = fac_advance(tab, nmat, chunk, cur, &FacEntry::usq_t0);
         const FacEntry& e = tab[cur];
-        const UsqArgs q{e.g, e.n, e.dv, e.w.a, e.w.b, e.w.upart, e.w.ticket, e.w.scal};
-        usq_tile(q, tile - e.usq_t0, e.ntiles, clip_d, &s_w[0], &s_last);
+        const UsqArgs q{e.g, e.n, e.dv, e.w.a, e.w.b, e.w.upart, e.w.ticket, e.w.scal, zero};
+        usq_chunk(q, chunk - e.usq_t0, clip_d, s_w, s_d, &s_last);
     }
 }
 
@@ -992,8 +1050,8 @@ static void second_moment_multi(const FacEntry* tab, const al_factored_info* inf
     sumsq_multi_kernel<0><<<(unsigned)info->sumsq_tiles, kThreads, 0, st>>>(tab, info->nmat, fs);
     factor_multi(tab, info->nmat, fs, 0, info->factor_tiles, st);
     scale_multi_kernel<<<(unsigned)info->scale_tiles, kThreads, 0, st>>>(tab, info->nmat, fs, 0);
-    usq_multi_kernel<<<persistent_grid((const void*)usq_multi_kernel, kThreads, 0, info->tiles),
-                       kThreads, 0, st>>>(tab, info->nmat, info->tiles, fs.clip_d);
+    usq_multi_kernel<<<persistent_grid((const void*)usq_multi_kernel, kThreads, 0, info->rms_chunks),
+                       kThreads, 0, st>>>(tab, info->nmat, info->rms_chunks, fs.clip_d, fs.zero);
 }
 
 static int check_multi_call(const void* plan_dev, const al_factored_info* info, int op) {
@@ -1086,13 +1144,14 @@ int al_factored_plan(int op, const al_factored_matrix* mats, int nmat, int v_bit
         e.fac_t0 = info->factor_tiles;
         e.fac2_t0 = info->factor2_tiles;
         e.sc_t0 = info->scale_tiles;
-        e.usq_t0 = info->tiles;
+        e.usq_t0 = info->rms_chunks;
         e.upd_t0 = info->tiles;
         info->sumsq_tiles += (int64_t)e.ncb * e.nrb;
         info->factor_tiles += blocks_of(m.rows, v_block) + blocks_of(m.cols, v_block);
         if (came) info->factor2_tiles += blocks_of(m.rows, c_block) + blocks_of(m.cols, c_block);
         info->scale_tiles += blocks_of(m.rows + m.cols, kThreads);
         info->tiles += e.ntiles;
+        info->rms_chunks += blocks_of(e.ntiles, kUsqChunk);
         info->total_params += e.n;
         memcpy(base + kFacEntryOffset + (size_t)i * sizeof(FacEntry), &e, sizeof(e));
     }
@@ -1134,6 +1193,7 @@ int al_adafactor_step_multi(const void* plan_dev, const al_factored_info* info,
     fs.omb1 = (float)(1.0 - (double)hp->beta1);
     fs.decay = (float)(1.0 - (double)hp->lr * (double)hp->weight_decay);
     fs.lr = hp->lr;
+    fs.one = 1.0f;
     second_moment_multi(tab, info, fs, st);
     if (info->has_momentum)
         update_multi<1>(tab, info->nmat, info->tiles, fs, st);
@@ -1171,6 +1231,7 @@ int al_came_step_multi(const void* plan_dev, const al_factored_info* info, const
     fs.omb1 = (float)(1.0 - (double)hp->beta1);
     fs.decay = (float)(1.0 - (double)hp->lr * (double)hp->weight_decay);
     fs.lr = hp->lr;
+    fs.one = 1.0f;
     second_moment_multi(tab, info, fs, st);
     // residual sums, confidence factors and their scales, update
     sumsq_multi_kernel<1><<<(unsigned)info->sumsq_tiles, kThreads, 0, st>>>(tab, info->nmat, fs);

@@ -467,21 +467,37 @@ __device__ __forceinline__ void ff_acc(float& hi, float& lo, float h, float l) {
     lo = lo + (e + l);
 }
 
-// Two-float accumulation of the exact squares of a pair of values (two
-// independent sums): x^2 = h + l with h = RN(x x) and -l = RN(h - x x)
-// (exact), then Knuth's TwoSum of hi and h; neg = (-1, -1). h is a fused
-// multiply-add with zero, a value the compiler cannot see (from the
-// kernel's parameters): a paired product feeding the sums could otherwise
-// be contracted into them.
-__device__ __forceinline__ void ff_acc_sq2(float2& hi, float2& lo, float2 x, float2 neg,
-                                           float2 zero) {
-    const float2 h = fma2(x, x, zero);
-    const float2 nl = fma2(mul2(x, neg), x, h);
+// Paired two-float accumulation (two independent sums): adds h + l, given
+// h and nl = -l, to (hi, lo) by Knuth's TwoSum of hi and h.
+__device__ __forceinline__ void ff_acc2(float2& hi, float2& lo, float2 h, float2 nl) {
     const float2 s = add2(hi, h);
     const float2 bb = sub2(s, hi);
     const float2 e = add2(sub2(hi, sub2(s, bb)), sub2(h, bb));
     hi = s;
     lo = add2(lo, sub2(e, nl));
+}
+
+// Exact squares of a pair of values: x^2 = h + l with h = RN(x x) and
+// nl = -l = RN(h - x x) (exact); neg = (-1, -1). h is a fused multiply-add
+// with zero, a value the compiler cannot see (from the kernel's parameters):
+// a paired product feeding the sums could otherwise be contracted into them.
+__device__ __forceinline__ void ff_sq2(float2 x, float2 neg, float2 zero, float2& h, float2& nl) {
+    h = fma2(x, x, zero);
+    nl = fma2(mul2(x, neg), x, h);
+}
+
+__device__ __forceinline__ void ff_acc_sq2(float2& hi, float2& lo, float2 x, float2 neg,
+                                           float2 zero) {
+    float2 h, nl;
+    ff_sq2(x, neg, zero, h, nl);
+    ff_acc2(hi, lo, h, nl);
+}
+
+// The two sums of a pair merged into one (hi, lo).
+__device__ __forceinline__ void ff_merge2(float2 hi2, float2 lo2, float& hi, float& lo) {
+    hi = hi2.x;
+    lo = lo2.x;
+    ff_acc(hi, lo, hi2.y, lo2.y);
 }
 
 __device__ __forceinline__ void ff_warp_sum(float& hi, float& lo) {

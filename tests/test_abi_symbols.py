@@ -102,6 +102,7 @@ def test_grouped_factored_plan_host_logic(lib):
     assert info.factor2_tiles == info.factor_tiles
     assert info.scale_tiles == sum(tiles(r + c, 256) for r, c in shapes)
     assert info.tiles == sum(tiles(r * c, 4096) for r, c in shapes)
+    assert info.rms_chunks == sum(tiles(tiles(r * c, 4096), 8) for r, c in shapes)
     assert lib.al_factored_plan(*args(2, arr, ws.value - 1)) == -4   # workspace too small
     assert lib.al_factored_plan(*args(3, arr, ws.value)) == -1       # not a factored op
     # momentum in some matrices only; CAME without momentum; no confidence
