@@ -74,7 +74,8 @@ static __device__ __noinline__ void store_codes_masked(int8_t* m_codes, void* v_
 // parameter space costs no registers.
 struct AdamWPairs {
     float2 decay, nstep, c2, omb1, omb2, beta1, beta2, eps;
-    float2 one;  // (1, 1), opaque to the compiler: f * one + c rounds as f + c
+    float2 one;   // (1, 1) and (0, 0), opaque to the compiler: f * one + c
+    float2 zero;  // rounds as f + c, fma(x, y, zero) as x y
     float log_floor;
 };
 
@@ -89,6 +90,7 @@ static AdamWPairs adamw_pairs(const AdamWScalars& s) {
     q.beta2 = make_float2(s.beta2, s.beta2);
     q.eps = make_float2(s.eps, s.eps);
     q.one = make_float2(1.0f, 1.0f);
+    q.zero = make_float2(0.0f, 0.0f);
     q.log_floor = s.log_floor;
     return q;
 }
@@ -113,13 +115,14 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
     constexpr int NBM = kCH / CPBM;
     constexpr int NE = 4 * kCH;
     constexpr float Lm2 = VBITS == 8 ? 254.0f : 65534.0f;
-    __shared__ __align__(16) float2 s_tab[kThreads / 32][NBV * 32];
+    __shared__ __align__(16) float2 s_tab[kThreads / 32][1][NBV * 32];
     __shared__ float s_val[kThreads / 32][VBITS == 8 ? NBV * 256 : 1];
     __shared__ uint32_t s_part[2][3][kThreads / 32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int wpbv = v_block > kASeg ? v_block / kASeg : 1;
     const int wpbm = m_block > kASeg ? m_block / kASeg : 1;
     const float kf = al8_table_k(lane);
+    const Opaque2 ok2{s.one, s.zero};
     const int G = gridDim.x;
     int cur = 0;
     int parity = 0;  // slot of the next cross-warp block reduction
@@ -181,7 +184,14 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
         // ---- decode the previous states
         float vh[NE];
         if constexpr (VBITS == 8) {
-            al8_build_values<NBV>(s_val[warp], s_tab[warp], olmin, odelta, kf);
+            if constexpr (NBV == 1) {
+                al8_build_values<1>(s_val[warp], s_tab[warp][0], olmin, odelta, kf);
+            } else {
+                // two blocks per segment: their levels in one paired pass
+                al8_build_tables2(s_tab[warp][0], s_tab[warp][0] + 32, olmin[0], odelta[0],
+                                  olmin[1], odelta[1], kf, ok2);
+                al8_values_from_tables<NBV>(s_val[warp], s_tab[warp][0], olmin, odelta);
+            }
 #pragma unroll
             for (int e = 0; e < NE; ++e)
                 vh[e] = s_val[warp][256 * (e / 4 / CPBV) + ((vw[e / 4] >> (8 * (e % 4))) & 0xFFu)];

@@ -85,7 +85,7 @@ al_encode_kernel(const float* __restrict__ x, int64_t n, int block, float log_fl
 template <int CPB, int BITS>
 __global__ void __launch_bounds__(kThreads)
 al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta, int64_t n,
-                 int block, float* __restrict__ out, int64_t ntiles) {
+                 int block, float* __restrict__ out, int64_t ntiles, Opaque2 k) {
     constexpr int NB = 4 / CPB;
     __shared__ __align__(16) float2 s_tab[kThreads / 32][NB * 32];
     __shared__ float s_val[kThreads / 32][BITS == 8 ? NB * 256 : 1];
@@ -118,7 +118,12 @@ al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta,
         }
         // AL8: the blocks' 256 exactly rounded values in shared memory, then
         // one lookup per element; AL16: each level directly
-        if constexpr (BITS == 8) al8_build_values<NB>(s_val[warp], s_tab[warp], lmin, delta, kf);
+        if constexpr (BITS == 8) {
+            if constexpr (NB >= 2)
+                al8_build_values_paired<NB>(s_val[warp], s_tab[warp], lmin, delta, kf, k);
+            else
+                al8_build_values<NB>(s_val[warp], s_tab[warp], lmin, delta, kf);
+        }
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
             const int b = c / CPB;
@@ -265,7 +270,9 @@ int al_decode(const void* codes, const float* meta, int64_t n, int block, int bi
     if (!aligned(out, 16) || !aligned(codes, 16) || !aligned(meta, 8)) return ALQ_ERR_ALIGN;
     const int64_t ntiles = blocks_of(n, kTile);
     cudaStream_t s = (cudaStream_t)stream;
-#define LAUNCH(k) k<<<grid_for(k, ntiles), kThreads, 0, s>>>(codes, meta, n, block, out, ntiles)
+#define LAUNCH(k)                                                                      \
+    k<<<grid_for(k, ntiles), kThreads, 0, s>>>(codes, meta, n, block, out, ntiles,         \
+                                               Opaque2{make_float2(1.0f, 1.0f), make_float2(0.0f, 0.0f)})
     if (bits == 8) {
         ALQ_DISPATCH_CPB(block, al_decode_kernel, , 8)
     } else {

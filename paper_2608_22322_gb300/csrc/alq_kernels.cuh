@@ -236,6 +236,107 @@ __device__ __forceinline__ bool al8_fast_ok(float lmin, float delta) {
     return delta > 0.0f && lmin >= -96.0f;
 }
 
+// ------------------------------------------- paired two-float AL levels --
+// al_level_ff (alq_numerics.h) for two (l_min, Delta) at once, step for step
+// in paired instructions: every rounding of the scalar routine happens here
+// too (the steps that routine documents as exact may fuse), so the results
+// are the scalar ones. A product that enters a sum is formed by a fused
+// multiply-add with zero, or enters it through a fused multiply-add by one,
+// both values the compiler cannot see (k.x, k.y from the kernel's
+// parameters): a paired product feeding a paired add could otherwise be
+// contracted. The table lookups and the integer parts stay scalar.
+struct Opaque2 {
+    float2 one, zero;
+};
+
+__device__ __forceinline__ float2 rint_small2(float2 x, const Opaque2& k, int& i0, int& i1) {
+    const float2 magic = make_float2(12582912.0f, 12582912.0f);
+    const float2 r = fma2(x, k.one, magic);
+    i0 = (int)(f2u(r.x) - 0x4B400000u);
+    i1 = (int)(f2u(r.y) - 0x4B400000u);
+    return sub2(r, magic);
+}
+
+__device__ __forceinline__ void two_sum2(float2 a, float2 b, float2& s, float2& e) {
+    s = add2(a, b);
+    const float2 bb = sub2(s, a);
+    e = add2(sub2(a, sub2(s, bb)), sub2(b, bb));
+}
+
+__device__ __forceinline__ void exp2_ff2(float2 fh, float2 fl, const Opaque2& k, float2& rh,
+                                         float2& rl, int& eo0, int& eo1) {
+    int n0, n1;
+    const float2 ns = rint_small2(mul2(fh, make_float2(1024.0f, 1024.0f)), k, n0, n1);
+    const float2 f0 = fma2(ns, make_float2(-1.0f / 1024.0f, -1.0f / 1024.0f), fh);  // exact
+    float2 gh, gl;
+    two_sum2(f0, fl, gh, gl);
+    const float2 ln2h = make_float2(ALQ_LN2_HI, ALQ_LN2_HI), ln2l = make_float2(ALQ_LN2_LO, ALQ_LN2_LO);
+    const float2 wh = fma2(gh, ln2h, k.zero);
+    const float2 nwh = mul2(gh, make_float2(-ALQ_LN2_HI, -ALQ_LN2_HI));
+    const float2 wl = add2(fma2(gh, ln2h, nwh), fma2(mul2(gh, ln2l), k.one, mul2(gl, ln2h)));
+    const float2 a = fma2(mul2(wh, make_float2(1.0f / 6.0f, 1.0f / 6.0f)), k.one,
+                          make_float2(0.5f, 0.5f));
+    const float2 c = fma2(mul2(mul2(wh, wh), a), k.one, wl);
+    const int j0 = n0 & 1023, j1 = n1 & 1023;
+    eo0 = n0 >> 10;
+    eo1 = n1 >> 10;
+    const float2 th = make_float2(ALQ_TAB(kExp2Hi, j0), ALQ_TAB(kExp2Hi, j1));
+    const float2 tl = make_float2(ALQ_TAB(kExp2Lo, j0), ALQ_TAB(kExp2Lo, j1));
+    const float2 ph = fma2(th, wh, k.zero);
+    const float2 pl = fma2(th, wh, mul2(th, make_float2(-wh.x, -wh.y)));
+    const float2 sh = fma2(ph, k.one, th);
+    const float2 sl = fma2(ph, k.one, sub2(th, sh));  // ph - (sh - th)
+    const float2 lo = add2(sl, add2(pl, add2(tl, fma2(mul2(tl, wh), k.one, mul2(th, c)))));
+    rh = add2(sh, lo);
+    rl = sub2(lo, sub2(rh, sh));
+}
+
+__device__ __forceinline__ void al_level_ff2(float2 lmin, float2 delta, float kf, float Lm2,
+                                             float inv_Lm2, const Opaque2& k, float2& rh,
+                                             float2& rl) {
+    int I00, I01, N0, N1;
+    const float2 I0f = rint_small2(lmin, k, I00, I01);
+    const float2 F0 = sub2(lmin, I0f);  // exact
+    const float2 kf2 = make_float2(kf, kf);
+    const float2 ph = fma2(kf2, delta, k.zero);
+    const float2 pl = fma2(kf2, delta, mul2(kf2, make_float2(-delta.x, -delta.y)));
+    const float2 inv = make_float2(inv_Lm2, inv_Lm2);
+    const float2 Nf = rint_small2(mul2(ph, inv), k, N0, N1);
+    const float2 r0 = fma2(Nf, make_float2(-Lm2, -Lm2), ph);  // exact
+    float2 Rh, Rl;
+    two_sum2(r0, pl, Rh, Rl);
+    const float2 q1 = fma2(Rh, inv, k.zero);
+    const float2 rem = fma2(mul2(Rh, make_float2(-inv_Lm2, -inv_Lm2)), make_float2(Lm2, Lm2), Rh);
+    const float2 q2 = fma2(add2(rem, Rl), inv, k.zero);
+    float2 Fh, Fe;
+    two_sum2(F0, q1, Fh, Fe);
+    const float2 Fl = add2(Fe, q2);
+    int eo0, eo1;
+    exp2_ff2(Fh, Fl, k, rh, rl, eo0, eo1);
+    const float2 sc = make_float2(pow2i(I00 + N0 + eo0), pow2i(I01 + N1 + eo1));
+    rh = mul2(rh, sc);
+    rl = mul2(rl, sc);
+}
+
+// The two-float level tables of two blocks, each lane one entry of each (the
+// layout of al8_build_tables); a block outside the fast range gets zeros.
+__device__ __forceinline__ void al8_build_tables2(float2* tab0, float2* tab1, float lmin0,
+                                                  float delta0, float lmin1, float delta1,
+                                                  float kf, const Opaque2& k) {
+    const int lane = threadIdx.x & 31;
+    const bool hi = lane >= 16;
+    const int slot = hi ? al8_hi_slot((uint32_t)(lane - 16)) : lane;
+    const bool f0 = al8_fast_ok(lmin0, delta0), f1 = al8_fast_ok(lmin1, delta1);
+    // blocks outside the fast range compute a harmless level and are zeroed
+    const float2 lm = make_float2(hi && f0 ? lmin0 : 0.0f, hi && f1 ? lmin1 : 0.0f);
+    const float2 dl = make_float2(f0 ? delta0 : 1.0f, f1 ? delta1 : 1.0f);
+    float2 rh, rl;
+    al_level_ff2(lm, dl, kf, 254.0f, 1.0f / 254.0f, k, rh, rl);
+    tab0[slot] = f0 ? make_float2(rh.x, rl.x) : make_float2(0.0f, 0.0f);
+    tab1[slot] = f1 ? make_float2(rh.y, rl.y) : make_float2(0.0f, 0.0f);
+    __syncwarp();
+}
+
 // al8_decode_pair (alq_numerics.h) on two values with the same low factor
 // (bh, bl), step for step in paired instructions (each component rounds as
 // the scalar operation does).
@@ -365,10 +466,9 @@ static __device__ __noinline__ void al8_values_fixup(float* vals, const float2* 
 // FP64 under one warp-uniform branch. An element decode is then a single
 // shared-memory load. tab must be 16-byte aligned.
 template <int NB>
-__device__ __forceinline__ void al8_build_values(float* vals, float2* tab,
-                                                 const float (&lmin)[NB],
-                                                 const float (&delta)[NB], float kf) {
-    al8_build_tables<NB>(tab, lmin, delta, kf);
+__device__ __forceinline__ void al8_values_from_tables(float* vals, const float2* tab,
+                                                       const float (&lmin)[NB],
+                                                       const float (&delta)[NB]) {
     const int lane = threadIdx.x & 31;
     bool any_fb = false;
 #pragma unroll
@@ -397,6 +497,28 @@ __device__ __forceinline__ void al8_build_values(float* vals, float2* tab,
         for (int b = 0; b < NB; ++b) al8_values_fixup(vals + 256 * b, tab + 32 * b, lmin[b], delta[b]);
     }
     __syncwarp();
+}
+
+template <int NB>
+__device__ __forceinline__ void al8_build_values(float* vals, float2* tab,
+                                                 const float (&lmin)[NB],
+                                                 const float (&delta)[NB], float kf) {
+    al8_build_tables<NB>(tab, lmin, delta, kf);
+    al8_values_from_tables<NB>(vals, tab, lmin, delta);
+}
+
+// The same for NB >= 2 blocks, their levels two blocks per paired pass.
+template <int NB>
+__device__ __forceinline__ void al8_build_values_paired(float* vals, float2* tab,
+                                                        const float (&lmin)[NB],
+                                                        const float (&delta)[NB], float kf,
+                                                        const Opaque2& k) {
+    static_assert(NB % 2 == 0, "pairs of blocks");
+#pragma unroll
+    for (int b = 0; b < NB; b += 2)
+        al8_build_tables2(tab + 32 * b, tab + 32 * (b + 1), lmin[b], delta[b], lmin[b + 1],
+                          delta[b + 1], kf, k);
+    al8_values_from_tables<NB>(vals, tab, lmin, delta);
 }
 
 // Element decode with the level computed directly in two-float form (any
