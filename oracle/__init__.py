@@ -66,7 +66,7 @@ _sig("ora_uf8_encode", None, _f32p, _i64, _int, _i8p, _f32p)
 _sig("ora_uf8_decode", None, _i8p, _f32p, _i64, _int, _f32p)
 _sig("ora_adamw_update_fp32", None, _f32p, _f32p, _f32p, _f32p, _i64,
      C.POINTER(AdamWHP), _i64)
-_sig("ora_adamw_step", None, _f32p, _f32p, _i8p, _f32p, _vp, _f32p, _i64,
+_sig("ora_adamw_step", None, _f32p, _f32p, _vp, _vp, _vp, _vp, _i64,
      _int, _int, _int, C.POINTER(AdamWHP), _i64, _vp, _vp)
 _sig("ora_adafactor_update_fp32", None, _f32p, _f32p, _i64, _i64, _f32p, _f32p,
      _vp, C.POINTER(AdafactorHP), _i64)
@@ -97,7 +97,8 @@ def _f32(a) -> np.ndarray:
 
 
 def code_dtype(bits: int):
-    return np.uint8 if bits <= 8 else np.uint16
+    """Storage type of a state of this role precision (32: unquantized fp32)."""
+    return np.uint8 if bits <= 8 else np.uint16 if bits <= 16 else np.float32
 
 
 def num_blocks(n: int, block: int) -> int:
@@ -173,10 +174,12 @@ def adamw_update_fp32(p, g, m, v, hp: dict, t: int):
 
 def adamw_step(p, g, m_codes, m_absmax, v_codes, v_meta, m_block, v_block,
                v_bits, hp: dict, t: int, want_fresh: bool = False):
-    """Quantized AdamW step in place; optionally return the fresh (m, v)."""
+    """Quantized AdamW step in place; optionally return the fresh (m, v).
+    v_bits 32: the unquantized reference (m_codes and v_codes are fp32 m and
+    v; m_absmax and v_meta are unused)."""
     mf = np.zeros(p.size, np.float32) if want_fresh else None
     vf = np.zeros(p.size, np.float32) if want_fresh else None
-    _lib.ora_adamw_step(p, _f32(g), m_codes, m_absmax, _ptr(v_codes), v_meta,
+    _lib.ora_adamw_step(p, _f32(g), _ptr(m_codes), _ptr(m_absmax), _ptr(v_codes), _ptr(v_meta),
                         p.size, m_block, v_block, v_bits,
                         C.byref(_hp(AdamWHP, hp)), t, _ptr(mf), _ptr(vf))
     return (mf, vf) if want_fresh else None

@@ -135,6 +135,25 @@ void ora_al_decode(const void* codes, const float* meta, int64_t n, int block,
     }
 }
 
+/* A state kept in a role's precision (Sec. 4.5, state policy): AL8/AL16
+ * codes with block metadata, or bits == 32, the unquantized fp32 state
+ * (codes then point to fp32 values; there is no metadata). */
+static void state_decode(const void* codes, const float* meta, int64_t n,
+                         int block, int bits, float* out) {
+    if (bits == 32)
+        memcpy(out, codes, sizeof(float) * (size_t)n);
+    else
+        ora_al_decode(codes, meta, n, block, bits, out);
+}
+
+static void state_encode(const float* x, int64_t n, int block, int bits,
+                         float log_floor, void* codes, float* meta) {
+    if (bits == 32)
+        memcpy(codes, x, sizeof(float) * (size_t)n);
+    else
+        ora_al_encode(x, n, block, bits, log_floor, codes, meta);
+}
+
 /* Eq. (7): code bytes plus two fp32 values per block. */
 int64_t ora_al_state_bytes(int64_t n, int block, int bits) {
     int64_t code_bytes = (bits <= 8) ? n : 2 * n;
@@ -209,15 +228,23 @@ void ora_adamw_step(float* p, const float* g, int8_t* m_codes,
                     int m_block, int v_block, int v_bits,
                     const ora_adamw_hp* hp, int64_t t, float* m_fresh,
                     float* v_fresh) {
+    /* v_bits == 32: the unquantized reference, m and v dense fp32 (m_codes
+     * and v_codes point to fp32 arrays; m_absmax and v_meta are unused) */
     float* m = (float*)malloc(sizeof(float) * (size_t)(n > 0 ? n : 1));
     float* v = (float*)malloc(sizeof(float) * (size_t)(n > 0 ? n : 1));
-    ora_uf8_decode(m_codes, m_absmax, n, m_block, m);
-    ora_al_decode(v_codes, v_meta, n, v_block, v_bits, v);
+    if (v_bits == 32)
+        memcpy(m, m_codes, sizeof(float) * (size_t)n);
+    else
+        ora_uf8_decode(m_codes, m_absmax, n, m_block, m);
+    state_decode(v_codes, v_meta, n, v_block, v_bits, v);
     ora_adamw_update_fp32(p, g, m, v, n, hp, t);
     if (m_fresh) memcpy(m_fresh, m, sizeof(float) * (size_t)n);
     if (v_fresh) memcpy(v_fresh, v, sizeof(float) * (size_t)n);
-    ora_uf8_encode(m, n, m_block, m_codes, m_absmax);
-    ora_al_encode(v, n, v_block, v_bits, hp->log_floor, v_codes, v_meta);
+    if (v_bits == 32)
+        memcpy(m_codes, m, sizeof(float) * (size_t)n);
+    else
+        ora_uf8_encode(m, n, m_block, m_codes, m_absmax);
+    state_encode(v, n, v_block, v_bits, hp->log_floor, v_codes, v_meta);
     free(m);
     free(v);
 }
@@ -330,15 +357,15 @@ void ora_adafactor_step(float* p, const float* g, int64_t rows, int64_t cols,
     float* R = (float*)xmalloc(sizeof(float) * (size_t)rows);
     float* C = (float*)xmalloc(sizeof(float) * (size_t)cols);
     float* M = m_codes ? (float*)xmalloc(sizeof(float) * (size_t)n) : NULL;
-    ora_al_decode(r_codes, r_meta, rows, fac_block, fac_bits, R);
-    ora_al_decode(c_codes, c_meta, cols, fac_block, fac_bits, C);
+    state_decode(r_codes, r_meta, rows, fac_block, fac_bits, R);
+    state_decode(c_codes, c_meta, cols, fac_block, fac_bits, C);
     if (M) ora_uf8_decode(m_codes, m_absmax, n, m_block, M);
     ora_adafactor_update_fp32(p, g, rows, cols, R, C, M, hp, t);
     if (R_fresh) memcpy(R_fresh, R, sizeof(float) * (size_t)rows);
     if (C_fresh) memcpy(C_fresh, C, sizeof(float) * (size_t)cols);
     if (M_fresh && M) memcpy(M_fresh, M, sizeof(float) * (size_t)n);
-    ora_al_encode(R, rows, fac_block, fac_bits, hp->log_floor, r_codes, r_meta);
-    ora_al_encode(C, cols, fac_block, fac_bits, hp->log_floor, c_codes, c_meta);
+    state_encode(R, rows, fac_block, fac_bits, hp->log_floor, r_codes, r_meta);
+    state_encode(C, cols, fac_block, fac_bits, hp->log_floor, c_codes, c_meta);
     if (M) ora_uf8_encode(M, n, m_block, m_codes, m_absmax);
     free(R); free(C); free(M);
 }
@@ -415,10 +442,10 @@ void ora_came_step(float* p, const float* g, int64_t rows, int64_t cols,
     float* Cr = (float*)xmalloc(sizeof(float) * (size_t)rows);
     float* Cc = (float*)xmalloc(sizeof(float) * (size_t)cols);
     float* M = (float*)xmalloc(sizeof(float) * (size_t)n);
-    ora_al_decode(vr_codes, vr_meta, rows, v_block, v_bits, Vr);
-    ora_al_decode(vc_codes, vc_meta, cols, v_block, v_bits, Vc);
-    ora_al_decode(cr_codes, cr_meta, rows, c_block, c_bits, Cr);
-    ora_al_decode(cc_codes, cc_meta, cols, c_block, c_bits, Cc);
+    state_decode(vr_codes, vr_meta, rows, v_block, v_bits, Vr);
+    state_decode(vc_codes, vc_meta, cols, v_block, v_bits, Vc);
+    state_decode(cr_codes, cr_meta, rows, c_block, c_bits, Cr);
+    state_decode(cc_codes, cc_meta, cols, c_block, c_bits, Cc);
     ora_uf8_decode(m_codes, m_absmax, n, m_block, M);
     ora_came_update_fp32(p, g, rows, cols, Vr, Vc, Cr, Cc, M, hp, t);
     if (fresh) {
@@ -429,10 +456,10 @@ void ora_came_step(float* p, const float* g, int64_t rows, int64_t cols,
         memcpy(f, Cc, sizeof(float) * (size_t)cols); f += cols;
         memcpy(f, M, sizeof(float) * (size_t)n);
     }
-    ora_al_encode(Vr, rows, v_block, v_bits, hp->log_floor_v, vr_codes, vr_meta);
-    ora_al_encode(Vc, cols, v_block, v_bits, hp->log_floor_v, vc_codes, vc_meta);
-    ora_al_encode(Cr, rows, c_block, c_bits, hp->log_floor_c, cr_codes, cr_meta);
-    ora_al_encode(Cc, cols, c_block, c_bits, hp->log_floor_c, cc_codes, cc_meta);
+    state_encode(Vr, rows, v_block, v_bits, hp->log_floor_v, vr_codes, vr_meta);
+    state_encode(Vc, cols, v_block, v_bits, hp->log_floor_v, vc_codes, vc_meta);
+    state_encode(Cr, rows, c_block, c_bits, hp->log_floor_c, cr_codes, cr_meta);
+    state_encode(Cc, cols, c_block, c_bits, hp->log_floor_c, cc_codes, cc_meta);
     ora_uf8_encode(M, n, m_block, m_codes, m_absmax);
     free(Vr); free(Vc); free(Cr); free(Cc); free(M);
 }

@@ -359,3 +359,90 @@ def test_quantized_adafactor_and_came_track_fp32():
     steps, _ = _came_fp32_run(Gs, hpc, rows, cols)
     pf = -hpc["lr"] * np.sum(steps, axis=0)
     assert ora.update_error(p, pf) < 0.02
+
+
+# ======================================================== FP32 state role ==
+# Sec. 4.5 (state policy): a state may stay unquantized (FP32) instead of
+# AL8 / AL16; with bits = 32 the steps keep it as plain fp32 values.
+def test_fp32_role_adamw_step_is_torch_adamw():
+    """v_bits = 32 (m and v dense fp32) through the step: torch.optim.AdamW
+    (float64) over 10 steps, as the fp32 update itself."""
+    w = wl.AdamWSingle(shape=(64, 512))
+    p = w.p0.ravel().copy()
+    m = np.zeros_like(p)
+    v = np.zeros_like(p)
+    tp = torch.tensor(w.p0.ravel(), dtype=torch.float64, requires_grad=True)
+    opt = torch.optim.AdamW([tp], lr=1e-3, betas=(0.9, 0.999), eps=1e-8,
+                            weight_decay=0.01, foreach=False)
+    p0 = p.copy()
+    for t in range(1, 11):
+        g = w.grad(t).ravel()
+        ora.adamw_step(p, g, m, None, v, None, 256, 256, 32, ADAMW_HP, t)
+        tp.grad = torch.tensor(g, dtype=torch.float64)
+        opt.step()
+    assert _rel(p - p0, tp.detach().numpy() - p0) < 1e-5
+    assert np.any(m != 0) and np.all(v >= 0)
+
+
+def test_fp32_role_adafactor_step_matches_torch():
+    """fac_bits = 32 through the step (no momentum): torch.optim.Adafactor's
+    update direction."""
+    rows, cols = 48, 80
+    hp = dict(lr=1e-3, eps1=1e-30, clip_d=1.0, decay_rate=-0.8, beta1=0.9,
+              weight_decay=0.0, log_floor=float(np.float32(math.log2(1e-30))))
+    Gs = [wl.lognormal_col_grad((rows, cols), 1e-3, 0.05, 300 + t) for t in range(6)]
+    p0 = wl.param_init((rows, cols), 9)
+    ref = _torch_adafactor_steps(Gs, p0, 1e-3, -0.8, 1.0)
+    p = p0.ravel().copy()
+    R = np.zeros(rows, np.float32)
+    Cc = np.zeros(cols, np.float32)
+    dummy = np.zeros(2, np.float32)
+    for t, G in enumerate(Gs, start=1):
+        before = p.copy()
+        ora.adafactor_step(p, G.ravel(), rows, cols, R, dummy, Cc, dummy, 32, 128, None, None,
+                           256, hp, t)
+        mine = -(p.astype(np.float64) - before) / hp["lr"]
+        assert _rel(mine, ref[t - 1].ravel()) < 2e-5, t
+    assert np.all(R > 0) and np.all(Cc > 0)
+
+
+def test_fp32_role_came_step_is_fp32_update():
+    """CAME with V and C in FP32 through the step equals the fp32 update on
+    plain arrays bit for bit; the paper's FP32-C variant (AL16 V, FP32 C)
+    tracks it."""
+    rows, cols = 40, 96
+    hp = dict(lr=1e-4, beta1=0.9, beta2=0.999, beta3=0.9999, eps1=1e-30, eps2=1e-16,
+              clip_d=1.0, weight_decay=0.0, log_floor_v=float(np.float32(math.log2(1e-30))),
+              log_floor_c=float(np.float32(math.log2(1e-16))))
+    p0 = wl.param_init((rows, cols), 13).ravel()
+    pa, pb, pc = p0.copy(), p0.copy(), p0.copy()
+    n = rows * cols
+    fa = [np.zeros(rows, np.float32), np.zeros(cols, np.float32), np.zeros(rows, np.float32),
+          np.zeros(cols, np.float32)]
+    fb = [x.copy() for x in fa]
+    Ma = np.zeros(n, np.float32)
+    mc = np.zeros(n, np.int8)
+    ma = np.zeros(n // 256 + 1, np.float32)
+    mc2, ma2 = mc.copy(), ma.copy()
+    dummy = np.zeros(2, np.float32)
+    vr16 = np.zeros(rows, np.uint16)
+    vr16m = np.zeros(2 * (rows // 128 + 1), np.float32)
+    vc16 = np.zeros(cols, np.uint16)
+    vc16m = np.zeros(2 * (cols // 128 + 1), np.float32)
+    cr, cc = np.zeros(rows, np.float32), np.zeros(cols, np.float32)
+    mc3, ma3 = mc.copy(), ma.copy()
+    for t in range(1, 6):
+        g = wl.student_t_grad((rows, cols), 1e-3, 3.0, 0.05, 70 + t).ravel()
+        # reference: fp32 update on plain states, momentum through UF8 as in the step
+        M = ora.uf8_decode(mc2, ma2, 256)
+        ora.came_update_fp32(pa, g, rows, cols, *fa, M, hp, t)
+        mc2, ma2 = ora.uf8_encode(M, 256)
+        ora.came_step(pb, g, rows, cols, fb[0], dummy, fb[1], dummy, 32, 128, fb[2], dummy,
+                      fb[3], dummy, 32, 128, mc, ma, 256, hp, t)
+        ora.came_step(pc, g, rows, cols, vr16, vr16m, vc16, vc16m, 16, 128, cr, dummy, cc,
+                      dummy, 32, 128, mc3, ma3, 256, hp, t)
+        assert np.array_equal(pa.view(np.uint32), pb.view(np.uint32)), t
+        for x, y in zip(fa, fb):
+            assert np.array_equal(x.view(np.uint32), y.view(np.uint32)), t
+    assert ora.update_error(pc - p0, pa - p0) < 0.03
+
