@@ -153,6 +153,11 @@ typedef struct {
  *   m_block, v_block  block sizes, powers of two in [128, 2048].
  *   v_codes  [n] uint8 (v_bits = 8) or uint16 (v_bits = 16) AL codes,
  *   v_meta   [2*ceil(n/v_block)] fp32.
+ *   v_bits = 32 is the unquantized FP32 role (Sec. 4.5, "AL8, AL16, or
+ *            FP32 according to state sensitivity"): m_codes and v_codes
+ *            then point to dense fp32 m and v [n], m_absmax, v_meta,
+ *            m_block and v_block are unused (m_absmax and v_meta may be
+ *            NULL), and the step is the same arithmetic without the codec.
  *   hp       host pointer; t >= 1.
  * Scalars computed on the host in double and rounded to fp32 once:
  *   decay = 1 - lr*wd, step = lr / (1 - beta1^t), c2 = 1 / sqrt(1 - beta2^t),
@@ -242,6 +247,10 @@ typedef struct {
  * "row and column statistics"; lr 1e-3 in Sec. 6.1) whose row factor R [rows]
  * and column factor C [cols] are AL-coded (fac_bits 8 or 16, fac_block), and
  * optional UF8 momentum. p and g are row-major [rows x cols] fp32.
+ * fac_bits = 32 keeps the factors unquantized (Sec. 4.5's FP32 role):
+ * r_codes and c_codes then point to fp32 factors, r_meta and c_meta are
+ * unused (may be NULL). The same holds for v_bits and c_bits of
+ * al_came_step (c_bits = 32 with AL-coded V is the paper's "FP32 C" CAME).
  *   r_i = mean_j(g_ij^2 + eps1), c_j = mean_i(g_ij^2 + eps1)  (exact sums,
  *         rounded once to fp32);
  *   R = rho*R_hat + (1-rho)*r,  C = rho*C_hat + (1-rho)*c;

@@ -364,6 +364,49 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
     }
 }
 
+// ------------------------------------------------ unquantized reference --
+// v_bits 32: AdamW with dense fp32 m and v (Sec. 4.5's FP32 state role, the
+// unquantized reference): the per-element arithmetic of the fused kernel
+// with m_hat = m and v_hat = v, no codec; 28 bytes per parameter. The same
+// tiles and descriptors (m_codes and v_codes hold fp32 m and v).
+__global__ void __launch_bounds__(kThreads)
+adamw_fp32_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t total_tiles,
+                  PlanEntry single, AdamWPairs s) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    int cur = 0;
+    for (int64_t tile = blockIdx.x; tile < total_tiles; tile += gridDim.x) {
+        const PlanEntry d = plan_entry(table, ntensors, single, tile, cur);
+        const int64_t e0 = (tile - d.first_tile) * kATile + (int64_t)warp * kASeg + 4 * lane;
+        float* m = reinterpret_cast<float*>(d.m_codes);
+        float* v = reinterpret_cast<float*>(d.v_codes);
+#pragma unroll
+        for (int c = 0; c < kCH; ++c) {
+            const int64_t idx = e0 + 128 * c;
+            if (idx >= d.n) continue;
+            const float4 g4 = load4f(d.g, idx, d.n), p4 = load4f(d.p, idx, d.n);
+            const float4 m4 = load4f(m, idx, d.n), v4 = load4f(v, idx, d.n);
+            float2 pn[2], mn[2], vn[2];
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+                const float2 gi = i == 0 ? make_float2(g4.x, g4.y) : make_float2(g4.z, g4.w);
+                const float2 pi = i == 0 ? make_float2(p4.x, p4.y) : make_float2(p4.z, p4.w);
+                const float2 mi = i == 0 ? make_float2(m4.x, m4.y) : make_float2(m4.z, m4.w);
+                const float2 vi = i == 0 ? make_float2(v4.x, v4.y) : make_float2(v4.z, v4.w);
+                const float2 p1 = mul2(pi, s.decay);
+                const float2 mm = fma2(s.beta1, mi, mul2(s.omb1, gi));
+                const float2 vv = fma2(s.beta2, vi, mul2(s.omb2, mul2(gi, gi)));
+                const float2 den = fma2(make_float2(sqrtf(vv.x), sqrtf(vv.y)), s.c2, s.eps);
+                pn[i] = fma2(s.nstep, make_float2(mm.x / den.x, mm.y / den.y), p1);
+                mn[i] = mm;
+                vn[i] = vv;
+            }
+            store4f(d.p, idx, d.n, make_float4(pn[0].x, pn[0].y, pn[1].x, pn[1].y));
+            store4f(m, idx, d.n, make_float4(mn[0].x, mn[0].y, mn[1].x, mn[1].y));
+            store4f(v, idx, d.n, make_float4(vn[0].x, vn[0].y, vn[1].x, vn[1].y));
+        }
+    }
+}
+
 // ------------------------------------------------------------- dispatch --
 static int cpb_of(int block) { return block >= kASeg ? kCH : block / 128; }
 static bool adamw_block_ok(int block) { return valid_block(block) && block <= kATile; }
@@ -396,6 +439,12 @@ static int launch_adamw(const PlanEntry* table, int ntensors, int64_t total_tile
                         const PlanEntry& single, int v_block, int m_block, int v_bits,
                         const al_adamw_hp* hp, int64_t t, cudaStream_t st) {
     const AdamWScalars s = adamw_scalars(hp, t);
+    if (v_bits == 32) {
+        const int grid = persistent_grid((const void*)adamw_fp32_kernel, kThreads, 0, total_tiles);
+        adamw_fp32_kernel<<<grid, kThreads, 0, st>>>(table, ntensors, total_tiles, single,
+                                                      adamw_pairs(s));
+        return check_launch();
+    }
     const int cv = cpb_of(v_block), cm = cpb_of(m_block);
     if (v_bits == 8)
         return launch_adamw_v<8>(cv, cm, table, ntensors, total_tiles, single, v_block, m_block, s, st);
@@ -410,16 +459,25 @@ static int check_hp(const al_adamw_hp* hp) {
     return ALQ_OK;
 }
 
+// v_bits 32: m_codes and v_codes are fp32 m and v; m_absmax and v_meta are
+// unused (may be NULL).
 static int check_tensor(const PlanEntry& e, int v_bits) {
     if (e.n < 0) return ALQ_ERR_INVALID_ARG;
     if (e.n == 0) return ALQ_OK;
-    if (!e.p || !e.g || !e.m_codes || !e.m_absmax || !e.v_codes || !e.v_meta)
+    const bool raw = v_bits == 32;
+    if (!e.p || !e.g || !e.m_codes || !e.v_codes || (!raw && (!e.m_absmax || !e.v_meta)))
         return ALQ_ERR_INVALID_ARG;
     if (!aligned(e.p, 16) || !aligned(e.g, 16) || !aligned(e.m_codes, 16) ||
-        !aligned(e.v_codes, 16) || !aligned(e.v_meta, 8) || !aligned(e.m_absmax, 4))
+        !aligned(e.v_codes, 16))
         return ALQ_ERR_ALIGN;
-    (void)v_bits;
+    if (!raw && (!aligned(e.v_meta, 8) || !aligned(e.m_absmax, 4))) return ALQ_ERR_ALIGN;
     return ALQ_OK;
+}
+
+// Bit widths and block sizes of a call: blocks are ignored for v_bits 32.
+static bool adamw_config_ok(int m_block, int v_block, int v_bits) {
+    if (v_bits == 32) return true;
+    return adamw_block_ok(m_block) && adamw_block_ok(v_block) && (v_bits == 8 || v_bits == 16);
 }
 
 }  // namespace alq
@@ -431,8 +489,7 @@ extern "C" {
 int al_adamw_step(float* p, const float* g, int8_t* m_codes, float* m_absmax, void* v_codes,
                   float* v_meta, int64_t n, int m_block, int v_block, int v_bits,
                   const al_adamw_hp* hp, int64_t t, void* stream) {
-    if (!adamw_block_ok(m_block) || !adamw_block_ok(v_block) || (v_bits != 8 && v_bits != 16))
-        return ALQ_ERR_UNSUPPORTED;
+    if (!adamw_config_ok(m_block, v_block, v_bits)) return ALQ_ERR_UNSUPPORTED;
     if (t < 1) return ALQ_ERR_INVALID_ARG;
     int st = check_hp(hp);
     if (st) return st;
@@ -447,8 +504,7 @@ int al_adamw_step(float* p, const float* g, int8_t* m_codes, float* m_absmax, vo
 int al_adamw_plan(const al_adamw_tensor* tensors, int ntensors, int m_block, int v_block,
                   int v_bits, void* plan_host, size_t plan_bytes, al_multi_info* info) {
     if (!tensors || ntensors <= 0 || !plan_host || !info) return ALQ_ERR_INVALID_ARG;
-    if (!adamw_block_ok(m_block) || !adamw_block_ok(v_block) || (v_bits != 8 && v_bits != 16))
-        return ALQ_ERR_UNSUPPORTED;
+    if (!adamw_config_ok(m_block, v_block, v_bits)) return ALQ_ERR_UNSUPPORTED;
     size_t need = 0;
     al_adamw_plan_bytes(ntensors, &need);
     if (plan_bytes < need) return ALQ_ERR_INVALID_ARG;
@@ -487,9 +543,7 @@ int al_adamw_step_multi(const void* plan_dev, const al_multi_info* info, const a
     if (!plan_dev || !info || t < 1) return ALQ_ERR_INVALID_ARG;
     if (!aligned(plan_dev, 16)) return ALQ_ERR_ALIGN;
     if (info->ntensors <= 0 || info->total_tiles < 0) return ALQ_ERR_INVALID_ARG;
-    if (!adamw_block_ok(info->m_block) || !adamw_block_ok(info->v_block) ||
-        (info->v_bits != 8 && info->v_bits != 16))
-        return ALQ_ERR_UNSUPPORTED;
+    if (!adamw_config_ok(info->m_block, info->v_block, info->v_bits)) return ALQ_ERR_UNSUPPORTED;
     int st = check_hp(hp);
     if (st) return st;
     if (info->total_tiles == 0) return ALQ_OK;

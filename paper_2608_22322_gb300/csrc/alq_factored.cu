@@ -274,7 +274,8 @@ __device__ __forceinline__ void factor_block(const FactorDesc& f, int64_t b,
     const bool first = rsum != nullptr;
     const int64_t lo = b * f.block;
     const int64_t hi = lo + f.block < f.len ? lo + f.block : f.len;
-    const float2 om = __ldg(reinterpret_cast<const float2*>(f.meta) + b);
+    const bool raw = f.bits == 32;  // the unquantized fp32 role: no metadata
+    const float2 om = raw ? make_float2(0.f, 0.f) : __ldg(reinterpret_cast<const float2*>(f.meta) + b);
     const float Lm2 = f.bits == 8 ? 254.0f : 65534.0f;
     float v[KPT];
     uint32_t vmin = 0xFFFFFFFFu, vmax = 0u;
@@ -296,7 +297,8 @@ __device__ __forceinline__ void factor_block(const FactorDesc& f, int64_t b,
             }
             for (; p < f.nparts; ++p) s += pp[(int64_t)p * f.len];
             const float stat = (float)(s / f.mean_len + f.add_eps);
-            const float old = al_decode_direct(fac_code(f, i), om.x, om.y, Lm2);
+            const float old = raw ? ((const float*)f.codes)[i]
+                                  : al_decode_direct(fac_code(f, i), om.x, om.y, Lm2);
             v[k] = f.beta * old + f.omb * stat;
             f.fresh[i] = v[k];
             const uint32_t vb = f2u(v[k]);
@@ -312,6 +314,21 @@ __device__ __forceinline__ void factor_block(const FactorDesc& f, int64_t b,
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xFFFFFFFFu, t, o);
         if ((threadIdx.x & 31) == 0) s_sum[threadIdx.x >> 5] = t;
+    }
+    if (raw) {
+        // the fresh factor is the stored state
+        __syncthreads();
+        if (first && threadIdx.x == 0) {
+            double t = 0.0;
+            for (int w = 0; w < kThreads / 32; ++w) t += s_sum[w];
+            rsum[b] = t;
+        }
+#pragma unroll
+        for (int k = 0; k < KPT; ++k) {
+            const int64_t i = lo + threadIdx.x + (int64_t)kThreads * k;
+            if (i < hi) ((float*)f.codes)[i] = v[k];
+        }
+        return;
     }
     vmin = __reduce_min_sync(0xFFFFFFFFu, vmin);
     vmax = __reduce_max_sync(0xFFFFFFFFu, vmax);
@@ -631,10 +648,12 @@ static int check_matrix(const float* p, const float* g, int64_t rows, int64_t co
     return ALQ_OK;
 }
 
+// bits 8 or 16: AL codes with block metadata; 32: the unquantized fp32 role
+// (codes point to fp32 values, meta is unused and may be NULL).
 static int check_factor(const void* codes, const float* meta, int bits, int block) {
-    if (!codes || !meta) return ALQ_ERR_INVALID_ARG;
-    if ((bits != 8 && bits != 16) || !valid_block(block)) return ALQ_ERR_UNSUPPORTED;
-    if (!aligned(codes, 16) || !aligned(meta, 8)) return ALQ_ERR_ALIGN;
+    if (!codes || (bits != 32 && !meta)) return ALQ_ERR_INVALID_ARG;
+    if ((bits != 8 && bits != 16 && bits != 32) || !valid_block(block)) return ALQ_ERR_UNSUPPORTED;
+    if (!aligned(codes, 16) || (bits != 32 && !aligned(meta, 8))) return ALQ_ERR_ALIGN;
     return ALQ_OK;
 }
 

@@ -194,3 +194,33 @@ def test_adamw_rejects_bad_arguments(B):
         B.al_adamw_step(x[1:], x[1:], c[1:], x, c[1:], x, 256, 256, 8, ADAMW_HP, 1)
     with pytest.raises(B.AlqError, match="INVALID_ARG"):
         B.al_adamw_step(x, x, c, x, c, x, 256, 256, 8, ADAMW_HP, 0)
+
+
+def test_adamw_fp32_role_single_and_plan(B):
+    """v_bits = 32 (dense fp32 m and v, Sec. 4.5's FP32 role): the kernel's
+    parameters and states equal the oracle's bit for bit, single tensor and
+    multi-tensor plan, ragged sizes."""
+    import torch
+    sizes = [41107, 5, 4096 * 3 + 17]
+    hs, ds, gds = [], [], []
+    for i, n in enumerate(sizes):
+        p0 = (wl.rng(500 + i).standard_normal(n) * 0.02).astype(np.float32)
+        h = dict(p=p0.copy(), m=np.zeros(n, np.float32), v=np.zeros(n, np.float32))
+        hs.append(h)
+        ds.append({k: torch.from_numpy(v.copy()).cuda() for k, v in h.items()})
+        gds.append(torch.zeros(n, dtype=torch.float32, device="cuda"))
+    plan = B.AdamWPlan([dict(p=d["p"], g=g, m_codes=d["m"], m_absmax=None, v_codes=d["v"],
+                             v_meta=None) for d, g in zip(ds[1:], gds[1:])], 256, 256, 32)
+    for t in range(1, 5):
+        for i, n in enumerate(sizes):
+            g = wl.gaussian_grad((n,), 1e-3, 600 + 10 * t + i, wl.zero_mask((n,), 0.05, 7 + i))
+            h = hs[i]
+            ora.adamw_step(h["p"], g, h["m"], None, h["v"], None, 256, 256, 32, ADAMW_HP, t)
+            gds[i].copy_(torch.from_numpy(g))
+        B.al_adamw_step(ds[0]["p"], gds[0], ds[0]["m"], None, ds[0]["v"], None, 256, 256, 32,
+                        ADAMW_HP, t)
+        plan.step(ADAMW_HP, t)
+        torch.cuda.synchronize()
+        for h, d in zip(hs, ds):
+            for k in ("p", "m", "v"):
+                assert bytes_equal(h[k], d[k].cpu().numpy()) == 0, (t, k, h["p"].size)

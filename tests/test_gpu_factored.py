@@ -217,3 +217,72 @@ def test_grouped_factored_step_matches_single(B, op, mom, bits, block):
                 a = dg[i][k].cpu().numpy()
                 b = ds[i][k].cpu().numpy()
                 assert bytes_equal(a, b) == 0, (op, t, i, k)
+
+
+@pytest.mark.parametrize("op,vb,cb", [("adafactor", 32, 0), ("came", 16, 32), ("came", 32, 32)])
+def test_fp32_factor_roles_match_oracle(B, op, vb, cb):
+    """Factors kept unquantized (bits 32, Sec. 4.5): Adafactor with fp32
+    factors, the paper's FP32-C CAME (AL16 V, fp32 C) and CAME with fp32 V
+    and C, against the oracle; and the grouped step equals the per-matrix
+    step bit for bit."""
+    import torch
+    rows, cols = 300, 772
+    came = op == "came"
+
+    def fac(ln, bits):
+        if bits == 32:
+            return np.zeros(ln, np.float32), None
+        return _state(ln, bits, 128)
+
+    p = wl.param_init((rows, cols), 17).ravel()
+    st = [fac(rows, vb), fac(cols, vb)] + ([fac(rows, cb), fac(cols, cb)] if came else [])
+    n = rows * cols
+    mc = np.zeros(n, np.int8)
+    ma = np.zeros((n + 255) // 256, np.float32)
+    dt = lambda a: None if a is None else _t(a)
+    d1 = dict(p=_t(p), st=[(dt(c), dt(m)) for c, m in st], mc=_t(mc), ma=_t(ma))
+    d2 = dict(p=_t(p), st=[(dt(c), dt(m)) for c, m in st], mc=_t(mc), ma=_t(ma))
+    g_dev = torch.zeros(n, dtype=torch.float32, device="cuda")
+    keys = ["vr", "vc", "cr", "cc"]
+    m = dict(p=d2["p"], g=g_dev, rows=rows, cols=cols, m_codes=d2["mc"], m_absmax=d2["ma"])
+    for k, (c, me) in zip(keys, d2["st"]):
+        m[k + "_codes"], m[k + "_meta"] = c, me
+    plan = B.FactoredPlan(B.AL_OP_CAME if came else B.AL_OP_ADAFACTOR, [m], vb, 128,
+                          cb if came else 16, 128, 256)
+    ws = torch.empty(B.al_workspace_size(B.AL_OP_CAME if came else B.AL_OP_ADAFACTOR, rows, cols),
+                     dtype=torch.uint8, device="cuda")
+    flips = 0
+    for t in range(1, 5):
+        g = wl.student_t_grad((rows, cols), 1e-3, 3.0, 0.05, 4400 + t).ravel()
+        g_dev.copy_(torch.from_numpy(g))
+        dummy = np.zeros(2, np.float32)
+        hm = lambda x: dummy if x is None else x
+        if came:
+            ora.came_step(p, g, rows, cols, st[0][0], hm(st[0][1]), st[1][0], hm(st[1][1]), vb,
+                          128, st[2][0], hm(st[2][1]), st[3][0], hm(st[3][1]), cb, 128, mc, ma,
+                          256, CAME_HP, t)
+            s_ = d1["st"]
+            B.al_came_step(d1["p"], g_dev, rows, cols, s_[0][0], s_[0][1], s_[1][0], s_[1][1], vb,
+                           128, s_[2][0], s_[2][1], s_[3][0], s_[3][1], cb, 128, d1["mc"],
+                           d1["ma"], 256, CAME_HP, t, ws)
+            plan.step(CAME_HP, t)
+        else:
+            ora.adafactor_step(p, g, rows, cols, st[0][0], hm(st[0][1]), st[1][0], hm(st[1][1]),
+                               32, 128, mc, ma, 256, ADA_HP, t)
+            s_ = d1["st"]
+            B.al_adafactor_step(d1["p"], g_dev, rows, cols, s_[0][0], s_[0][1], s_[1][0],
+                                s_[1][1], 32, 128, d1["mc"], d1["ma"], 256, ADA_HP, t, ws)
+            plan.step(ADA_HP, t)
+        torch.cuda.synchronize()
+        _cmp_p(p, d1["p"], f"step {t}")
+        for (c, _), (dc, _), bits in zip(st, d1["st"], [vb, vb, cb, cb]):
+            if bits == 32:
+                got = dc.cpu().numpy()
+                assert np.max(np.abs(got - c) / np.maximum(np.abs(c), 1e-38)) < 1e-5
+            else:
+                flips += _cmp_codes("factor codes", c, dc, bits)
+        flips += _cmp_codes("M codes", mc, d1["mc"], 8)
+        for a, b in zip([d1["p"], d1["mc"], d1["ma"]] + [x for x, _ in d1["st"]],
+                        [d2["p"], d2["mc"], d2["ma"]] + [x for x, _ in d2["st"]]):
+            assert bytes_equal(a.cpu().numpy(), b.cpu().numpy()) == 0, t
+    print(f"{op} v{vb} c{cb}: code flips = {flips}")
