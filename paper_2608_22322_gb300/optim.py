@@ -10,12 +10,18 @@ the parameters into launches and follows torch.optim's conventions
 (param_groups, state_dict / load_state_dict, closures, learning-rate
 schedulers changing group["lr"]).
 
-Per-role precision (Sec. 6.2, "AL8 second moments with UF8 momentum", "AL16
-for both V and C"): each param group chooses the bit width of its AL-coded
-states (v_bits, c_bits, fac_bits) and block sizes; migrate_bits() re-codes a
-trained state from AL8 to AL16 or back through the codec. Parameters that a
-method cannot take (APOLLO needs matrices) are routed to the quantized AdamW
-step, as the paper routes embeddings and norms separately (Sec. 6.1).
+Per-role precision (Sec. 4.5; Sec. 6.2, "AL8 second moments with UF8
+momentum", "AL16 for both V and C"): each param group chooses the bit width
+of its states (v_bits, c_bits, fac_bits: 8 or 16 for AL codes, 32 for the
+unquantized FP32 role; AdamW's v_bits 32 keeps m in fp32 too) and block
+sizes; migrate_bits() re-codes a trained AL state from AL8 to AL16 or back
+through the codec. Parameter grouping (Sec. 6.1): G0 gives every parameter
+the selected configuration; g1_param_groups() builds G1, which keeps the
+states of one-dimensional tensors, biases, normalization parameters, token
+embeddings and the language-model head unquantized. Parameters that a method
+cannot take (APOLLO needs matrices) are routed to the quantized AdamW step.
+The factored optimizers step each param group's matrices in grouped
+launches (al_adafactor_step_multi / al_came_step_multi).
 """
 from __future__ import annotations
 
@@ -25,7 +31,7 @@ import torch
 
 from . import binding as B
 
-__all__ = ["AdamW", "Adafactor", "CAME", "Apollo"]
+__all__ = ["AdamW", "Adafactor", "CAME", "Apollo", "g1_param_groups"]
 
 
 def _log2_floor(x: float) -> float:
@@ -36,7 +42,35 @@ def _log2_floor(x: float) -> float:
 
 
 def _code_dtype(bits: int):
-    return torch.uint8 if bits == 8 else torch.int16  # AL16 codes travel as int16 bits
+    """Storage dtype of a state of this width (AL16 codes travel as int16
+    bits; 32 is the unquantized fp32 state)."""
+    return torch.uint8 if bits == 8 else torch.int16 if bits == 16 else torch.float32
+
+
+def _check_bits(bits: int, what: str):
+    if bits not in (8, 16, 32):
+        raise ValueError(f"{what} must be 8, 16 or 32")
+
+
+def g1_param_groups(named_parameters, protected: dict, others: dict = None,
+                    patterns=("bias", "norm", "embed", "lm_head", "wte", "wpe")):
+    """Sec. 6.1's G1 grouping: one-dimensional tensors, biases, normalization
+    parameters, token embeddings and the language-model head (by name: any of
+    `patterns` in the parameter's name) form a protected group whose options
+    are `protected` (e.g. dict(v_bits=32) for AdamW, dict(fac_bits=32) for
+    Adafactor: states unquantized); the remaining tensors keep `others` (the
+    selected low-precision path). Returns param groups for the optimizers of
+    this module. G0 is simply all parameters in one group."""
+    prot, rest = [], []
+    for name, p in named_parameters:
+        low = name.lower()
+        (prot if p.dim() <= 1 or any(k in low for k in patterns) else rest).append(p)
+    groups = []
+    if rest:
+        groups.append(dict(params=rest, **(others or {})))
+    if prot:
+        groups.append(dict(params=prot, **protected))
+    return groups
 
 
 def _check_param(p: torch.Tensor, what: str):
@@ -57,6 +91,8 @@ class _Base(torch.optim.Optimizer):
 
     # state key -> group key holding its bit width (None: UF8 int8 codes)
     _CODES: dict = {}
+    # group key whose value 32 keeps the momentum in fp32 too (AdamW)
+    _M_FOLLOWS = None
     # AL state key -> (metadata key, group key of its block size)
     _AL: dict = {}
 
@@ -69,7 +105,11 @@ class _Base(torch.optim.Optimizer):
                     continue
                 for key, bits_key in self._CODES.items():
                     if key in st:
-                        dt = torch.int8 if bits_key is None else _code_dtype(group[bits_key])
+                        if bits_key is None:
+                            raw = self._M_FOLLOWS and group[self._M_FOLLOWS] == 32
+                            dt = torch.float32 if raw else torch.int8
+                        else:
+                            dt = _code_dtype(group[bits_key])
                         st[key] = st[key].to(dtype=dt)
 
     @torch.no_grad()
@@ -83,6 +123,8 @@ class _Base(torch.optim.Optimizer):
             old = group[bits_key]
             if old == new_bits:
                 continue
+            if old == 32:
+                raise ValueError("migrate_bits re-codes AL8/AL16 states; an FP32 group stays FP32")
             for p in group["params"]:
                 st = self.state.get(p)
                 if not st:
@@ -107,16 +149,17 @@ class _Base(torch.optim.Optimizer):
 class AdamW(_Base):
     """AdamW (Sec. 3.1, Eq. (1)) with UF8 momentum and AL-coded second moment;
     one fused launch per group and step over every parameter with a gradient
-    (al_adamw_step_multi). v_bits 8 or 16, blocks powers of two in
-    [128, 2048]; log_floor defaults to log2(eps^2)."""
+    (al_adamw_step_multi). v_bits 8 or 16 (AL8/AL16 V, UF8 M) or 32 (m and
+    v unquantized fp32), blocks powers of two in [128, 2048]; log_floor
+    defaults to log2(eps^2)."""
 
     _CODES = {"m_codes": None, "v_codes": "v_bits"}
     _AL = {"v_codes": ("v_meta", "v_block")}
+    _M_FOLLOWS = "v_bits"
 
     def __init__(self, params, lr=1e-3, betas=(0.9, 0.999), eps=1e-8, weight_decay=1e-2,
                  v_bits=8, v_block=256, m_block=256, log_floor=None):
-        if v_bits not in (8, 16):
-            raise ValueError("v_bits must be 8 or 16")
+        _check_bits(v_bits, "v_bits")
         defaults = dict(lr=lr, betas=betas, eps=eps, weight_decay=weight_decay, v_bits=v_bits,
                         v_block=v_block, m_block=m_block,
                         log_floor=log_floor if log_floor is not None else _log2_floor(eps * eps))
@@ -127,12 +170,13 @@ class AdamW(_Base):
         n = p.numel()
         st = self.state[p]
         st["step"] = 0
-        st["m_codes"] = torch.zeros(n, dtype=torch.int8, device=p.device)
-        st["m_absmax"] = torch.zeros(_blocks(n, group["m_block"]), dtype=torch.float32,
-                                     device=p.device)
+        raw = group["v_bits"] == 32
+        st["m_codes"] = torch.zeros(n, dtype=torch.float32 if raw else torch.int8, device=p.device)
+        st["m_absmax"] = torch.zeros(0 if raw else _blocks(n, group["m_block"]),
+                                     dtype=torch.float32, device=p.device)
         st["v_codes"] = torch.zeros(n, dtype=_code_dtype(group["v_bits"]), device=p.device)
-        st["v_meta"] = torch.zeros(2 * _blocks(n, group["v_block"]), dtype=torch.float32,
-                                   device=p.device)
+        st["v_meta"] = torch.zeros(0 if raw else 2 * _blocks(n, group["v_block"]),
+                                   dtype=torch.float32, device=p.device)
 
     def _plan(self, tensors, group):
         key = (tuple((t["p"].data_ptr(), t["g"].data_ptr(), t["v_codes"].data_ptr(),
@@ -185,45 +229,38 @@ def _as_matrix(p: torch.Tensor):
     return 1, p.numel()
 
 
-class _Workspace:
-    """A growing scratch buffer shared by the per-matrix calls of one step."""
-
-    def __init__(self):
-        self.buf = None
-
-    def get(self, nbytes: int, device):
-        if self.buf is None or self.buf.numel() < nbytes or self.buf.device != device:
-            self.buf = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=device)
-        return self.buf
-
-
 class Adafactor(_Base):
     """Adafactor (Sec. 3.1: factored second moment) with AL-coded row/column
-    factors (fac_bits 8 or 16, fac_block) and optional UF8 momentum
-    (beta1 > 0); rho_t = 1 - t^decay_rate, RMS clip d. Vectors are treated as
-    1 x n matrices."""
+    factors (fac_bits 8 or 16, fac_block; 32: unquantized fp32 factors) and
+    optional UF8 momentum (beta1 > 0); rho_t = 1 - t^decay_rate, RMS clip d.
+    Vectors are treated as 1 x n matrices. Each group's matrices step in one
+    grouped launch per pass."""
 
     _CODES = {"r_codes": "fac_bits", "c_codes": "fac_bits", "m_codes": None}
     _AL = {"r_codes": ("r_meta", "fac_block"), "c_codes": ("c_meta", "fac_block")}
 
     def __init__(self, params, lr=1e-3, eps1=1e-30, clip_d=1.0, decay_rate=-0.8, beta1=0.9,
                  weight_decay=0.0, fac_bits=16, fac_block=128, m_block=256, log_floor=None):
+        _check_bits(fac_bits, "fac_bits")
         defaults = dict(lr=lr, eps1=eps1, clip_d=clip_d, decay_rate=decay_rate, beta1=beta1,
                         weight_decay=weight_decay, fac_bits=fac_bits, fac_block=fac_block,
                         m_block=m_block,
                         log_floor=log_floor if log_floor is not None else _log2_floor(eps1))
         super().__init__(params, defaults)
-        self._ws = _Workspace()
+        self._plans: dict = {}
 
     def _init_state(self, p, group):
         rows, cols = _as_matrix(p)
         dev, fb = p.device, group["fac_block"]
         st = self.state[p]
         st["step"] = 0
+        raw = group["fac_bits"] == 32
         st["r_codes"] = torch.zeros(rows, dtype=_code_dtype(group["fac_bits"]), device=dev)
-        st["r_meta"] = torch.zeros(2 * _blocks(rows, fb), dtype=torch.float32, device=dev)
+        st["r_meta"] = torch.zeros(0 if raw else 2 * _blocks(rows, fb), dtype=torch.float32,
+                                   device=dev)
         st["c_codes"] = torch.zeros(cols, dtype=_code_dtype(group["fac_bits"]), device=dev)
-        st["c_meta"] = torch.zeros(2 * _blocks(cols, fb), dtype=torch.float32, device=dev)
+        st["c_meta"] = torch.zeros(0 if raw else 2 * _blocks(cols, fb), dtype=torch.float32,
+                                   device=dev)
         if group["beta1"] > 0:
             st["m_codes"] = torch.zeros(p.numel(), dtype=torch.int8, device=dev)
             st["m_absmax"] = torch.zeros(_blocks(p.numel(), group["m_block"]),
@@ -238,6 +275,7 @@ class Adafactor(_Base):
         for group in self.param_groups:
             hp = {k: group[k] for k in ("lr", "eps1", "clip_d", "decay_rate", "beta1",
                                         "weight_decay", "log_floor")}
+            buckets: dict = {}
             for p in group["params"]:
                 if p.grad is None:
                     continue
@@ -247,18 +285,37 @@ class Adafactor(_Base):
                 st = self.state[p]
                 st["step"] += 1
                 rows, cols = _as_matrix(p)
-                ws = self._ws.get(B.al_workspace_size(B.AL_OP_ADAFACTOR, rows, cols), p.device)
-                B.al_adafactor_step(p, p.grad, rows, cols, st["r_codes"], st["r_meta"],
-                                    st["c_codes"], st["c_meta"], group["fac_bits"],
-                                    group["fac_block"], st.get("m_codes"), st.get("m_absmax"),
-                                    group["m_block"], hp, st["step"], ws)
+                buckets.setdefault(st["step"], []).append(
+                    dict(p=p, g=p.grad, rows=rows, cols=cols, vr_codes=st["r_codes"],
+                         vr_meta=st["r_meta"], vc_codes=st["c_codes"], vc_meta=st["c_meta"],
+                         m_codes=st.get("m_codes"), m_absmax=st.get("m_absmax")))
+            for t, mats in buckets.items():
+                _grouped_plan(self._plans, B.AL_OP_ADAFACTOR, mats, group["fac_bits"],
+                              group["fac_block"], 16, 128, group["m_block"]).step(hp, t)
         return loss
+
+
+def _grouped_plan(cache: dict, op, mats, v_bits, v_block, c_bits, c_block, m_block):
+    """A cached FactoredPlan over these matrices (plans bind pointers)."""
+    key = (op, v_bits, v_block, c_bits, c_block, m_block,
+           tuple(tuple(0 if m.get(k) is None else m[k].data_ptr()
+                       for k in ("p", "g", "vr_codes", "vc_codes", "cr_codes", "cc_codes",
+                                 "m_codes")) for m in mats))
+    plan = cache.get(key)
+    if plan is None:
+        if len(cache) > 64:
+            cache.clear()
+        plan = B.FactoredPlan(op, mats, v_bits, v_block, c_bits, c_block, m_block)
+        cache[key] = plan
+    return plan
 
 
 class CAME(_Base):
     """CAME (Sec. 3.1: dense momentum, factored second moment and factored
     confidence; beta3 0.9999 in Sec. 6.1) with AL-coded factors (v_bits and
-    c_bits, 8 or 16) and UF8 momentum."""
+    c_bits, 8 or 16; 32: unquantized fp32 factors, e.g. the paper's FP32-C
+    variant c_bits=32) and UF8 momentum. Each group's matrices step in one
+    grouped launch per pass."""
 
     _CODES = {"vr_codes": "v_bits", "vc_codes": "v_bits", "cr_codes": "c_bits",
               "cc_codes": "c_bits", "m_codes": None}
@@ -268,12 +325,14 @@ class CAME(_Base):
     def __init__(self, params, lr=1e-4, betas=(0.9, 0.999, 0.9999), eps=(1e-30, 1e-16),
                  clip_d=1.0, weight_decay=0.0, v_bits=16, v_block=128, c_bits=16, c_block=128,
                  m_block=256):
+        _check_bits(v_bits, "v_bits")
+        _check_bits(c_bits, "c_bits")
         defaults = dict(lr=lr, betas=betas, eps=eps, clip_d=clip_d, weight_decay=weight_decay,
                         v_bits=v_bits, v_block=v_block, c_bits=c_bits, c_block=c_block,
                         m_block=m_block, log_floor_v=_log2_floor(eps[0]),
                         log_floor_c=_log2_floor(eps[1]))
         super().__init__(params, defaults)
-        self._ws = _Workspace()
+        self._plans: dict = {}
 
     def _floor_key(self, state_key: str) -> str:
         return "log_floor_c" if state_key.startswith("c") else "log_floor_v"
@@ -287,8 +346,8 @@ class CAME(_Base):
                                ("c", group["c_bits"], group["c_block"])):
             for side, m in (("r", rows), ("c", cols)):
                 st[f"{pre}{side}_codes"] = torch.zeros(m, dtype=_code_dtype(bits), device=dev)
-                st[f"{pre}{side}_meta"] = torch.zeros(2 * _blocks(m, blk), dtype=torch.float32,
-                                                      device=dev)
+                st[f"{pre}{side}_meta"] = torch.zeros(0 if bits == 32 else 2 * _blocks(m, blk),
+                                                      dtype=torch.float32, device=dev)
         st["m_codes"] = torch.zeros(p.numel(), dtype=torch.int8, device=dev)
         st["m_absmax"] = torch.zeros(_blocks(p.numel(), group["m_block"]), dtype=torch.float32,
                                      device=dev)
@@ -305,6 +364,7 @@ class CAME(_Base):
             hp = dict(lr=group["lr"], beta1=b1, beta2=b2, beta3=b3, eps1=e1, eps2=e2,
                       clip_d=group["clip_d"], weight_decay=group["weight_decay"],
                       log_floor_v=group["log_floor_v"], log_floor_c=group["log_floor_c"])
+            buckets: dict = {}
             for p in group["params"]:
                 if p.grad is None:
                     continue
@@ -314,12 +374,14 @@ class CAME(_Base):
                 st = self.state[p]
                 st["step"] += 1
                 rows, cols = _as_matrix(p)
-                ws = self._ws.get(B.al_workspace_size(B.AL_OP_CAME, rows, cols), p.device)
-                B.al_came_step(p, p.grad, rows, cols, st["vr_codes"], st["vr_meta"],
-                               st["vc_codes"], st["vc_meta"], group["v_bits"], group["v_block"],
-                               st["cr_codes"], st["cr_meta"], st["cc_codes"], st["cc_meta"],
-                               group["c_bits"], group["c_block"], st["m_codes"],
-                               st["m_absmax"], group["m_block"], hp, st["step"], ws)
+                m = dict(p=p, g=p.grad, rows=rows, cols=cols, m_codes=st["m_codes"],
+                         m_absmax=st["m_absmax"])
+                for k in ("vr", "vc", "cr", "cc"):
+                    m[k + "_codes"], m[k + "_meta"] = st[k + "_codes"], st[k + "_meta"]
+                buckets.setdefault(st["step"], []).append(m)
+            for t, mats in buckets.items():
+                _grouped_plan(self._plans, B.AL_OP_CAME, mats, group["v_bits"], group["v_block"],
+                              group["c_bits"], group["c_block"], group["m_block"]).step(hp, t)
         return loss
 
 

@@ -213,3 +213,60 @@ def test_wrappers_reject_cpu_parameters(mods):
     p.grad = torch.zeros(16)
     with pytest.raises(ValueError):
         optim.AdamW([p]).step()
+
+
+def test_g1_grouping_fp32_roles(mods):
+    """Sec. 6.1's G1: 1-D tensors, biases, norms, embeddings and the LM head
+    get unquantized states (v_bits 32: fp32 m and v; fac_bits 32: fp32
+    factors), the rest the AL path; the FP32 AdamW group equals the oracle's
+    unquantized step bit for bit."""
+    import torch
+    import oracle as ora
+    B, optim = mods
+
+    class Tiny(torch.nn.Module):
+        def __init__(self):
+            super().__init__()
+            self.embed_tokens = torch.nn.Embedding(64, 32)
+            self.proj = torch.nn.Linear(32, 48)
+            self.norm = torch.nn.LayerNorm(48)
+            self.lm_head = torch.nn.Linear(48, 64, bias=False)
+
+    torch.manual_seed(0)
+    model = Tiny().cuda()
+    groups = optim.g1_param_groups(model.named_parameters(), dict(v_bits=32))
+    names = {id(p): n for n, p in model.named_parameters()}
+    assert [names[id(p)] for p in groups[0]["params"]] == ["proj.weight"]
+    assert len(groups[1]["params"]) == 5 and groups[1]["v_bits"] == 32
+    opt = optim.AdamW(groups, lr=1e-3, weight_decay=0.01)
+    ref = {n: p.detach().cpu().numpy().ravel().copy() for n, p in model.named_parameters()}
+    mv = {n: (np.zeros(r.size, np.float32), np.zeros(r.size, np.float32)) for n, r in ref.items()}
+    for t in (1, 2, 3):
+        for i, p in enumerate(model.parameters()):
+            p.grad = torch.from_numpy(wl.gaussian_grad(tuple(p.shape), 1e-3, 50 * t + i)).cuda()
+        for n, p in model.named_parameters():
+            if n != "proj.weight":
+                g = p.grad.cpu().numpy().ravel()
+                ora.adamw_step(ref[n], g, mv[n][0], None, mv[n][1], None, 256, 256, 32,
+                               dict(ADAMW_HP, lr=1e-3), t)
+        opt.step()
+        torch.cuda.synchronize()
+        for n, p in model.named_parameters():
+            if n != "proj.weight":
+                assert np.array_equal(ref[n].view(np.uint32),
+                                      p.detach().cpu().numpy().ravel().view(np.uint32)), (n, t)
+    st = opt.state[model.norm.weight]
+    assert st["m_codes"].dtype == torch.float32 and st["v_codes"].dtype == torch.float32
+    assert opt.state[model.proj.weight]["v_codes"].dtype == torch.uint8
+    # Adafactor G1: fp32 factors for the protected group
+    opt2 = optim.Adafactor(optim.g1_param_groups(model.named_parameters(), dict(fac_bits=32)),
+                           beta1=0.0)
+    opt2.step()
+    assert opt2.state[model.lm_head.weight]["r_codes"].dtype == torch.float32
+    assert opt2.state[model.proj.weight]["r_codes"].dtype == torch.int16
+    # CAME FP32-C: confidence factors fp32, second moment AL16
+    opt3 = optim.CAME(model.parameters(), c_bits=32)
+    opt3.step()
+    st3 = opt3.state[model.proj.weight]
+    assert st3["cr_codes"].dtype == torch.float32 and st3["vr_codes"].dtype == torch.int16
+    assert torch.all(st3["cr_codes"] > 0)
