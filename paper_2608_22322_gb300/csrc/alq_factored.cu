@@ -25,6 +25,7 @@
 // the grouped ones (one launch per pass over many matrices, tiles never
 // crossing a matrix) call the same functions, so a matrix's results do not
 // depend on which path stepped it.
+#include "alq_async.cuh"
 #include "alq_kernels.cuh"
 
 namespace alq {
@@ -101,14 +102,56 @@ struct ResidualArgs {
 // MODE 0: terms g^2 (exact two-float squares). MODE 1: terms CAME's
 // residual (u_hat - m)^2 + eps2 rounded to fp32 as the update defines it.
 // One 64-row x 512-column tile (bx over columns, by over rows); every
-// thread of the CTA calls it, with the CTA's shared scratch s_col.
+// thread of the CTA calls it, with the CTA's dynamic shared memory (see
+// SumsqSmem). Each warp walks its eight rows two at a time; the next pair's
+// loads go to shared memory by per-thread asynchronous copies while the
+// current pair is summed (each thread reads back only what it copied, so no
+// barrier is needed), which keeps the loads of two row pairs in flight
+// without holding them in registers.
+template <int MODE>
+struct SumsqSmem {
+    // per stage, warp, row of the pair, chunk and lane: g (16 bytes), and for
+    // MODE 1 the momentum codes and the block absmax (4 bytes each)
+    static constexpr int kSlots = 2 * (kThreads / 32) * 2 * 4 * 32;
+    static constexpr size_t kG = sizeof(float4) * kSlots;
+    static constexpr size_t kBytes = kG + (MODE == 1 ? 2 * sizeof(uint32_t) * kSlots : 0);
+    static_assert(kBytes >= sizeof(float2) * (kThreads / 32) * kFC, "s_col aliases the stages");
+};
+
 template <int MODE>
 __device__ __forceinline__ void sumsq_tile(const float* __restrict__ g, int rows, int cols,
                                            const ResidualArgs& ra, double* __restrict__ rowpart,
                                            double* __restrict__ colpart, int bx, int by,
-                                           float2 (*s_col)[kFC]) {
+                                           unsigned char* smem) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int c0 = bx * kFC, r0 = by * kFR;
+    float4* sg = reinterpret_cast<float4*>(smem);
+    uint32_t* sm = reinterpret_cast<uint32_t*>(smem + SumsqSmem<MODE>::kG);
+    uint32_t* sa = sm + SumsqSmem<MODE>::kSlots;
+    // this thread's slot of (stage, row q of the pair, chunk k)
+    auto slot = [&](int st, int q, int k) {
+        return (((st * (kThreads / 32) + warp) * 2 + q) * 4 + k) * 32 + lane;
+    };
+    // copies of the row pair starting at warp row 2 * it into stage it & 1
+    auto issue = [&](int it) {
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const int row = r0 + warp + 8 * (2 * it + q);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int col = c0 + 128 * k + 4 * lane;
+                const bool ok = row < rows && col < cols;
+                const int64_t idx = ok ? (int64_t)row * cols + col : 0;
+                const int sl = slot(it & 1, q, k);
+                cp_async16(smem_u32(sg + sl), g + idx, ok);
+                if (MODE == 1) {
+                    cp_async4(smem_u32(sm + sl), ra.m_codes + idx, ok);
+                    cp_async4(smem_u32(sa + sl), ra.m_absmax + (idx >> ra.m_shift), ok);
+                }
+            }
+        }
+        cp_async_commit();
+    };
     // column sums of this lane's 16 columns as 8 pairs; each row's sum as
     // two (even and odd elements) merged before the warp sum
     float2 ch[8], cl[8];
@@ -130,46 +173,33 @@ __device__ __forceinline__ void sumsq_tile(const float* __restrict__ g, int rows
     // this warp's eight row sums, row k's in lane k, converted to fp64 in
     // one instruction at the end (FP64 is slow on this part)
     float keep_h = 0.0f, keep_l = 0.0f;
-    // two rows per pass: all loads first (zero past the matrix), then the
-    // terms in row order
-    for (int rr = 0; rr < kFR / 8; rr += 2) {
-        float4 gv[2][4];
-        uint32_t mw[2][4];
-        float dm[2][4], ai[2];
+    constexpr int kIters = kFR / 16;  // row pairs per warp
+    issue(0);
+    for (int it = 0; it < kIters; ++it) {
+        if (it + 1 < kIters) issue(it + 1); else cp_async_commit();
+        cp_async_wait<1>();
 #pragma unroll
         for (int q = 0; q < 2; ++q) {
-            const int row = r0 + warp + 8 * (rr + q);
-            ai[q] = (MODE == 1 && row < rows) ? __ldg(ra.a + row) : 0.0f;
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const int col = c0 + 128 * k + 4 * lane;
-                gv[q][k] = make_float4(0.f, 0.f, 0.f, 0.f);
-                mw[q][k] = 0u;
-                dm[q][k] = 0.0f;
-                if (row < rows && col < cols) {
-                    const int64_t idx = (int64_t)row * cols + col;
-                    gv[q][k] = __ldcs(reinterpret_cast<const float4*>(g + idx));
-                    if (MODE == 1) {
-                        mw[q][k] = __ldcs(reinterpret_cast<const unsigned int*>(ra.m_codes + idx));
-                        dm[q][k] = __ldg(ra.m_absmax + (idx >> ra.m_shift)) / 127.0f;
-                    }
-                }
-            }
-        }
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-            const int row = r0 + warp + 8 * (rr + q);
+            const int row = r0 + warp + 8 * (2 * it + q);
+            const float ai = (MODE == 1 && row < rows) ? __ldg(ra.a + row) : 0.0f;
             float2 rh2 = make_float2(0.0f, 0.0f), rl2 = make_float2(0.0f, 0.0f);
             if (row < rows) {
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
                     const int col = c0 + 128 * k + 4 * lane;
                     if (col < cols) {
-                        const uint32_t mx = mw[q][k] ^ 0x80808080u;
+                        const int sl = slot(it & 1, q, k);
+                        const float4 gv = sg[sl];
+                        uint32_t mx = 0;
+                        float dm = 0.0f;
+                        if (MODE == 1) {
+                            mx = sm[sl] ^ 0x80808080u;
+                            dm = __uint_as_float(sa[sl]) / 127.0f;
+                        }
 #pragma unroll
                         for (int jp = 0; jp < 2; ++jp) {
-                            const float2 x = jp == 0 ? make_float2(gv[q][k].x, gv[q][k].y)
-                                                     : make_float2(gv[q][k].z, gv[q][k].w);
+                            const float2 x = jp == 0 ? make_float2(gv.x, gv.y)
+                                                     : make_float2(gv.z, gv.w);
                             float2 h, nl;
                             if (MODE == 0) {
                                 ff_sq2(x, neg, zero, h, nl);
@@ -178,13 +208,13 @@ __device__ __forceinline__ void sumsq_tile(const float* __restrict__ g, int rows
                                 // before it enters a sum (opaque one)
                                 const float2 bj = jp == 0 ? make_float2(bv[k].x, bv[k].y)
                                                           : make_float2(bv[k].z, bv[k].w);
-                                const float2 u = mul2(mul2(x, make_float2(ai[q], ai[q])), bj);
+                                const float2 u = mul2(mul2(x, make_float2(ai, ai)), bj);
                                 const float2 uh = mul2(u, make_float2(icf, icf));
                                 const float2 qf = make_float2(
                                     u2f(__byte_perm(mx, 0x4B400000u, 0x7640u | (2 * jp))),
                                     u2f(__byte_perm(mx, 0x4B400000u, 0x7640u | (2 * jp + 1))));
                                 const float2 mh = mul2(add2(qf, make_float2(-12583040.0f, -12583040.0f)),
-                                                       make_float2(dm[q][k], dm[q][k]));
+                                                       make_float2(dm, dm));
                                 const float2 nmk = fma2(mul2(make_float2(-ra.beta1, -ra.beta1), mh), one,
                                                         mul2(make_float2(-ra.omb1, -ra.omb1), uh));
                                 const float2 d = fma2(uh, one, nmk);  // uh - mk
@@ -200,19 +230,22 @@ __device__ __forceinline__ void sumsq_tile(const float* __restrict__ g, int rows
             float rh, rl;
             ff_merge2(rh2, rl2, rh, rl);
             ff_warp_sum(rh, rl);
-            if (lane == rr + q) {
+            if (lane == 2 * it + q) {
                 keep_h = rh;
                 keep_l = rl;
             }
         }
     }
+    cp_async_wait<0>();
     {
         const int row = r0 + warp + 8 * lane;  // lane k holds row warp + 8 k
         if (lane < kFR / 8 && row < rows)
             rowpart[(int64_t)bx * rows + row] = (double)keep_h + (double)keep_l;
     }
     // column sums: the warps' two-float sums merged in warp order, one fp64
-    // conversion per column
+    // conversion per column (the merge buffer reuses the stages)
+    float2 (*s_col)[kFC] = reinterpret_cast<float2 (*)[kFC]>(smem);
+    __syncthreads();
 #pragma unroll
     for (int k = 0; k < 4; ++k)
 #pragma unroll
@@ -235,8 +268,8 @@ template <int MODE>
 __global__ void __launch_bounds__(kThreads)
 sumsq_kernel(const float* __restrict__ g, int rows, int cols, ResidualArgs ra,
              double* __restrict__ rowpart, double* __restrict__ colpart) {
-    __shared__ float2 s_col[kThreads / 32][kFC];
-    sumsq_tile<MODE>(g, rows, cols, ra, rowpart, colpart, blockIdx.x, blockIdx.y, s_col);
+    extern __shared__ __align__(16) unsigned char s_sumsq[];
+    sumsq_tile<MODE>(g, rows, cols, ra, rowpart, colpart, blockIdx.x, blockIdx.y, s_sumsq);
 }
 
 // ---------------------------------------------------------------- factor --
@@ -625,6 +658,21 @@ update_kernel(UpdateArgs u, int64_t ntiles) {
 }
 
 // ------------------------------------------------------------- host side --
+// The sums kernels' dynamic shared memory (above the 48 KB default: one
+// opt-in per kernel; a refusal shows up as a failed launch).
+template <typename K>
+static size_t sumsq_smem_optin(K kernel, size_t bytes) {
+    cudaFuncSetAttribute((const void*)kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)bytes);
+    return bytes;
+}
+
+template <int MODE>
+static void launch_sumsq(dim3 grid, const float* g, int rows, int cols, const ResidualArgs& ra,
+                         double* rowpart, double* colpart, cudaStream_t st) {
+    static const size_t smem = sumsq_smem_optin(sumsq_kernel<MODE>, SumsqSmem<MODE>::kBytes);
+    sumsq_kernel<MODE><<<grid, kThreads, smem, st>>>(g, rows, cols, ra, rowpart, colpart);
+}
 static int cpb_of(int block) { return block >= 512 ? 4 : block / 128; }
 
 template <int MODE>
@@ -706,8 +754,7 @@ static int second_moment_passes(const float* g, int64_t rows, int64_t cols, cons
     const int ncb = (int)blocks_of(cols, kFC), nrb = (int)blocks_of(rows, kFR);
     ResidualArgs none{};
     none.one = 1.0f;
-    sumsq_kernel<0><<<dim3(ncb, nrb), kThreads, 0, st>>>(g, (int)rows, (int)cols, none,
-                                                        w.rowpart, w.colpart);
+    launch_sumsq<0>(dim3(ncb, nrb), g, (int)rows, (int)cols, none, w.rowpart, w.colpart, st);
     const int nb0 = (int)blocks_of(rows, fr.block);
     launch_factor(fr, fc, w.rsum, st);
     scale_kernel<<<(unsigned)blocks_of(rows + cols, kThreads), kThreads, 0, st>>>(
@@ -819,8 +866,7 @@ int al_came_step(float* p, const float* g, int64_t rows, int64_t cols, void* vr_
     // confidence (beta3) and the confidence scales
     ResidualArgs ra{m_codes, m_absmax, 0, w.a, w.b, w.scal, hp->beta1, omb1, hp->eps2, 1.0f, 0.0f};
     while ((1 << ra.m_shift) < m_block) ++ra.m_shift;
-    sumsq_kernel<1><<<dim3(ncb, nrb), kThreads, 0, s>>>(g, (int)rows, (int)cols, ra, w.rowpart,
-                                                       w.colpart);
+    launch_sumsq<1>(dim3(ncb, nrb), g, (int)rows, (int)cols, ra, w.rowpart, w.colpart, s);
     FactorDesc cr = factor_desc(w.rowpart, ncb, rows, cols, 0.0, hp->beta3, omb3, cr_codes,
                                 cr_meta, c_bits, c_block, hp->log_floor_c, w.fr2);
     FactorDesc cc = factor_desc(w.colpart, nrb, cols, rows, 0.0, hp->beta3, omb3, cc_codes,
@@ -923,7 +969,7 @@ __device__ __forceinline__ int fac_advance(const FacEntry* __restrict__ tab, int
 template <int MODE>
 __global__ void __launch_bounds__(kThreads)
 sumsq_multi_kernel(const FacEntry* __restrict__ tab, int nmat, FacStep fs) {
-    __shared__ float2 s_col[kThreads / 32][kFC];
+    extern __shared__ __align__(16) unsigned char s_sumsq[];
     const FacEntry& e = fac_entry(tab, nmat, blockIdx.x, &FacEntry::sq_t0);
     const int64_t lt = blockIdx.x - e.sq_t0;
     ResidualArgs ra{};
@@ -933,7 +979,7 @@ sumsq_multi_kernel(const FacEntry* __restrict__ tab, int nmat, FacStep fs) {
     ra.one = fs.one;
     ra.zero = fs.zero;
     sumsq_tile<MODE>(e.g, (int)e.rows, (int)e.cols, ra, e.w.rowpart, e.w.colpart,
-                     (int)(lt % e.ncb), (int)(lt / e.ncb), s_col);
+                     (int)(lt % e.ncb), (int)(lt / e.ncb), s_sumsq);
 }
 
 // which = 0: the second-moment factors; 1: CAME's confidence factors.
@@ -1066,7 +1112,8 @@ static void update_multi(const FacEntry* tab, int nmat, int64_t tiles, const Fac
 // scales (which also zero the RMS tickets), the RMS pass.
 static void second_moment_multi(const FacEntry* tab, const al_factored_info* info,
                                 const FacStep& fs, cudaStream_t st) {
-    sumsq_multi_kernel<0><<<(unsigned)info->sumsq_tiles, kThreads, 0, st>>>(tab, info->nmat, fs);
+    static const size_t smem0 = sumsq_smem_optin(sumsq_multi_kernel<0>, SumsqSmem<0>::kBytes);
+    sumsq_multi_kernel<0><<<(unsigned)info->sumsq_tiles, kThreads, smem0, st>>>(tab, info->nmat, fs);
     factor_multi(tab, info->nmat, fs, 0, info->factor_tiles, st);
     scale_multi_kernel<<<(unsigned)info->scale_tiles, kThreads, 0, st>>>(tab, info->nmat, fs, 0);
     usq_multi_kernel<<<persistent_grid((const void*)usq_multi_kernel, kThreads, 0, info->rms_chunks),
@@ -1253,7 +1300,8 @@ int al_came_step_multi(const void* plan_dev, const al_factored_info* info, const
     fs.one = 1.0f;
     second_moment_multi(tab, info, fs, st);
     // residual sums, confidence factors and their scales, update
-    sumsq_multi_kernel<1><<<(unsigned)info->sumsq_tiles, kThreads, 0, st>>>(tab, info->nmat, fs);
+    static const size_t smem1 = sumsq_smem_optin(sumsq_multi_kernel<1>, SumsqSmem<1>::kBytes);
+    sumsq_multi_kernel<1><<<(unsigned)info->sumsq_tiles, kThreads, smem1, st>>>(tab, info->nmat, fs);
     factor_multi(tab, info->nmat, fs, 1, info->factor2_tiles, st);
     scale_multi_kernel<<<(unsigned)info->scale_tiles, kThreads, 0, st>>>(tab, info->nmat, fs, 1);
     update_multi<2>(tab, info->nmat, info->tiles, fs, st);
