@@ -31,7 +31,8 @@
 namespace alq {
 
 constexpr int kFR = 64;   // rows per sumsq tile
-constexpr int kFC = 512;  // columns per sumsq tile
+constexpr int kFC = 256;  // columns per sumsq tile
+constexpr int kFCH = kFC / 128;  // 4-column chunks per lane
 constexpr int kUsqChunk = 8;  // tiles of kTile elements per RMS partial
 
 // ------------------------------------------------------------ workspace --
@@ -101,7 +102,7 @@ struct ResidualArgs {
 // ----------------------------------------------------------------- sumsq --
 // MODE 0: terms g^2 (exact two-float squares). MODE 1: terms CAME's
 // residual (u_hat - m)^2 + eps2 rounded to fp32 as the update defines it.
-// One 64-row x 512-column tile (bx over columns, by over rows); every
+// One 64-row x kFC-column tile (bx over columns, by over rows); every
 // thread of the CTA calls it, with the CTA's dynamic shared memory (see
 // SumsqSmem). Each warp walks its eight rows two at a time; the next pair's
 // loads go to shared memory by per-thread asynchronous copies while the
@@ -112,7 +113,7 @@ template <int MODE>
 struct SumsqSmem {
     // per stage, warp, row of the pair, chunk and lane: g (16 bytes), and for
     // MODE 1 the momentum codes and the block absmax (4 bytes each)
-    static constexpr int kSlots = 2 * (kThreads / 32) * 2 * 4 * 32;
+    static constexpr int kSlots = 2 * (kThreads / 32) * 2 * kFCH * 32;
     static constexpr size_t kG = sizeof(float4) * kSlots;
     static constexpr size_t kBytes = kG + (MODE == 1 ? 2 * sizeof(uint32_t) * kSlots : 0);
     static_assert(kBytes >= sizeof(float2) * (kThreads / 32) * kFC, "s_col aliases the stages");
@@ -130,7 +131,7 @@ __device__ __forceinline__ void sumsq_tile(const float* __restrict__ g, int rows
     uint32_t* sa = sm + SumsqSmem<MODE>::kSlots;
     // this thread's slot of (stage, row q of the pair, chunk k)
     auto slot = [&](int st, int q, int k) {
-        return (((st * (kThreads / 32) + warp) * 2 + q) * 4 + k) * 32 + lane;
+        return (((st * (kThreads / 32) + warp) * 2 + q) * kFCH + k) * 32 + lane;
     };
     // copies of the row pair starting at warp row 2 * it into stage it & 1
     auto issue = [&](int it) {
@@ -138,7 +139,7 @@ __device__ __forceinline__ void sumsq_tile(const float* __restrict__ g, int rows
         for (int q = 0; q < 2; ++q) {
             const int row = r0 + warp + 8 * (2 * it + q);
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
+            for (int k = 0; k < kFCH; ++k) {
                 const int col = c0 + 128 * k + 4 * lane;
                 const bool ok = row < rows && col < cols;
                 const int64_t idx = ok ? (int64_t)row * cols + col : 0;
@@ -152,19 +153,19 @@ __device__ __forceinline__ void sumsq_tile(const float* __restrict__ g, int rows
         }
         cp_async_commit();
     };
-    // column sums of this lane's 16 columns as 8 pairs; each row's sum as
+    // column sums of this lane's 4 kFCH columns as pairs; each row's sum as
     // two (even and odd elements) merged before the warp sum
-    float2 ch[8], cl[8];
+    float2 ch[2 * kFCH], cl[2 * kFCH];
 #pragma unroll
-    for (int k = 0; k < 8; ++k) ch[k] = cl[k] = make_float2(0.0f, 0.0f);
+    for (int k = 0; k < 2 * kFCH; ++k) ch[k] = cl[k] = make_float2(0.0f, 0.0f);
     const float2 one = make_float2(ra.one, ra.one), zero = make_float2(ra.zero, ra.zero);
     const float2 neg = make_float2(-1.0f, -1.0f);
     float icf = 0.0f;
-    float4 bv[4];  // column scales of this lane's columns (CAME residual)
+    float4 bv[kFCH];  // column scales of this lane's columns (CAME residual)
     if (MODE == 1) {
         icf = __ldg(ra.scal);
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
+        for (int k = 0; k < kFCH; ++k) {
             const int col = c0 + 128 * k + 4 * lane;
             bv[k] = col < cols ? __ldg(reinterpret_cast<const float4*>(ra.b + col))
                                : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -185,7 +186,7 @@ __device__ __forceinline__ void sumsq_tile(const float* __restrict__ g, int rows
             float2 rh2 = make_float2(0.0f, 0.0f), rl2 = make_float2(0.0f, 0.0f);
             if (row < rows) {
 #pragma unroll
-                for (int k = 0; k < 4; ++k) {
+                for (int k = 0; k < kFCH; ++k) {
                     const int col = c0 + 128 * k + 4 * lane;
                     if (col < cols) {
                         const int sl = slot(it & 1, q, k);
@@ -247,7 +248,7 @@ __device__ __forceinline__ void sumsq_tile(const float* __restrict__ g, int rows
     float2 (*s_col)[kFC] = reinterpret_cast<float2 (*)[kFC]>(smem);
     __syncthreads();
 #pragma unroll
-    for (int k = 0; k < 4; ++k)
+    for (int k = 0; k < kFCH; ++k)
 #pragma unroll
         for (int jp = 0; jp < 2; ++jp) {
             const float2 h = ch[2 * k + jp], l = cl[2 * k + jp];

@@ -97,7 +97,7 @@ def test_grouped_factored_plan_host_logic(lib):
     tiles = lambda n, t: -(-n // t)
     assert info.nmat == 3 and info.op == 2 and info.has_momentum == 1
     assert info.total_params == sum(r * c for r, c in shapes)
-    assert info.sumsq_tiles == sum(tiles(c, 512) * tiles(r, 64) for r, c in shapes)
+    assert info.sumsq_tiles == sum(tiles(c, 256) * tiles(r, 64) for r, c in shapes)
     assert info.factor_tiles == sum(tiles(r, 128) + tiles(c, 128) for r, c in shapes)
     assert info.factor2_tiles == info.factor_tiles
     assert info.scale_tiles == sum(tiles(r + c, 256) for r, c in shapes)
