@@ -5,7 +5,7 @@
 // Launch sequence of one step:
 //   project   R = bf16(G) * P^T on the tensor cores: four converter warps
 //             read 128-channel tiles of G (fp32) and write them as bf16
-//             (round to nearest even) into a 4-stage shared-memory ring in
+//             (round to nearest even) into a 2-stage shared-memory ring in
 //             the 128-byte-swizzled K-major layout, transposing when the
 //             channels are G's columns; TMA loads the matching P tiles; one
 //             thread issues tcgen05.mma (bf16 x bf16 -> fp32) into a
@@ -29,7 +29,7 @@ namespace alq {
 
 constexpr int kGM = 128;      // UMMA M (rows of A per CTA)
 constexpr int kGK = 64;       // K per stage (64 bf16 = one 128-byte swizzle row)
-constexpr int kStages = 4;
+constexpr int kStages = 2;  // two CTAs per SM: one drains its accumulator while the other streams
 constexpr int kAStage = kGM * kGK * 2;     // 16 KB
 constexpr int kBStage = 256 * kGK * 2;     // 32 KB (rank <= 256)
 constexpr int kGemmSmem = kStages * (kAStage + kBStage) + 1024 + 256;
@@ -241,19 +241,15 @@ __device__ __forceinline__ bool conv_stage(const float (&v)[64], int kb, uint8_t
     return true;
 }
 
-// All K blocks of a converter warp, the loads of block kb + 1 in flight
-// while block kb is converted and stored.
+// All K blocks of a converter warp (the other CTA on the SM keeps the
+// loads flowing while this one converts).
 template <bool RS>
 __device__ __forceinline__ bool conv_all(const GemmArgs& a, int m0, uint8_t* sA, uint32_t afull0,
                                          uint32_t empty0, int c, int lane) {
-    float va[64], vb[64];
-    conv_load<RS>(a, m0, 0, c, lane, va);
-    for (int kb = 0; kb < a.kblocks; kb += 2) {
-        if (kb + 1 < a.kblocks) conv_load<RS>(a, m0, kb + 1, c, lane, vb);
+    float va[64];
+    for (int kb = 0; kb < a.kblocks; ++kb) {
+        conv_load<RS>(a, m0, kb, c, lane, va);
         if (!conv_stage<RS>(va, kb, sA, afull0, empty0, c, lane)) return false;
-        if (kb + 1 >= a.kblocks) break;
-        if (kb + 2 < a.kblocks) conv_load<RS>(a, m0, kb + 2, c, lane, va);
-        if (!conv_stage<RS>(vb, kb + 1, sA, afull0, empty0, c, lane)) return false;
     }
     return true;
 }
@@ -268,7 +264,7 @@ __device__ __forceinline__ void project_tile(const CUtensorMap* tmB, const GemmA
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t* sA = smem;
     uint8_t* sB = smem + kStages * kAStage;
-    uint64_t* bars = (uint64_t*)(sB + kStages * kBStage);  // bfull[4], afull[4], empty[4], accum
+    uint64_t* bars = (uint64_t*)(sB + kStages * kBStage);  // bfull, afull, empty per stage; accum
     uint32_t* tmem_slot = (uint32_t*)(bars + 3 * kStages + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t bfull0 = smem_u32(bars), afull0 = smem_u32(bars + kStages);
@@ -368,7 +364,7 @@ __device__ __forceinline__ void project_tile(const CUtensorMap* tmB, const GemmA
                      : "memory");
 }
 
-__global__ void __launch_bounds__(kProjThreads, 1)
+__global__ void __launch_bounds__(kProjThreads, 2)
 apollo_project_kernel(const __grid_constant__ CUtensorMap tmB, GemmArgs a) {
     extern __shared__ uint8_t smem_raw[];
     project_tile(&tmB, a, blockIdx.x * kGM, smem_raw);
@@ -778,7 +774,7 @@ __device__ __forceinline__ int entry_for(const ApEntry* __restrict__ tab, int nm
     return cur;
 }
 
-__global__ void __launch_bounds__(kProjThreads, 1)
+__global__ void __launch_bounds__(kProjThreads, 2)
 apollo_project_multi_kernel(const ApEntry* __restrict__ tab, const uint16_t* __restrict__ tile_mat,
                             int rank, int* err) {
     extern __shared__ uint8_t smem_raw[];
