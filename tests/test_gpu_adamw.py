@@ -224,3 +224,56 @@ def test_adamw_fp32_role_single_and_plan(B):
         for h, d in zip(hs, ds):
             for k in ("p", "m", "v"):
                 assert bytes_equal(h[k], d[k].cpu().numpy()) == 0, (t, k, h["p"].size)
+
+
+def test_adamw_beyond_2_31_elements_sampled(B):
+    """One tensor of 2^31 + 4099 parameters (64-bit indexing in the kernel):
+    sampled blocks below and above 2^31, and the ragged last block, against
+    the oracle re-run from a snapshot of each block (blocks are independent).
+    An empty tensor next to it in a plan is a no-op."""
+    import torch
+    n = (1 << 31) + 4099
+    nb = (n + 255) // 256
+    p = torch.empty(n, dtype=torch.float32, device="cuda")
+    wl.torch_device_normal_(p, 0.02, 77)
+    g = torch.empty(n, dtype=torch.float32, device="cuda")
+    d = dict(p=p, g=g, m_codes=torch.zeros(n, dtype=torch.int8, device="cuda"),
+             m_absmax=torch.zeros(nb, dtype=torch.float32, device="cuda"),
+             v_codes=torch.zeros(n, dtype=torch.uint8, device="cuda"),
+             v_meta=torch.zeros(2 * nb, dtype=torch.float32, device="cuda"))
+    e = {k: torch.zeros(0, dtype=v.dtype, device="cuda") for k, v in d.items()}
+    plan = B.AdamWPlan([e, d], 256, 256, 8)
+    assert plan.info.total_elems == n
+    picks = [0, 3, (1 << 23) - 1, 1 << 23, (1 << 23) + 1, nb - 2, nb - 1]
+    for t in (1, 2):
+        wl.torch_device_normal_(g, 1e-3, 500 + t)
+        wl.torch_device_zero_(g, 0.01, 600 + t)
+        snap = []
+        for b in picks:
+            lo, hi = 256 * b, min(256 * (b + 1), n)
+            snap.append(dict(p=p[lo:hi].cpu().numpy(), g=g[lo:hi].cpu().numpy(),
+                             mc=d["m_codes"][lo:hi].cpu().numpy(),
+                             ma=d["m_absmax"][b:b + 1].cpu().numpy(),
+                             vc=d["v_codes"][lo:hi].cpu().numpy(),
+                             vm=d["v_meta"][2 * b:2 * b + 2].cpu().numpy()))
+        plan.step(ADAMW_HP, t)
+        torch.cuda.synchronize()
+        for b, s in zip(picks, snap):
+            ora.adamw_step(s["p"], s["g"], s["mc"], s["ma"], s["vc"], s["vm"], 256, 256, 8,
+                           ADAMW_HP, t)
+            lo, hi = 256 * b, min(256 * (b + 1), n)
+            for k, got in (("p", p[lo:hi]), ("mc", d["m_codes"][lo:hi]),
+                           ("ma", d["m_absmax"][b:b + 1]), ("vc", d["v_codes"][lo:hi]),
+                           ("vm", d["v_meta"][2 * b:2 * b + 2])):
+                assert bytes_equal(s[k], got.cpu().numpy()) == 0, (b, k, t)
+    assert (nb - 1) * 256 > (1 << 31) and n - (nb - 1) * 256 == 3  # ragged last block
+    del d, p, g, plan
+    torch.cuda.empty_cache()
+
+
+def test_adamw_empty_tensor_is_a_noop(B):
+    import torch
+    z = torch.zeros(0, device="cuda")
+    zc = torch.zeros(0, dtype=torch.int8, device="cuda")
+    B.al_adamw_step(z, z, zc, z, zc, z, 256, 256, 8, ADAMW_HP, 1)
+    torch.cuda.synchronize()

@@ -89,7 +89,7 @@ def _rel(a, b):
 
 
 @pytest.mark.parametrize("rows,cols", [(256, 512), (512, 256), (384, 640), (200, 332),
-                                       (332, 200)])
+                                       (332, 200), (8, 8), (16, 8), (8, 36)])
 def test_projection_matches_double_product(B, rows, cols):
     """The tcgen05 GEMM (G converted to bf16 inside the projection, both
     channel layouts, ragged K and channel tiles) against the double product

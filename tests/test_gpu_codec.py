@@ -159,3 +159,25 @@ def test_encode_fast_path_every_mantissa(B):
     torch.cuda.synchronize()
     assert bytes_equal(meta, tm.cpu().numpy()) == 0
     assert int(np.sum(tc.cpu().numpy() != codes)) == 0
+
+
+def test_codec_empty_and_tiny_inputs(B):
+    """n = 0 is a no-op; n = 1..7 (one partial block, shorter than a
+    vector) round-trips exactly as the oracle codes it."""
+    import torch
+    z = torch.zeros(0, device="cuda")
+    B.al_encode(z, 256, 8, FLOOR, torch.zeros(0, dtype=torch.uint8, device="cuda"), z)
+    B.al_decode(torch.zeros(0, dtype=torch.uint8, device="cuda"), z, 256, 8, z)
+    for n in range(1, 8):
+        x = state_mix(n, 256, seed=900 + n)
+        x[0] = 3.5e-7
+        codes, meta = ora.al_encode(x, 256, 8, FLOOR)
+        tc = torch.zeros(n, dtype=torch.uint8, device="cuda")
+        tm = torch.zeros(2, dtype=torch.float32, device="cuda")
+        B.al_encode(_dev(x), 256, 8, FLOOR, tc, tm)
+        out = torch.empty(n, dtype=torch.float32, device="cuda")
+        B.al_decode(tc, tm, 256, 8, out)
+        torch.cuda.synchronize()
+        assert bytes_equal(meta, tm.cpu().numpy()) == 0, n
+        assert np.array_equal(tc.cpu().numpy(), codes), n
+        assert bytes_equal(ora.al_decode(codes, meta, 256, 8), out.cpu().numpy()) == 0, n
