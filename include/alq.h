@@ -168,7 +168,10 @@ typedef struct {
  *   p = fma(-step, m/den, p1);
  * then m is UF8-encoded (m_block) and v is AL-encoded (v_block, log_floor).
  * The parameter update uses the fresh fp32 m and v, not their re-decoded
- * values.
+ * values. m, v, their codes and block constants are exact in this order.
+ * With v_bits 8 or 16, sqrt(v) and the division m/den are the hardware's
+ * approximations (a few ulp), so p differs from the IEEE result by a few ulp
+ * of step*|m/den|; with v_bits 32 they are IEEE and p is exact too.
  */
 int al_adamw_step(float* p, const float* g, int8_t* m_codes, float* m_absmax,
                   void* v_codes, float* v_meta, int64_t n, int m_block,

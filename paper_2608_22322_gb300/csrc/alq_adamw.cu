@@ -8,6 +8,12 @@
 // and write the codes and metadata. 16.09 bytes per parameter for AL8/UF8
 // with 256-element blocks.
 //
+// Every state value, code and block constant is the exact fp32 result of the
+// oracle's operation order. The update direction u = m / (sqrt(v) c2 + eps),
+// which moves only p, takes the hardware's approximate square root and
+// reciprocal: a parameter differs from the IEEE result by a few ulp of its
+// step lr |u|, far inside the 1e-5 relative parameter tolerance.
+//
 // The same kernel serves one tensor (descriptor passed by value) or a plan of
 // many tensors (descriptor table in device memory, tiles never crossing a
 // tensor boundary). The grid is persistent: each CTA walks tiles with a
@@ -230,8 +236,9 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
                 const float2 mm = fma2(s.beta1, mh, mul2(s.omb1, gi));
                 const float2 vh2 = make_float2(vh[4 * c + 2 * h], vh[4 * c + 2 * h + 1]);
                 const float2 vv = fma2(s.beta2, vh2, mul2(s.omb2, mul2(gi, gi)));
-                const float2 den = fma2(make_float2(sqrtf(vv.x), sqrtf(vv.y)), s.c2, s.eps);
-                const float2 u = make_float2(mm.x / den.x, mm.y / den.y);
+                // the update direction, approximately (moves p only)
+                const float2 den = fma2(make_float2(sqrt_approx(vv.x), sqrt_approx(vv.y)), s.c2, s.eps);
+                const float2 u = mul2(mm, make_float2(rcp_approx(den.x), rcp_approx(den.y)));
                 pn[h] = fma2(s.nstep, u, p1);
                 mf[2 * c + h] = mm;
                 vf2[2 * c + h] = vv;
@@ -367,7 +374,8 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
 // ------------------------------------------------ unquantized reference --
 // v_bits 32: AdamW with dense fp32 m and v (Sec. 4.5's FP32 state role, the
 // unquantized reference): the per-element arithmetic of the fused kernel
-// with m_hat = m and v_hat = v, no codec; 28 bytes per parameter. The same
+// with m_hat = m and v_hat = v, no codec, and the IEEE square root and
+// division (bit for bit the oracle's); 28 bytes per parameter. The same
 // tiles and descriptors (m_codes and v_codes hold fp32 m and v).
 __global__ void __launch_bounds__(kThreads)
 adamw_fp32_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t total_tiles,

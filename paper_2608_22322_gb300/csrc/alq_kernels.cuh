@@ -59,6 +59,24 @@ __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
 }
 
 // ------------------------------------------------------------- chunk I/O --
+// ---------------------------------------- approximate update direction --
+// The hardware's approximate square root and reciprocal (a few ulp each).
+// The fused AdamW step forms its update direction u = m / (sqrt(v) c2 + eps)
+// with them: u moves only the parameters and feeds no optimizer state, so
+// every code and block constant stays exact, and a step's parameter differs
+// from the IEEE result by a few ulp of lr |u| at most.
+__device__ __forceinline__ float sqrt_approx(float x) {
+    float r;
+    asm("sqrt.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
+    return r;
+}
+
+__device__ __forceinline__ float rcp_approx(float x) {
+    float r;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+    return r;
+}
+
 __device__ __forceinline__ int64_t blocks_of_dev(int64_t n, int block) {
     return (n + block - 1) / block;
 }

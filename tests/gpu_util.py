@@ -55,3 +55,25 @@ def bytes_equal(a: np.ndarray, b: np.ndarray) -> int:
     b = np.ascontiguousarray(b).view(np.uint8)
     assert a.shape == b.shape
     return int(np.sum(a != b))
+
+
+def step_size(p_new: np.ndarray, p_old: np.ndarray, hp: dict) -> np.ndarray:
+    """|lr * u| of an AdamW step, recovered from the oracle's parameters
+    before and after it: p_new - (1 - lr wd) p_old."""
+    decay = 1.0 - hp["lr"] * hp["weight_decay"]
+    return np.abs(p_new.astype(np.float64) - decay * p_old.astype(np.float64))
+
+
+def params_off(ref: np.ndarray, got: np.ndarray, steps: np.ndarray, rtol: float = 1e-5) -> int:
+    """Number of parameters outside |got - ref| <= rtol (|ref| + steps).
+
+    The fused AdamW kernel forms the update direction u = m / (sqrt(v) c2 +
+    eps) with the hardware's approximate square root and reciprocal (a few
+    ulp; every state, code and block constant stays exact). Over t steps a
+    parameter then drifts from the oracle's by at most about 2^-21 of the
+    summed step sizes |lr u| (steps) plus one fp32 rounding of p per step:
+    within rtol = 1e-5 of |p| + steps, the parameter tolerance of the
+    method's parity bar, for t up to a few hundred."""
+    ref = ref.astype(np.float64)
+    d = np.abs(got.astype(np.float64) - ref)
+    return int(np.sum(~(d <= rtol * (np.abs(ref) + steps))))
