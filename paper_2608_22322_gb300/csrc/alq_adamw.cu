@@ -299,7 +299,8 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
             }
         }
 
-        float vmn[NBV], vmx[NBV], nlmin[NBV], ndelta[NBV], K[NBV], E[NBV];
+        float vmn[NBV], vmx[NBV], nlmin[NBV], ndelta[NBV];
+        AlEncConsts ek[NBV];
 #pragma unroll
         for (int b = 0; b < NBV; ++b) {
             vmn[b] = u2f(bvmin[b] + 1u);
@@ -307,7 +308,7 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
         }
         al_blocks_params<NBV>(vmn, vmx, s.log_floor, nlmin, ndelta);
 #pragma unroll
-        for (int b = 0; b < NBV; ++b) al_encode_consts(ndelta[b], Lm2, K[b], E[b]);
+        for (int b = 0; b < NBV; ++b) ek[b] = al_encode_consts(nlmin[b], ndelta[b], Lm2);
         float ms[NBM], msc[NBM], minv[NBM];
 #pragma unroll
         for (int b = 0; b < NBM; ++b) {
@@ -319,7 +320,7 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
 
         // ---- encode and write the codes and block constants
         uint32_t qv[NE];
-        al_encode_chunks<VBITS, CPBV, NBV, kCH>(vf, vmn, nlmin, ndelta, K, E, qv);
+        al_encode_chunks<VBITS, CPBV, NBV, kCH, true>(vf, vmn, nlmin, ndelta, ek, qv);
 #pragma unroll
         for (int c = 0; c < kCH; ++c) {
             const int bm = c / CPBM;

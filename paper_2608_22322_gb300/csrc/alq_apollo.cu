@@ -560,7 +560,8 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
         ff_warp_sum(nrhs[b], nrls[b]);
         ff_warp_sum(nghs[b], ngls[b]);
     }
-    float vmn[NB], vmx[NB], nlmin[NB], ndelta[NB], K[NB], E[NB], ms[NB], sc[NB], inv[NB];
+    float vmn[NB], vmx[NB], nlmin[NB], ndelta[NB], ms[NB], sc[NB], inv[NB];
+    AlEncConsts ek[NB];
 #pragma unroll
     for (int b = 0; b < NB; ++b) {
         vmn[b] = u2f(bvmin[b] + 1u);
@@ -572,9 +573,9 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
     }
     al_blocks_params<NB>(vmn, vmx, m.log_floor, nlmin, ndelta);
 #pragma unroll
-    for (int b = 0; b < NB; ++b) al_encode_consts(ndelta[b], Lm2, K[b], E[b]);
+    for (int b = 0; b < NB; ++b) ek[b] = al_encode_consts(nlmin[b], ndelta[b], Lm2);
     uint32_t qv[NE];
-    al_encode_chunks<VBITS, CPB, NB, kMCH>(vf, vmn, nlmin, ndelta, K, E, qv);
+    al_encode_chunks<VBITS, CPB, NB, kMCH, true>(vf, vmn, nlmin, ndelta, ek, qv);
 #pragma unroll
     for (int c = 0; c < kMCH; ++c) {
         const int b = c / CPB;

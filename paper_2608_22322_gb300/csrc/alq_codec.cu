@@ -47,7 +47,8 @@ al_encode_kernel(const float* __restrict__ x, int64_t n, int block, float log_fl
             bmin[0] = cta_group_reduce<false>(bmin[0], s_part[0], wpb);
             bmax[0] = cta_group_reduce<true>(bmax[0], s_part[1], wpb);
         }
-        float mn[NB], mx[NB], lmin[NB], delta[NB], K[NB], E[NB];
+        float mn[NB], mx[NB], lmin[NB], delta[NB];
+        AlEncConsts ek[NB];
 #pragma unroll
         for (int b = 0; b < NB; ++b) {
             mn[b] = u2f(bmin[b] + 1u);
@@ -55,12 +56,12 @@ al_encode_kernel(const float* __restrict__ x, int64_t n, int block, float log_fl
         }
         al_blocks_params<NB>(mn, mx, log_floor, lmin, delta);
 #pragma unroll
-        for (int b = 0; b < NB; ++b) al_encode_consts(delta[b], Lm2, K[b], E[b]);
+        for (int b = 0; b < NB; ++b) ek[b] = al_encode_consts(lmin[b], delta[b], Lm2);
         float xv[16];
 #pragma unroll
         for (int e = 0; e < 16; ++e) xv[e] = f4get(v[e / 4], e % 4);
         uint32_t q[16];
-        al_encode_chunks<BITS, CPB, NB, 4>(xv, mn, lmin, delta, K, E, q);
+        al_encode_chunks<BITS, CPB, NB, 4>(xv, mn, lmin, delta, ek, q);
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
             const int64_t idx = chunk_index(seg0, c, lane);

@@ -373,9 +373,9 @@ __device__ __forceinline__ void factor_block(const FactorDesc& f, int64_t b,
         for (int w = 0; w < kThreads / 32; ++w) t += s_sum[w];
         rsum[b] = t;
     }
-    float lmin, delta, K, E;
+    float lmin, delta;
     al_block_params(u2f(vmin + 1u), u2f(vmax), f.log_floor, lmin, delta);
-    al_encode_consts(delta, Lm2, K, E);
+    const AlEncConsts ek = al_encode_consts(lmin, delta, Lm2);
 #pragma unroll
     for (int k = 0; k < KPT; ++k) {
         const int64_t i = lo + threadIdx.x + (int64_t)kThreads * k;
@@ -383,7 +383,7 @@ __device__ __forceinline__ void factor_block(const FactorDesc& f, int64_t b,
             uint32_t q = 0;
             if (v[k] != 0.0f) {
                 bool fb;
-                q = al_quantize_fast(v[k], lmin, K, E, Lm2, fb);
+                q = al_quantize_fast(v[k], ek, Lm2, fb);
                 if (fb) q = al_quantize_fp64(v[k], lmin, delta, (double)Lm2);
             }
             if (f.bits == 8)

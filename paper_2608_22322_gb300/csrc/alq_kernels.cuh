@@ -382,14 +382,14 @@ struct Arr {
 // in FP64.
 template <int BITS, int CPB, int NB, int CH>
 static __device__ __noinline__ Arr<uint32_t, 4 * CH> al_encode_fixup(
-    Arr<float, 4 * CH> x, Arr<float, NB> lmin, Arr<float, NB> delta, Arr<float, NB> K,
-    Arr<float, NB> E, Arr<uint32_t, 4 * CH> q) {
+    Arr<float, 4 * CH> x, Arr<float, NB> lmin, Arr<float, NB> delta, Arr<AlEncConsts, NB> k,
+    Arr<uint32_t, 4 * CH> q) {
     constexpr float Lm2 = BITS == 8 ? 254.0f : 65534.0f;
 #pragma unroll
     for (int e = 0; e < 4 * CH; ++e) {
         const int b = e / 4 / CPB;
         bool fb;
-        al_quantize_fast(x.v[e], lmin.v[b], K.v[b], E.v[b], Lm2, fb);
+        al_quantize_fast(x.v[e], k.v[b], Lm2, fb);
         if (x.v[e] == 0.0f)
             q.v[e] = 0u;
         else if (fb)
@@ -399,46 +399,54 @@ static __device__ __noinline__ Arr<uint32_t, 4 * CH> al_encode_fixup(
 }
 
 // Eq. (4) for the 4 CH values of a lane's chunks: al_quantize_fast on pairs
-// of values in paired instructions, branch-free, with the same fixup in
-// FP64 for values near a half-integer of t. mn is each block's minimum
-// positive value (0 for a block without one); a block with a subnormal
-// minimum sends the whole segment through the fixup, so that the fast path
-// needs no per-value subnormal test. Zero (and -0) codes as 0: its biased
-// exponent 0 gives t <= -K < 0 (l_min >= -126 without subnormals), so
-// q = rint(clip(t)) + [x != 0] = 0.
-template <int BITS, int CPB, int NB, int CH>
+// of values in paired instructions (the clamping fused multiply-adds
+// scalar), branch-free, with the same fixup in FP64 for values near a
+// half-integer of t. mn is each block's minimum positive value (0 for a
+// block without one); a block with a subnormal minimum sends the whole
+// segment through the fixup, so that the fast path needs no per-value
+// subnormal test. Zero codes as 0: its exponent field 0 gives tau <=
+// -(127 + l_min) / Delta < 0 (l_min >= -126 without subnormals), so
+// q = rint(Lm2 clip(tau)) + [x != 0] = 0. POS: every x has its sign bit
+// clear (no -0), so the exponent field needs no mask.
+template <int BITS, int CPB, int NB, int CH, bool POS = false>
 __device__ __forceinline__ void al_encode_chunks(const float (&x)[4 * CH], const float (&mn)[NB],
                                                  const float (&lmin)[NB],
-                                                 const float (&delta)[NB], const float (&K)[NB],
-                                                 const float (&E)[NB], uint32_t (&q)[4 * CH]) {
+                                                 const float (&delta)[NB],
+                                                 const AlEncConsts (&k)[NB],
+                                                 uint32_t (&q)[4 * CH]) {
     constexpr float Lm2 = BITS == 8 ? 254.0f : 65534.0f;
     bool any_fb = false;
 #pragma unroll
     for (int b = 0; b < NB; ++b) any_fb |= (mn[b] > 0.0f) & (mn[b] < 0x1p-126f);
-    const float2 e0 = make_float2(8388735.0f, 8388735.0f);  // 2^23 + 127
     const float2 rc = make_float2(12582912.0f, 12582912.0f);  // 1.5 * 2^23
+    const float2 l2 = make_float2(Lm2, Lm2);
 #pragma unroll
     for (int e = 0; e < 4 * CH; e += 2) {
         const int b = e / 4 / CPB;
         const uint32_t x0 = f2u(x[e]), x1 = f2u(x[e + 1]);
-        const float2 eb = make_float2(u2f(0x4B000000u | ((x0 >> 23) & 0xFFu)),
-                                      u2f(0x4B000000u | ((x1 >> 23) & 0xFFu)));
+        // 2^23 + the biased exponent: one funnel shift when the sign is clear
+        const float2 eb = POS ? make_float2(u2f(__funnelshift_r(x0, 0x4B000000u >> 9, 23)),
+                                            u2f(__funnelshift_r(x1, 0x4B000000u >> 9, 23)))
+                              : make_float2(u2f(0x4B000000u | ((x0 >> 23) & 0xFFu)),
+                                            u2f(0x4B000000u | ((x1 >> 23) & 0xFFu)));
         const float2 lg = make_float2(lg2_mant(u2f((x0 & 0x007FFFFFu) | 0x3F800000u)),
                                       lg2_mant(u2f((x1 & 0x007FFFFFu) | 0x3F800000u)));
-        const float2 d = add2(sub2(sub2(eb, e0), make_float2(lmin[b], lmin[b])), lg);
-        const float2 t = mul2(d, make_float2(K[b], K[b]));
-        const float2 tc = make_float2(fminf(fmaxf(t.x, 0.0f), Lm2), fminf(fmaxf(t.y, 0.0f), Lm2));
-        const float2 rr = add2(tc, rc);
-        const float2 df = sub2(tc, sub2(rr, rc));
-        const float h = 0.5f - E[b];
+        const float2 iD = make_float2(k[b].iD, k[b].iD);
+        const float2 s1 = sub2(eb, make_float2(k[b].e0p, k[b].e0p));  // e - I, exact
+        const float2 u = fma2(lg, iD, make_float2(k[b].nFiD, k[b].nFiD));
+        const float2 t1 = make_float2(fma_sat(s1.x, iD.x, u.x), fma_sat(s1.y, iD.y, u.y));
+        const float2 rr = fma2(t1, l2, rc);  // rint(Lm2 t1) + 1.5 * 2^23
+        const float2 df = fma2(t1, l2, sub2(rc, rr));
+        const float h = 0.5f - k[b].E;
         any_fb |= (fabsf(df.x) > h) | (fabsf(df.y) > h);
-        q[e] = (f2u(rr.x) - 0x4B400000u) + min(x0 << 1, 1u);
-        q[e + 1] = (f2u(rr.y) - 0x4B400000u) + min(x1 << 1, 1u);
+        q[e] = (f2u(rr.x) - 0x4B400000u) + (POS ? min(x0, 1u) : min(x0 << 1, 1u));
+        q[e + 1] = (f2u(rr.y) - 0x4B400000u) + (POS ? min(x1, 1u) : min(x1 << 1, 1u));
     }
     if (__builtin_expect(__any_sync(0xFFFFFFFFu, any_fb), 0)) {
         Arr<float, 4 * CH> xa;
         Arr<uint32_t, 4 * CH> qa;
-        Arr<float, NB> la, da, ka, ea;
+        Arr<float, NB> la, da;
+        Arr<AlEncConsts, NB> ka;
 #pragma unroll
         for (int e = 0; e < 4 * CH; ++e) {
             xa.v[e] = x[e];
@@ -448,10 +456,9 @@ __device__ __forceinline__ void al_encode_chunks(const float (&x)[4 * CH], const
         for (int b = 0; b < NB; ++b) {
             la.v[b] = lmin[b];
             da.v[b] = delta[b];
-            ka.v[b] = K[b];
-            ea.v[b] = E[b];
+            ka.v[b] = k[b];
         }
-        qa = al_encode_fixup<BITS, CPB, NB, CH>(xa, la, da, ka, ea, qa);
+        qa = al_encode_fixup<BITS, CPB, NB, CH>(xa, la, da, ka, qa);
 #pragma unroll
         for (int e = 0; e < 4 * CH; ++e) q[e] = qa.v[e];
     }
@@ -559,11 +566,11 @@ __device__ __forceinline__ float al16_decode(uint32_t q, float lmin, float delta
 // Eq. (4) element encode with the FP64 fallback near rounding boundaries.
 template <int BITS>
 __device__ __forceinline__ uint32_t al_encode_elem(float x, float lmin, float delta,
-                                                   float K, float E) {
+                                                   const AlEncConsts& k) {
     if (x == 0.0f) return 0u;
     constexpr float Lm2 = BITS == 8 ? 254.0f : 65534.0f;
     bool fb;
-    uint32_t q = al_quantize_fast(x, lmin, K, E, Lm2, fb);
+    uint32_t q = al_quantize_fast(x, k, Lm2, fb);
     if (fb) q = al_quantize_fp64(x, lmin, delta, (double)Lm2);
     return q;
 }

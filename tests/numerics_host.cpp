@@ -42,12 +42,11 @@ void alqn_al8_decode(const uint8_t* q, int64_t n, float lmin, float delta,
 void alqn_al_quantize(const float* x, int64_t n, float lmin, float delta,
                       int bits, uint32_t* codes, int64_t* fb_count) {
     float Lm2 = (float)((1u << bits) - 2u);
-    float K, E;
-    al_encode_consts(delta, Lm2, K, E);
+    const AlEncConsts ek = al_encode_consts(lmin, delta, Lm2);
     for (int64_t i = 0; i < n; ++i) {
         if (x[i] == 0.0f) { codes[i] = 0; continue; }
         bool fb;
-        uint32_t q = al_quantize_fast(x[i], lmin, K, E, Lm2, fb);
+        uint32_t q = al_quantize_fast(x[i], ek, Lm2, fb);
         if (fb) {
             ++*fb_count;
             q = al_quantize_fp64(x[i], lmin, delta, (double)Lm2);
