@@ -384,7 +384,7 @@ __device__ __forceinline__ void factor_block(const FactorDesc& f, int64_t b,
             if (v[k] != 0.0f) {
                 bool fb;
                 q = al_quantize_fast(v[k], ek, Lm2, fb);
-                if (fb) q = al_quantize_fp64(v[k], lmin, delta, (double)Lm2);
+                if (fb) q = al_quantize_refine(v[k], lmin, delta, Lm2);
             }
             if (f.bits == 8)
                 ((uint8_t*)f.codes)[i] = (uint8_t)q;

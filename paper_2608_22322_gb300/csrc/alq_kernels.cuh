@@ -364,7 +364,7 @@ __device__ __forceinline__ float2 al8_decode_pair2(float2 ah, float2 al, float2 
     const float2 r = fma2(ah, bh, c);
     const float2 t = fma2(ah, nbh, r);
     const float2 res = sub2(c, t);
-    const float2 z = fma2(res, make_float2(1.0f + 0x1p-15f, 1.0f + 0x1p-15f), r);
+    const float2 z = fma2(res, make_float2(kZivFactor, kZivFactor), r);
     fb0 = z.x != r.x;
     fb1 = z.y != r.y;
     return r;
@@ -379,7 +379,7 @@ struct Arr {
 
 // Rare path of al_encode_chunks, out of line: zero codes for zeros, redo the
 // boundary tests (with the subnormal test) and recompute the flagged codes
-// in FP64.
+// in two-float arithmetic (FP64 for the few that cannot be decided so).
 template <int BITS, int CPB, int NB, int CH>
 static __device__ __noinline__ Arr<uint32_t, 4 * CH> al_encode_fixup(
     Arr<float, 4 * CH> x, Arr<float, NB> lmin, Arr<float, NB> delta, Arr<AlEncConsts, NB> k,
@@ -393,7 +393,7 @@ static __device__ __noinline__ Arr<uint32_t, 4 * CH> al_encode_fixup(
         if (x.v[e] == 0.0f)
             q.v[e] = 0u;
         else if (fb)
-            q.v[e] = al_quantize_fp64(x.v[e], lmin.v[b], delta.v[b], (double)Lm2);
+            q.v[e] = al_quantize_refine(x.v[e], lmin.v[b], delta.v[b], Lm2);
     }
     return q;
 }
@@ -571,7 +571,7 @@ __device__ __forceinline__ uint32_t al_encode_elem(float x, float lmin, float de
     constexpr float Lm2 = BITS == 8 ? 254.0f : 65534.0f;
     bool fb;
     uint32_t q = al_quantize_fast(x, k, Lm2, fb);
-    if (fb) q = al_quantize_fp64(x, lmin, delta, (double)Lm2);
+    if (fb) q = al_quantize_refine(x, lmin, delta, Lm2);
     return q;
 }
 

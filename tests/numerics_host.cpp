@@ -49,6 +49,23 @@ void alqn_al_quantize(const float* x, int64_t n, float lmin, float delta,
         uint32_t q = al_quantize_fast(x[i], ek, Lm2, fb);
         if (fb) {
             ++*fb_count;
+            q = al_quantize_refine(x[i], lmin, delta, Lm2);
+        }
+        codes[i] = q;
+    }
+}
+
+// Two-float Eq. (4) alone for every nonzero value (FP64 where it cannot
+// decide); undecided counts those.
+void alqn_al_quantize_ff(const float* x, int64_t n, float lmin, float delta, int bits,
+                         uint32_t* codes, int64_t* undecided) {
+    float Lm2 = (float)((1u << bits) - 2u);
+    for (int64_t i = 0; i < n; ++i) {
+        if (x[i] == 0.0f) { codes[i] = 0; continue; }
+        bool ok;
+        uint32_t q = al_quantize_ff(x[i], lmin, delta, Lm2, ok);
+        if (!ok) {
+            ++*undecided;
             q = al_quantize_fp64(x[i], lmin, delta, (double)Lm2);
         }
         codes[i] = q;

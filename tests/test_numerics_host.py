@@ -47,6 +47,7 @@ def lib():
                                   C.c_float, f32p, C.POINTER(C.c_int64)]
     L.alqn_al_quantize.argtypes = [f32p, C.c_int64, C.c_float, C.c_float, C.c_int,
                                    np.ctypeslib.ndpointer(np.uint32), C.POINTER(C.c_int64)]
+    L.alqn_al_quantize_ff.argtypes = L.alqn_al_quantize.argtypes
     return L
 
 
@@ -133,3 +134,30 @@ def test_al_quantize_fast_matches_oracle(lib, bits):
         n_total += 512
     limit = 2e-3 if bits == 8 else 0.2  # AL16's 65534 levels exceed fp32 resolution
     assert fb.value < n_total * limit, (fb.value, n_total)
+
+
+@pytest.mark.parametrize("bits", [8, 16])
+def test_al_quantize_two_float_matches_oracle(lib, bits):
+    """The two-float Eq. (4) that refines the values the fp32 fast path
+    cannot decide, on values placed within 1e-4 of the half-integers of t
+    (where the fast path gives up) and on random ones, equals the oracle's
+    double expression; it leaves a tiny fraction to FP64."""
+    r = wl.rng(40 + bits)
+    Lm2 = (1 << bits) - 2
+    floor_ = np.float32(math.log2(1e-16))
+    und = C.c_int64(0)
+    n_total = 0
+    for _ in range(300):
+        spread = float(r.choice([0.5, 5.0, 20.0, 60.0]))
+        lo = float(r.uniform(-60, -20))
+        x = np.exp2(r.uniform(lo, lo + spread, 512)).astype(np.float32)
+        lm, de, _ = ora.al_block_meta(x, float(floor_))
+        # half of them next to a code boundary: t = k + 0.5 +- 1e-4
+        k = r.integers(0, Lm2, 256) + 0.5 + r.uniform(-1e-4, 1e-4, 256)
+        x[:256] = np.exp2(float(lm) + k * float(de) / Lm2).astype(np.float32)
+        q = np.zeros(512, np.uint32)
+        lib.alqn_al_quantize_ff(x, 512, float(lm), float(de), bits, q, C.byref(und))
+        want = np.array([ora.al_quantize(float(v), lm, de, bits) for v in x], np.uint32)
+        np.testing.assert_array_equal(q, want)
+        n_total += 512
+    assert und.value < n_total * 1e-3, (und.value, n_total)
