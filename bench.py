@@ -575,13 +575,15 @@ def _row_came(torch, np, wl, B, dev):
              cr_meta=m["cr"][1], cc_codes=m["cc"][0], cc_meta=m["cc"][1], m_codes=m["mc"],
              m_absmax=m["ma"]) for m in grp], 16, vb, 16, cb, 256) for grp in groups]
         for k in range(2)]
-    streams = [torch.cuda.Stream(device=dev) for _ in range(ngroups)]
+    nstreams = int(os.environ.get("ALQ_BENCH_STREAMS", str(ngroups)))
+    streams = [torch.cuda.Stream(device=dev) for _ in range(nstreams)]
 
     def step(t):
         main = torch.cuda.current_stream(dev)
-        for st, plan in zip(streams, plans[t % 2]):
+        for st in streams:
             st.wait_stream(main)
-            plan.step(hp, t, stream=st)
+        for i, plan in enumerate(plans[t % 2]):
+            plan.step(hp, t, stream=streams[i % nstreams])
         for st in streams:
             main.wait_stream(st)
 
@@ -606,7 +608,7 @@ def _row_came(torch, np, wl, B, dev):
     return dict(step=step, n=nm * n1, bytes=nbytes, launches=8 * ngroups, oracle=oracle_sample,
                 workload=f"CAME {nm} x {rows}x{cols}, AL16 factored V and C block 128, "
                          f"UF8 momentum block 256, grouped steps (al_came_step_multi) over "
-                         f"{ngroups} groups of matrices on {ngroups} streams",
+                         f"{ngroups} groups of matrices on {nstreams} streams",
                 bytes_note="algorithmic minimum 14.03 B/param (G read once)")
 
 

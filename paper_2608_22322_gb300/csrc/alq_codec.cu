@@ -13,8 +13,11 @@ static int grid_for(Kernel kernel, int64_t ntiles) {
 }
 
 // ------------------------------------------------------------- AL encode --
+// Three CTAs per SM (at most 80 registers; four, 64 registers, for blocks of
+// 512): the per-block chain (reduction, two-float log2, constants) is
+// latency bound, and more resident warps hide more of it.
 template <int CPB, int BITS>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, CPB == 4 ? 4 : 3)
 al_encode_kernel(const float* __restrict__ x, int64_t n, int block, float log_floor,
                  void* __restrict__ codes, float* __restrict__ meta, int64_t ntiles) {
     constexpr int NB = 4 / CPB;
