@@ -275,8 +275,9 @@ sumsq_kernel(const float* __restrict__ g, int rows, int cols, ResidualArgs ra,
 
 // ---------------------------------------------------------------- factor --
 // One factor vector's update: stat_i = sum_p part[p][i] / mean_len + add_eps
-// (fp64, fixed order, rounded once), fresh = beta * decode(old) + omb * stat,
-// then AL re-encoding of each block.
+// (fp64, fixed order: partial p into accumulator p mod 4, the four added
+// pairwise; rounded once), fresh = beta * decode(old) + omb * stat, then AL
+// re-encoding of each block.
 struct FactorDesc {
     const double* part;
     int nparts;
@@ -318,18 +319,29 @@ __device__ __forceinline__ void factor_block(const FactorDesc& f, int64_t b,
         const int64_t i = lo + threadIdx.x + (int64_t)kThreads * k;
         v[k] = 0.0f;
         if (i < hi) {
-            // partials in index order; loads issued eight at a time
-            double s = 0.0;
+            // partials in a fixed order: loads issued 32 at a time (one
+            // memory round trip per 32 partials), summed into four
+            // accumulators (partial p into accumulator p mod 4, in index
+            // order), which are then added as (a0 + a1) + (a2 + a3)
+            double a[4] = {0.0, 0.0, 0.0, 0.0};
             const double* pp = f.part + i;
             int p = 0;
-            for (; p + 8 <= f.nparts; p += 8) {
-                double t8[8];
+            for (; p + 32 <= f.nparts; p += 32) {
+                double t32[32];
 #pragma unroll
-                for (int q = 0; q < 8; ++q) t8[q] = pp[(int64_t)(p + q) * f.len];
+                for (int q = 0; q < 32; ++q) t32[q] = pp[(int64_t)(p + q) * f.len];
 #pragma unroll
-                for (int q = 0; q < 8; ++q) s += t8[q];
+                for (int q = 0; q < 32; ++q) a[q & 3] += t32[q];
             }
-            for (; p < f.nparts; ++p) s += pp[(int64_t)p * f.len];
+            for (; p + 4 <= f.nparts; p += 4) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) a[q] += pp[(int64_t)(p + q) * f.len];
+            }
+            // p is a multiple of 4 here: the last 0-3 partials
+#pragma unroll
+            for (int q = 0; q < 3; ++q)
+                if (p + q < f.nparts) a[q] += pp[(int64_t)(p + q) * f.len];
+            const double s = (a[0] + a[1]) + (a[2] + a[3]);
             const float stat = (float)(s / f.mean_len + f.add_eps);
             const float old = raw ? ((const float*)f.codes)[i]
                                   : al_decode_direct(fac_code(f, i), om.x, om.y, Lm2);
