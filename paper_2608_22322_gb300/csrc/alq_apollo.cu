@@ -524,9 +524,11 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
             const float2 vh2 = make_float2(vh[4 * c + 2 * i], vh[4 * c + 2 * i + 1]);
             const float2 mq = fma2(mul2(b1, mh), one, mul2(o1, rv));
             const float2 vq = fma2(mul2(b2, vh2), one, mul2(o2, mul2(rv, rv)));
-            const float2 den = fma2(mul2(make_float2(sqrtf(vq.x), sqrtf(vq.y)), c2), one, eps);
+            // the bias-corrected ratio feeds only the channel scales (so
+            // only p): approximate square root and reciprocal
+            const float2 den = fma2(mul2(make_float2(sqrt_approx(vq.x), sqrt_approx(vq.y)), c2), one, eps);
             const float2 num = mul2(mq, ic1);
-            const float2 rt = make_float2(num.x / den.x, num.y / den.y);
+            const float2 rt = mul2(num, make_float2(rcp_approx(den.x), rcp_approx(den.y)));
             mf2[2 * c + i] = mq;
             vf[4 * c + 2 * i] = vq.x;
             vf[4 * c + 2 * i + 1] = vq.y;
