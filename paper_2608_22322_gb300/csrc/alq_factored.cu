@@ -476,23 +476,39 @@ __device__ __forceinline__ double usq_chunk_sum(const UsqArgs& q, int64_t chunk,
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const float2 zero = make_float2(q.zero, q.zero), neg = make_float2(-1.0f, -1.0f);
     float2 hi2 = make_float2(0.0f, 0.0f), lo2 = make_float2(0.0f, 0.0f);
-    for (int k = 0; k < kUsqChunk; ++k) {
-        const int64_t seg0 = (chunk * kUsqChunk + k) * kTile + (int64_t)warp * kSeg;
-        if (seg0 >= q.n) break;
+    // the gradient loads of two tiles in flight per step (the row and column
+    // scales, small and cached, are read as they are used), accumulated in
+    // tile, chunk and element order: the order of one tile at a time
+    for (int k = 0; k < kUsqChunk; k += 2) {
+        float4 gv[2][4];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            const int64_t idx = chunk_index(seg0, c, lane);
-            if (idx < q.n) {
-                const uint32_t row = divide((uint32_t)idx, q.dv);
-                const uint32_t col = (uint32_t)idx - row * q.dv.d;
-                const float4 gv = __ldcs(reinterpret_cast<const float4*>(q.g + idx));
-                const float4 bv = __ldg(reinterpret_cast<const float4*>(q.b + col));
-                const float2 ai = make_float2(__ldg(q.a + row), __ldg(q.a + row));
+        for (int kk = 0; kk < 2; ++kk) {
+            const int64_t seg0 = (chunk * kUsqChunk + k + kk) * kTile + (int64_t)warp * kSeg;
 #pragma unroll
-                for (int jp = 0; jp < 2; ++jp) {
-                    const float2 x = jp == 0 ? make_float2(gv.x, gv.y) : make_float2(gv.z, gv.w);
-                    const float2 bj = jp == 0 ? make_float2(bv.x, bv.y) : make_float2(bv.z, bv.w);
-                    ff_acc_sq2(hi2, lo2, mul2(mul2(x, ai), bj), neg, zero);  // u = (g a_i) b_j
+            for (int c = 0; c < 4; ++c) {
+                const int64_t idx = chunk_index(seg0, c, lane);
+                gv[kk][c] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (idx < q.n) gv[kk][c] = __ldcs(reinterpret_cast<const float4*>(q.g + idx));
+            }
+        }
+#pragma unroll
+        for (int kk = 0; kk < 2; ++kk) {
+            const int64_t seg0 = (chunk * kUsqChunk + k + kk) * kTile + (int64_t)warp * kSeg;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                const int64_t idx = chunk_index(seg0, c, lane);
+                if (idx < q.n) {
+                    const uint32_t row = divide((uint32_t)idx, q.dv);
+                    const uint32_t col = (uint32_t)idx - row * q.dv.d;
+                    const float4 bv = __ldg(reinterpret_cast<const float4*>(q.b + col));
+                    const float2 ai = make_float2(__ldg(q.a + row), __ldg(q.a + row));
+                    const float4& g4 = gv[kk][c];
+#pragma unroll
+                    for (int jp = 0; jp < 2; ++jp) {
+                        const float2 x = jp == 0 ? make_float2(g4.x, g4.y) : make_float2(g4.z, g4.w);
+                        const float2 bj = jp == 0 ? make_float2(bv.x, bv.y) : make_float2(bv.z, bv.w);
+                        ff_acc_sq2(hi2, lo2, mul2(mul2(x, ai), bj), neg, zero);  // u = (g a_i) b_j
+                    }
                 }
             }
         }
