@@ -112,7 +112,9 @@ __device__ __forceinline__ PlanEntry plan_entry(const PlanEntry* table, int nten
 // Four CTAs per SM (64 registers): the step is bound by the latency of each
 // warp's dependent chains more than by issue slots, and 32 resident warps
 // hide more of it than 24 do, despite a few spilled registers.
-template <int CPBV, int CPBM, int VBITS>
+// WIDE: AL8 blocks wider than a segment (512 .. 2048 elements), whose value
+// table is built once per block by the warps that share it.
+template <int CPBV, int CPBM, int VBITS, bool WIDE = false>
 __global__ void __launch_bounds__(kThreads, 4)
 adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t total_tiles,
                    PlanEntry single, int v_block, int m_block, AdamWPairs s) {
@@ -190,7 +192,15 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
         // ---- decode the previous states
         float vh[NE];
         if constexpr (VBITS == 8) {
-            if constexpr (NBV == 1) {
+            if constexpr (WIDE) {
+                // the group's first warp computes the block's levels, then
+                // every warp of the group its share of the 255 values
+                const int g0 = (warp / wpbv) * wpbv;
+                if (warp == g0) al8_build_tables<1>(s_tab[g0][0], olmin, odelta, kf);
+                __syncthreads();
+                al8_values_part(s_val[g0], s_tab[g0][0], olmin[0], odelta[0], warp - g0, wpbv);
+                __syncthreads();
+            } else if constexpr (NBV == 1) {
                 al8_build_values<1>(s_val[warp], s_tab[warp][0], olmin, odelta, kf);
             } else {
                 // two blocks per segment: their levels in one paired pass
@@ -198,9 +208,10 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
                                   olmin[1], odelta[1], kf, ok2);
                 al8_values_from_tables<NBV>(s_val[warp], s_tab[warp][0], olmin, odelta);
             }
+            const float* vt = s_val[WIDE ? (warp / wpbv) * wpbv : warp];
 #pragma unroll
             for (int e = 0; e < NE; ++e)
-                vh[e] = s_val[warp][256 * (e / 4 / CPBV) + ((vw[e / 4] >> (8 * (e % 4))) & 0xFFu)];
+                vh[e] = vt[256 * (e / 4 / CPBV) + ((vw[e / 4] >> (8 * (e % 4))) & 0xFFu)];
         } else {
 #pragma unroll
             for (int e = 0; e < NE; ++e)
@@ -424,7 +435,9 @@ template <int CPBV, int CPBM, int VBITS>
 static int launch_adamw_t(const PlanEntry* table, int ntensors, int64_t total_tiles,
                           const PlanEntry& single, int v_block, int m_block,
                           const AdamWScalars& s, cudaStream_t stream) {
-    auto k = adamw_fused_kernel<CPBV, CPBM, VBITS>;
+    constexpr bool kWideOk = VBITS == 8 && CPBV == kCH;
+    auto k = kWideOk && v_block > kASeg ? adamw_fused_kernel<CPBV, CPBM, VBITS, kWideOk>
+                                        : adamw_fused_kernel<CPBV, CPBM, VBITS, false>;
     const int grid = persistent_grid((const void*)k, kThreads, 0, total_tiles);
     k<<<grid, kThreads, 0, stream>>>(table, ntensors, total_tiles, single, v_block, m_block,
                                      adamw_pairs(s));

@@ -524,6 +524,68 @@ __device__ __forceinline__ void al8_values_from_tables(float* vals, const float2
     __syncwarp();
 }
 
+// Rare path of al8_values_part: this warp's share of codes (steps j0 ..
+// j0 + nsteps - 1, halves in hmask) recomputed in FP64 where the product
+// could not be certified or the block is outside the fast range.
+static __device__ __noinline__ void al8_values_part_fixup(float* vals, const float2* tab,
+                                                          float lmin, float delta, int j0,
+                                                          int nsteps, uint32_t hmask) {
+    const int lane = threadIdx.x & 31;
+    const bool fast = al8_fast_ok(lmin, delta);
+    for (int j = j0; j < j0 + nsteps; ++j) {
+        for (int h = 0; h < 2; ++h) {
+            if (!((hmask >> h) & 1u)) continue;
+            const uint32_t q = (uint32_t)(lane + 64 * j + 32 * h);
+            const float2 A = tab[al8_hi_slot(q >> 4)];
+            const float2 Bt = tab[q & 15u];
+            bool fb;
+            al8_decode_pair(A.x, A.y, Bt.x, Bt.y, fb);
+            if ((q != 0u) && (fb || !fast)) vals[q] = al_dequantize_fp64(q, lmin, delta, 254.0);
+        }
+    }
+}
+
+// One block's value table shared by the wpb (2, 4 or 8) warps whose segments
+// it spans: warp r of the group computes its share of the pair steps of
+// al8_values_from_tables (step j covers codes l + 64 j and l + 64 j + 32;
+// wpb 2: steps 2 r, 2 r + 1; wpb 4: step r; wpb 8: one half of step r / 2),
+// from the block's level tables in tab, with the same products, the same
+// certification and the same FP64 recomputation, so every value is the one
+// al8_values_from_tables stores. The caller synchronises the group before
+// and after.
+__device__ __forceinline__ void al8_values_part(float* vals, const float2* tab, float lmin,
+                                                float delta, int r, int wpb) {
+    const int lane = threadIdx.x & 31;
+    const int nsteps = wpb == 2 ? 2 : 1;
+    const int j0 = wpb == 8 ? (r >> 1) : r * nsteps;
+    const uint32_t hmask = wpb == 8 ? (1u << (r & 1)) : 3u;
+    const float2 Bt = tab[lane & 15];
+    const float2 bh = make_float2(Bt.x, Bt.x), bl = make_float2(Bt.y, Bt.y);
+    const float2 nbh = make_float2(-Bt.x, -Bt.x);
+    const float4* A4 = reinterpret_cast<const float4*>(tab + 16 + 8 * (lane >> 4));
+    bool any_fb = !al8_fast_ok(lmin, delta);
+#pragma unroll
+    for (int s = 0; s < 2; ++s) {
+        if (s >= nsteps) break;
+        const int j = j0 + s;
+        const float4 a = A4[j];
+        bool f0, f1;
+        const float2 v = al8_decode_pair2(make_float2(a.x, a.z), make_float2(a.y, a.w), bh, bl,
+                                          nbh, f0, f1);
+        const uint32_t q0 = (uint32_t)(lane + 64 * j);
+        if (hmask & 1u) {
+            vals[q0] = q0 == 0u ? 0.0f : v.x;
+            any_fb |= (q0 != 0u) & f0;
+        }
+        if (hmask & 2u) {
+            vals[q0 + 32] = v.y;
+            any_fb |= f1;
+        }
+    }
+    if (__builtin_expect(__any_sync(0xFFFFFFFFu, any_fb), 0))
+        al8_values_part_fixup(vals, tab, lmin, delta, j0, nsteps, hmask);
+}
+
 template <int NB>
 __device__ __forceinline__ void al8_build_values(float* vals, float2* tab,
                                                  const float (&lmin)[NB],
