@@ -123,7 +123,9 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
     constexpr int NBM = kCH / CPBM;
     constexpr int NE = 4 * kCH;
     constexpr float Lm2 = VBITS == 8 ? 254.0f : 65534.0f;
-    __shared__ __align__(16) float2 s_tab[kThreads / 32][1][NBV * 32];
+    // level tables; one block per segment: two slots, alternating between
+    // iterations, written by the even warp of each pair
+    __shared__ __align__(16) float2 s_tab[kThreads / 32][NBV == 1 ? 2 : 1][NBV * 32];
     __shared__ float s_val[kThreads / 32][VBITS == 8 ? NBV * 256 : 1];
     __shared__ uint32_t s_part[2][3][kThreads / 32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -134,6 +136,7 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
     const int G = gridDim.x;
     int cur = 0;
     int parity = 0;  // slot of the next cross-warp block reduction
+    int tslot = 0;   // level-table slot of this iteration
     for (int64_t tile = blockIdx.x; tile < total_tiles; tile += G) {
         const PlanEntry d = plan_entry(table, ntensors, single, tile, cur);
         const int64_t n = d.n;
@@ -201,7 +204,24 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
                 al8_values_part(s_val[g0], s_tab[g0][0], olmin[0], odelta[0], warp - g0, wpbv);
                 __syncthreads();
             } else if constexpr (NBV == 1) {
-                al8_build_values<1>(s_val[warp], s_tab[warp][0], olmin, odelta, kf);
+                // warps 2k and 2k + 1 hold adjacent blocks of one tensor: the
+                // even warp computes both blocks' levels in one paired pass
+                // (the scalar pass's roundings, so the same entries) and the
+                // pair meets at a 64-thread barrier. The slots alternate, so
+                // the even warp never overwrites a table the odd one reads.
+                if ((warp & 1) == 0) {
+                    float l1 = 0.0f, d1 = 0.0f;
+                    if (seg0 + kASeg < n) {
+                        const float2 mt = __ldg(reinterpret_cast<const float2*>(d.v_meta) + vb0 + 1);
+                        l1 = mt.x;
+                        d1 = mt.y;
+                    }
+                    al8_build_tables2(s_tab[warp][tslot], s_tab[warp + 1][tslot], olmin[0],
+                                      odelta[0], l1, d1, kf, ok2);
+                }
+                asm volatile("bar.sync %0, 64;" ::"r"(1 + (warp >> 1)) : "memory");
+                al8_values_from_tables<1>(s_val[warp], s_tab[warp][tslot], olmin, odelta);
+                tslot ^= 1;
             } else {
                 // two blocks per segment: their levels in one paired pass
                 al8_build_tables2(s_tab[warp][0], s_tab[warp][0] + 32, olmin[0], odelta[0],
