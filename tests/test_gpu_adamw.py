@@ -110,20 +110,23 @@ def test_adamw_al16(B, m_block, v_block):
     _run_single(B, w, m_block, v_block, 16, 4)
 
 
-def test_adamw_plan_many_tensors(B):
-    """Multi-tensor plan: tiny, ragged and multi-tile tensors in one launch."""
+@pytest.mark.parametrize("v_block", [2048, 256])
+def test_adamw_plan_many_tensors(B, v_block):
+    """Multi-tensor plan: tiny, ragged and multi-tile tensors in one launch
+    (V blocks of 2048 shared by a CTA's warps; of 256, one per warp with
+    the warp pairs' shared level pass)."""
     import torch
     sizes = [1, 5, 4095, 4097, 300, 2 * 4096 + 511, 17, 64 * 1024]
     pairs, gens = [], []
     for i, n in enumerate(sizes):
         p0 = wl.param_init((n,), 40 + i, norm_vector_value=0.5) if i % 2 else \
             (wl.rng(40 + i).standard_normal(n) * 0.02).astype(np.float32)
-        pairs.append(Pair(p0, 256, 2048, 8))
+        pairs.append(Pair(p0, 256, v_block, 8))
         gens.append(lambda t, n=n, i=i: wl.gaussian_grad((n,), 1e-3, 900 + 31 * i + t,
                                                          wl.zero_mask((n,), 0.1, 77 + i)))
     gdev = [torch.zeros(n, dtype=torch.float32, device="cuda") for n in sizes]
     plan = B.AdamWPlan([dict(g=gdev[i], **pr.dev_args()) for i, pr in enumerate(pairs)],
-                       256, 2048, 8)
+                       256, v_block, 8)
     for t in range(1, 4):
         for i, pr in enumerate(pairs):
             g = gens[i](t)
