@@ -137,6 +137,8 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
     int cur = 0;
     int parity = 0;  // slot of the next cross-warp block reduction
     int tslot = 0;   // level-table slot of this iteration
+    int wit = 0;     // WIDE: this iteration's index within its look-ahead round
+    int curL = 0;    // WIDE: descriptor cursor of the look-ahead lookups
     for (int64_t tile = blockIdx.x; tile < total_tiles; tile += G) {
         const PlanEntry d = plan_entry(table, ntensors, single, tile, cur);
         const int64_t n = d.n;
@@ -196,13 +198,33 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
         float vh[NE];
         if constexpr (VBITS == 8) {
             if constexpr (WIDE) {
-                // the group's first warp computes the block's levels, then
-                // every warp of the group its share of the 255 values
-                const int g0 = (warp / wpbv) * wpbv;
-                if (warp == g0) al8_build_tables<1>(s_tab[g0][0], olmin, odelta, kf);
+                // every wpbv iterations, warp r of a group computes the levels
+                // of the group's block at tile + r G (all at once, one
+                // barrier); every iteration, each warp of the group its share
+                // of the 255 values. A block's constants change only when
+                // its own tile is processed, after they have been used.
+                const int g0 = (warp / wpbv) * wpbv, r = warp - g0;
+                if (wit == 0) {
+                    float la[1] = {olmin[0]}, da[1] = {odelta[0]};
+                    if (r > 0) {
+                        la[0] = da[0] = 0.0f;
+                        const int64_t tx = tile + (int64_t)r * G;
+                        if (tx < total_tiles) {
+                            const PlanEntry dx = plan_entry(table, ntensors, single, tx, curL);
+                            const int64_t sx = (tx - dx.first_tile) * kATile + (int64_t)g0 * kASeg;
+                            if (sx < dx.n) {
+                                const float2 mt = __ldg(reinterpret_cast<const float2*>(dx.v_meta) + (sx >> v_shift));
+                                la[0] = mt.x;
+                                da[0] = mt.y;
+                            }
+                        }
+                    }
+                    al8_build_tables<1>(s_tab[warp][0], la, da, kf);
+                    __syncthreads();
+                }
+                al8_values_part(s_val[g0], s_tab[g0 + wit][0], olmin[0], odelta[0], r, wpbv);
                 __syncthreads();
-                al8_values_part(s_val[g0], s_tab[g0][0], olmin[0], odelta[0], warp - g0, wpbv);
-                __syncthreads();
+                wit = wit + 1 == wpbv ? 0 : wit + 1;
             } else if constexpr (NBV == 1) {
                 // warps 2k and 2k + 1 hold adjacent blocks of one tensor: the
                 // even warp computes both blocks' levels in one paired pass
