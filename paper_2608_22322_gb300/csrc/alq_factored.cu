@@ -30,6 +30,40 @@
 
 namespace alq {
 
+// ------------------------------------------- programmatic dependent launch --
+// The passes of a step form a dependent chain on one stream. Each is launched
+// with programmatic stream serialization: every CTA first allows the next
+// pass to be launched (its CTAs take SM slots as this pass's CTAs retire, and
+// its launch latency overlaps this pass), then waits until the previous
+// grid has completed and its memory operations are visible. Every memory
+// access of a pass comes after that wait, so the order of reads and writes
+// is the order of the stream.
+__device__ __forceinline__ void pdl_entry() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// The grouped passes (several matrices per launch, groups on several
+// streams) launch without the attribute: there, dependent CTAs waiting on SM
+// slots took them from the other streams' passes (measured slower); the
+// instructions of pdl_entry() are then no-ops.
+template <typename... KArgs, typename... Args>
+static void pdl_launch(bool dependent, void (*k)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = dependent ? 1 : 0;
+    cudaLaunchKernelEx(&cfg, k, args...);  // errors surface through check_launch()
+}
+
+
 constexpr int kFR = 64;   // rows per sumsq tile
 constexpr int kFC = 256;  // columns per sumsq tile
 constexpr int kFCH = kFC / 128;  // 4-column chunks per lane
@@ -269,6 +303,7 @@ template <int MODE>
 __global__ void __launch_bounds__(kThreads)
 sumsq_kernel(const float* __restrict__ g, int rows, int cols, ResidualArgs ra,
              double* __restrict__ rowpart, double* __restrict__ colpart) {
+    pdl_entry();
     extern __shared__ __align__(16) unsigned char s_sumsq[];
     sumsq_tile<MODE>(g, rows, cols, ra, rowpart, colpart, blockIdx.x, blockIdx.y, s_sumsq);
 }
@@ -411,6 +446,7 @@ __device__ __forceinline__ void factor_block(const FactorDesc& f, int64_t b,
 template <int KPT>
 __global__ void __launch_bounds__(kThreads)
 factor_kernel(FactorDesc f0, FactorDesc f1, int nb0, double* __restrict__ rsum) {
+    pdl_entry();
     const bool first = (int)blockIdx.x < nb0;
     factor_block<KPT>(first ? f0 : f1, first ? blockIdx.x : blockIdx.x - nb0,
                       first ? rsum : nullptr);
@@ -445,6 +481,7 @@ __global__ void __launch_bounds__(kThreads)
 scale_kernel(const float* __restrict__ R, int rows, const float* __restrict__ C, int cols,
              const double* __restrict__ rsum, int nrb, float* __restrict__ a,
              float* __restrict__ b, unsigned int* __restrict__ ticket) {
+    pdl_entry();
     scale_tile(R, rows, C, cols, rsum, nrb, a, b, ticket, blockIdx.x);
 }
 
@@ -561,6 +598,7 @@ __device__ __forceinline__ void usq_chunk(const UsqArgs& q, int64_t chunk, float
 
 __global__ void __launch_bounds__(kThreads)
 usq_kernel(UsqArgs q, float clip_d) {
+    pdl_entry();
     __shared__ float2 s_w[kThreads / 32];
     __shared__ double s_d[kThreads];
     __shared__ bool s_last;
@@ -681,6 +719,7 @@ __device__ __forceinline__ void update_tile(const UpdateArgs& u, int64_t tile, u
 template <int MODE, int CPBM>
 __global__ void __launch_bounds__(kThreads)
 update_kernel(UpdateArgs u, int64_t ntiles) {
+    pdl_entry();
     __shared__ uint32_t s_part[kThreads / 32];
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x)
         update_tile<MODE, CPBM>(u, tile, s_part);
@@ -700,7 +739,8 @@ template <int MODE>
 static void launch_sumsq(dim3 grid, const float* g, int rows, int cols, const ResidualArgs& ra,
                          double* rowpart, double* colpart, cudaStream_t st) {
     static const size_t smem = sumsq_smem_optin(sumsq_kernel<MODE>, SumsqSmem<MODE>::kBytes);
-    sumsq_kernel<MODE><<<grid, kThreads, smem, st>>>(g, rows, cols, ra, rowpart, colpart);
+    pdl_launch(true, sumsq_kernel<MODE>, dim3(grid), dim3(kThreads), smem, st, g, rows, cols, ra,
+               rowpart, colpart);
 }
 static int cpb_of(int block) { return block >= 512 ? 4 : block / 128; }
 
@@ -712,9 +752,11 @@ static int launch_update(const UpdateArgs& u, cudaStream_t st) {
                   : cpb == 2 ? (const void*)update_kernel<MODE, 2>
                              : (const void*)update_kernel<MODE, 4>;
     const int grid = persistent_grid(k, kThreads, 0, ntiles);
-    if (cpb == 1) update_kernel<MODE, 1><<<grid, kThreads, 0, st>>>(u, ntiles);
-    else if (cpb == 2) update_kernel<MODE, 2><<<grid, kThreads, 0, st>>>(u, ntiles);
-    else update_kernel<MODE, 4><<<grid, kThreads, 0, st>>>(u, ntiles);
+    if (cpb == 1) pdl_launch(true, update_kernel<MODE, 1>, dim3(grid), dim3(kThreads), 0, st, u,
+                             ntiles);
+    else if (cpb == 2) pdl_launch(true, update_kernel<MODE, 2>, dim3(grid), dim3(kThreads), 0, st,
+                                  u, ntiles);
+    else pdl_launch(true, update_kernel<MODE, 4>, dim3(grid), dim3(kThreads), 0, st, u, ntiles);
     return check_launch();
 }
 
@@ -768,11 +810,16 @@ static void launch_factor(const FactorDesc& fr, const FactorDesc& fc, double* rs
     const int kpt = fr.block <= kThreads ? 1 : fr.block / kThreads;
     const unsigned grid = (unsigned)(nb0 + nb1);
     switch (kpt) {
-        case 1: factor_kernel<1><<<grid, kThreads, 0, st>>>(fr, fc, nb0, rsum); break;
-        case 2: factor_kernel<2><<<grid, kThreads, 0, st>>>(fr, fc, nb0, rsum); break;
-        case 4: factor_kernel<4><<<grid, kThreads, 0, st>>>(fr, fc, nb0, rsum); break;
-        case 8: factor_kernel<8><<<grid, kThreads, 0, st>>>(fr, fc, nb0, rsum); break;
-        default: factor_kernel<16><<<grid, kThreads, 0, st>>>(fr, fc, nb0, rsum); break;
+        case 1: pdl_launch(true, factor_kernel<1>, dim3(grid), dim3(kThreads), 0, st, fr, fc, nb0,
+                           rsum); break;
+        case 2: pdl_launch(true, factor_kernel<2>, dim3(grid), dim3(kThreads), 0, st, fr, fc, nb0,
+                           rsum); break;
+        case 4: pdl_launch(true, factor_kernel<4>, dim3(grid), dim3(kThreads), 0, st, fr, fc, nb0,
+                           rsum); break;
+        case 8: pdl_launch(true, factor_kernel<8>, dim3(grid), dim3(kThreads), 0, st, fr, fc, nb0,
+                           rsum); break;
+        default: pdl_launch(true, factor_kernel<16>, dim3(grid), dim3(kThreads), 0, st, fr, fc, nb0,
+                            rsum); break;
     }
 }
 
@@ -786,14 +833,16 @@ static int second_moment_passes(const float* g, int64_t rows, int64_t cols, cons
     launch_sumsq<0>(dim3(ncb, nrb), g, (int)rows, (int)cols, none, w.rowpart, w.colpart, st);
     const int nb0 = (int)blocks_of(rows, fr.block);
     launch_factor(fr, fc, w.rsum, st);
-    scale_kernel<<<(unsigned)blocks_of(rows + cols, kThreads), kThreads, 0, st>>>(
-        fr.fresh, (int)rows, fc.fresh, (int)cols, w.rsum, nb0, a, b, w.ticket);
+    pdl_launch(true, scale_kernel, dim3((unsigned)blocks_of(rows + cols, kThreads)),
+               dim3(kThreads), 0, st, fr.fresh, (int)rows, fc.fresh, (int)cols, w.rsum, nb0, a, b,
+               w.ticket);
     const int64_t n = rows * cols;
     const int64_t ntiles = blocks_of(n, kTile);
     const UsqArgs q{g, n, make_divider((uint32_t)cols), a, b, w.upart, w.ticket, w.scal, 0.0f};
     const int64_t nchunks = blocks_of(ntiles, kUsqChunk);
-    usq_kernel<<<persistent_grid((const void*)usq_kernel, kThreads, 0, nchunks), kThreads, 0, st>>>(
-        q, clip_d);
+    pdl_launch(true, usq_kernel,
+               dim3(persistent_grid((const void*)usq_kernel, kThreads, 0, nchunks)),
+               dim3(kThreads), 0, st, q, clip_d);
     return check_launch();
 }
 
@@ -902,9 +951,9 @@ int al_came_step(float* p, const float* g, int64_t rows, int64_t cols, void* vr_
                                 cc_meta, c_bits, c_block, hp->log_floor_c, w.fc2);
     const int nb0 = (int)blocks_of(rows, c_block), nb1 = (int)blocks_of(cols, c_block);
     launch_factor(cr, cc, w.rsum2, s);
-    scale_kernel<<<(unsigned)blocks_of(rows + cols, kThreads), kThreads, 0, s>>>(
-        w.fr2, (int)rows, w.fc2, (int)cols, w.rsum2, (int)blocks_of(rows, cr.block), w.a2, w.b2,
-        nullptr);
+    pdl_launch(true, scale_kernel, dim3((unsigned)blocks_of(rows + cols, kThreads)),
+               dim3(kThreads), 0, s, w.fr2, (int)rows, w.fc2, (int)cols, w.rsum2,
+               (int)blocks_of(rows, cr.block), w.a2, w.b2, nullptr);
     st = check_launch();
     if (st) return st;
 
@@ -998,6 +1047,7 @@ __device__ __forceinline__ int fac_advance(const FacEntry* __restrict__ tab, int
 template <int MODE>
 __global__ void __launch_bounds__(kThreads)
 sumsq_multi_kernel(const FacEntry* __restrict__ tab, int nmat, FacStep fs) {
+    pdl_entry();
     extern __shared__ __align__(16) unsigned char s_sumsq[];
     const FacEntry& e = fac_entry(tab, nmat, blockIdx.x, &FacEntry::sq_t0);
     const int64_t lt = blockIdx.x - e.sq_t0;
@@ -1015,6 +1065,7 @@ sumsq_multi_kernel(const FacEntry* __restrict__ tab, int nmat, FacStep fs) {
 template <int KPT>
 __global__ void __launch_bounds__(kThreads)
 factor_multi_kernel(const FacEntry* __restrict__ tab, int nmat, FacStep fs, int which) {
+    pdl_entry();
     const FacEntry& e = fac_entry(tab, nmat, blockIdx.x, which ? &FacEntry::fac2_t0 : &FacEntry::fac_t0);
     const int64_t lt = blockIdx.x - (which ? e.fac2_t0 : e.fac_t0);
     const int block = which ? fs.c_block : fs.v_block;
@@ -1040,6 +1091,7 @@ factor_multi_kernel(const FacEntry* __restrict__ tab, int nmat, FacStep fs, int 
 
 __global__ void __launch_bounds__(kThreads)
 scale_multi_kernel(const FacEntry* __restrict__ tab, int nmat, FacStep fs, int which) {
+    pdl_entry();
     const FacEntry& e = fac_entry(tab, nmat, blockIdx.x, &FacEntry::sc_t0);
     const int lt = (int)(blockIdx.x - e.sc_t0);
     if (which == 0)
@@ -1053,6 +1105,7 @@ scale_multi_kernel(const FacEntry* __restrict__ tab, int nmat, FacStep fs, int w
 __global__ void __launch_bounds__(kThreads)
 usq_multi_kernel(const FacEntry* __restrict__ tab, int nmat, int64_t nchunks, float clip_d,
                  float zero) {
+    pdl_entry();
     __shared__ float2 s_w[kThreads / 32];
     __shared__ double s_d[kThreads];
     __shared__ bool s_last;
@@ -1068,6 +1121,7 @@ usq_multi_kernel(const FacEntry* __restrict__ tab, int nmat, int64_t nchunks, fl
 template <int MODE, int CPBM>
 __global__ void __launch_bounds__(kThreads)
 update_multi_kernel(const FacEntry* __restrict__ tab, int nmat, int64_t ntiles, FacStep fs) {
+    pdl_entry();
     __shared__ uint32_t s_part[kThreads / 32];
     int cur = 0;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
@@ -1108,7 +1162,8 @@ static int check_factored_matrices(const al_factored_matrix* mats, int nmat) {
 template <int KPT>
 static void launch_factor_multi(const FacEntry* tab, int nmat, const FacStep& fs, int which,
                                 int64_t tiles, cudaStream_t st) {
-    factor_multi_kernel<KPT><<<(unsigned)tiles, kThreads, 0, st>>>(tab, nmat, fs, which);
+    pdl_launch(false, factor_multi_kernel<KPT>, dim3((unsigned)tiles), dim3(kThreads), 0, st, tab,
+               nmat, fs, which);
 }
 
 static void factor_multi(const FacEntry* tab, int nmat, const FacStep& fs, int which,
@@ -1132,9 +1187,12 @@ static void update_multi(const FacEntry* tab, int nmat, int64_t tiles, const Fac
                   : cpb == 2 ? (const void*)update_multi_kernel<MODE, 2>
                              : (const void*)update_multi_kernel<MODE, 4>;
     const int grid = persistent_grid(k, kThreads, 0, tiles);
-    if (cpb == 1) update_multi_kernel<MODE, 1><<<grid, kThreads, 0, st>>>(tab, nmat, tiles, fs);
-    else if (cpb == 2) update_multi_kernel<MODE, 2><<<grid, kThreads, 0, st>>>(tab, nmat, tiles, fs);
-    else update_multi_kernel<MODE, 4><<<grid, kThreads, 0, st>>>(tab, nmat, tiles, fs);
+    if (cpb == 1) pdl_launch(false, update_multi_kernel<MODE, 1>, dim3(grid), dim3(kThreads), 0, st,
+                             tab, nmat, tiles, fs);
+    else if (cpb == 2) pdl_launch(false, update_multi_kernel<MODE, 2>, dim3(grid), dim3(kThreads),
+                                  0, st, tab, nmat, tiles, fs);
+    else pdl_launch(false, update_multi_kernel<MODE, 4>, dim3(grid), dim3(kThreads), 0, st, tab,
+                    nmat, tiles, fs);
 }
 
 // The passes both optimizers share: g^2 sums, second-moment factors, their
@@ -1142,11 +1200,13 @@ static void update_multi(const FacEntry* tab, int nmat, int64_t tiles, const Fac
 static void second_moment_multi(const FacEntry* tab, const al_factored_info* info,
                                 const FacStep& fs, cudaStream_t st) {
     static const size_t smem0 = sumsq_smem_optin(sumsq_multi_kernel<0>, SumsqSmem<0>::kBytes);
-    sumsq_multi_kernel<0><<<(unsigned)info->sumsq_tiles, kThreads, smem0, st>>>(tab, info->nmat, fs);
+    pdl_launch(false, sumsq_multi_kernel<0>,
+               dim3((unsigned)info->sumsq_tiles), dim3(kThreads), smem0, st, tab, info->nmat, fs);
     factor_multi(tab, info->nmat, fs, 0, info->factor_tiles, st);
-    scale_multi_kernel<<<(unsigned)info->scale_tiles, kThreads, 0, st>>>(tab, info->nmat, fs, 0);
-    usq_multi_kernel<<<persistent_grid((const void*)usq_multi_kernel, kThreads, 0, info->rms_chunks),
-                       kThreads, 0, st>>>(tab, info->nmat, info->rms_chunks, fs.clip_d, fs.zero);
+    pdl_launch(false, scale_multi_kernel,
+               dim3((unsigned)info->scale_tiles), dim3(kThreads), 0, st, tab, info->nmat, fs, 0);
+    pdl_launch(false, usq_multi_kernel,
+               dim3(persistent_grid((const void*)usq_multi_kernel, kThreads, 0, info->rms_chunks)), dim3(kThreads), 0, st, tab, info->nmat, info->rms_chunks, fs.clip_d, fs.zero);
 }
 
 static int check_multi_call(const void* plan_dev, const al_factored_info* info, int op) {
@@ -1330,9 +1390,11 @@ int al_came_step_multi(const void* plan_dev, const al_factored_info* info, const
     second_moment_multi(tab, info, fs, st);
     // residual sums, confidence factors and their scales, update
     static const size_t smem1 = sumsq_smem_optin(sumsq_multi_kernel<1>, SumsqSmem<1>::kBytes);
-    sumsq_multi_kernel<1><<<(unsigned)info->sumsq_tiles, kThreads, smem1, st>>>(tab, info->nmat, fs);
+    pdl_launch(false, sumsq_multi_kernel<1>,
+               dim3((unsigned)info->sumsq_tiles), dim3(kThreads), smem1, st, tab, info->nmat, fs);
     factor_multi(tab, info->nmat, fs, 1, info->factor2_tiles, st);
-    scale_multi_kernel<<<(unsigned)info->scale_tiles, kThreads, 0, st>>>(tab, info->nmat, fs, 1);
+    pdl_launch(false, scale_multi_kernel,
+               dim3((unsigned)info->scale_tiles), dim3(kThreads), 0, st, tab, info->nmat, fs, 1);
     update_multi<2>(tab, info->nmat, info->tiles, fs, st);
     return check_launch();
 }
