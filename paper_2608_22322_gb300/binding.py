@@ -114,6 +114,7 @@ _sig("alq_status_string", C.c_char_p, _int)
 _sig("alq_last_cuda_error", C.c_char_p)
 _sig("alq_version", _int)
 _sig("al_num_blocks", _i64, _i64, _int)
+_sig("al_meta_count", _i64, _i64, _int)
 _sig("al_state_bytes", _i64, _i64, _int, _int)
 _sig("al_encode", _int, _vp, _i64, _int, _int, _flt, _vp, _vp, _vp)
 _sig("al_decode", _int, _vp, _vp, _i64, _int, _int, _vp, _vp)
@@ -185,6 +186,10 @@ def al_num_blocks(n: int, block: int) -> int:
     return lib.al_num_blocks(n, block)
 
 
+def al_meta_count(n: int, block: int) -> int:
+    return lib.al_meta_count(n, block)
+
+
 def al_state_bytes(n: int, block: int, bits: int) -> int:
     return lib.al_state_bytes(n, block, bits)
 
@@ -225,30 +230,66 @@ def al_adamw_step(p, g, m_codes, m_absmax, v_codes, v_meta, m_block, v_block, v_
         p.numel(), m_block, v_block, v_bits, C.byref(h), t, _stream(stream)))
 
 
-class AdamWPlan:
+class _BoundPlan:
+    """Gradient rebinding shared by the plans. A plan binds device pointers;
+    it keeps the optimizer's own arrays (parameters, states, workspace)
+    alive but holds no gradient tensor: a training loop that frees its
+    gradients every step (zero_grad(set_to_none=True)) passes the current
+    ones to step(grads=...), and the host image is rebuilt with their
+    addresses and copied to the plan's device buffer, in stream order, only
+    when an address changed. A plan stepped without grads uses the
+    gradients it was built with, which the caller must keep alive."""
+
+    def _rebind(self, grads, stream):
+        ptrs = [_ptr(g) for g in grads]
+        if len(ptrs) != len(self._gptrs):
+            raise ValueError(f"{type(self).__name__}.step: {len(ptrs)} gradients for "
+                             f"{len(self._gptrs)} bound arrays")
+        if ptrs == self._gptrs:
+            return
+        for i, p in enumerate(ptrs):
+            self._arr[i].g = p
+        self._build()
+        self._gptrs = ptrs
+        if stream is None:
+            self.dev.copy_(self._host)
+        else:
+            with torch.cuda.stream(stream):
+                self.dev.copy_(self._host)
+
+
+class AdamWPlan(_BoundPlan):
     """Device copy of a multi-tensor AdamW plan (al_adamw_plan) and its host
     summary. `tensors` is a list of dicts with keys p, g, m_codes, m_absmax,
-    v_codes, v_meta (torch CUDA tensors)."""
+    v_codes, v_meta (torch CUDA tensors); see _BoundPlan for g."""
 
     def __init__(self, tensors, m_block, v_block, v_bits, device=None):
         nt = len(tensors)
-        arr = (AdamWTensor * nt)()
+        self._arr = (AdamWTensor * nt)()
         for i, t in enumerate(tensors):
-            arr[i] = AdamWTensor(_ptr(t["p"]), _ptr(t["g"]), _ptr(t["m_codes"]),
-                                 _ptr(t["m_absmax"]), _ptr(t["v_codes"]),
-                                 _ptr(t["v_meta"]), t["p"].numel())
+            self._arr[i] = AdamWTensor(_ptr(t["p"]), _ptr(t["g"]), _ptr(t["m_codes"]),
+                                       _ptr(t["m_absmax"]), _ptr(t["v_codes"]),
+                                       _ptr(t["v_meta"]), t["p"].numel())
+        self._gptrs = [_ptr(t["g"]) for t in tensors]
+        self._cfg = (m_block, v_block, v_bits)
         nbytes = C.c_size_t(0)
         _check("al_adamw_plan_bytes", lib.al_adamw_plan_bytes(nt, C.byref(nbytes)))
-        host = torch.zeros(nbytes.value, dtype=torch.uint8)
+        self._host = torch.zeros(nbytes.value, dtype=torch.uint8)
         self.info = MultiInfo()
-        _check("al_adamw_plan", lib.al_adamw_plan(arr, nt, m_block, v_block, v_bits,
-                                                  host.data_ptr(), nbytes.value,
-                                                  C.byref(self.info)))
+        self._build()
         dev = device if device is not None else tensors[0]["p"].device
-        self.dev = host.to(dev)
-        self.tensors = tensors  # keep the arrays alive while the plan is used
+        self.dev = self._host.to(dev)
+        # keep the optimizer's arrays alive while the plan is used (not g)
+        self.tensors = [{k: v for k, v in t.items() if k != "g"} for t in tensors]
 
-    def step(self, hp: dict, t: int, stream=None):
+    def _build(self):
+        _check("al_adamw_plan", lib.al_adamw_plan(self._arr, len(self._arr), *self._cfg,
+                                                  self._host.data_ptr(), self._host.numel(),
+                                                  C.byref(self.info)))
+
+    def step(self, hp: dict, t: int, stream=None, grads=None):
+        if grads is not None:
+            self._rebind(grads, stream)
         h = _hp(AdamWHP, hp)
         _check("al_adamw_step_multi", lib.al_adamw_step_multi(
             _ptr(self.dev), C.byref(self.info), C.byref(h), t, _stream(stream)))
@@ -304,14 +345,14 @@ def al_apollo_step(p, g, rows, cols, proj, m_codes, m_absmax, m_block, v_codes, 
         _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
-class FactoredPlan:
+class FactoredPlan(_BoundPlan):
     """A grouped Adafactor or CAME step over many matrices (al_factored_plan
     / al_adafactor_step_multi / al_came_step_multi): owns the workspace and
     the device copy of the plan. `op` is AL_OP_ADAFACTOR or AL_OP_CAME;
     `mats` is a list of dicts with keys p, g, rows, cols, vr_codes, vr_meta,
     vc_codes, vc_meta, and for CAME cr_codes, cr_meta, cc_codes, cc_meta,
     and optionally (always for CAME) m_codes, m_absmax (torch CUDA
-    tensors)."""
+    tensors); see _BoundPlan for g."""
 
     _KEYS = ("vr_codes", "vr_meta", "vc_codes", "vc_meta", "cr_codes", "cr_meta", "cc_codes",
              "cc_meta", "m_codes", "m_absmax")
@@ -319,27 +360,37 @@ class FactoredPlan:
     def __init__(self, op, mats, v_bits, v_block, c_bits=16, c_block=128, m_block=256,
                  device=None):
         nm = len(mats)
-        arr = (FactoredMatrix * nm)()
+        self._arr = (FactoredMatrix * nm)()
         for i, m in enumerate(mats):
-            arr[i] = FactoredMatrix(_ptr(m["p"]), _ptr(m["g"]), m["rows"], m["cols"],
-                                    *[_ptr(m.get(k)) for k in self._KEYS])
+            self._arr[i] = FactoredMatrix(_ptr(m["p"]), _ptr(m["g"]), m["rows"], m["cols"],
+                                          *[_ptr(m.get(k)) for k in self._KEYS])
+        self._gptrs = [_ptr(m["g"]) for m in mats]
         dev = device if device is not None else mats[0]["p"].device
         ws = C.c_size_t(0)
         _check("al_factored_workspace_multi",
-               lib.al_factored_workspace_multi(arr, nm, C.byref(ws)))
+               lib.al_factored_workspace_multi(self._arr, nm, C.byref(ws)))
         self.workspace = torch.zeros(ws.value, dtype=torch.uint8, device=dev)
         nbytes = C.c_size_t(0)
-        _check("al_factored_plan_bytes", lib.al_factored_plan_bytes(arr, nm, C.byref(nbytes)))
-        host = torch.zeros(nbytes.value, dtype=torch.uint8)
+        _check("al_factored_plan_bytes",
+               lib.al_factored_plan_bytes(self._arr, nm, C.byref(nbytes)))
+        self._host = torch.zeros(nbytes.value, dtype=torch.uint8)
         self.info = FactoredInfo()
-        _check("al_factored_plan", lib.al_factored_plan(
-            op, arr, nm, v_bits, v_block, c_bits, c_block, m_block, _ptr(self.workspace),
-            ws.value, host.data_ptr(), nbytes.value, C.byref(self.info)))
         self.op = op
-        self.dev = host.to(dev)
-        self.mats = mats  # keep the arrays alive while the plan is used
+        self._cfg = (v_bits, v_block, c_bits, c_block, m_block)
+        self._build()
+        self.dev = self._host.to(dev)
+        # keep the optimizer's arrays alive while the plan is used (not g)
+        self.mats = [{k: v for k, v in m.items() if k != "g"} for m in mats]
 
-    def step(self, hp: dict, t: int, stream=None):
+    def _build(self):
+        _check("al_factored_plan", lib.al_factored_plan(
+            self.op, self._arr, len(self._arr), *self._cfg, _ptr(self.workspace),
+            self.workspace.numel(), self._host.data_ptr(), self._host.numel(),
+            C.byref(self.info)))
+
+    def step(self, hp: dict, t: int, stream=None, grads=None):
+        if grads is not None:
+            self._rebind(grads, stream)
         if self.op == AL_OP_ADAFACTOR:
             h = _hp(AdafactorHP, hp)
             _check("al_adafactor_step_multi", lib.al_adafactor_step_multi(
@@ -350,35 +401,46 @@ class FactoredPlan:
                 _ptr(self.dev), C.byref(self.info), C.byref(h), t, _stream(stream)))
 
 
-class ApolloPlan:
+class ApolloPlan(_BoundPlan):
     """A grouped APOLLO step over many matrices (al_apollo_plan /
     al_apollo_step_multi): owns the workspace and the device copy of the
     plan. `mats` is a list of dicts with keys p, g, rows, cols, proj, m_codes,
-    m_absmax, v_codes, v_meta (torch CUDA tensors; proj holds bf16 bits)."""
+    m_absmax, v_codes, v_meta (torch CUDA tensors; proj holds bf16 bits);
+    see _BoundPlan for g."""
 
     def __init__(self, mats, rank, v_bits, device=None):
         nm = len(mats)
-        arr = (ApolloMatrix * nm)()
+        self._arr = (ApolloMatrix * nm)()
         for i, m in enumerate(mats):
-            arr[i] = ApolloMatrix(_ptr(m["p"]), _ptr(m["g"]), m["rows"], m["cols"],
-                                  _ptr(m["proj"]), _ptr(m["m_codes"]), _ptr(m["m_absmax"]),
-                                  _ptr(m["v_codes"]), _ptr(m["v_meta"]))
+            self._arr[i] = ApolloMatrix(_ptr(m["p"]), _ptr(m["g"]), m["rows"], m["cols"],
+                                        _ptr(m["proj"]), _ptr(m["m_codes"]),
+                                        _ptr(m["m_absmax"]), _ptr(m["v_codes"]),
+                                        _ptr(m["v_meta"]))
+        self._gptrs = [_ptr(m["g"]) for m in mats]
         dev = device if device is not None else mats[0]["p"].device
         ws = C.c_size_t(0)
         _check("al_apollo_workspace_multi",
-               lib.al_apollo_workspace_multi(arr, nm, rank, C.byref(ws)))
+               lib.al_apollo_workspace_multi(self._arr, nm, rank, C.byref(ws)))
         self.workspace = torch.zeros(ws.value, dtype=torch.uint8, device=dev)
         nbytes = C.c_size_t(0)
-        _check("al_apollo_plan_bytes", lib.al_apollo_plan_bytes(arr, nm, C.byref(nbytes)))
-        host = torch.zeros(nbytes.value, dtype=torch.uint8)
+        _check("al_apollo_plan_bytes", lib.al_apollo_plan_bytes(self._arr, nm, C.byref(nbytes)))
+        self._host = torch.zeros(nbytes.value, dtype=torch.uint8)
         self.info = ApolloInfo()
-        _check("al_apollo_plan", lib.al_apollo_plan(
-            arr, nm, rank, v_bits, _ptr(self.workspace), ws.value, host.data_ptr(),
-            nbytes.value, C.byref(self.info)))
-        self.dev = host.to(dev)
-        self.mats = mats  # keep the arrays alive while the plan is used
+        self._cfg = (rank, v_bits)
+        self._build()
+        self.dev = self._host.to(dev)
+        # keep the optimizer's arrays alive while the plan is used (not g)
+        self.mats = [{k: v for k, v in m.items() if k != "g"} for m in mats]
 
-    def step(self, hp: dict, t: int, stream=None):
+    def _build(self):
+        _check("al_apollo_plan", lib.al_apollo_plan(
+            self._arr, len(self._arr), *self._cfg, _ptr(self.workspace),
+            self.workspace.numel(), self._host.data_ptr(), self._host.numel(),
+            C.byref(self.info)))
+
+    def step(self, hp: dict, t: int, stream=None, grads=None):
+        if grads is not None:
+            self._rebind(grads, stream)
         h = _hp(ApolloHP, hp)
         _check("al_apollo_step_multi", lib.al_apollo_step_multi(
             _ptr(self.dev), C.byref(self.info), C.byref(h), t, _stream(stream)))

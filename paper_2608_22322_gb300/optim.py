@@ -179,8 +179,10 @@ class AdamW(_Base):
                                    dtype=torch.float32, device=p.device)
 
     def _plan(self, tensors, group):
-        key = (tuple((t["p"].data_ptr(), t["g"].data_ptr(), t["v_codes"].data_ptr(),
-                      t["m_codes"].data_ptr()) for t in tensors),
+        """A cached plan over these tensors, keyed on the addresses of the
+        parameters and states only: gradients are rebound at every step
+        (the plan holds none, so freed gradients are not kept alive)."""
+        key = (_state_key(tensors, ("p", "m_codes", "m_absmax", "v_codes", "v_meta")),
                group["m_block"], group["v_block"], group["v_bits"])
         plan = self._plans.get(key)
         if plan is None:
@@ -213,12 +215,19 @@ class AdamW(_Base):
             hp = dict(lr=group["lr"], beta1=b1, beta2=b2, eps=group["eps"],
                       weight_decay=group["weight_decay"], log_floor=group["log_floor"])
             for t, tensors in buckets.items():
-                self._plan(tensors, group).step(hp, t)
+                self._plan(tensors, group).step(hp, t, grads=[x["g"] for x in tensors])
         return loss
 
     def migrate_bits(self, bits_key: str = "v_bits", new_bits: int = 16):
         self._plans.clear()
         super().migrate_bits(bits_key, new_bits)
+
+
+def _state_key(items, keys):
+    """Plan cache key: the addresses of the parameters and states a plan
+    binds (never the gradients')."""
+    return tuple(tuple(0 if it.get(k) is None else it[k].data_ptr() for k in keys)
+                 for it in items)
 
 
 def _as_matrix(p: torch.Tensor):
@@ -291,16 +300,18 @@ class Adafactor(_Base):
                          m_codes=st.get("m_codes"), m_absmax=st.get("m_absmax")))
             for t, mats in buckets.items():
                 _grouped_plan(self._plans, B.AL_OP_ADAFACTOR, mats, group["fac_bits"],
-                              group["fac_block"], 16, 128, group["m_block"]).step(hp, t)
+                              group["fac_block"], 16, 128, group["m_block"]).step(
+                                  hp, t, grads=[m["g"] for m in mats])
         return loss
 
 
 def _grouped_plan(cache: dict, op, mats, v_bits, v_block, c_bits, c_block, m_block):
-    """A cached FactoredPlan over these matrices (plans bind pointers)."""
+    """A cached FactoredPlan over these matrices (plans bind pointers; the
+    key holds parameter and state addresses, gradients are rebound at each
+    step)."""
     key = (op, v_bits, v_block, c_bits, c_block, m_block,
-           tuple(tuple(0 if m.get(k) is None else m[k].data_ptr()
-                       for k in ("p", "g", "vr_codes", "vc_codes", "cr_codes", "cc_codes",
-                                 "m_codes")) for m in mats))
+           _state_key(mats, ("p", "vr_codes", "vr_meta", "vc_codes", "vc_meta", "cr_codes",
+                             "cr_meta", "cc_codes", "cc_meta", "m_codes", "m_absmax")))
     plan = cache.get(key)
     if plan is None:
         if len(cache) > 64:
@@ -381,7 +392,8 @@ class CAME(_Base):
                 buckets.setdefault(st["step"], []).append(m)
             for t, mats in buckets.items():
                 _grouped_plan(self._plans, B.AL_OP_CAME, mats, group["v_bits"], group["v_block"],
-                              group["c_bits"], group["c_block"], group["m_block"]).step(hp, t)
+                              group["c_bits"], group["c_block"], group["m_block"]).step(
+                                  hp, t, grads=[m["g"] for m in mats])
         return loss
 
 
@@ -475,16 +487,15 @@ class Apollo(_Base):
                       alpha=group["alpha"], weight_decay=group["weight_decay"],
                       norm_growth_gamma=0.0, log_floor=group["log_floor"], rank=group["rank"])
             for t, mats in buckets.items():
-                key = (tuple((m["p"].data_ptr(), m["g"].data_ptr(), m["v_codes"].data_ptr(),
-                              m["m_codes"].data_ptr()) for m in mats),
-                       group["rank"], group["v_bits"])
+                key = (_state_key(mats, ("p", "proj", "m_codes", "m_absmax", "v_codes",
+                                         "v_meta")), group["rank"], group["v_bits"])
                 plan = self._plans.get(key)
                 if plan is None:
                     if len(self._plans) > 8:
                         self._plans.clear()
                     plan = B.ApolloPlan(mats, group["rank"], group["v_bits"])
                     self._plans[key] = plan
-                plan.step(hp, t)
+                plan.step(hp, t, grads=[m["g"] for m in mats])
         return loss
 
     def state_dict(self):

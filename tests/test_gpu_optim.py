@@ -270,3 +270,36 @@ def test_g1_grouping_fp32_roles(mods):
     st3 = opt3.state[model.proj.weight]
     assert st3["cr_codes"].dtype == torch.float32 and st3["vr_codes"].dtype == torch.int16
     assert torch.all(st3["cr_codes"] > 0)
+
+
+@pytest.mark.parametrize("kind", ["AdamW", "CAME", "Apollo", "Adafactor"])
+def test_wrappers_hold_no_gradients(mods, kind):
+    """A training loop that frees its gradients every step
+    (zero_grad(set_to_none=True), torch's default) gets fresh gradient
+    tensors at new addresses: the cached plans are keyed on parameter and
+    state addresses and rebind the gradients, so over 100 steps no plan is
+    added and device memory stays flat after the second step."""
+    import torch
+    _, optim = mods
+    shapes = [(256, 512), (128, 256), (512,)] if kind != "Apollo" else [(256, 512), (128, 256)]
+    params = _params(shapes, 40)
+    opt = {"AdamW": lambda: optim.AdamW(params),
+           "CAME": lambda: optim.CAME(params),
+           "Adafactor": lambda: optim.Adafactor(params),
+           "Apollo": lambda: optim.Apollo(params, rank=128)}[kind]()
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(5)
+    base = None
+    for step in range(1, 101):
+        opt.zero_grad(set_to_none=True)
+        for p in params:
+            p.grad = torch.randn(p.shape, device="cuda", generator=gen) * 1e-3
+        opt.step()
+        if step == 2:
+            torch.cuda.synchronize()
+            base = torch.cuda.memory_allocated()
+            nplans = len(opt._plans)
+    torch.cuda.synchronize()
+    assert torch.cuda.memory_allocated() == base
+    assert len(opt._plans) == nplans <= 1
+    assert all(torch.isfinite(p).all() for p in params)
