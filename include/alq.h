@@ -27,7 +27,12 @@
  *  - Quantization blocks are consecutive runs of `block` elements of one
  *    tensor; the last block of a tensor may be partial, and elements past the
  *    end never enter a block statistic. `block` must be a power of two in
- *    [128, 4096].
+ *    [128, 4096] (the fused AdamW step: [128, 2048]). The paper's block
+ *    sizes (256 and 2048, Sec. 6.2; 128 for the AL16 factors) are all of
+ *    this form. The kernels give each lane whole 4-element chunks of 128
+ *    consecutive elements per warp and locate blocks by shifts, so a block
+ *    never splits a chunk; other sizes return ALQ_ERR_UNSUPPORTED (the
+ *    oracle accepts any size).
  *  - AL metadata is two fp32 values per block, interleaved:
  *    meta[2b] = l_min, meta[2b+1] = Delta (Sec. 4.1, "each block also stores
  *    l_min and Delta"). An all-zero block stores (0, 0) and all-zero codes.
@@ -65,12 +70,21 @@ extern "C" {
 #define ALQ_ERR_WORKSPACE (-4)   /* workspace missing or smaller than required */
 #define ALQ_ERR_CUDA (-5)        /* a CUDA runtime call or launch failed       */
 
+/* The same status codes under the AL_ prefix. */
+#define AL_OK ALQ_OK
+#define AL_ERR_INVALID_ARG ALQ_ERR_INVALID_ARG
+#define AL_ERR_UNSUPPORTED ALQ_ERR_UNSUPPORTED
+#define AL_ERR_ALIGN ALQ_ERR_ALIGN
+#define AL_ERR_WORKSPACE ALQ_ERR_WORKSPACE
+#define AL_ERR_CUDA ALQ_ERR_CUDA
+
 /* Human-readable name of a status code (static string). */
 const char* alq_status_string(int status);
 
 /* Text of the last CUDA error seen by this library on the calling thread, or
- * "" if none. */
+ * "" if none. al_last_cuda_error is the same function under the al_ prefix. */
 const char* alq_last_cuda_error(void);
+const char* al_last_cuda_error(void);
 
 /* Library ABI version: 100 * major + minor. */
 int alq_version(void);
@@ -78,6 +92,11 @@ int alq_version(void);
 /* Number of quantization blocks of `block` elements covering n elements,
  * ceil(n / block). Host-only; returns -1 for invalid arguments. */
 int64_t al_num_blocks(int64_t n, int block);
+
+/* Number of fp32 metadata values of an AL-coded state of n elements: two
+ * (l_min, Delta) per block, 2 * ceil(n / block). Host-only; returns -1 for
+ * invalid arguments. */
+int64_t al_meta_count(int64_t n, int block);
 
 /* Logical storage of one AL-coded state of n elements in bytes: codes plus
  * 8 bytes of metadata per block (Sec. 4.4, Eq. (7): c_AL8 = 1 + 8/B bytes per
@@ -283,9 +302,11 @@ int al_adafactor_step(float* p, const float* g, int64_t rows, int64_t cols,
  * results are exactly those of al_adafactor_step without the workspace.
  *   - Every GPU that loads the library reserves that array until the process
  *     exits.
- *   - The first call on each device looks up the array's device address
- *     (cudaGetSymbolAddress, with that device current); make that first call
- *     before capturing any stream.
+ *   - Every call looks up the array's device address (cudaGetSymbolAddress,
+ *     with the calling thread's current device and context), so the address
+ *     stays valid after cudaDeviceReset or under another context on the same
+ *     device. The first call on a device may load the library's device code:
+ *     make that first call before capturing any stream.
  *   - Every call on a device shares the one array: calls that may run
  *     concurrently on the GPU (different streams, no ordering between them)
  *     race and corrupt each other's results. Serialise them on one stream.

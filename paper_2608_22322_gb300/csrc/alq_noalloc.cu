@@ -12,11 +12,12 @@
 //
 // The array is a file-scope __device__ variable: every GPU that loads this
 // library holds kNoAllocScratchBytes of device memory for it until the
-// process exits. Host code cannot use the array's name as a device address,
-// so the first call on each device looks the address up with
-// cudaGetSymbolAddress (with that device current) and caches it.
-#include <mutex>
-
+// process exits. Host code cannot use the array's name as a device address:
+// each call looks the address up with cudaGetSymbolAddress, with the
+// calling thread's device and context current. The lookup is a host-side
+// table read once the library's device code is loaded (the first call on a
+// device may load it), and doing it per call means the address can never be
+// stale after cudaDeviceReset or under another context on the same device.
 #include "alq_internal.h"
 
 namespace alq {
@@ -24,22 +25,12 @@ namespace alq {
 constexpr size_t kNoAllocScratchBytes = size_t(4) << 20;  // 4 MiB
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
-constexpr int kMaxDevices = 64;
-
-// Device address of g_noalloc_scratch on the current device, looked up once
-// per device. Returns nullptr (and records the CUDA error) on failure.
+// Device address of g_noalloc_scratch in the current context. Returns
+// nullptr (and records the CUDA error) on failure.
 static void* scratch_address() {
-    static std::mutex mu;
-    static void* addr[kMaxDevices] = {};
-    int dev = 0;
-    if (record_cuda(cudaGetDevice(&dev)) != ALQ_OK || dev < 0 || dev >= kMaxDevices) return nullptr;
-    std::lock_guard<std::mutex> lock(mu);
-    if (!addr[dev]) {
-        void* p = nullptr;
-        if (record_cuda(cudaGetSymbolAddress(&p, g_noalloc_scratch)) != ALQ_OK) return nullptr;
-        addr[dev] = p;
-    }
-    return addr[dev];
+    void* p = nullptr;
+    if (record_cuda(cudaGetSymbolAddress(&p, g_noalloc_scratch)) != ALQ_OK) return nullptr;
+    return p;
 }
 
 }  // namespace alq
