@@ -111,11 +111,18 @@ const char* alq_status_string(int status) {
 
 const char* alq_last_cuda_error(void) { return g_last_error; }
 
+const char* al_last_cuda_error(void) { return g_last_error; }
+
 int alq_version(void) { return 100; }
 
 int64_t al_num_blocks(int64_t n, int block) {
     if (n < 0 || block <= 0) return -1;
     return blocks_of(n, block);
+}
+
+int64_t al_meta_count(int64_t n, int block) {
+    if (n < 0 || block <= 0) return -1;
+    return 2 * blocks_of(n, block);
 }
 
 int64_t al_state_bytes(int64_t n, int block, int bits) {

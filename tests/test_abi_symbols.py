@@ -48,6 +48,25 @@ def test_host_helpers(lib):
     assert lib.al_num_blocks(0, 256) == 0
     assert lib.al_state_bytes(1 << 30, 2048, 8) == (1 << 30) + 8 * (1 << 19)
     assert lib.al_state_bytes(10, 256, 3) == -1
+    lib.al_meta_count.restype = C.c_int64
+    lib.al_meta_count.argtypes = [C.c_int64, C.c_int]
+    assert lib.al_meta_count(1000, 256) == 8
+    assert lib.al_meta_count(0, 256) == 0
+    assert lib.al_meta_count(-1, 256) == -1
+    lib.al_last_cuda_error.restype = C.c_char_p
+    lib.alq_last_cuda_error.restype = C.c_char_p
+    assert lib.al_last_cuda_error() == lib.alq_last_cuda_error() == b""
+
+
+def test_status_aliases_match():
+    """The AL_ status names are the ALQ_ codes."""
+    text = open(HEADER).read()
+    codes = dict(re.findall(r"#define (ALQ_\w+) \(?(-?\d+)\)?", text))
+    aliases = dict(re.findall(r"#define (AL_\w+) (ALQ_\w+)", text))
+    assert set(aliases) == {"AL_OK", "AL_ERR_INVALID_ARG", "AL_ERR_UNSUPPORTED", "AL_ERR_ALIGN",
+                            "AL_ERR_WORKSPACE", "AL_ERR_CUDA"}
+    for a, target in aliases.items():
+        assert a[3:] == target[4:] and target in codes
 
 
 def test_validation_rejects_before_launch(lib):
