@@ -2,21 +2,26 @@
 channel-wise scale) with the oracle.
 
 Sec. 3.1 (projected moments give a channel-wise scale of the original
-gradient), Sec. 6.1 (rank 256, channel-wise). The projection R = P bf16(G)
-runs on the tensor cores with fp32 accumulation, so it is not bit-exact: the
-test bounds it against the double-precision product of the same bf16
-operands (the oracle's projection) at 1e-5 of each channel's norm.
-Everything after the projection follows the oracle's arithmetic exactly,
-except the bias-corrected ratio M/(sqrt(V) + eps) behind the channel scales,
-which takes the approximate square root and reciprocal (it moves p only):
-fed the GPU's own R (teacher-forced), the oracle must reproduce the
-projected-moment codes and their block metadata bit for bit, and the
-parameters within 1e-5 of |p| plus the step size.
-Free-running, the parameters must stay within 1e-5 relative after 10 steps
-(the benchmark spec's bound). The projected states themselves can differ by more
-than one code free-running: AL's block interval starts at the channel's
-smallest |R|^2, whose relative error under fp32 accumulation is large, so a
-whole block's levels can shift; that is counted and reported.
+gradient), Sec. 6.1 (rank 256, channel-wise), at the TinyLlama matrix
+shapes (2048 x 2048, 5632 x 2048, 2048 x 5632, 256 x 2048) and smaller,
+ragged ones. The projection R = P bf16(G) runs on the tensor cores with
+fp32 accumulation, so it is not bit-exact: the test bounds it against the
+double-precision product of the same bf16 operands (the oracle's
+projection) at 1e-5 of each channel's norm. Everything after the
+projection follows the oracle's arithmetic exactly, except the
+bias-corrected ratio M/(sqrt(V) + eps) behind the channel scales, which
+takes the approximate square root and reciprocal (it moves p only): fed the
+GPU's own R (teacher-forced), the oracle must reproduce the projected-moment
+codes and their block constants bit for bit, and the parameters within 1e-5
+of |p| plus the step size.
+Free-running, the two trajectories see different R (fp32 against double
+accumulation), and each channel's AL block starts at its smallest R^2,
+whose relative error is the largest: block constants shift, codes move by
+a level, and the difference in the parameters' displacement is bounded by
+the codec's own error. Bar: the displacement (p_t - p_0) within 1e-4
+relative of the oracle's after 10 steps (the AL8 codec's displacement
+error against fp32 states is ~6e-4 at these ranks), parameters within 1e-5
+relative; code and constant differences are reported.
 """
 import math
 
@@ -110,7 +115,11 @@ def test_projection_matches_double_product(B, rows, cols):
     assert _rel(Rg, Ro) < 1e-5
 
 
-@pytest.mark.parametrize("rows,cols,steps", [(256, 1024, 6), (1024, 512, 6), (1024, 2816, 2)])
+CONFIG5 = [(2048, 2048), (5632, 2048), (2048, 5632), (256, 2048)]
+
+
+@pytest.mark.parametrize("rows,cols,steps", [(256, 1024, 6), (1024, 512, 6), (1024, 2816, 2)]
+                         + [(r, c, 3) for r, c in CONFIG5])
 def test_apollo_teacher_forced_exact_states(B, rows, cols, steps):
     """Each step from the GPU's own pre-step state and its own R: codes and
     metadata agree with the oracle bit for bit, parameters within 1e-5 of
@@ -125,6 +134,7 @@ def test_apollo_teacher_forced_exact_states(B, rows, cols, steps):
                            a.d["vc"], a.d["vm"], 8, 256, a.dprev, a.hp, t, a.ws)
         torch.cuda.synchronize()
         R = a.device_R()
+        assert np.all(np.isfinite(R)), "projection pipeline reported a failure (NaN)"
         ora.apollo_step_given_R(snap["p"], g, rows, cols, R, snap["mc"], snap["ma"], 256,
                                 snap["vc"], snap["vm"], 8, 256, 0.0, a.hp, t)
         p_dev = a.d["p"].cpu().numpy()
@@ -136,23 +146,35 @@ def test_apollo_teacher_forced_exact_states(B, rows, cols, steps):
         assert bad == 0, f"step {t}: {bad} parameters outside the tolerance"
 
 
-@pytest.mark.parametrize("rows,cols,steps", [(256, 1024, 10), (1024, 512, 10)])
+@pytest.mark.parametrize("rows,cols,steps", [(256, 1024, 10), (1024, 512, 10)]
+                         + [(r, c, 10) for r, c in CONFIG5])
 def test_apollo_free_running(B, rows, cols, steps):
     import torch
     a = Apollo(B, rows, cols, HP, seed=21)
     p0 = a.h["p"].copy()
+    R_err = 0.0
     for t in range(1, steps + 1):
         g = wl.gaussian_grad((rows, cols), 1e-3, 300 + t).ravel()
         a.step(g, t)
+        if t == 1:
+            torch.cuda.synchronize()
+            Rg = a.device_R().reshape(a.L, 256)
+            Ro = ora.apollo_project(g, rows, cols, a.P, 256).reshape(a.L, 256)
+            per_ch = np.linalg.norm(Ro.astype(np.float64), axis=1, keepdims=True)
+            R_err = float(np.max(np.abs(Rg - Ro) / per_ch))
+            assert R_err < 1e-5
     torch.cuda.synchronize()
     pd = a.d["p"].cpu().numpy()
     assert _rel(pd, a.h["p"]) < 1e-5
     disp = _rel(pd - p0, a.h["p"] - p0)
-    flips = sum(int(np.sum(a.d[k].cpu().numpy().astype(np.int64) != a.h[k].astype(np.int64)))
-                for k in ("mc", "vc"))
-    print(f"apollo {rows}x{cols}: relative displacement error {disp:.2e}, "
-          f"projected-code differences {flips} of {2 * a.L * 256}")
-    assert disp < 5e-3
+    n_codes = a.L * 256
+    diff = {k: int(np.sum(a.d[k].cpu().numpy().view(np.uint8) != a.h[k].view(np.uint8)))
+            for k in ("mc", "vc", "vm")}
+    print(f"apollo {rows}x{cols}, {steps} steps: R error {R_err:.1e} of the channel norm; "
+          f"relative displacement error {disp:.2e}; differing M^P codes {diff['mc']}, "
+          f"V^P codes {diff['vc']} of {n_codes}, V^P constant bytes {diff['vm']} of "
+          f"{8 * a.L}")
+    assert disp < 1e-4
 
 
 def test_apollo_norm_growth_limiter(B):
