@@ -16,6 +16,8 @@ import numpy as np
 from . import build as _build
 
 _lib = C.CDLL(_build.build())
+_lib_plain = _lib
+_lib_threaded = None
 
 _f32p = np.ctypeslib.ndpointer(np.float32, flags="C_CONTIGUOUS")
 _i8p = np.ctypeslib.ndpointer(np.int8, flags="C_CONTIGUOUS")
@@ -49,11 +51,52 @@ class ApolloHP(C.Structure):
                   "norm_growth_gamma", "log_floor")] + [("rank", C.c_int32)])
 
 
+_SIGS = []
+
+
 def _sig(name, res, *args):
+    _SIGS.append((name, res, list(args)))
     fn = getattr(_lib, name)
     fn.restype = res
     fn.argtypes = list(args)
     return fn
+
+
+def use_threads(on: bool = True) -> int:
+    """Switch every function of this module to the OpenMP build of the same
+    source (all host cores; the same results bit for bit) or back to the
+    plain single-threaded build. Returns the number of threads the next
+    calls use (1 when the compiler has no OpenMP)."""
+    global _lib, _lib_threaded
+    if not on:
+        _lib = _lib_plain
+        return 1
+    if _lib_threaded is None:
+        path = _build.build_threaded()
+        if path is None:
+            return 1
+        lib = C.CDLL(path)
+        for name, res, args in _SIGS:
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib_threaded = lib
+    _lib = _lib_threaded
+    return threads()
+
+
+def threads() -> int:
+    """Threads the current build runs its parallel loops on (OpenMP's
+    default: OMP_NUM_THREADS, else the cores this process may run on)."""
+    import os
+    if _lib is _lib_plain:
+        return 1
+    if os.environ.get("OMP_NUM_THREADS", "").isdigit():
+        return int(os.environ["OMP_NUM_THREADS"])
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
 
 
 _sig("ora_al_block_meta", _int, _f32p, _i64, _flt, C.POINTER(_flt), C.POINTER(_flt))

@@ -26,6 +26,13 @@
  *                     scaling in Sec. 6.1.
  *   update error      Sec. 3.2, Eq. (2).
  *
+ * Threads: the file also builds with -fopenmp (the benchmark's all-core CPU
+ * baseline). Only loops whose iterations are independent carry an OpenMP
+ * pragma -- blocks, elements, rows, columns, channels, each summed in its
+ * own fixed order -- and every reduction across them stays a sequential
+ * loop, so both builds give the same bits; without -fopenmp the pragmas are
+ * ignored.
+ *
  * Every function is pinned by tests that do not re-derive it: invariants and
  * closed forms of the paper (exact zero, endpoint codes, half-step round-trip
  * bound, monotone codes, brute force at 4 bits, storage numbers printed in
@@ -112,6 +119,7 @@ float ora_al_dequantize(uint32_t q, float lmin, float delta, int bits) {
 void ora_al_encode(const float* x, int64_t n, int block, int bits,
                    float log_floor, void* codes, float* meta) {
     int64_t nb = nblocks_of(n, block);
+#pragma omp parallel for schedule(static)
     for (int64_t b = 0; b < nb; ++b) {
         int64_t lo = b * block;
         int64_t len = (n - lo < block) ? (n - lo) : block;
@@ -128,6 +136,7 @@ void ora_al_encode(const float* x, int64_t n, int block, int bits,
 
 void ora_al_decode(const void* codes, const float* meta, int64_t n, int block,
                    int bits, float* out) {
+#pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < n; ++i) {
         int64_t b = i / block;
         out[i] = ora_al_dequantize(code_get(codes, bits, i), meta[2 * b],
@@ -167,6 +176,7 @@ int64_t ora_al_state_bytes(int64_t n, int block, int bits) {
 void ora_uf8_encode(const float* m, int64_t n, int block, int8_t* codes,
                     float* absmax) {
     int64_t nb = nblocks_of(n, block);
+#pragma omp parallel for schedule(static)
     for (int64_t b = 0; b < nb; ++b) {
         int64_t lo = b * block;
         int64_t len = (n - lo < block) ? (n - lo) : block;
@@ -191,6 +201,7 @@ void ora_uf8_encode(const float* m, int64_t n, int block, int8_t* codes,
 
 void ora_uf8_decode(const int8_t* codes, const float* absmax, int64_t n,
                     int block, float* out) {
+#pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < n; ++i) {
         float d = absmax[i / block] / 127.0f;
         out[i] = (float)codes[i] * d;
@@ -209,6 +220,7 @@ void ora_adamw_update_fp32(float* p, const float* g, float* m, float* v,
     const float omb1 = (float)(1.0 - (double)hp->beta1);
     const float omb2 = (float)(1.0 - (double)hp->beta2);
     const float b1 = hp->beta1, b2 = hp->beta2, eps = hp->eps;
+#pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < n; ++i) {
         float gi = g[i];
         /* Eq. (1) in fp32; a product that is added is fused with the sum
@@ -254,6 +266,7 @@ void ora_adamw_step(float* p, const float* g, int8_t* m_codes,
 /* mean_j(g_ij^2 + eps1) for every row, exact squares summed in double. */
 static void row_sq_means(const float* g, int64_t rows, int64_t cols,
                          float eps1, float* r) {
+#pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < rows; ++i) {
         double s = 0.0;
         for (int64_t j = 0; j < cols; ++j) {
@@ -266,6 +279,7 @@ static void row_sq_means(const float* g, int64_t rows, int64_t cols,
 
 static void col_sq_means(const float* g, int64_t rows, int64_t cols,
                          float eps1, float* c) {
+#pragma omp parallel for schedule(static)
     for (int64_t j = 0; j < cols; ++j) {
         double s = 0.0;
         for (int64_t i = 0; i < rows; ++i) {
@@ -295,13 +309,11 @@ static void inv_sqrt_factors(const float* R, int64_t rows, const float* C,
 static float scaled_update(const float* g, int64_t rows, int64_t cols,
                            const float* a, const float* b, float clip_d,
                            float* u) {
-    double ss = 0.0;
+#pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < rows; ++i)
-        for (int64_t j = 0; j < cols; ++j) {
-            float x = (g[i * cols + j] * a[i]) * b[j];
-            u[i * cols + j] = x;
-            ss += (double)x * (double)x;
-        }
+        for (int64_t j = 0; j < cols; ++j) u[i * cols + j] = (g[i * cols + j] * a[i]) * b[j];
+    double ss = 0.0;  /* in element order */
+    for (int64_t k = 0; k < rows * cols; ++k) ss += (double)u[k] * (double)u[k];
     double rms = sqrt(ss / ((double)rows * (double)cols));
     double cf = rms / (double)clip_d;
     if (cf < 1.0) cf = 1.0;
@@ -334,6 +346,7 @@ void ora_adafactor_update_fp32(float* p, const float* g, int64_t rows,
     for (int64_t j = 0; j < cols; ++j) C[j] = rho * C[j] + omr * c[j];
     inv_sqrt_factors(R, rows, C, cols, a, b);
     const float icf = scaled_update(g, rows, cols, a, b, hp->clip_d, u);
+#pragma omp parallel for schedule(static)
     for (int64_t k = 0; k < n; ++k) {
         float uh = u[k] * icf;
         float upd = uh;
@@ -398,6 +411,7 @@ void ora_came_update_fp32(float* p, const float* g, int64_t rows, int64_t cols,
     const float icf = scaled_update(g, rows, cols, a, b, hp->clip_d, u);
 
     /* momentum of the clipped update and its residual */
+#pragma omp parallel for schedule(static)
     for (int64_t k = 0; k < n; ++k) {
         float uh = u[k] * icf;
         float mk = hp->beta1 * M[k] + omb1 * uh;
@@ -407,11 +421,13 @@ void ora_came_update_fp32(float* p, const float* g, int64_t rows, int64_t cols,
     }
 
     /* confidence factors: beta3-EMAs of the residual's row/column means */
+#pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < rows; ++i) {
         double s = 0.0;
         for (int64_t j = 0; j < cols; ++j) s += (double)res[i * cols + j];
         r[i] = (float)(s / (double)cols);
     }
+#pragma omp parallel for schedule(static)
     for (int64_t j = 0; j < cols; ++j) {
         double s = 0.0;
         for (int64_t i = 0; i < rows; ++i) s += (double)res[i * cols + j];
@@ -421,6 +437,7 @@ void ora_came_update_fp32(float* p, const float* g, int64_t rows, int64_t cols,
     for (int64_t j = 0; j < cols; ++j) Cc[j] = hp->beta3 * Cc[j] + omb3 * c[j];
     inv_sqrt_factors(Cr, rows, Cc, cols, a, b);
 
+#pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < rows; ++i)
         for (int64_t j = 0; j < cols; ++j) {
             int64_t k = i * cols + j;
@@ -483,23 +500,34 @@ float ora_bf16_to_f32(uint16_t b) {
 
 /* If rows <= cols the rows are the short side: R[j][k] = sum_i P[k][i] g[i][j]
  * with channels j over the columns; otherwise R[j][k] = sum_i P[k][i] g[j][i]
- * with channels over the rows. */
+ * with channels over the rows. Both operands are rounded to bf16 once, into
+ * double copies laid out with the short side contiguous; every sum runs over
+ * i in ascending order. */
 void ora_apollo_project(const float* g, int64_t rows, int64_t cols,
                         const uint16_t* proj, int rank, float* R) {
     const int rows_short = rows <= cols;
     const int64_t s = rows_short ? rows : cols;
     const int64_t L = rows_short ? cols : rows;
+    double* gb = (double*)malloc(sizeof(double) * (size_t)(L * s));   /* [L][s] */
+    double* pb = (double*)malloc(sizeof(double) * (size_t)(rank * s)); /* [rank][s] */
+    for (int64_t j = 0; j < L; ++j)
+        for (int64_t i = 0; i < s; ++i) {
+            float gv = rows_short ? g[i * cols + j] : g[j * cols + i];
+            gb[j * s + i] = (double)ora_bf16_to_f32(ora_f32_to_bf16(gv));
+        }
+    for (int64_t q = 0; q < (int64_t)rank * s; ++q)
+        pb[q] = (double)ora_bf16_to_f32(proj[q]);
+#pragma omp parallel for schedule(static)
     for (int64_t j = 0; j < L; ++j)
         for (int k = 0; k < rank; ++k) {
+            const double* gj = gb + j * s;
+            const double* pk = pb + (int64_t)k * s;
             double acc = 0.0;
-            for (int64_t i = 0; i < s; ++i) {
-                float gv = rows_short ? g[i * cols + j] : g[j * cols + i];
-                double gb = (double)ora_bf16_to_f32(ora_f32_to_bf16(gv));
-                double pb = (double)ora_bf16_to_f32(proj[(int64_t)k * s + i]);
-                acc += pb * gb;
-            }
+            for (int64_t i = 0; i < s; ++i) acc += pk[i] * gj[i];
             R[j * rank + k] = (float)acc;
         }
+    free(gb);
+    free(pb);
 }
 
 /* Everything after the projection, for a given R [c x rank]. */
@@ -521,6 +549,7 @@ void ora_apollo_update_given_R(float* p, const float* g, int64_t rows,
     const float lr_a = (float)((double)hp->lr * (double)hp->alpha);
 
     float* s = (float*)xmalloc(sizeof(float) * (size_t)L);
+#pragma omp parallel for schedule(static)
     for (int64_t j = 0; j < L; ++j) {
         double nr = 0.0, ng = 0.0;
         for (int k = 0; k < rank; ++k) {
@@ -558,6 +587,7 @@ void ora_apollo_update_given_R(float* p, const float* g, int64_t rows,
         }
     }
 
+#pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < rows; ++i)
         for (int64_t j = 0; j < cols; ++j) {
             int64_t k = i * cols + j;
