@@ -303,3 +303,169 @@ def test_wrappers_hold_no_gradients(mods, kind):
     assert torch.cuda.memory_allocated() == base
     assert len(opt._plans) == nplans <= 1
     assert all(torch.isfinite(p).all() for p in params)
+
+
+# -------------------------------------------------- wrappers vs the oracle --
+def _np(t):
+    import torch
+    x = t.detach().cpu()
+    if x.dtype == torch.int16:
+        return x.numpy().view(np.uint16)
+    return x.numpy()
+
+
+def _set_grads(params, t, seed):
+    import torch
+    gs = []
+    for i, p in enumerate(params):
+        g = wl.student_t_grad(tuple(p.shape), 1e-3, 3.0, 0.05, seed + 100 * t + i)
+        p.grad = torch.from_numpy(g).cuda()
+        gs.append(g.ravel())
+    return gs
+
+
+def test_adamw_wrapper_with_g1_grouping_matches_oracle(mods):
+    """optim.AdamW over G1 groups (Sec. 6.1: one-dimensional tensors, biases,
+    norms and embeddings keep fp32 states, the rest AL8 V + UF8 M), 10 steps
+    against the oracle's step per tensor: AL8/UF8 codes and block constants
+    bit for bit, fp32-role states and parameters bit for bit, AL-path
+    parameters within 1e-5 of |p| plus the step sizes."""
+    import torch
+    import oracle as ora
+    from gpu_util import params_off, step_size
+    _, optim = mods
+    named = [("layer.weight", (64, 300)), ("layer.bias", (300,)), ("norm.weight", (512,)),
+             ("embed.weight", (100, 64)), ("mlp.weight", (37, 111))]
+    params = _params([s for _, s in named], 60)
+    groups = optim.g1_param_groups(zip([n for n, _ in named], params), dict(v_bits=32))
+    opt = optim.AdamW(groups, lr=1e-3, weight_decay=0.01)
+    protected = {id(p) for g in groups if g.get("v_bits") == 32 for p in g["params"]}
+    assert len(protected) == 3
+    host = []
+    for p in params:
+        n = p.numel()
+        raw = id(p) in protected
+        host.append(dict(p=_np(p).ravel().copy(), raw=raw,
+                         m=np.zeros(n, np.float32 if raw else np.int8),
+                         ma=None if raw else np.zeros((n + 255) // 256, np.float32),
+                         v=np.zeros(n, np.float32 if raw else np.uint8),
+                         vm=None if raw else np.zeros(2 * ((n + 255) // 256), np.float32),
+                         steps=np.zeros(n)))
+    for t in range(1, 11):
+        gs = _set_grads(params, t, 3000)
+        opt.step()
+        for h, g in zip(host, gs):
+            before = h["p"].copy()
+            ora.adamw_step(h["p"], g, h["m"], h["ma"], h["v"], h["vm"], 256, 256,
+                           32 if h["raw"] else 8, ADAMW_HP, t)
+            h["steps"] += step_size(h["p"], before, ADAMW_HP)
+    torch.cuda.synchronize()
+    for p, h in zip(params, host):
+        st = opt.state[p]
+        if h["raw"]:
+            for want, got in ((h["p"], p), (h["m"], st["m_codes"]), (h["v"], st["v_codes"])):
+                assert np.array_equal(want.view(np.uint8), _np(got).ravel().view(np.uint8))
+        else:
+            for want, key in ((h["m"], "m_codes"), (h["ma"], "m_absmax"), (h["v"], "v_codes"),
+                              (h["vm"], "v_meta")):
+                assert np.array_equal(want.view(np.uint8), _np(st[key]).view(np.uint8)), key
+            assert params_off(h["p"], _np(p).ravel(), h["steps"]) == 0
+
+
+@pytest.mark.parametrize("kind", ["Adafactor", "CAME"])
+def test_factored_wrappers_match_oracle(mods, kind):
+    """optim.Adafactor (AL16 factors, UF8 momentum) and optim.CAME (AL16 V
+    and C, UF8 momentum) over two matrices and a vector (a 1 x n matrix),
+    10 steps against the oracle's step per matrix: every code, block
+    constant and parameter bit for bit."""
+    import torch
+    import oracle as ora
+    _, optim = mods
+    shapes = [(64, 300), (300,), (256, 128)]
+    params = _params(shapes, 70)
+    opt = optim.CAME(params) if kind == "CAME" else optim.Adafactor(params)
+    g0 = opt.param_groups[0]
+    host = []
+    for p, s in zip(params, shapes):
+        rows, cols = (s[0], s[1]) if len(s) == 2 else (1, s[0])
+        n = rows * cols
+        h = dict(p=_np(p).ravel().copy(), rows=rows, cols=cols,
+                 mc=np.zeros(n, np.int8), ma=np.zeros((n + 255) // 256, np.float32))
+        for k, ln in (("vr", rows), ("vc", cols), ("cr", rows), ("cc", cols)):
+            h[k] = np.zeros(ln, np.uint16)
+            h[k + "m"] = np.zeros(2 * ((ln + 127) // 128), np.float32)
+        host.append(h)
+    for t in range(1, 11):
+        gs = _set_grads(params, t, 5000)
+        opt.step()
+        for h, g in zip(host, gs):
+            if kind == "CAME":
+                b1, b2, b3 = g0["betas"]
+                hp = dict(lr=g0["lr"], beta1=b1, beta2=b2, beta3=b3, eps1=g0["eps"][0],
+                          eps2=g0["eps"][1], clip_d=g0["clip_d"],
+                          weight_decay=g0["weight_decay"], log_floor_v=g0["log_floor_v"],
+                          log_floor_c=g0["log_floor_c"])
+                ora.came_step(h["p"], g, h["rows"], h["cols"], h["vr"], h["vrm"], h["vc"],
+                              h["vcm"], 16, 128, h["cr"], h["crm"], h["cc"], h["ccm"], 16, 128,
+                              h["mc"], h["ma"], 256, hp, t)
+            else:
+                hp = {k: g0[k] for k in ("lr", "eps1", "clip_d", "decay_rate", "beta1",
+                                          "weight_decay", "log_floor")}
+                ora.adafactor_step(h["p"], g, h["rows"], h["cols"], h["vr"], h["vrm"], h["vc"],
+                                   h["vcm"], 16, 128, h["mc"], h["ma"], 256, hp, t)
+    torch.cuda.synchronize()
+    keys = ({"vr": "vr_codes", "vrm": "vr_meta", "vc": "vc_codes", "vcm": "vc_meta",
+             "cr": "cr_codes", "crm": "cr_meta", "cc": "cc_codes", "ccm": "cc_meta"}
+            if kind == "CAME" else
+            {"vr": "r_codes", "vrm": "r_meta", "vc": "c_codes", "vcm": "c_meta"})
+    keys.update(mc="m_codes", ma="m_absmax")
+    for p, h in zip(params, host):
+        st = opt.state[p]
+        assert np.array_equal(h["p"].view(np.uint32), _np(p).ravel().view(np.uint32))
+        for hk, sk in keys.items():
+            assert np.array_equal(h[hk].view(np.uint8), _np(st[sk]).view(np.uint8)), (kind, sk)
+
+
+def test_apollo_wrapper_matches_oracle(mods):
+    """optim.Apollo: a matrix stepped through the grouped APOLLO launch with
+    the wrapper's own seeded projection, against the oracle's quantized
+    APOLLO step with that projection over 10 steps (displacement within
+    1e-4 of the oracle's: the projections accumulate differently, as in the
+    direct tests), and a vector routed to the quantized AdamW step (codes
+    and block constants bit for bit)."""
+    import torch
+    import oracle as ora
+    from gpu_util import params_off, step_size
+    _, optim = mods
+    params = _params([(256, 512), (512,)], 80)
+    opt = optim.Apollo(params, rank=128, lr=1e-4)
+    mat, vec = params
+    hp = dict(lr=1e-4, beta1=0.9, beta2=0.999, eps=1e-8, alpha=1.0, weight_decay=0.0,
+              norm_growth_gamma=0.0, log_floor=opt.param_groups[0]["log_floor"], rank=128)
+    hm = dict(p=_np(mat).ravel().copy(), mc=np.zeros(512 * 128, np.int8),
+              ma=np.zeros(512, np.float32), vc=np.zeros(512 * 128, np.uint8),
+              vm=np.zeros(1024, np.float32))
+    p0 = hm["p"].copy()
+    hv = dict(p=_np(vec).ravel().copy(), mc=np.zeros(512, np.int8), ma=np.zeros(2, np.float32),
+              vc=np.zeros(512, np.uint8), vm=np.zeros(4, np.float32), steps=np.zeros(512))
+    ahp = dict(ADAMW_HP, lr=1e-4, weight_decay=0.0)
+    for t in range(1, 11):
+        gs = _set_grads(params, t, 7000)
+        opt.step()
+        P = _np(opt.state[mat]["proj"]).copy()
+        ora.apollo_step(hm["p"], gs[0], 256, 512, P, hm["mc"], hm["ma"], 128, hm["vc"],
+                        hm["vm"], 8, 128, 0.0, hp, t)
+        before = hv["p"].copy()
+        ora.adamw_step(hv["p"], gs[1], hv["mc"], hv["ma"], hv["vc"], hv["vm"], 256, 256, 8,
+                       ahp, t)
+        hv["steps"] += step_size(hv["p"], before, ahp)
+    torch.cuda.synchronize()
+    pm = _np(mat).ravel().astype(np.float64)
+    disp = np.linalg.norm(pm - p0) and (np.linalg.norm((pm - p0) - (hm["p"] - p0))
+                                        / np.linalg.norm(hm["p"] - p0))
+    assert disp < 1e-4, disp
+    st = opt._adamw.state[vec]
+    for want, key in ((hv["mc"], "m_codes"), (hv["ma"], "m_absmax"), (hv["vc"], "v_codes"),
+                      (hv["vm"], "v_meta")):
+        assert np.array_equal(want.view(np.uint8), _np(st[key]).view(np.uint8)), key
+    assert params_off(hv["p"], _np(vec).ravel(), hv["steps"]) == 0
