@@ -72,35 +72,47 @@ def single_step_update_error(regime: str, block: int = 2048, bits: int = 8,
 
 def ema_drift(steps: int = 5000, block: int = 2048, bits: int = 8, n: int = 1 << 20,
               regime: str = "medium", beta1: float = 0.9, beta2: float = 0.999,
-              eps: float = 1e-8, seed: int = 0, device="cuda"):
+              eps: float = 1e-8, seed: int = 0, device="cuda", grad_fn=None,
+              return_state: bool = False):
     """A `steps`-long Adam-style EMA of fresh gradients whose per-block scale
     follows the regime (Sec. 5.6): the quantized second moment comes from the
-    fused AdamW step (lr = 0, AL-coded V, UF8 M), the reference from fp32
-    EMAs. Returns (V drift, steady-state update error) in the sense of
+    fused AdamW step (lr = 0, AL-coded V, UF8 M), the reference from float64
+    EMAs of the same gradients. Returns (V drift, steady-state update error) in the sense of
     Eq. (2): ||V_hat - V|| / ||V|| and the relative error of
-    M / (sqrt(V) + eps) with fp32 M against the same with V_hat."""
+    M / (sqrt(V) + eps) with fp32 M against the same with V_hat.
+    grad_fn(t), if given, supplies step t's gradient (a device tensor of n
+    fp32 values) instead of the regime's draws; return_state adds the final
+    (m_codes, m_absmax, v_codes, v_meta)."""
     nb = (n + block - 1) // block
-    scale = lognormal_state(nb, regime, seed, 1, device).sqrt().repeat_interleave(block)[:n]
+    scale = (None if grad_fn is not None else
+             lognormal_state(nb, regime, seed, 1, device).sqrt().repeat_interleave(block)[:n])
     p = torch.zeros(n, dtype=torch.float32, device=device)
     mc = torch.zeros(n, dtype=torch.int8, device=device)
     ma = torch.zeros((n + 255) // 256, dtype=torch.float32, device=device)
     vc = torch.zeros(n, dtype=torch.uint8 if bits == 8 else torch.int16, device=device)
     vm = torch.zeros(2 * nb, dtype=torch.float32, device=device)
-    v = torch.zeros(n, dtype=torch.float32, device=device)
-    m = torch.zeros(n, dtype=torch.float32, device=device)
+    v = torch.zeros(n, dtype=torch.float64, device=device)
+    m = torch.zeros(n, dtype=torch.float64, device=device)
     g = torch.empty(n, dtype=torch.float32, device=device)
     hp = dict(lr=0.0, beta1=beta1, beta2=beta2, eps=eps, weight_decay=0.0,
               log_floor=float(torch.tensor(math.log2(eps * eps), dtype=torch.float32)))
     gen = _gen(seed + 7, device)
     for t in range(1, steps + 1):
-        g.normal_(0.0, 1.0, generator=gen).mul_(scale)
+        if grad_fn is not None:
+            g = grad_fn(t)
+        else:
+            g.normal_(0.0, 1.0, generator=gen).mul_(scale)
         B.al_adamw_step(p, g, mc, ma, vc, vm, 256, block, bits, hp, t)
-        v.mul_(beta2).add_(g * g, alpha=1.0 - beta2)
-        m.mul_(beta1).add_(g, alpha=1.0 - beta1)
-    v_hat = torch.empty_like(v)
+        gd = g.double()
+        v.mul_(beta2).add_(gd * gd, alpha=1.0 - beta2)
+        m.mul_(beta1).add_(gd, alpha=1.0 - beta1)
+    v_hat = torch.empty(n, dtype=torch.float32, device=device)
     B.al_decode(vc, vm, block, bits, v_hat)
+    v_hat = v_hat.double()
     drift = update_error(v_hat, v)
     upd = update_error(m / (v_hat.sqrt() + eps), m / (v.sqrt() + eps))
+    if return_state:
+        return drift, upd, (mc, ma, vc, vm)
     return drift, upd
 
 
@@ -112,7 +124,7 @@ def main():
         e16 = single_step_update_error(r, 2048, 16)
         print(f"{r:8s} {100 * e8:8.3f} {100 * e16:10.5f}")
     print("5K-step EMA (beta2 = 0.999), medium regime: V drift %, update error %")
-    for blk in (256, 2048):
+    for blk in (256, 512, 1024, 2048):
         d, u = ema_drift(5000, blk, 8)
         print(f"block {blk:5d}  AL8  drift {100 * d:7.3f}  update {100 * u:7.3f}")
 
