@@ -490,8 +490,11 @@ int al_apollo_step(float* p, const float* g, int64_t rows, int64_t cols,
  * every step. The plan records the matrices' pointers, the workspace and the
  * TMA descriptors of the projections: rebuild it if any of them
  * changes (a refreshed projection written into the same proj buffer needs no
- * rebuild). The norm-growth limiter is not available here
- * (hp->norm_growth_gamma > 0 returns ALQ_ERR_UNSUPPORTED).
+ * rebuild). The norm-growth limiter (hp->norm_growth_gamma > 0) limits
+ * every matrix by its own previous norm (prev_norm, one device scalar per
+ * matrix, as in al_apollo_step); it returns ALQ_ERR_INVALID_ARG when a
+ * matrix of the plan has no prev_norm. Each matrix's results, limiter
+ * included, are bit for bit those of al_apollo_step.
  */
 typedef struct {
     float* p;              /* [rows x cols] fp32, as in al_apollo_step      */
@@ -502,17 +505,21 @@ typedef struct {
     float* m_absmax;
     void* v_codes;         /* [max(rows, cols) x rank] AL8 or AL16          */
     float* v_meta;
+    float* prev_norm;      /* device scalar, the limiter's previous norm
+                              (nullable when the limiter is never used)     */
 } al_apollo_matrix;
 
 /* Summary of a grouped plan (host struct, filled by al_apollo_plan). */
 typedef struct {
-    int32_t nmat, rank, v_bits, reserved;
+    int32_t nmat, rank, v_bits;
+    int32_t limiter_ok;     /* 1 when every matrix has a prev_norm           */
     int64_t total_params;   /* sum of rows * cols                            */
     int64_t total_channels; /* sum of max(rows, cols)                        */
     int64_t gemm_tiles;     /* 128-channel tiles of the grouped projection   */
     int64_t mom_tiles;      /* 2048-value tiles of the moments pass          */
     int64_t upd_tiles;      /* 4096-parameter tiles of the update pass       */
     void* workspace;        /* the workspace the plan is bound to            */
+    int64_t norm_chunks;    /* limiter partial sums (8 update tiles each)    */
 } al_apollo_info;
 
 /* Bytes of a plan over these matrices (host and device copies alike). */

@@ -67,14 +67,16 @@ class AdamWTensor(C.Structure):
 class ApolloMatrix(C.Structure):
     _fields_ = [("p", C.c_void_p), ("g", C.c_void_p), ("rows", C.c_int64),
                 ("cols", C.c_int64), ("proj", C.c_void_p), ("m_codes", C.c_void_p),
-                ("m_absmax", C.c_void_p), ("v_codes", C.c_void_p), ("v_meta", C.c_void_p)]
+                ("m_absmax", C.c_void_p), ("v_codes", C.c_void_p), ("v_meta", C.c_void_p),
+                ("prev_norm", C.c_void_p)]
 
 
 class ApolloInfo(C.Structure):
     _fields_ = [("nmat", C.c_int32), ("rank", C.c_int32), ("v_bits", C.c_int32),
-                ("reserved", C.c_int32), ("total_params", C.c_int64),
+                ("limiter_ok", C.c_int32), ("total_params", C.c_int64),
                 ("total_channels", C.c_int64), ("gemm_tiles", C.c_int64), ("mom_tiles", C.c_int64),
-                ("upd_tiles", C.c_int64), ("workspace", C.c_void_p)]
+                ("upd_tiles", C.c_int64), ("workspace", C.c_void_p),
+                ("norm_chunks", C.c_int64)]
 
 
 class FactoredMatrix(C.Structure):
@@ -405,8 +407,10 @@ class ApolloPlan(_BoundPlan):
     """A grouped APOLLO step over many matrices (al_apollo_plan /
     al_apollo_step_multi): owns the workspace and the device copy of the
     plan. `mats` is a list of dicts with keys p, g, rows, cols, proj, m_codes,
-    m_absmax, v_codes, v_meta (torch CUDA tensors; proj holds bf16 bits);
-    see _BoundPlan for g."""
+    m_absmax, v_codes, v_meta (torch CUDA tensors; proj holds bf16 bits) and
+    optionally prev_norm (a one-element fp32 tensor: the norm-growth
+    limiter's state, needed on every matrix when hp's norm_growth_gamma >
+    0); see _BoundPlan for g."""
 
     def __init__(self, mats, rank, v_bits, device=None):
         nm = len(mats)
@@ -415,7 +419,7 @@ class ApolloPlan(_BoundPlan):
             self._arr[i] = ApolloMatrix(_ptr(m["p"]), _ptr(m["g"]), m["rows"], m["cols"],
                                         _ptr(m["proj"]), _ptr(m["m_codes"]),
                                         _ptr(m["m_absmax"]), _ptr(m["v_codes"]),
-                                        _ptr(m["v_meta"]))
+                                        _ptr(m["v_meta"]), _ptr(m.get("prev_norm")))
         self._gptrs = [_ptr(m["g"]) for m in mats]
         dev = device if device is not None else mats[0]["p"].device
         ws = C.c_size_t(0)

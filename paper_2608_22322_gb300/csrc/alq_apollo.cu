@@ -14,7 +14,11 @@
 //   moments   per channel (one quantization block = rank values): decode
 //             UF8 M^P and AL8 V^P, Adam EMAs with bias correction, channel
 //             norms of Rt and R (exact two-float sums) -> s_j, re-encode.
-//   limiter   (optional) ||G s|| and the norm-growth cap.
+//   limiter   (optional) ||G s|| and the norm-growth cap: sums of squares
+//             per chunk of kNormChunk update tiles (a partition of each
+//             matrix that does not depend on the grid), summed in chunk
+//             order by the limiter kernel, so the grouped step limits every
+//             matrix exactly as the single-matrix step does.
 //   update    p = p (1 - lr wd) - (lr alpha) g s_j.
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -38,12 +42,17 @@ constexpr int kGemmSmem = kStages * (kAStage + kBStage) + 1024 + 256;
 struct ApWs {
     float* R;        // [L][rank]
     float* scale;    // [L]
-    double* npart;   // [kMaxNormParts] limiter partials
+    double* npart;   // [norm_chunks(n)] limiter partials
     float* lim;      // [2]: limiter factor
     int* err;        // [1]: projection pipeline timeout flag
     size_t bytes;
 };
-constexpr int kMaxNormParts = 4096;
+
+// Limiter partials: one per chunk of kNormChunk update tiles of a matrix.
+constexpr int kNormChunk = 8;
+static __host__ __device__ int64_t norm_chunks(int64_t n) {
+    return (((n + kTile - 1) / kTile) + kNormChunk - 1) / kNormChunk;
+}
 
 static size_t r256(size_t x) { return (x + 255) & ~(size_t)255; }
 
@@ -60,7 +69,7 @@ static ApWs ap_layout(void* base, int64_t rows, int64_t cols, int rank) {
     (void)s;
     w.R = (float*)take(4 * (size_t)L * rank);
     w.scale = (float*)take(4 * (size_t)L);
-    w.npart = (double*)take(8 * (size_t)kMaxNormParts);
+    w.npart = (double*)take(8 * (size_t)norm_chunks(rows * cols));
     w.lim = (float*)take(8);
     w.err = (int*)take(4);
     w.bytes = off;
@@ -642,12 +651,17 @@ struct ApUpdateArgs {
     float decay, lr_a;
 };
 
-__global__ void __launch_bounds__(kThreads)
-apollo_gnorm_kernel(ApUpdateArgs u, int64_t ntiles, double* __restrict__ part) {
-    __shared__ double s_w[kThreads / 32];
+// Sum of (g s_j)^2 over chunk `chunk` (update tiles chunk * kNormChunk ..
+// + kNormChunk - 1 of a matrix of ntiles tiles), computed by the whole CTA
+// in a fixed order (each warp its segments tile by tile in two-float, the
+// warps merged in order in double) and written to part[chunk]. s_w holds
+// kThreads / 32 doubles; every thread of the CTA calls this.
+__device__ __forceinline__ void gnorm_chunk(const ApUpdateArgs& u, int64_t chunk, int64_t ntiles,
+                                            double* __restrict__ part, double* s_w) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     float hi = 0.0f, lo = 0.0f;
-    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+    const int64_t t1 = min(ntiles, (chunk + 1) * kNormChunk);
+    for (int64_t tile = chunk * kNormChunk; tile < t1; ++tile) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
@@ -660,8 +674,8 @@ apollo_gnorm_kernel(ApUpdateArgs u, int64_t ntiles, double* __restrict__ part) {
             if (u.rows_short) {
                 sv = __ldg(reinterpret_cast<const float4*>(u.scale + col));
             } else {
-                const float s = __ldg(u.scale + row);
-                sv = make_float4(s, s, s, s);
+                const float sc = __ldg(u.scale + row);
+                sv = make_float4(sc, sc, sc, sc);
             }
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
@@ -673,20 +687,29 @@ apollo_gnorm_kernel(ApUpdateArgs u, int64_t ntiles, double* __restrict__ part) {
         }
     }
     ff_warp_sum(hi, lo);
+    __syncthreads();  // s_w of the previous chunk has been read
     if (lane == 0) s_w[warp] = (double)hi + (double)lo;
     __syncthreads();
     if (threadIdx.x == 0) {
-        double s = 0.0;
-        for (int w = 0; w < kThreads / 32; ++w) s += s_w[w];
-        part[blockIdx.x] = s;
+        double sum = 0.0;
+        for (int w = 0; w < kThreads / 32; ++w) sum += s_w[w];
+        part[chunk] = sum;
     }
 }
 
-__global__ void apollo_limit_kernel(const double* __restrict__ part, int nparts, float gamma,
-                                    float* __restrict__ prev_norm, float* __restrict__ lim) {
-    if (threadIdx.x != 0) return;
+__global__ void __launch_bounds__(kThreads)
+apollo_gnorm_kernel(ApUpdateArgs u, int64_t ntiles, int64_t nchunks, double* __restrict__ part) {
+    __shared__ double s_w[kThreads / 32];
+    for (int64_t c = blockIdx.x; c < nchunks; c += gridDim.x) gnorm_chunk(u, c, ntiles, part, s_w);
+}
+
+// The limiter of one matrix from its chunk partials (summed in chunk order):
+// ||G s|| against gamma times the previous norm.
+__device__ __forceinline__ void limit_one(const double* __restrict__ part, int64_t nparts,
+                                          float gamma, float* __restrict__ prev_norm,
+                                          float* __restrict__ lim) {
     double ss = 0.0;
-    for (int i = 0; i < nparts; ++i) ss += part[i];
+    for (int64_t i = 0; i < nparts; ++i) ss += part[i];
     const double nt = sqrt(ss);
     const double prev = (double)*prev_norm;
     const double cap = (double)gamma * prev;
@@ -697,6 +720,11 @@ __global__ void apollo_limit_kernel(const double* __restrict__ part, int nparts,
         lim[0] = 1.0f;
         *prev_norm = (float)nt;
     }
+}
+
+__global__ void apollo_limit_kernel(const double* __restrict__ part, int64_t nparts, float gamma,
+                                    float* __restrict__ prev_norm, float* __restrict__ lim) {
+    if (threadIdx.x == 0) limit_one(part, nparts, gamma, prev_norm, lim);
 }
 
 // One tile (kTile parameters) of p = p (1 - lr wd) - (lr alpha) lim (g s_j).
@@ -747,7 +775,9 @@ struct ApPlanHeader {
     int32_t nmat, rank, v_bits;
     int64_t gemm_tiles, mom_tiles, upd_tiles;
     int64_t total_params, total_channels;
-    int64_t reserved[3];
+    int64_t norm_chunks;
+    int32_t limiter_ok, reserved0;
+    int64_t reserved;
 };
 static_assert(sizeof(ApPlanHeader) == 80, "plan header layout");
 
@@ -765,6 +795,10 @@ struct ApEntry {  // aligned as CUtensorMap (at least 64 bytes)
     Divider dv;
     int32_t rows_short, kblocks;
     int64_t gemm_t0, mom_t0, upd_t0;  // first tile of each pass
+    int64_t nrm_t0;                   // first limiter chunk
+    double* npart;                    // limiter partials [norm_chunks(n)]
+    float* lim;                       // limiter factor
+    float* prev_norm;                 // previous update norm (device scalar)
 };
 
 constexpr size_t kApEntryOffset = 128;  // header rounded up to the entry alignment
@@ -818,9 +852,10 @@ apollo_moments_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t n
     ps.flush();
 }
 
+// limited: every matrix's update is scaled by its limiter factor.
 __global__ void __launch_bounds__(kThreads)
 apollo_update_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t ntiles,
-                           ApUpdateArgs base) {
+                           ApUpdateArgs base, int limited) {
     int cur = 0;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         cur = entry_for(tab, nmat, tile, cur, &ApEntry::upd_t0);
@@ -832,8 +867,37 @@ apollo_update_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t nt
         u.dv = e.dv;
         u.rows_short = e.rows_short;
         u.scale = e.scale;
-        update_tile(u, tile - e.upd_t0, 1.0f);
+        u.lim = limited ? e.lim : nullptr;
+        update_tile(u, tile - e.upd_t0, limited ? __ldg(e.lim) : 1.0f);
     }
+}
+
+// Limiter partials of every matrix: one chunk per iteration, the chunks of
+// all matrices in one launch.
+__global__ void __launch_bounds__(kThreads)
+apollo_gnorm_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t nchunks) {
+    __shared__ double s_w[kThreads / 32];
+    int cur = 0;
+    for (int64_t c = blockIdx.x; c < nchunks; c += gridDim.x) {
+        cur = entry_for(tab, nmat, c, cur, &ApEntry::nrm_t0);
+        const ApEntry& e = tab[cur];
+        ApUpdateArgs u{};
+        u.g = e.g;
+        u.n = e.n;
+        u.dv = e.dv;
+        u.rows_short = e.rows_short;
+        u.scale = e.scale;
+        gnorm_chunk(u, c - e.nrm_t0, (e.n + kTile - 1) / kTile, e.npart, s_w);
+    }
+}
+
+// One thread per matrix: its limiter factor and new previous norm.
+__global__ void apollo_limit_multi_kernel(const ApEntry* __restrict__ tab, int nmat,
+                                          float gamma) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= nmat) return;
+    const ApEntry& e = tab[i];
+    limit_one(e.npart, norm_chunks(e.n), gamma, e.prev_norm, e.lim);
 }
 
 // ------------------------------------------------------------- host side --
@@ -981,10 +1045,10 @@ extern "C" int al_apollo_step(float* p, const float* g, int64_t rows, int64_t co
     u.lr_a = (float)((double)hp->lr * (double)hp->alpha);
     const int64_t ntiles = blocks_of(u.n, kTile);
     if (hp->norm_growth_gamma > 0.0f) {
-        int grid = persistent_grid((const void*)apollo_gnorm_kernel, kThreads, 0, ntiles);
-        if (grid > kMaxNormParts) grid = kMaxNormParts;
-        apollo_gnorm_kernel<<<grid, kThreads, 0, st>>>(u, ntiles, w.npart);
-        apollo_limit_kernel<<<1, 32, 0, st>>>(w.npart, grid, hp->norm_growth_gamma, prev_norm,
+        const int64_t nch = norm_chunks(u.n);
+        apollo_gnorm_kernel<<<persistent_grid((const void*)apollo_gnorm_kernel, kThreads, 0, nch),
+                              kThreads, 0, st>>>(u, ntiles, nch, w.npart);
+        apollo_limit_kernel<<<1, 32, 0, st>>>(w.npart, nch, hp->norm_growth_gamma, prev_norm,
                                                w.lim);
         u.lim = w.lim;
     }
@@ -1010,10 +1074,12 @@ static ApShape ap_shape(const al_apollo_matrix& m) {
     return a;
 }
 
-// Per-matrix scratch of a grouped step: R, scale, each 256-byte aligned.
+// Per-matrix scratch of a grouped step: R, scale, limiter partials and
+// factor, each 256-byte aligned.
 static size_t multi_ws_bytes(const al_apollo_matrix& m, int rank) {
     const ApShape a = ap_shape(m);
-    return r256(4 * (size_t)a.L * rank) + r256(4 * (size_t)a.L);
+    return r256(4 * (size_t)a.L * rank) + r256(4 * (size_t)a.L) +
+           r256(8 * (size_t)norm_chunks(a.n)) + r256(8);
 }
 
 static int check_matrices(const al_apollo_matrix* mats, int nmat) {
@@ -1076,6 +1142,7 @@ extern "C" int al_apollo_plan(const al_apollo_matrix* mats, int nmat, int rank, 
     char* ws = (char*)workspace + 256;  // first 256 bytes: timeout flag
     ApPlanHeader h{};
     h.magic = kApPlanMagic;
+    h.limiter_ok = 1;
     h.nmat = nmat;
     h.rank = rank;
     h.v_bits = v_bits;
@@ -1092,6 +1159,9 @@ extern "C" int al_apollo_plan(const al_apollo_matrix* mats, int nmat, int rank, 
         e.v_meta = m.v_meta;
         e.R = (float*)ws;
         e.scale = (float*)(ws + r256(4 * (size_t)a.L * rank));
+        e.npart = (double*)(ws + r256(4 * (size_t)a.L * rank) + r256(4 * (size_t)a.L));
+        e.lim = (float*)((char*)e.npart + r256(8 * (size_t)norm_chunks(a.n)));
+        e.prev_norm = m.prev_norm;
         ws += multi_ws_bytes(m, rank);
         e.rows = m.rows;
         e.cols = m.cols;
@@ -1105,6 +1175,7 @@ extern "C" int al_apollo_plan(const al_apollo_matrix* mats, int nmat, int rank, 
         e.gemm_t0 = h.gemm_tiles;
         e.mom_t0 = h.mom_tiles;
         e.upd_t0 = h.upd_tiles;
+        e.nrm_t0 = h.norm_chunks;
         if (!make_map(&e.tmB, m.proj, (uint64_t)a.s, (uint64_t)rank, (uint32_t)rank))
             return record_cuda(cudaErrorInvalidValue);
         const int64_t gt = blocks_of(a.L, kGM);
@@ -1112,6 +1183,8 @@ extern "C" int al_apollo_plan(const al_apollo_matrix* mats, int nmat, int rank, 
         h.gemm_tiles += gt;
         h.mom_tiles += blocks_of(e.npj, kMTile);
         h.upd_tiles += blocks_of(a.n, kTile);
+        h.norm_chunks += norm_chunks(a.n);
+        if (!m.prev_norm) h.limiter_ok = 0;
         h.total_params += a.n;
         h.total_channels += a.L;
         memcpy(base + kApEntryOffset + (size_t)i * sizeof(ApEntry), &e, sizeof(e));
@@ -1120,7 +1193,8 @@ extern "C" int al_apollo_plan(const al_apollo_matrix* mats, int nmat, int rank, 
     info->nmat = nmat;
     info->rank = rank;
     info->v_bits = v_bits;
-    info->reserved = 0;
+    info->limiter_ok = h.limiter_ok;
+    info->norm_chunks = h.norm_chunks;
     info->total_params = h.total_params;
     info->total_channels = h.total_channels;
     info->gemm_tiles = h.gemm_tiles;
@@ -1136,7 +1210,8 @@ extern "C" int al_apollo_step_multi(const void* plan_dev, const al_apollo_info* 
         return ALQ_ERR_INVALID_ARG;
     if (!aligned(plan_dev, 64)) return ALQ_ERR_ALIGN;
     if (hp->rank != info->rank) return ALQ_ERR_INVALID_ARG;
-    if (hp->norm_growth_gamma > 0.0f) return ALQ_ERR_UNSUPPORTED;
+    const bool limited = hp->norm_growth_gamma > 0.0f;
+    if (limited && !info->limiter_ok) return ALQ_ERR_INVALID_ARG;  // a matrix has no prev_norm
     cudaStream_t st = (cudaStream_t)stream;
     const ApEntry* tab = (const ApEntry*)((const char*)plan_dev + kApEntryOffset);
     const uint16_t* tile_mat = (const uint16_t*)((const char*)plan_dev + kApEntryOffset +
@@ -1171,12 +1246,23 @@ extern "C" int al_apollo_step_multi(const void* plan_dev, const al_apollo_info* 
     rc = check_launch();
     if (rc) return rc;
 
+    if (limited) {
+        const int64_t nch = info->norm_chunks;
+        apollo_gnorm_multi_kernel<<<persistent_grid((const void*)apollo_gnorm_multi_kernel,
+                                                    kThreads, 0, nch),
+                                    kThreads, 0, st>>>(tab, info->nmat, nch);
+        apollo_limit_multi_kernel<<<(info->nmat + 127) / 128, 128, 0, st>>>(
+            tab, info->nmat, hp->norm_growth_gamma);
+        rc = check_launch();
+        if (rc) return rc;
+    }
     ApUpdateArgs u{};
     u.lim = nullptr;
     u.decay = (float)(1.0 - (double)hp->lr * (double)hp->weight_decay);
     u.lr_a = (float)((double)hp->lr * (double)hp->alpha);
     apollo_update_multi_kernel<<<persistent_grid((const void*)apollo_update_multi_kernel,
                                                  kThreads, 0, info->upd_tiles),
-                                 kThreads, 0, st>>>(tab, info->nmat, info->upd_tiles, u);
+                                 kThreads, 0, st>>>(tab, info->nmat, info->upd_tiles, u,
+                                                    limited ? 1 : 0);
     return check_launch();
 }

@@ -412,19 +412,24 @@ class Apollo(_Base):
     V^P (v_bits), stepped for all matrices of a group in one grouped launch
     sequence (al_apollo_step_multi). The projection of each matrix is drawn
     from N(0, 1/rank) (seeded by `seed` and the parameter's index, redrawn
-    every proj_gap steps) and rounded to bf16. Parameters that are not
-    eligible matrices (vectors, shapes the kernels do not take) are stepped by
-    the quantized AdamW with the same lr, betas, eps and weight decay."""
+    every proj_gap steps) and rounded to bf16. norm_growth_gamma > 0 turns on
+    the norm-growth limiter (each matrix's scaled-gradient norm may grow by at
+    most that factor per step; per-matrix state "prev_norm"). Parameters that
+    are not eligible matrices (vectors, shapes the kernels do not take) are
+    stepped by the quantized AdamW with the same lr, betas, eps and weight
+    decay."""
 
     _CODES = {"m_codes": None, "v_codes": "v_bits"}
     _AL = {"v_codes": ("v_meta", "rank")}
 
     def __init__(self, params, lr=1e-4, betas=(0.9, 0.999), eps=1e-8, alpha=1.0,
-                 weight_decay=0.0, rank=256, v_bits=8, proj_gap=200, seed=0, log_floor=None):
+                 weight_decay=0.0, rank=256, v_bits=8, proj_gap=200, seed=0, log_floor=None,
+                 norm_growth_gamma=0.0):
         if rank not in (128, 256):
             raise ValueError("rank must be 128 or 256")
         defaults = dict(lr=lr, betas=betas, eps=eps, alpha=alpha, weight_decay=weight_decay,
                         rank=rank, v_bits=v_bits, proj_gap=proj_gap, seed=seed,
+                        norm_growth_gamma=norm_growth_gamma,
                         log_floor=log_floor if log_floor is not None else _log2_floor(eps * eps))
         super().__init__(params, defaults)
         others = [p for g in self.param_groups for p in g["params"] if not _apollo_ok(p, rank)]
@@ -445,6 +450,7 @@ class Apollo(_Base):
         st["m_absmax"] = torch.zeros(npj // r, dtype=torch.float32, device=dev)
         st["v_codes"] = torch.zeros(npj, dtype=_code_dtype(group["v_bits"]), device=dev)
         st["v_meta"] = torch.zeros(2 * (npj // r), dtype=torch.float32, device=dev)
+        st["prev_norm"] = torch.zeros(1, dtype=torch.float32, device=dev)
 
     def _draw_projection(self, p, group, st):
         gen = torch.Generator(device=p.device)
@@ -478,17 +484,22 @@ class Apollo(_Base):
                 if (st["step"] - 1) % group["proj_gap"] == 0:
                     self._draw_projection(p, group, st)
                 rows, cols = p.shape
+                if "prev_norm" not in st:  # a state saved before the limiter existed
+                    st["prev_norm"] = torch.zeros(1, dtype=torch.float32, device=p.device)
                 buckets.setdefault(st["step"], []).append(
                     dict(p=p, g=p.grad, rows=rows, cols=cols, proj=st["proj"],
                          m_codes=st["m_codes"], m_absmax=st["m_absmax"],
-                         v_codes=st["v_codes"], v_meta=st["v_meta"]))
+                         v_codes=st["v_codes"], v_meta=st["v_meta"],
+                         prev_norm=st["prev_norm"]))
             b1, b2 = group["betas"]
             hp = dict(lr=group["lr"], beta1=b1, beta2=b2, eps=group["eps"],
                       alpha=group["alpha"], weight_decay=group["weight_decay"],
-                      norm_growth_gamma=0.0, log_floor=group["log_floor"], rank=group["rank"])
+                      norm_growth_gamma=group.get("norm_growth_gamma", 0.0),
+                      log_floor=group["log_floor"], rank=group["rank"])
             for t, mats in buckets.items():
                 key = (_state_key(mats, ("p", "proj", "m_codes", "m_absmax", "v_codes",
-                                         "v_meta")), group["rank"], group["v_bits"])
+                                         "v_meta", "prev_norm")), group["rank"],
+                       group["v_bits"])
                 plan = self._plans.get(key)
                 if plan is None:
                     if len(self._plans) > 8:

@@ -245,12 +245,76 @@ def test_apollo_grouped_step_matches_single(B, rank, v_bits):
     assert info.gemm_tiles == sum((max(r, c) + 127) // 128 for r, c in shapes)
 
 
-def test_apollo_grouped_rejects_limiter_and_bad_arguments(B):
+@pytest.mark.parametrize("rank", [128, 256])
+def test_apollo_grouped_limiter_matches_single(B, rank):
+    """The norm-growth limiter in the grouped step (per-matrix chunk
+    partials of ||G s||^2, one limiter thread per matrix) gives every matrix
+    bit for bit the single-matrix step's parameters, states and previous
+    norm over four steps; the previous norms follow the oracle's within
+    1e-5. The scaled update G s does not grow with the gradient's scale
+    (s_j normalises each channel), so the cap is engaged by channels that
+    wake up: every other channel has a zero gradient at steps 1 and 2 (s_j =
+    0) and all are active from step 3, when ||G s|| grows by about sqrt(2)."""
+    import torch
+    shapes = [(64, 256), (384, 128), (136, 1000), (1000, 136), (512, 2048)]
+    hp = dict(HP, rank=rank, norm_growth_gamma=1.01)
+    single, grouped, host = [], [], []
+    for i, (rows, cols) in enumerate(shapes):
+        st = _mat_state(rows, cols, rank, 8, 500 + 11 * i)
+        host.append(dict({k: v.copy() for k, v in st.items()}, prev=np.float32(0.0)))
+        single.append({k: _t(v) for k, v in st.items()})
+        grouped.append({k: _t(v) for k, v in st.items()})
+        single[-1]["prev"] = torch.zeros(1, dtype=torch.float32, device="cuda")
+        grouped[-1]["prev_norm"] = torch.zeros(1, dtype=torch.float32, device="cuda")
+    grads = [torch.zeros(r * c, dtype=torch.float32, device="cuda") for r, c in shapes]
+    plan = B.ApolloPlan([dict(grouped[i], g=grads[i], rows=r, cols=c)
+                         for i, (r, c) in enumerate(shapes)], rank, 8)
+    assert plan.info.limiter_ok == 1
+    capped = 0
+    for t in range(1, 5):
+        for i, (rows, cols) in enumerate(shapes):
+            g = wl.gaussian_grad((rows, cols), 1e-3, 9500 + 13 * i + t)
+            if t < 3:  # every other channel dormant
+                if rows <= cols:
+                    g[:, ::2] = 0.0
+                else:
+                    g[::2, :] = 0.0
+            g = g.ravel()
+            grads[i].copy_(torch.from_numpy(g))
+            d = single[i]
+            ws = torch.zeros(B.al_workspace_size(B.AL_OP_APOLLO, rows, cols, rank),
+                             dtype=torch.uint8, device="cuda")
+            B.al_apollo_step(d["p"], grads[i], rows, cols, d["proj"], d["m_codes"],
+                             d["m_absmax"], rank, d["v_codes"], d["v_meta"], 8, rank, d["prev"],
+                             hp, t, ws)
+            h = host[i]
+            before = h["prev"]
+            _, h["prev"] = ora.apollo_step(h["p"], g, rows, cols, h["proj"], h["m_codes"],
+                                           h["m_absmax"], rank, h["v_codes"], h["v_meta"], 8,
+                                           rank, h["prev"], hp, t)
+            if t == 3:  # the woken channels: the norm is capped at 1.01 x the last
+                capped += int(abs(float(h["prev"]) - 1.01 * float(before))
+                              <= 1e-6 * float(h["prev"]))
+        plan.step(hp, t)
+        torch.cuda.synchronize()
+        for i in range(len(shapes)):
+            for k in ("p", "m_codes", "m_absmax", "v_codes", "v_meta"):
+                a = single[i][k].cpu().numpy().view(np.uint8)
+                b = grouped[i][k].cpu().numpy().view(np.uint8)
+                assert np.array_equal(a, b), (shapes[i], k, t)
+            assert single[i]["prev"].item() == grouped[i]["prev_norm"].item(), (shapes[i], t)
+            assert abs(grouped[i]["prev_norm"].item() - float(host[i]["prev"])) <= \
+                1e-5 * float(host[i]["prev"]), (shapes[i], t)
+    assert capped == len(shapes)  # the spike at t = 3 engaged every matrix's cap
+
+
+def test_apollo_grouped_rejects_limiter_without_state_and_bad_arguments(B):
     import torch
     st = {k: _t(v) for k, v in _mat_state(64, 256, 128, 8, 5).items()}
     g = torch.zeros(64 * 256, dtype=torch.float32, device="cuda")
     plan = B.ApolloPlan([dict(st, g=g, rows=64, cols=256)], 128, 8)
-    with pytest.raises(B.AlqError):
+    assert plan.info.limiter_ok == 0
+    with pytest.raises(B.AlqError, match="INVALID_ARG"):  # no prev_norm for the limiter
         plan.step(dict(HP, rank=128, norm_growth_gamma=1.01), 1)
     with pytest.raises(B.AlqError):
         plan.step(dict(HP, rank=256), 1)  # rank differs from the plan's
