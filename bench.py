@@ -15,8 +15,12 @@ region), SM clocks sampled during the timed region, and the kernel launch
 count. With N > 1 (torchrun) every rank runs an independent replica (the
 AdamW step has no cross-rank exchange); value = params of all ranks / max
 rank time. --impl reference times the CPU oracle instead (the reference arm).
---workload adafactor|came|apollo|codec times the other hot-path rows instead,
-one JSON line each (see run_rows).
+The same default run then times the other hot-path rows (Adafactor 4096 x
+4096, CAME 22 x 2048 x 5632, APOLLO over the 154 TinyLlama matrices, the
+AL8/UF8 codec on 2^28 elements) and reports them under "rows", each with its
+own clock record, an L2 flush between timed steps and the oracle on a
+bounded sample (--no-rows skips them). --workload adafactor|came|apollo|codec
+times one of those rows alone, as its own JSON line.
 """
 from __future__ import annotations
 
@@ -58,6 +62,8 @@ def parse_args():
     ap.add_argument("--v-block", type=int, default=256,
                     help="AdamW second-moment block size (256 is the benchmark's "
                          "configuration; 2048 is the paper's core AdamW setting)")
+    ap.add_argument("--no-rows", action="store_true",
+                    help="skip the other hot-path rows after the headline step")
     ap.add_argument("--workload", default="adamw",
                     choices=["adamw", "adafactor", "came", "apollo", "codec"],
                     help="adamw: the headline TinyLlama AdamW step (default); the others "
@@ -93,6 +99,34 @@ def measured_peaks():
             return json.load(f), "measured"
     except OSError:
         return {"hbm_gbs": 6800.0}, "fallback"
+
+
+def host_info():
+    """The host cores the CPU baselines run on: nproc and the CPU model."""
+    model = None
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                model = line.split(":", 1)[1].strip()
+                break
+    except (OSError, subprocess.SubprocessError):
+        pass
+    if model is None:
+        try:
+            for line in open("/proc/cpuinfo"):
+                if line.lower().startswith(("model name", "cpu part")):
+                    model = line.split(":", 1)[1].strip()
+                    break
+        except OSError:
+            pass
+    return {"nproc": os.cpu_count(), "cpu_model": model}
+
+
+def oracle_threads(ora, want: bool) -> int:
+    """Switch the oracle to its OpenMP build (all host cores, the same
+    results bit for bit) or back; returns the thread count in use."""
+    return ora.use_threads(want)
 
 
 class ClockSampler:
@@ -209,14 +243,18 @@ def algorithmic_bytes(arrs):
     return tot
 
 
-def cpu_baseline(torch, ora, arrs, hp, t, max_params=180_000_000, v_block=256):
-    """The oracle (single-threaded C) on a bounded sample: the first tensors
-    of the plan, up to max_params parameters, from the device state."""
-    import numpy as np
+def cpu_baseline(torch, ora, arrs, hp, t, v_block=256):
+    """The oracle on the host cores: its OpenMP build (parallel over blocks
+    and elements; the same results as the single-threaded build) over the
+    whole parameter set for one step, or, where the compiler has no OpenMP,
+    the single-threaded build over the first tensors (up to 180M
+    parameters)."""
+    threads = oracle_threads(ora, True)
+    max_params = None if threads > 1 else 180_000_000
     sample, taken = [], 0
     for a in arrs:
         n = a["p"].numel()
-        if taken + n > max_params and taken > 0:
+        if max_params is not None and taken + n > max_params and taken > 0:
             break
         sample.append(a)
         taken += n
@@ -228,9 +266,11 @@ def cpu_baseline(torch, ora, arrs, hp, t, max_params=180_000_000, v_block=256):
     for h in host:
         ora.adamw_step(h["p"], h["g"], h["mc"], h["ma"], h["vc"], h["vm"], 256, v_block, 8, hp, t)
     dt = time.perf_counter() - t0
-    return {"value": taken / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"one step over the first {len(sample)} TinyLlama tensors "
-                      f"({taken} params, {dt:.1f} s, single thread)"}
+    oracle_threads(ora, False)
+    what = ("all" if len(sample) == len(arrs) else f"the first {len(sample)}")
+    return dict({"value": taken / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
+                 "sample": f"one step over {what} TinyLlama tensors ({taken} params, {dt:.1f} s "
+                           f"on {threads} thread{'s' if threads > 1 else ''})"}, **host_info())
 
 
 def run_ours(args):
@@ -304,6 +344,20 @@ def run_ours(args):
         import oracle as ora
         cpu = cpu_baseline(torch, ora, arrs, hp, t + 1, v_block=args.v_block)
 
+    rows = None
+    if rank == 0 and world == 1 and not args.no_rows and not args.tensors:
+        # the other rows are single-GPU measurements of their own workloads
+        del arrs, plans
+        import gc
+        gc.collect()
+        torch.cuda.empty_cache()
+        rows = {}
+        for name in ("adafactor", "came", "apollo", "codec"):
+            rows[name] = measure_row(name, args, dev, warmup=5, min_steps=20,
+                                     with_cpu=not args.no_cpu, summary=True)
+            gc.collect()
+            torch.cuda.empty_cache()
+
     if world > 1:
         dist.destroy_process_group()
     if rank != 0:
@@ -325,6 +379,8 @@ def run_ours(args):
                      "peak_source": f"{peak_src} hbm_gbs", "kernel": "adamw_fused_kernel"},
         "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "gpu_launches": launches,
     }
+    if rows is not None:
+        line["rows"] = rows
     print(json.dumps(line), flush=True)
 
 
@@ -421,9 +477,11 @@ def run_e2e(torch, B, arrs, hp, t, steps, n_params, dev, nchunks=32):
 # ---------------------------------------------------------- reference arm --
 def run_reference(args):
     """The CPU oracle as the reference arm: each step is one oracle AdamW step
-    over a bounded sample of the workload (a slice of up to 16M parameters
-    with the TinyLlama draws, sized so warmup + steps take about 100 s of
-    single-thread time), on this host's cores."""
+    over a bounded sample of the workload (a slice of the TinyLlama draws,
+    sized from a calibration step so that warmup + steps take about 100 s,
+    between 1M and 256M parameters), on this host's cores (the oracle's
+    OpenMP build where the compiler has OpenMP: the same results as the
+    single-threaded build)."""
     import numpy as np
 
     import oracle as ora
@@ -432,16 +490,25 @@ def run_reference(args):
     world = int(os.environ.get("WORLD_SIZE", "1"))
     if rank != 0:
         return
-    n = int(100 * 2.6e7 / max(1, args.steps + args.warmup)) // 4096 * 4096
-    n = max(1 << 20, min(1 << 24, n))
-    p = (wl.rng(1).standard_normal(n) * 0.02).astype(np.float32)
-    gs = [wl.gaussian_grad((n,), 1e-3, 10 + k, wl.zero_mask((n,), 0.01, 20 + k)) for k in range(2)]
-    mc = np.zeros(n, np.int8)
-    ma = np.zeros(n // 256, np.float32)
-    vc = np.zeros(n, np.uint8)
-    vm = np.zeros(2 * n // 256, np.float32)
+    threads = oracle_threads(ora, True)
     hp = dict(lr=1e-3, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.01,
               log_floor=float(np.float32(np.log2(1e-16))))
+
+    def state(n):
+        p = (wl.rng(1).standard_normal(n) * 0.02).astype(np.float32)
+        gs = [wl.gaussian_grad((n,), 1e-3, 10 + k, wl.zero_mask((n,), 0.01, 20 + k))
+              for k in range(2)]
+        return (p, gs, np.zeros(n, np.int8), np.zeros(n // 256, np.float32),
+                np.zeros(n, np.uint8), np.zeros(2 * n // 256, np.float32))
+
+    n0 = 1 << 22
+    p, gs, mc, ma, vc, vm = state(n0)
+    t0 = time.perf_counter()
+    ora.adamw_step(p, gs[1], mc, ma, vc, vm, 256, 256, 8, hp, 1)
+    rate = n0 / (time.perf_counter() - t0)
+    n = int(100.0 * rate / max(1, args.steps + args.warmup)) // 4096 * 4096
+    n = max(1 << 20, min(1 << 28, n))
+    p, gs, mc, ma, vc, vm = state(n)
     t = 0
     for _ in range(args.warmup):
         t += 1
@@ -451,6 +518,7 @@ def run_reference(args):
         t += 1
         ora.adamw_step(p, gs[t % 2], mc, ma, vc, vm, 256, 256, 8, hp, t)
     dt = (time.perf_counter() - t0) / args.steps
+    oracle_threads(ora, False)
     v = n / dt
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT,
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
@@ -458,8 +526,10 @@ def run_reference(args):
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {"workload": "tinyllama-1.1b AdamW, AL8 second moment + UF8 momentum, "
                                    "blocks 256", "sample": f"{n} params per step"},
-            "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
-                             "sample": f"one oracle step over {n} params per timed step"},
+            "cpu_baseline": dict({"value": v, "unit": UNIT, "cores": threads, "kind": "oracle",
+                                  "sample": f"one oracle step over {n} params per timed step "
+                                            f"on {threads} thread{'s' if threads > 1 else ''}"},
+                                 **host_info()),
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -540,7 +610,7 @@ def _row_adafactor(torch, np, wl, B, dev):
         t0 = time.perf_counter()
         ora.adafactor_step(ph, gh, rows, cols, rc, rm, cc, cm, fbits, fb, mch, mah, 256, hp, t)
         dt = time.perf_counter() - t0
-        return n / dt, f"one step of the whole {rows}x{cols} matrix ({dt:.1f} s, single thread)"
+        return n / dt, f"one step of the whole {rows}x{cols} matrix ({dt:.2f} s)"
 
     return dict(step=step, n=n, bytes=nbytes, launches=6, oracle=oracle_sample,
                 workload=f"Adafactor {rows}x{cols}, AL16 factors block 128, UF8 momentum block 256",
@@ -623,9 +693,10 @@ def _row_came(torch, np, wl, B, dev):
         t0 = time.perf_counter()
         ora.came_step(ph, gh, rows, cols, *args, hp, t)
         dt = time.perf_counter() - t0
-        return n1 / dt, f"one step of one {rows}x{cols} matrix ({dt:.1f} s, single thread)"
+        return n1 / dt, f"one step of one {rows}x{cols} matrix ({dt:.2f} s)"
 
     return dict(step=step, n=nm * n1, bytes=nbytes, launches=8 * ngroups, oracle=oracle_sample,
+                cpu_threads=True,
                 workload=f"CAME {nm} x {rows}x{cols}, AL16 factored V and C block 128, "
                          f"UF8 momentum block 256, grouped steps (al_came_step_multi) over "
                          f"{ngroups} groups of matrices on {nstreams} streams",
@@ -690,9 +761,9 @@ def _row_apollo(torch, np, wl, B, dev):
                         h(m["ma"]), 256, h(m["vc"]), h(m["vm"]), 8, 256, np.float32(0.0), hp, t)
         dt = time.perf_counter() - t0
         return rows * cols / dt, (f"one step of one {rows}x{cols} matrix incl. the rank-{r} "
-                                  f"projection in double ({dt:.1f} s, single thread)")
+                                  f"projection in double ({dt:.2f} s)")
 
-    return dict(step=step, n=n_tot, bytes=nbytes, flops=flops, launches=3,
+    return dict(step=step, n=n_tot, bytes=nbytes, flops=flops, launches=3, cpu_threads=True,
                 oracle=oracle_sample,
                 workload=f"APOLLO TinyLlama-1.1B {len(mats)} matrices (one grouped step), "
                          f"rank {r}, UF8 M^P, AL8 V^P block 256",
@@ -733,78 +804,132 @@ def _row_codec(torch, np, wl, B, dev):
         codes, meta = ora.al_encode(xh, 256, 8, floor)
         ora.al_decode(codes, meta, 256, 8)
         dt = time.perf_counter() - t0
-        return k / dt, f"AL8 encode + decode of {k} elements ({dt:.1f} s, single thread)"
+        return k / dt, f"AL8 encode + decode of {k} elements ({dt:.2f} s)"
 
-    return dict(step=step, n=n, bytes=nbytes, launches=4, oracle=oracle_sample,
+    return dict(step=step, n=n, bytes=nbytes, launches=4, oracle=oracle_sample, cpu_threads=True,
                 workload="codec 2^28 elements, AL8 encode+decode and UF8 encode+decode, block 256",
                 bytes_note="20 B/element + block constants")
 
 
-def run_rows(args):
-    """One JSON line for a non-headline hot-path row: device time of whole
-    steps (all of the row's launches) with CUDA events, bytes/time against the
-    measured HBM copy peak, the oracle on a bounded sample, SM clocks."""
+class L2Flush:
+    """Writes a buffer twice the L2's size between timed steps, so that no
+    step starts with the previous step's data in L2."""
+
+    def __init__(self, torch, dev):
+        props = torch.cuda.get_device_properties(dev)
+        l2 = int(getattr(props, "L2_cache_size", 0) or (129 << 20))
+        self.buf = torch.empty(2 * l2 // 4, dtype=torch.float32, device=dev)
+
+    def __call__(self):
+        self.buf.zero_()
+
+
+def measure_row(name, args, dev, warmup, min_steps, with_cpu, summary):
+    """Times one non-headline hot-path row: whole steps (all of the row's
+    launches) with CUDA events around each step and an L2 flush between
+    steps (outside the events), at least min_steps steps and enough to fill
+    about 0.6 s, with nvidia-smi clock samples over the timed loop; bytes
+    per step over time against the measured HBM copy peak; the oracle on a
+    bounded sample (its OpenMP build for the multi-matrix rows)."""
     import numpy as np
     import torch
 
-    from paper_2608_22322_gb300 import build_lib
-    build_lib.build()
     from paper_2608_22322_gb300 import binding as B
     from paper_2608_22322_gb300 import workloads as wl
 
-    if int(os.environ.get("RANK", "0")) != 0:
-        return  # the rows are single-GPU measurements
-    dev = torch.device("cuda", 0)
     build = {"adafactor": _row_adafactor, "came": _row_came, "apollo": _row_apollo,
-             "codec": _row_codec}[args.workload]
+             "codec": _row_codec}[name]
     w = build(torch, np, wl, B, dev)
+    flush = L2Flush(torch, dev)
+    stream = torch.cuda.current_stream(dev)
     t = 0
-    for _ in range(args.warmup):
+    for _ in range(max(3, warmup)):
         t += 1
         w["step"](t)
-    torch.cuda.synchronize(dev)
-    props = torch.cuda.get_device_properties(dev)
-    sampler = ClockSampler(str(getattr(props, "uuid", "") or "").replace("GPU-", ""))
-    sampler.start()
-    time.sleep(0.3)
-    stream = torch.cuda.current_stream(dev)
+    # calibrate the step count to fill about 0.6 s of timed steps
     ev0 = torch.cuda.Event(enable_timing=True)
     ev1 = torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize(dev)
     ev0.record(stream)
-    for _ in range(args.steps):
+    for _ in range(3):
         t += 1
         w["step"](t)
     ev1.record(stream)
     torch.cuda.synchronize(dev)
-    ms_step = ev0.elapsed_time(ev1) / args.steps
+    est = ev0.elapsed_time(ev1) / 3
+    steps = max(min_steps, args.steps if not summary else 0, int(600.0 / max(est, 1e-3)))
+    steps = min(steps, 20000)
+    props = torch.cuda.get_device_properties(dev)
+    sampler = ClockSampler(str(getattr(props, "uuid", "") or "").replace("GPU-", ""))
+    sampler.start()
+    time.sleep(0.3)
+    pairs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+             for _ in range(steps)]
+    torch.cuda.synchronize(dev)
+    for a, b in pairs:
+        flush()
+        t += 1
+        a.record(stream)
+        w["step"](t)
+        b.record(stream)
+    torch.cuda.synchronize(dev)
     clocks = sampler.stop()
+    ms_step = sum(a.elapsed_time(b) for a, b in pairs) / steps
     peaks, peak_src = measured_peaks()
     peak = float(peaks.get("hbm_gbs", 6800.0))
     achieved = w["bytes"] / (ms_step * 1e-3) / 1e9
+    unit = "params/s" if name != "codec" else "elements/s"
     cpu = None
-    if not args.no_cpu:
+    if with_cpu:
         import oracle as ora
+        threads = oracle_threads(ora, w.get("cpu_threads", False))
         v, sample = w["oracle"](ora, t + 1)
-        cpu = {"value": v, "unit": "params/s" if args.workload != "codec" else "elements/s",
-               "cores": 1, "kind": "oracle", "sample": sample}
+        oracle_threads(ora, False)
+        cpu = dict({"value": v, "unit": unit, "cores": threads, "kind": "oracle",
+                    "sample": f"{sample} on {threads} thread{'s' if threads > 1 else ''}"},
+                   **host_info())
+    roof = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+            "frac": achieved / peak, "traffic": None, "peak_source": f"{peak_src} hbm_gbs",
+            "kernel": "whole step (all launches; per-kernel shares in profiles/)"}
+    l2 = "L2 flushed (a write of twice its size) between timed steps, outside the events"
+    if summary:
+        out = {"workload": w["workload"], "value": w["n"] / (ms_step * 1e-3), "unit": unit,
+               "ms_per_step": ms_step, "steps": steps, "warmup": max(3, warmup),
+               "params_per_step": w["n"], "bytes_per_step": w["bytes"], "bytes": w["bytes_note"],
+               "roofline": roof, "clocks": clocks, "gpu_launches": w["launches"] * steps,
+               "l2": l2, "cpu_baseline": cpu}
+        if "flops" in w:
+            out["projection_tflops"] = w["flops"] / (ms_step * 1e-3) / 1e12
+            out["projection_note"] = "2 r s L flop per matrix over the whole step's time"
+        del w
+        return out
     line = {
-        "metric": ROW_METRICS[args.workload], "value": w["n"] / (ms_step * 1e-3),
-        "unit": "params/s" if args.workload != "codec" else "elements/s", "n_gpus": 1,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-        "data": "synthetic",
-        "config": {"workload": w["workload"], "params_per_gpu": w["n"], "bytes_per_step": w["bytes"],
-                   "bytes": w["bytes_note"], "parallelism": "single GPU"},
-        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": None,
-                     "peak_source": f"{peak_src} hbm_gbs",
-                     "kernel": "whole step (all launches; per-kernel shares in profiles/)"},
-        "cpu_baseline": cpu, "e2e": None, "clocks": clocks,
-        "gpu_launches": w["launches"] * args.steps,
+        "metric": ROW_METRICS[name], "value": w["n"] / (ms_step * 1e-3),
+        "unit": unit, "n_gpus": 1, "steps": steps, "warmup": max(3, warmup),
+        "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32", "data": "synthetic",
+        "config": {"workload": w["workload"], "params_per_gpu": w["n"],
+                   "bytes_per_step": w["bytes"], "bytes": w["bytes_note"], "l2": l2,
+                   "parallelism": "single GPU"},
+        "roofline": roof, "cpu_baseline": cpu, "e2e": None, "clocks": clocks,
+        "gpu_launches": w["launches"] * steps,
     }
     if "flops" in w:
         line["projection_tflops"] = w["flops"] / (ms_step * 1e-3) / 1e12
+    return line
+
+
+def run_rows(args):
+    """One JSON line for a non-headline hot-path row (--workload)."""
+    import torch
+
+    from paper_2608_22322_gb300 import build_lib
+    build_lib.build()
+    if int(os.environ.get("RANK", "0")) != 0:
+        return  # the rows are single-GPU measurements
+    dev = torch.device("cuda", 0)
+    line = measure_row(args.workload, args, dev, warmup=args.warmup, min_steps=args.steps,
+                       with_cpu=not args.no_cpu, summary=False)
     print(json.dumps(line), flush=True)
 
 
