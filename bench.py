@@ -682,18 +682,21 @@ def _row_came(torch, np, wl, B, dev):
     nbytes = nm * (14 * n1 + 8 * ((n1 + 255) // 256) + facb)
 
     def oracle_sample(ora, t):
+        """One oracle step of every matrix (the whole workload)."""
         import numpy as np_
-        m = mats[0]
         h = lambda x: x.cpu().numpy().copy()
         u16 = lambda x: x.cpu().numpy().view(np_.uint16).copy()
-        ph, gh = h(m["p"]), m["gs"][0].cpu().numpy()
-        args = [u16(m["vr"][0]), h(m["vr"][1]), u16(m["vc"][0]), h(m["vc"][1]), 16, vb,
-                u16(m["cr"][0]), h(m["cr"][1]), u16(m["cc"][0]), h(m["cc"][1]), 16, cb,
-                h(m["mc"]), h(m["ma"]), 256]
+        host = []
+        for m in mats:
+            host.append((h(m["p"]), m["gs"][0].cpu().numpy(),
+                         [u16(m["vr"][0]), h(m["vr"][1]), u16(m["vc"][0]), h(m["vc"][1]), 16, vb,
+                          u16(m["cr"][0]), h(m["cr"][1]), u16(m["cc"][0]), h(m["cc"][1]), 16, cb,
+                          h(m["mc"]), h(m["ma"]), 256]))
         t0 = time.perf_counter()
-        ora.came_step(ph, gh, rows, cols, *args, hp, t)
+        for ph, gh, args in host:
+            ora.came_step(ph, gh, rows, cols, *args, hp, t)
         dt = time.perf_counter() - t0
-        return n1 / dt, f"one step of one {rows}x{cols} matrix ({dt:.2f} s)"
+        return nm * n1 / dt, f"one step of all {nm} {rows}x{cols} matrices ({dt:.2f} s)"
 
     return dict(step=step, n=nm * n1, bytes=nbytes, launches=8 * ngroups, oracle=oracle_sample,
                 cpu_threads=True,
@@ -752,16 +755,22 @@ def _row_apollo(torch, np, wl, B, dev):
         plans[t % 2].step(hp, t)
 
     def oracle_sample(ora, t):
-        m = mats[0]
-        rows, cols = m["rows"], m["cols"]
+        """One oracle step of layer 0's seven matrices (q, k, v, o, gate, up,
+        down: 44M parameters), the projections in double."""
         h = lambda x: x.cpu().numpy().copy()
-        Ph = m["P"].cpu().numpy().view(np.uint16).copy()
+        host = []
+        for m in mats[:7]:
+            host.append((m["rows"], m["cols"], h(m["p"]), m["gs"][0].cpu().numpy(),
+                         m["P"].cpu().numpy().view(np.uint16).copy(), h(m["mc"]), h(m["ma"]),
+                         h(m["vc"]), h(m["vm"])))
         t0 = time.perf_counter()
-        ora.apollo_step(h(m["p"]), m["gs"][0].cpu().numpy(), rows, cols, Ph, h(m["mc"]),
-                        h(m["ma"]), 256, h(m["vc"]), h(m["vm"]), 8, 256, np.float32(0.0), hp, t)
+        for rows, cols, ph, gh, Ph, mch, mah, vch, vmh in host:
+            ora.apollo_step(ph, gh, rows, cols, Ph, mch, mah, 256, vch, vmh, 8, 256,
+                            np.float32(0.0), hp, t)
         dt = time.perf_counter() - t0
-        return rows * cols / dt, (f"one step of one {rows}x{cols} matrix incl. the rank-{r} "
-                                  f"projection in double ({dt:.2f} s)")
+        n = sum(x[0] * x[1] for x in host)
+        return n / dt, (f"one step of layer 0's 7 matrices ({n} params) incl. the rank-{r} "
+                        f"projections in double ({dt:.2f} s)")
 
     return dict(step=step, n=n_tot, bytes=nbytes, flops=flops, launches=3, cpu_threads=True,
                 oracle=oracle_sample,
@@ -798,7 +807,7 @@ def _row_codec(torch, np, wl, B, dev):
     nbytes = 20 * n + 2 * (8 * (n // 256)) + 2 * (4 * (n // 256))
 
     def oracle_sample(ora, t):
-        k = 1 << 24
+        k = n
         xh = x[:k].cpu().numpy()
         t0 = time.perf_counter()
         codes, meta = ora.al_encode(xh, 256, 8, floor)
