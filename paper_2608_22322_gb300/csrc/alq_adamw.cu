@@ -18,6 +18,9 @@
 // many tensors (descriptor table in device memory, tiles never crossing a
 // tensor boundary). The grid is persistent: each CTA walks tiles with a
 // stride of gridDim.x and a forward-only cursor into the descriptor table.
+// The exp2/log2 tables of the codec's two-float levels and block bounds are
+// read from shared memory in this translation unit (copied once per CTA).
+#define ALQ_SMEM_TABLES 1
 #include "alq_kernels.cuh"
 
 namespace alq {
@@ -128,12 +131,26 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
     __shared__ __align__(16) float2 s_tab[kThreads / 32][NBV == 1 ? 2 : 1][NBV * 32];
     __shared__ float s_val[kThreads / 32][VBITS == 8 ? NBV * 256 : 1];
     __shared__ uint32_t s_part[2][3][kThreads / 32];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // the warp index through a shuffle from lane 0: the compiler then knows it
+    // is the same for the whole warp, and every branch on the segment's
+    // position is a uniform one
+    const int warp = __shfl_sync(0xFFFFFFFFu, (int)(threadIdx.x >> 5), 0), lane = threadIdx.x & 31;
     const int wpbv = v_block > kASeg ? v_block / kASeg : 1;
     const int wpbm = m_block > kASeg ? m_block / kASeg : 1;
     const float kf = al8_table_k(lane);
     const Opaque2 ok2{s.one, s.zero};
     const int G = gridDim.x;
+    // the 2^(j/1024) and log2 reduction tables of the level and bound
+    // computations, 20 KB, into shared memory (their lookups sit on the
+    // level pass's dependent chain)
+    for (int i = threadIdx.x; i < 1024; i += kThreads) {
+        s_kExp2Hi[i] = kExp2HiD[i];
+        s_kExp2Lo[i] = kExp2LoD[i];
+        s_kLog2C[i] = kLog2CD[i];
+        s_kLog2Hi[i] = kLog2HiD[i];
+        s_kLog2Lo[i] = kLog2LoD[i];
+    }
+    __syncthreads();
     int cur = 0;
     int parity = 0;  // slot of the next cross-warp block reduction
     int tslot = 0;   // level-table slot of this iteration
@@ -238,11 +255,14 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
                         l1 = mt.x;
                         d1 = mt.y;
                     }
-                    al8_build_tables2(s_tab[warp][tslot], s_tab[warp + 1][tslot], olmin[0],
-                                      odelta[0], l1, d1, kf, ok2);
+                    al8_build_tables2_soa(reinterpret_cast<float*>(s_tab[warp][tslot]),
+                                          reinterpret_cast<float*>(s_tab[warp + 1][tslot]),
+                                          olmin[0], odelta[0], l1, d1, kf, ok2);
                 }
                 asm volatile("bar.sync %0, 64;" ::"r"(1 + (warp >> 1)) : "memory");
-                al8_values_from_tables<1>(s_val[warp], s_tab[warp][tslot], olmin, odelta);
+                al8_values_from_tables_soa(s_val[warp],
+                                           reinterpret_cast<const float*>(s_tab[warp][tslot]),
+                                           olmin[0], odelta[0]);
                 tslot ^= 1;
             } else {
                 // two blocks per segment: their levels in one paired pass

@@ -193,7 +193,10 @@ __device__ __forceinline__ uint32_t cta_group_reduce(uint32_t v, uint32_t* s_par
 // ------------------------------------------------------- AL block constants --
 // (l_min, Delta) of the NB blocks of a segment from their minimum positive
 // value mn and maximum mx (Eq. (3)). The 2 NB fp32-rounded logs are spread
-// over the lanes (one log per lane) and exchanged by shuffles.
+// over the lanes (one log per lane) and exchanged by shuffles; each is
+// first taken from the hardware log2 with its rounding certified
+// (log2_rn_fast), and the lanes it cannot certify (about one in ten) take
+// the two-float log2_rn under one warp-uniform branch.
 template <int NB>
 __device__ __forceinline__ void al_blocks_params(const float (&mn)[NB], const float (&mx)[NB],
                                                  float log_floor, float (&lmin)[NB],
@@ -206,7 +209,11 @@ __device__ __forceinline__ void al_blocks_params(const float (&mn)[NB], const fl
         if (v == 2 * b) x = mn[b];
         if (v == 2 * b + 1) x = mx[b];
     }
-    const float L = (x > 0.0f) ? log2_rn(x) : 0.0f;
+    bool ok;
+    float L = log2_rn_fast(x > 0.0f ? x : 1.0f, ok);
+    ok = ok || !(x > 0.0f);
+    L = (x > 0.0f) ? L : 0.0f;
+    if (__builtin_expect(__any_sync(0xFFFFFFFFu, !ok), 0)) L = log2_rn_fixup(x, L, ok);
 #pragma unroll
     for (int b = 0; b < NB; ++b) {
         const float l0 = __shfl_sync(0xFFFFFFFFu, L, 2 * b);
@@ -368,6 +375,66 @@ __device__ __forceinline__ float2 al8_decode_pair2(float2 ah, float2 al, float2 
     fb0 = z.x != r.x;
     fb1 = z.y != r.y;
     return r;
+}
+
+
+// ------------------------------------------ AL8 level tables, SoA layout --
+// The same two 16-entry level tables as al8_build_tables2 / al8_values_from_
+// tables, stored as 64 floats: the high parts at [slot], the low parts at
+// [32 + slot] (slots as in al8_hi_slot), so that the paired products read
+// the high parts of two entries, and their low parts, as adjacent pairs.
+__device__ __forceinline__ void al8_build_tables2_soa(float* tab0, float* tab1, float lmin0,
+                                                      float delta0, float lmin1, float delta1,
+                                                      float kf, const Opaque2& k) {
+    const int lane = threadIdx.x & 31;
+    const bool hi = lane >= 16;
+    const int slot = hi ? al8_hi_slot((uint32_t)(lane - 16)) : lane;
+    const bool f0 = al8_fast_ok(lmin0, delta0), f1 = al8_fast_ok(lmin1, delta1);
+    const float2 lm = make_float2(hi && f0 ? lmin0 : 0.0f, hi && f1 ? lmin1 : 0.0f);
+    const float2 dl = make_float2(f0 ? delta0 : 1.0f, f1 ? delta1 : 1.0f);
+    float2 rh, rl;
+    al_level_ff2(lm, dl, kf, 254.0f, 1.0f / 254.0f, k, rh, rl);
+    tab0[slot] = f0 ? rh.x : 0.0f;
+    tab0[32 + slot] = f0 ? rl.x : 0.0f;
+    tab1[slot] = f1 ? rh.y : 0.0f;
+    tab1[32 + slot] = f1 ? rl.y : 0.0f;
+    __syncwarp();
+}
+
+static __device__ __noinline__ void al8_values_fixup_soa(float* vals, const float* tab, float lmin,
+                                                         float delta) {
+    const int lane = threadIdx.x & 31;
+    const bool fast = al8_fast_ok(lmin, delta);
+    for (int k = 0; k < 8; ++k) {
+        const uint32_t q = (uint32_t)(lane + 32 * k);
+        const int sa = al8_hi_slot(q >> 4), sb = (int)(q & 15u);
+        bool fb;
+        al8_decode_pair(tab[sa], tab[32 + sa], tab[sb], tab[32 + sb], fb);
+        if ((q != 0u) && (fb || !fast)) vals[q] = al_dequantize_fp64(q, lmin, delta, 254.0);
+    }
+}
+
+__device__ __forceinline__ void al8_values_from_tables_soa(float* vals, const float* tab,
+                                                           float lmin, float delta) {
+    const int lane = threadIdx.x & 31;
+    const bool fast = al8_fast_ok(lmin, delta);
+    const float bv = tab[lane & 15], blv = tab[32 + (lane & 15)];
+    const float2 bh = make_float2(bv, bv), bl = make_float2(blv, blv);
+    const float2 nbh = make_float2(-bv, -bv);
+    const float2* Ah = reinterpret_cast<const float2*>(tab + 16 + 8 * (lane >> 4));
+    const float2* Al = reinterpret_cast<const float2*>(tab + 48 + 8 * (lane >> 4));
+    bool any_fb = !fast;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        bool f0, f1;
+        const float2 r = al8_decode_pair2(Ah[j], Al[j], bh, bl, nbh, f0, f1);
+        const uint32_t q0 = (uint32_t)(lane + 64 * j);
+        vals[q0] = q0 == 0u ? 0.0f : r.x;
+        vals[q0 + 32] = r.y;
+        any_fb |= ((q0 != 0u) & f0) | f1;
+    }
+    if (__builtin_expect(__any_sync(0xFFFFFFFFu, any_fb), 0)) al8_values_fixup_soa(vals, tab, lmin, delta);
+    __syncwarp();
 }
 
 // Fixed-size arrays passed by value to the out-of-line rare paths (so that

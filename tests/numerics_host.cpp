@@ -9,6 +9,14 @@ extern "C" {
 
 float alqn_log2_rn(float x) { return log2_rn(x); }
 
+// The certified fast path alone: ok = 1 when it vouches for its result.
+float alqn_log2_rn_fast(float x, int* ok) {
+    bool o;
+    const float r = log2_rn_fast(x, o);
+    *ok = o ? 1 : 0;
+    return r;
+}
+
 void alqn_block_params(float mn, float mx, float floor_, float* lmin, float* delta) {
     al_block_params(mn, mx, floor_, *lmin, *delta);
 }

@@ -39,6 +39,8 @@ def lib():
     f32p = np.ctypeslib.ndpointer(np.float32, flags="C_CONTIGUOUS")
     L.alqn_log2_rn.restype = C.c_float
     L.alqn_log2_rn.argtypes = [C.c_float]
+    L.alqn_log2_rn_fast.restype = C.c_float
+    L.alqn_log2_rn_fast.argtypes = [C.c_float, C.POINTER(C.c_int)]
     L.alqn_block_params.argtypes = [C.c_float, C.c_float, C.c_float,
                                     C.POINTER(C.c_float), C.POINTER(C.c_float)]
     L.alqn_level.argtypes = [C.c_float, C.c_float, C.c_int, C.c_float,
@@ -61,6 +63,35 @@ def test_log2_rn_matches_double_rounding(lib):
     ])
     for x in xs:
         assert lib.alqn_log2_rn(float(x)) == np.float32(math.log2(float(x))), x
+
+
+def test_log2_rn_fast_certifies_only_correct_roundings(lib):
+    """The hardware-log2 fast path of the block bounds: whenever it certifies
+    its result, the result is (float)log2((double)x); it certifies most
+    values of the second-moment range (|log2 x| in [16, 64)) and declines
+    near 1, for subnormals and for ties it cannot separate."""
+    r = wl.rng(2)
+    xs = np.concatenate([
+        np.exp2(r.uniform(-126, 127, 200000)).astype(np.float32),
+        np.exp2(r.uniform(-64, -16, 100000)).astype(np.float32),
+        (1 + r.uniform(-1e-3, 1e-3, 20000)).astype(np.float32),
+        np.float32(2.0) ** np.arange(-126, 127, dtype=np.float32),
+        np.array([1e-42, 3e-39, 1.0], np.float32),
+    ])
+    ok = C.c_int(0)
+    certified = in_range = cert_in_range = 0
+    for x in xs:
+        got = lib.alqn_log2_rn_fast(float(x), C.byref(ok))
+        want = np.float32(math.log2(float(x)))
+        if ok.value:
+            certified += 1
+            assert got == want, x
+        if 16.0 <= abs(float(want)) < 64.0:
+            in_range += 1
+            cert_in_range += ok.value
+        if x < np.float32(2.0) ** -126 or abs(float(x) - 1.0) < 1e-3:
+            assert not ok.value, x
+    assert cert_in_range > 0.8 * in_range, (cert_in_range, in_range)
 
 
 def test_block_params_match_oracle(lib):
