@@ -386,9 +386,19 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
 #pragma unroll
         for (int b = 0; b < NBM; ++b) {
             ms[b] = u2f(bmabs[b]);
-            msc[b] = 1.0f;
-            minv[b] = 0.0f;
-            if (ms[b] > 0.0f) uf8_encode_consts(ms[b], msc[b], minv[b]);
+            uf8_encode_consts(ms[b] > 0.0f ? ms[b] : 1.0f, msc[b], minv[b]);
+            minv[b] = ms[b] > 0.0f ? minv[b] : 0.0f;  // an all-zero block codes as 0
+        }
+        // (m sc) inv: sc is 1 except in blocks whose absmax is below 2^-120,
+        // where the fresh m values are scaled (exactly) first
+#pragma unroll
+        for (int c = 0; c < kCH; ++c) {
+            const int bm = c / CPBM;
+            if (__builtin_expect(msc[bm] != 1.0f, 0)) {
+                const float2 sc2 = make_float2(msc[bm], msc[bm]);
+                mf[2 * c] = mul2(mf[2 * c], sc2);
+                mf[2 * c + 1] = mul2(mf[2 * c + 1], sc2);
+            }
         }
 
         // ---- encode and write the codes and block constants
@@ -402,11 +412,11 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
             // two's complement byte for q < 0; all codes are 0 when the
             // block's absmax is 0 (inv = 0). The rounding add is a fused
             // multiply-add by the opaque one, so the product rounds first.
-            const float2 sc2 = make_float2(msc[bm], msc[bm]), inv2 = make_float2(minv[bm], minv[bm]);
+            const float2 inv2 = make_float2(minv[bm], minv[bm]);
             uint32_t rb[4];
 #pragma unroll
             for (int i = 0; i < 2; ++i) {
-                const float2 f = mul2(mul2(mf[2 * c + i], sc2), inv2);
+                const float2 f = mul2(mf[2 * c + i], inv2);
                 const float2 r = fma2(f, s.one, make_float2(12582912.0f, 12582912.0f));
                 rb[2 * i] = f2u(r.x);
                 rb[2 * i + 1] = f2u(r.y);

@@ -485,8 +485,17 @@ __device__ __forceinline__ void al_encode_chunks(const float (&x)[4 * CH], const
     bool any_fb = false;
 #pragma unroll
     for (int b = 0; b < NB; ++b) any_fb |= (mn[b] > 0.0f) & (mn[b] < 0x1p-126f);
-    const float2 rc = make_float2(12582912.0f, 12582912.0f);  // 1.5 * 2^23
+    // POS: q = rint(Lm2 t1) + 1 comes out of the rounding constant
+    // 1.5 * 2^23 + 1 (exact ties, where that constant could round the other
+    // way, always take the fixup), and min(q, bits of x) makes a zero 0
+    // (every positive x the fast path codes is normal: bits >= 2^23 > q)
+    const float cr = POS ? 12582913.0f : 12582912.0f;
+    const uint32_t cb = POS ? 0x4B400000u : 0x4B400000u;
+    const float2 rc = make_float2(cr, cr);
     const float2 l2 = make_float2(Lm2, Lm2);
+    float dmax[NB];  // the largest |t - rint(t)| distance to the tie of each block
+#pragma unroll
+    for (int b = 0; b < NB; ++b) dmax[b] = 0.0f;
 #pragma unroll
     for (int e = 0; e < 4 * CH; e += 2) {
         const int b = e / 4 / CPB;
@@ -502,13 +511,19 @@ __device__ __forceinline__ void al_encode_chunks(const float (&x)[4 * CH], const
         const float2 s1 = sub2(eb, make_float2(k[b].e0p, k[b].e0p));  // e - I, exact
         const float2 u = fma2(lg, iD, make_float2(k[b].nFiD, k[b].nFiD));
         const float2 t1 = make_float2(fma_sat(s1.x, iD.x, u.x), fma_sat(s1.y, iD.y, u.y));
-        const float2 rr = fma2(t1, l2, rc);  // rint(Lm2 t1) + 1.5 * 2^23
+        const float2 rr = fma2(t1, l2, rc);  // rint(Lm2 t1) + the rounding constant
         const float2 df = fma2(t1, l2, sub2(rc, rr));
-        const float h = 0.5f - k[b].E;
-        any_fb |= (fabsf(df.x) > h) | (fabsf(df.y) > h);
-        q[e] = (f2u(rr.x) - 0x4B400000u) + (POS ? min(x0, 1u) : min(x0 << 1, 1u));
-        q[e + 1] = (f2u(rr.y) - 0x4B400000u) + (POS ? min(x1, 1u) : min(x1 << 1, 1u));
+        dmax[b] = fmaxf(dmax[b], fmaxf(fabsf(df.x), fabsf(df.y)));
+        if (POS) {
+            q[e] = min(f2u(rr.x) - cb, x0);
+            q[e + 1] = min(f2u(rr.y) - cb, x1);
+        } else {
+            q[e] = (f2u(rr.x) - cb) + min(x0 << 1, 1u);
+            q[e + 1] = (f2u(rr.y) - cb) + min(x1 << 1, 1u);
+        }
     }
+#pragma unroll
+    for (int b = 0; b < NB; ++b) any_fb |= dmax[b] > 0.5f - k[b].E;
     if (__builtin_expect(__any_sync(0xFFFFFFFFu, any_fb), 0)) {
         Arr<float, 4 * CH> xa;
         Arr<uint32_t, 4 * CH> qa;
