@@ -866,8 +866,10 @@ def measure_row(name, args, dev, warmup, min_steps, with_cpu, summary):
     ev1.record(stream)
     torch.cuda.synchronize(dev)
     est = ev0.elapsed_time(ev1) / 3
-    steps = max(min_steps, args.steps if not summary else 0, int(600.0 / max(est, 1e-3)))
-    steps = min(steps, 20000)
+    # the default run's rows fill about 0.6 s of timed steps (enough clock
+    # samples); a row timed alone (--workload) runs exactly --steps steps
+    steps = (min(20000, max(min_steps, int(600.0 / max(est, 1e-3)))) if summary
+             else max(1, args.steps))
     props = torch.cuda.get_device_properties(dev)
     sampler = ClockSampler(str(getattr(props, "uuid", "") or "").replace("GPU-", ""))
     sampler.start()
