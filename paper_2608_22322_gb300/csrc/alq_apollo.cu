@@ -27,6 +27,8 @@
 #include <mutex>
 
 #include "alq_async.cuh"
+// the level and bound passes' exp2/log2 tables from per-CTA shared copies
+#define ALQ_SMEM_TABLES 1
 #include "alq_kernels.cuh"
 
 namespace alq {
@@ -448,7 +450,7 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
     constexpr int NB = kMCH / CPB;
     constexpr int NE = 4 * kMCH;
     constexpr float Lm2 = VBITS == 8 ? 254.0f : 65534.0f;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int warp = __shfl_sync(0xFFFFFFFFu, (int)(threadIdx.x >> 5), 0), lane = threadIdx.x & 31;
     const float kf = al8_table_k(lane);
     const int64_t nblk = blocks_of_dev(m.n, m.block);
     const int bshift = __ffs(m.block) - 1;
@@ -485,7 +487,16 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
     // previous V: AL8 through the blocks' tables of exactly rounded values
     float vh[NE];
     if constexpr (VBITS == 8) {
-        al8_build_values<NB>(vals, tab, olmin, odelta, kf);
+        float* ts = reinterpret_cast<float*>(tab);  // 64 floats per block (SoA)
+        if constexpr (NB == 2) {
+            const Opaque2 ok2{make_float2(m.one, m.one), make_float2(m.zero, m.zero)};
+            al8_build_tables2_soa(ts, ts + 64, olmin[0], odelta[0], olmin[1], odelta[1], kf, ok2);
+        } else {
+            al8_build_tables_soa(ts, olmin[0], odelta[0], kf);
+        }
+#pragma unroll
+        for (int b = 0; b < NB; ++b)
+            al8_values_from_tables_soa(vals + 256 * b, ts + 64 * b, olmin[b], odelta[b]);
 #pragma unroll
         for (int e = 0; e < NE; ++e)
             vh[e] = vals[256 * (e / 4 / CPB) + ((vw[e / 4] >> (8 * (e % 4))) & 0xFFu)];
@@ -578,9 +589,18 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
         vmn[b] = u2f(bvmin[b] + 1u);
         vmx[b] = u2f(bvmax[b]);
         ms[b] = u2f(bmabs[b]);
-        sc[b] = 1.0f;
-        inv[b] = 0.0f;
-        if (ms[b] > 0.0f) uf8_encode_consts(ms[b], sc[b], inv[b]);
+        uf8_encode_consts(ms[b] > 0.0f ? ms[b] : 1.0f, sc[b], inv[b]);
+        inv[b] = ms[b] > 0.0f ? inv[b] : 0.0f;  // an all-zero block codes as 0
+    }
+    // (m sc) inv: sc is 1 except in blocks whose absmax is below 2^-120
+#pragma unroll
+    for (int c = 0; c < kMCH; ++c) {
+        const int b = c / CPB;
+        if (__builtin_expect(sc[b] != 1.0f, 0)) {
+            const float2 s2 = make_float2(sc[b], sc[b]);
+            mf2[2 * c] = mul2(mf2[2 * c], s2);
+            mf2[2 * c + 1] = mul2(mf2[2 * c + 1], s2);
+        }
     }
     al_blocks_params<NB>(vmn, vmx, m.log_floor, nlmin, ndelta);
 #pragma unroll
@@ -593,11 +613,11 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
         const int64_t idx = chunk_index(seg0, c, lane);
         // q = rint((m sc) inv) as the low byte of 1.5 * 2^23 + q (two's
         // complement for q < 0); the rounding add by the opaque one
-        const float2 sc2 = make_float2(sc[b], sc[b]), inv2 = make_float2(inv[b], inv[b]);
+        const float2 inv2 = make_float2(inv[b], inv[b]);
         uint32_t rb[4];
 #pragma unroll
         for (int i = 0; i < 2; ++i) {
-            const float2 f = mul2(mul2(mf2[2 * c + i], sc2), inv2);
+            const float2 f = mul2(mf2[2 * c + i], inv2);
             const float2 rr = fma2(f, one, make_float2(12582912.0f, 12582912.0f));
             rb[2 * i] = f2u(rr.x);
             rb[2 * i + 1] = f2u(rr.y);
@@ -633,6 +653,14 @@ apollo_moments_kernel(MomentArgs m, int64_t ntiles) {
     __shared__ __align__(16) float2 s_tab[kThreads / 32][NB * 32];
     __shared__ float s_val[kThreads / 32][VBITS == 8 ? NB * 256 : 1];
     const int warp = threadIdx.x >> 5;
+    for (int i = threadIdx.x; i < 1024; i += kThreads) {
+        s_kExp2Hi[i] = kExp2HiD[i];
+        s_kExp2Lo[i] = kExp2LoD[i];
+        s_kLog2C[i] = kLog2CD[i];
+        s_kLog2Hi[i] = kLog2HiD[i];
+        s_kLog2Lo[i] = kLog2LoD[i];
+    }
+    __syncthreads();
     PendingScales ps;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x)
         moments_tile<CPB, VBITS>(m, tile, s_tab[warp], s_val[warp], ps);
@@ -834,6 +862,14 @@ apollo_moments_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t n
     __shared__ __align__(16) float2 s_tab[kThreads / 32][NB * 32];
     __shared__ float s_val[kThreads / 32][VBITS == 8 ? NB * 256 : 1];
     const int warp = threadIdx.x >> 5;
+    for (int i = threadIdx.x; i < 1024; i += kThreads) {
+        s_kExp2Hi[i] = kExp2HiD[i];
+        s_kExp2Lo[i] = kExp2LoD[i];
+        s_kLog2C[i] = kLog2CD[i];
+        s_kLog2Hi[i] = kLog2HiD[i];
+        s_kLog2Lo[i] = kLog2LoD[i];
+    }
+    __syncthreads();
     PendingScales ps;
     int cur = 0;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {

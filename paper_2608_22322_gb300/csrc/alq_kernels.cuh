@@ -401,6 +401,20 @@ __device__ __forceinline__ void al8_build_tables2_soa(float* tab0, float* tab1, 
     __syncwarp();
 }
 
+// One block's level tables in the SoA layout, one level per lane (scalar).
+__device__ __forceinline__ void al8_build_tables_soa(float* tab, float lmin, float delta,
+                                                     float kf) {
+    const int lane = threadIdx.x & 31;
+    const bool hi = lane >= 16;
+    const int slot = hi ? al8_hi_slot((uint32_t)(lane - 16)) : lane;
+    float rh = 0.0f, rl = 0.0f;
+    if (al8_fast_ok(lmin, delta))
+        al_level_ff(hi ? lmin : 0.0f, delta, kf, 254.0f, 1.0f / 254.0f, rh, rl);
+    tab[slot] = rh;
+    tab[32 + slot] = rl;
+    __syncwarp();
+}
+
 static __device__ __noinline__ void al8_values_fixup_soa(float* vals, const float* tab, float lmin,
                                                          float delta) {
     const int lane = threadIdx.x & 31;
