@@ -3,6 +3,8 @@
 // reduces each block's minimum positive value and maximum with warp
 // reductions, derives (l_min, Delta) once per block and writes codes and
 // metadata; the decoder rebuilds each block's level tables and writes fp32.
+// the level and bound passes' exp2/log2 tables from per-CTA shared copies
+#define ALQ_SMEM_TABLES 1
 #include "alq_kernels.cuh"
 
 namespace alq {
@@ -23,10 +25,18 @@ al_encode_kernel(const float* __restrict__ x, int64_t n, int block, float log_fl
     constexpr int NB = 4 / CPB;
     constexpr float Lm2 = BITS == 8 ? 254.0f : 65534.0f;
     __shared__ uint32_t s_part[2][kThreads / 32];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int warp = __shfl_sync(0xFFFFFFFFu, (int)(threadIdx.x >> 5), 0), lane = threadIdx.x & 31;
     const int wpb = block > kSeg ? block / kSeg : 1;
     const int64_t nblk = blocks_of_dev(n, block);
     const int bshift = __ffs(block) - 1;
+    for (int i = threadIdx.x; i < 1024; i += kThreads) {
+        s_kExp2Hi[i] = kExp2HiD[i];
+        s_kExp2Lo[i] = kExp2LoD[i];
+        s_kLog2C[i] = kLog2CD[i];
+        s_kLog2Hi[i] = kLog2HiD[i];
+        s_kLog2Lo[i] = kLog2LoD[i];
+    }
+    __syncthreads();
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
         float4 v[4];
@@ -93,10 +103,18 @@ al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta,
     constexpr int NB = 4 / CPB;
     __shared__ __align__(16) float2 s_tab[kThreads / 32][NB * 32];
     __shared__ float s_val[kThreads / 32][BITS == 8 ? NB * 256 : 1];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int warp = __shfl_sync(0xFFFFFFFFu, (int)(threadIdx.x >> 5), 0), lane = threadIdx.x & 31;
     const float kf = al8_table_k(lane);
     const int64_t nblk = blocks_of_dev(n, block);
     const int bshift = __ffs(block) - 1;
+    for (int i = threadIdx.x; i < 1024; i += kThreads) {
+        s_kExp2Hi[i] = kExp2HiD[i];
+        s_kExp2Lo[i] = kExp2LoD[i];
+        s_kLog2C[i] = kLog2CD[i];
+        s_kLog2Hi[i] = kLog2HiD[i];
+        s_kLog2Lo[i] = kLog2LoD[i];
+    }
+    __syncthreads();
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
         uint32_t w[4 * BITS / 8];
@@ -123,10 +141,18 @@ al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta,
         // AL8: the blocks' 256 exactly rounded values in shared memory, then
         // one lookup per element; AL16: each level directly
         if constexpr (BITS == 8) {
-            if constexpr (NB >= 2)
-                al8_build_values_paired<NB>(s_val[warp], s_tab[warp], lmin, delta, kf, k);
-            else
-                al8_build_values<NB>(s_val[warp], s_tab[warp], lmin, delta, kf);
+            float* ts = reinterpret_cast<float*>(s_tab[warp]);  // 64 floats per block (SoA)
+            if constexpr (NB >= 2) {
+#pragma unroll
+                for (int b = 0; b < NB; b += 2)
+                    al8_build_tables2_soa(ts + 64 * b, ts + 64 * (b + 1), lmin[b], delta[b],
+                                          lmin[b + 1], delta[b + 1], kf, k);
+            } else {
+                al8_build_tables_soa(ts, lmin[0], delta[0], kf);
+            }
+#pragma unroll
+            for (int b = 0; b < NB; ++b)
+                al8_values_from_tables_soa(s_val[warp] + 256 * b, ts + 64 * b, lmin[b], delta[b]);
         }
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
