@@ -525,7 +525,7 @@ __device__ __forceinline__ double usq_chunk_sum(const UsqArgs& q, int64_t chunk,
             for (int c = 0; c < 4; ++c) {
                 const int64_t idx = chunk_index(seg0, c, lane);
                 gv[kk][c] = make_float4(0.f, 0.f, 0.f, 0.f);
-                if (idx < q.n) gv[kk][c] = __ldcs(reinterpret_cast<const float4*>(q.g + idx));
+                if (idx < q.n) gv[kk][c] = __ldcg(reinterpret_cast<const float4*>(q.g + idx));
             }
         }
 #pragma unroll
