@@ -623,8 +623,9 @@ def _row_came(torch, np, wl, B, dev):
     gradients 1e-3 * Student-t(3) with 5% exact zeros. Algorithmic bytes: G
     read once (4), p read and written (8), momentum codes read and written
     (2), absmax and the four factor states; the library's passes read G four
-    times and the momentum codes twice, which is not counted. One grouped step
-    over the 22 matrices (al_came_step_multi: eight launches)."""
+    times and the momentum codes twice (from L2 where a matrix's gradient
+    stays there between its passes), which is not counted. Per-matrix steps
+    on three streams by default (see below)."""
     cfg = wl.CONFIGS["came"]
     rows, cols = cfg["shape"]
     nm = cfg["n_mats"]
@@ -653,27 +654,40 @@ def _row_came(torch, np, wl, B, dev):
         mats.append(dict(p=p, gs=gs, vr=fac(rows, vb), vc=fac(cols, vb), cr=fac(rows, cb),
                          cc=fac(cols, cb), mc=torch.zeros(n1, dtype=torch.int8, device=dev),
                          ma=torch.zeros((n1 + 255) // 256, dtype=torch.float32, device=dev)))
-    # grouped steps (one launch per pass over a group of matrices), the
-    # groups on their own streams so that one group's latency-bound passes
-    # overlap another's streaming ones; one plan per group and gradient
-    # buffer (a plan binds its gradients)
+    # per-matrix steps (al_came_step: eight passes chained by programmatic
+    # dependent launch) on three streams, so that three matrices' gradients
+    # (138 MB) share the L2 while their passes run (1.51 ms against 1.61 ms
+    # for grouped steps over 4 groups on 4 streams, on one box);
+    # ALQ_BENCH_CAME_SINGLE=0 times grouped steps instead (one launch per
+    # pass over a group of matrices, ALQ_BENCH_GROUPS groups on
+    # ALQ_BENCH_STREAMS streams; one plan per group and gradient buffer)
+    single = os.environ.get("ALQ_BENCH_CAME_SINGLE", "1") == "1"
     ngroups = int(os.environ.get("ALQ_BENCH_GROUPS", "4"))
     groups = [mats[i::ngroups] for i in range(ngroups)]
-    plans = [[B.FactoredPlan(B.AL_OP_CAME, [
+    plans = [] if single else [[B.FactoredPlan(B.AL_OP_CAME, [
         dict(p=m["p"], g=m["gs"][k], rows=rows, cols=cols, vr_codes=m["vr"][0],
              vr_meta=m["vr"][1], vc_codes=m["vc"][0], vc_meta=m["vc"][1], cr_codes=m["cr"][0],
              cr_meta=m["cr"][1], cc_codes=m["cc"][0], cc_meta=m["cc"][1], m_codes=m["mc"],
              m_absmax=m["ma"]) for m in grp], 16, vb, 16, cb, 256) for grp in groups]
         for k in range(2)]
-    nstreams = int(os.environ.get("ALQ_BENCH_STREAMS", str(ngroups)))
+    nstreams = int(os.environ.get("ALQ_BENCH_STREAMS", "3" if single else str(ngroups)))
     streams = [torch.cuda.Stream(device=dev) for _ in range(nstreams)]
+    wss = ([torch.empty(B.al_workspace_size(B.AL_OP_CAME, rows, cols), dtype=torch.uint8,
+                        device=dev) for _ in range(nm)] if single else None)
 
     def step(t):
         main = torch.cuda.current_stream(dev)
         for st in streams:
             st.wait_stream(main)
-        for i, plan in enumerate(plans[t % 2]):
-            plan.step(hp, t, stream=streams[i % nstreams])
+        if single:
+            for i, m in enumerate(mats):
+                B.al_came_step(m["p"], m["gs"][t % 2], rows, cols, m["vr"][0], m["vr"][1],
+                               m["vc"][0], m["vc"][1], 16, vb, m["cr"][0], m["cr"][1],
+                               m["cc"][0], m["cc"][1], 16, cb, m["mc"], m["ma"], 256, hp, t,
+                               wss[i], stream=streams[i % nstreams])
+        else:
+            for i, plan in enumerate(plans[t % 2]):
+                plan.step(hp, t, stream=streams[i % nstreams])
         for st in streams:
             main.wait_stream(st)
 
@@ -698,11 +712,13 @@ def _row_came(torch, np, wl, B, dev):
         dt = time.perf_counter() - t0
         return nm * n1 / dt, f"one step of all {nm} {rows}x{cols} matrices ({dt:.2f} s)"
 
-    return dict(step=step, n=nm * n1, bytes=nbytes, launches=8 * ngroups, oracle=oracle_sample,
-                cpu_threads=True,
+    sched = (f"per-matrix steps (al_came_step) on {nstreams} streams" if single else
+             f"grouped steps (al_came_step_multi) over {ngroups} groups of matrices on "
+             f"{nstreams} streams")
+    return dict(step=step, n=nm * n1, bytes=nbytes, launches=8 * (nm if single else ngroups),
+                oracle=oracle_sample, cpu_threads=True,
                 workload=f"CAME {nm} x {rows}x{cols}, AL16 factored V and C block 128, "
-                         f"UF8 momentum block 256, grouped steps (al_came_step_multi) over "
-                         f"{ngroups} groups of matrices on {nstreams} streams",
+                         f"UF8 momentum block 256, {sched}",
                 bytes_note="algorithmic minimum 14.03 B/param (G read once)")
 
 
