@@ -46,6 +46,7 @@ KERNEL_SOURCES = ["paper_2608_22322_gb300/csrc/alq_adamw.cu",
                   "paper_2608_22322_gb300/csrc/alq_numerics.h"]
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "adamw_fused_tinyllama.md")
 HP = None  # filled in main (needs numpy)
+MATS = 0  # --mats: CAME and APOLLO rows on their first K matrices
 
 
 def parse_args():
@@ -62,6 +63,8 @@ def parse_args():
     ap.add_argument("--v-block", type=int, default=256,
                     help="AdamW second-moment block size (256 is the benchmark's "
                          "configuration; 2048 is the paper's core AdamW setting)")
+    ap.add_argument("--mats", type=int, default=0,
+                    help="CAME and APOLLO rows: only the first K matrices (profiling runs)")
     ap.add_argument("--no-rows", action="store_true",
                     help="skip the other hot-path rows after the headline step")
     ap.add_argument("--workload", default="adamw",
@@ -628,7 +631,7 @@ def _row_came(torch, np, wl, B, dev):
     on three streams by default (see below)."""
     cfg = wl.CONFIGS["came"]
     rows, cols = cfg["shape"]
-    nm = cfg["n_mats"]
+    nm = min(cfg["n_mats"], MATS) if MATS else cfg["n_mats"]
     n1 = rows * cols
     hp = dict(lr=cfg["lr"], beta1=cfg["beta1"], beta2=cfg["beta2"], beta3=cfg["beta3"],
               eps1=cfg["eps1"], eps2=cfg["eps2"], clip_d=cfg["clip_d"],
@@ -737,7 +740,10 @@ def _row_apollo(torch, np, wl, B, dev):
               alpha=cfg["alpha"], weight_decay=cfg["weight_decay"], norm_growth_gamma=0.0,
               log_floor=float(np.float32(np.log2(1e-16))), rank=r)
     mats, nbytes, flops, n_tot = [], 0, 0, 0
-    for i, (_, (rows, cols)) in enumerate(wl.tinyllama_matrices()):
+    shapes = wl.tinyllama_matrices()
+    if MATS:
+        shapes = shapes[:MATS]
+    for i, (_, (rows, cols)) in enumerate(shapes):
         n1 = rows * cols
         s_, L = min(rows, cols), max(rows, cols)
         p = torch.empty(n1, dtype=torch.float32, device=dev)
@@ -961,7 +967,9 @@ def run_rows(args):
 
 
 def main():
+    global MATS
     args = parse_args()
+    MATS = args.mats
     if args.workload != "adamw":
         run_rows(args)
     elif args.impl == "reference":
