@@ -112,9 +112,9 @@ __device__ __forceinline__ PlanEntry plan_entry(const PlanEntry* table, int nten
     return table[cur];
 }
 
-// Four CTAs per SM (64 registers): the step is bound by the latency of each
-// warp's dependent chains more than by issue slots, and 32 resident warps
-// hide more of it than 24 do, despite a few spilled registers.
+// Four CTAs per SM (64 registers, no spills): the step is bound by the
+// latency of each warp's dependent chains more than by issue slots, and 32
+// resident warps hide more of it than 24 do.
 // WIDE: AL8 blocks wider than a segment (512 .. 2048 elements), whose value
 // table is built once per block by the warps that share it.
 template <int CPBV, int CPBM, int VBITS, bool WIDE = false>
@@ -236,10 +236,11 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
                             }
                         }
                     }
-                    al8_build_tables<1>(s_tab[warp][0], la, da, kf);
+                    al8_build_tables_soa(reinterpret_cast<float*>(s_tab[warp][0]), la[0], da[0], kf);
                     __syncthreads();
                 }
-                al8_values_part(s_val[g0], s_tab[g0 + wit][0], olmin[0], odelta[0], r, wpbv);
+                al8_values_part_soa(s_val[g0], reinterpret_cast<const float*>(s_tab[g0 + wit][0]),
+                                    olmin[0], odelta[0], r, wpbv);
                 __syncthreads();
                 wit = wit + 1 == wpbv ? 0 : wit + 1;
             } else if constexpr (NBV == 1) {
@@ -266,9 +267,13 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
                 tslot ^= 1;
             } else {
                 // two blocks per segment: their levels in one paired pass
-                al8_build_tables2(s_tab[warp][0], s_tab[warp][0] + 32, olmin[0], odelta[0],
-                                  olmin[1], odelta[1], kf, ok2);
-                al8_values_from_tables<NBV>(s_val[warp], s_tab[warp][0], olmin, odelta);
+                float* ts = reinterpret_cast<float*>(s_tab[warp][0]);
+                al8_build_tables2_soa(ts, ts + 64, olmin[0], odelta[0], olmin[1], odelta[1], kf,
+                                      ok2);
+#pragma unroll
+                for (int b = 0; b < NBV; ++b)
+                    al8_values_from_tables_soa(s_val[warp] + 256 * b, ts + 64 * b, olmin[b],
+                                               odelta[b]);
             }
             const float* vt = s_val[WIDE ? (warp / wpbv) * wpbv : warp];
 #pragma unroll

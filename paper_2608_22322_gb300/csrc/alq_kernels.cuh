@@ -241,22 +241,6 @@ __device__ __forceinline__ int al8_hi_slot(uint32_t a) {
     return 16 + (int)((a & 1u) << 3) + (int)(a >> 1);
 }
 
-template <int NB>
-__device__ __forceinline__ void al8_build_tables(float2* tab, const float (&lmin)[NB],
-                                                 const float (&delta)[NB], float kf) {
-    const int lane = threadIdx.x & 31;
-    const bool hi = lane >= 16;
-    const int slot = hi ? al8_hi_slot((uint32_t)(lane - 16)) : lane;
-#pragma unroll
-    for (int b = 0; b < NB; ++b) {
-        float rh = 0.0f, rl = 0.0f;
-        if (delta[b] > 0.0f && lmin[b] >= -96.0f)
-            al_level_ff(hi ? lmin[b] : 0.0f, delta[b], kf, 254.0f, 1.0f / 254.0f, rh, rl);
-        tab[32 * b + slot] = make_float2(rh, rl);
-    }
-    __syncwarp();
-}
-
 __device__ __forceinline__ bool al8_fast_ok(float lmin, float delta) {
     return delta > 0.0f && lmin >= -96.0f;
 }
@@ -343,25 +327,6 @@ __device__ __forceinline__ void al_level_ff2(float2 lmin, float2 delta, float kf
     rl = mul2(rl, sc);
 }
 
-// The two-float level tables of two blocks, each lane one entry of each (the
-// layout of al8_build_tables); a block outside the fast range gets zeros.
-__device__ __forceinline__ void al8_build_tables2(float2* tab0, float2* tab1, float lmin0,
-                                                  float delta0, float lmin1, float delta1,
-                                                  float kf, const Opaque2& k) {
-    const int lane = threadIdx.x & 31;
-    const bool hi = lane >= 16;
-    const int slot = hi ? al8_hi_slot((uint32_t)(lane - 16)) : lane;
-    const bool f0 = al8_fast_ok(lmin0, delta0), f1 = al8_fast_ok(lmin1, delta1);
-    // blocks outside the fast range compute a harmless level and are zeroed
-    const float2 lm = make_float2(hi && f0 ? lmin0 : 0.0f, hi && f1 ? lmin1 : 0.0f);
-    const float2 dl = make_float2(f0 ? delta0 : 1.0f, f1 ? delta1 : 1.0f);
-    float2 rh, rl;
-    al_level_ff2(lm, dl, kf, 254.0f, 1.0f / 254.0f, k, rh, rl);
-    tab0[slot] = f0 ? make_float2(rh.x, rl.x) : make_float2(0.0f, 0.0f);
-    tab1[slot] = f1 ? make_float2(rh.y, rl.y) : make_float2(0.0f, 0.0f);
-    __syncwarp();
-}
-
 // al8_decode_pair (alq_numerics.h) on two values with the same low factor
 // (bh, bl), step for step in paired instructions (each component rounds as
 // the scalar operation does).
@@ -378,11 +343,14 @@ __device__ __forceinline__ float2 al8_decode_pair2(float2 ah, float2 al, float2 
 }
 
 
-// ------------------------------------------ AL8 level tables, SoA layout --
-// The same two 16-entry level tables as al8_build_tables2 / al8_values_from_
-// tables, stored as 64 floats: the high parts at [slot], the low parts at
-// [32 + slot] (slots as in al8_hi_slot), so that the paired products read
-// the high parts of two entries, and their low parts, as adjacent pairs.
+// ------------------------------------------------------ AL8 level tables --
+// An AL8 block's codes q = 16 a + b factor through two 16-entry tables of
+// two-float levels (the high factor T_hi[a] and the low factor T_lo[b]),
+// stored as 64 floats: the high parts at [slot], the low parts at
+// [32 + slot] (slots 0-15 the low factors, al8_hi_slot(a) the high ones), so
+// that the paired products read the high parts of two entries, and their
+// low parts, as adjacent pairs. Each lane computes one entry; a block
+// outside the fast range gets zeros. Two blocks per paired pass:
 __device__ __forceinline__ void al8_build_tables2_soa(float* tab0, float* tab1, float lmin0,
                                                       float delta0, float lmin1, float delta1,
                                                       float kf, const Opaque2& k) {
@@ -401,7 +369,7 @@ __device__ __forceinline__ void al8_build_tables2_soa(float* tab0, float* tab1, 
     __syncwarp();
 }
 
-// One block's level tables in the SoA layout, one level per lane (scalar).
+// One block's level tables in the same layout, one level per lane (scalar).
 __device__ __forceinline__ void al8_build_tables_soa(float* tab, float lmin, float delta,
                                                      float kf) {
     const int lane = threadIdx.x & 31;
@@ -415,6 +383,9 @@ __device__ __forceinline__ void al8_build_tables_soa(float* tab, float lmin, flo
     __syncwarp();
 }
 
+// Rare path of al8_values_from_tables_soa, out of line so that the hot loop
+// stays compact: redo this lane's eight boundary tests of one block and
+// recompute the flagged values in FP64.
 static __device__ __noinline__ void al8_values_fixup_soa(float* vals, const float* tab, float lmin,
                                                          float delta) {
     const int lane = threadIdx.x & 31;
@@ -428,6 +399,14 @@ static __device__ __noinline__ void al8_values_fixup_soa(float* vals, const floa
     }
 }
 
+// The 256 decoded values of one block (Eq. (5), code 0 -> 0), exactly as
+// the double expression rounds them, in shared memory: lane l computes codes
+// l, l + 32, ..., l + 224 from the block's level tables (T_hi[q >> 4] *
+// T_lo[q & 15], two codes per paired step: T_lo[l & 15] is the same for all
+// eight); entries whose two-float product lies too close to an fp32 rounding
+// boundary, and blocks outside the fast range, are recomputed in FP64 under
+// one warp-uniform branch. An element decode is then a single shared-memory
+// load. tab must be 8-byte aligned.
 __device__ __forceinline__ void al8_values_from_tables_soa(float* vals, const float* tab,
                                                            float lmin, float delta) {
     const int lane = threadIdx.x & 31;
@@ -560,82 +539,21 @@ __device__ __forceinline__ void al_encode_chunks(const float (&x)[4 * CH], const
     }
 }
 
-// Rare path of al8_build_values, out of line so that the hot loop stays
-// compact: redo this lane's eight boundary tests of one block and recompute
-// the flagged values in FP64.
-static __device__ __noinline__ void al8_values_fixup(float* vals, const float2* tab, float lmin,
-                                                     float delta) {
-    const int lane = threadIdx.x & 31;
-    const bool fast = al8_fast_ok(lmin, delta);
-    for (int k = 0; k < 8; ++k) {
-        const uint32_t q = (uint32_t)(lane + 32 * k);
-        const float2 A = tab[al8_hi_slot(q >> 4)];
-        const float2 Bt = tab[q & 15u];
-        bool fb;
-        al8_decode_pair(A.x, A.y, Bt.x, Bt.y, fb);
-        if ((q != 0u) && (fb || !fast)) vals[q] = al_dequantize_fp64(q, lmin, delta, 254.0);
-    }
-}
-
-// The 256 decoded values of each of the NB blocks of a segment (Eq. (5), code
-// 0 -> 0), exactly as the double expression rounds them, in shared memory:
-// lane l computes codes l, l + 32, ..., l + 224 from the block's two-float
-// level tables (T_hi[q >> 4] * T_lo[q & 15], two codes per paired step:
-// T_lo[l & 15] is the same for all eight, the T_hi factors are read four at
-// a time); entries whose two-float product lies too close to an fp32
-// rounding boundary, and blocks outside the fast range, are recomputed in
-// FP64 under one warp-uniform branch. An element decode is then a single
-// shared-memory load. tab must be 16-byte aligned.
-template <int NB>
-__device__ __forceinline__ void al8_values_from_tables(float* vals, const float2* tab,
-                                                       const float (&lmin)[NB],
-                                                       const float (&delta)[NB]) {
-    const int lane = threadIdx.x & 31;
-    bool any_fb = false;
-#pragma unroll
-    for (int b = 0; b < NB; ++b) {
-        const bool fast = al8_fast_ok(lmin[b], delta[b]);
-        const float2 Bt = tab[32 * b + (lane & 15)];
-        const float2 bh = make_float2(Bt.x, Bt.x), bl = make_float2(Bt.y, Bt.y);
-        const float2 nbh = make_float2(-Bt.x, -Bt.x);
-        const float4* A4 = reinterpret_cast<const float4*>(tab + 32 * b + 16 + 8 * (lane >> 4));
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            // codes q0 = l + 64 j and q0 + 32: factors T_hi[4 j + (l >> 4)]
-            // and T_hi[4 j + 2 + (l >> 4)]
-            const float4 a = A4[j];
-            bool f0, f1;
-            const float2 r = al8_decode_pair2(make_float2(a.x, a.z), make_float2(a.y, a.w), bh,
-                                              bl, nbh, f0, f1);
-            const uint32_t q0 = (uint32_t)(lane + 64 * j);
-            vals[256 * b + q0] = q0 == 0u ? 0.0f : r.x;
-            vals[256 * b + q0 + 32] = r.y;
-            any_fb |= ((q0 != 0u) & f0) | f1 | !fast;
-        }
-    }
-    if (__builtin_expect(__any_sync(0xFFFFFFFFu, any_fb), 0)) {
-#pragma unroll
-        for (int b = 0; b < NB; ++b) al8_values_fixup(vals + 256 * b, tab + 32 * b, lmin[b], delta[b]);
-    }
-    __syncwarp();
-}
-
-// Rare path of al8_values_part: this warp's share of codes (steps j0 ..
+// Rare path of al8_values_part_soa: this warp's share of codes (steps j0 ..
 // j0 + nsteps - 1, halves in hmask) recomputed in FP64 where the product
 // could not be certified or the block is outside the fast range.
-static __device__ __noinline__ void al8_values_part_fixup(float* vals, const float2* tab,
-                                                          float lmin, float delta, int j0,
-                                                          int nsteps, uint32_t hmask) {
+static __device__ __noinline__ void al8_values_part_fixup_soa(float* vals, const float* tab,
+                                                              float lmin, float delta, int j0,
+                                                              int nsteps, uint32_t hmask) {
     const int lane = threadIdx.x & 31;
     const bool fast = al8_fast_ok(lmin, delta);
     for (int j = j0; j < j0 + nsteps; ++j) {
         for (int h = 0; h < 2; ++h) {
             if (!((hmask >> h) & 1u)) continue;
             const uint32_t q = (uint32_t)(lane + 64 * j + 32 * h);
-            const float2 A = tab[al8_hi_slot(q >> 4)];
-            const float2 Bt = tab[q & 15u];
+            const int sa = al8_hi_slot(q >> 4), sb = (int)(q & 15u);
             bool fb;
-            al8_decode_pair(A.x, A.y, Bt.x, Bt.y, fb);
+            al8_decode_pair(tab[sa], tab[32 + sa], tab[sb], tab[32 + sb], fb);
             if ((q != 0u) && (fb || !fast)) vals[q] = al_dequantize_fp64(q, lmin, delta, 254.0);
         }
     }
@@ -643,31 +561,29 @@ static __device__ __noinline__ void al8_values_part_fixup(float* vals, const flo
 
 // One block's value table shared by the wpb (2, 4 or 8) warps whose segments
 // it spans: warp r of the group computes its share of the pair steps of
-// al8_values_from_tables (step j covers codes l + 64 j and l + 64 j + 32;
+// al8_values_from_tables_soa (step j covers codes l + 64 j and l + 64 j + 32;
 // wpb 2: steps 2 r, 2 r + 1; wpb 4: step r; wpb 8: one half of step r / 2),
-// from the block's level tables in tab, with the same products, the same
-// certification and the same FP64 recomputation, so every value is the one
-// al8_values_from_tables stores. The caller synchronises the group before
-// and after.
-__device__ __forceinline__ void al8_values_part(float* vals, const float2* tab, float lmin,
-                                                float delta, int r, int wpb) {
+// with the same products, the same certification and the same FP64
+// recomputation, so every value is the one al8_values_from_tables_soa
+// stores. The caller synchronises the group before and after.
+__device__ __forceinline__ void al8_values_part_soa(float* vals, const float* tab, float lmin,
+                                                    float delta, int r, int wpb) {
     const int lane = threadIdx.x & 31;
     const int nsteps = wpb == 2 ? 2 : 1;
     const int j0 = wpb == 8 ? (r >> 1) : r * nsteps;
     const uint32_t hmask = wpb == 8 ? (1u << (r & 1)) : 3u;
-    const float2 Bt = tab[lane & 15];
-    const float2 bh = make_float2(Bt.x, Bt.x), bl = make_float2(Bt.y, Bt.y);
-    const float2 nbh = make_float2(-Bt.x, -Bt.x);
-    const float4* A4 = reinterpret_cast<const float4*>(tab + 16 + 8 * (lane >> 4));
+    const float bv = tab[lane & 15], blv = tab[32 + (lane & 15)];
+    const float2 bh = make_float2(bv, bv), bl = make_float2(blv, blv);
+    const float2 nbh = make_float2(-bv, -bv);
+    const float2* Ah = reinterpret_cast<const float2*>(tab + 16 + 8 * (lane >> 4));
+    const float2* Al = reinterpret_cast<const float2*>(tab + 48 + 8 * (lane >> 4));
     bool any_fb = !al8_fast_ok(lmin, delta);
 #pragma unroll
     for (int s = 0; s < 2; ++s) {
         if (s >= nsteps) break;
         const int j = j0 + s;
-        const float4 a = A4[j];
         bool f0, f1;
-        const float2 v = al8_decode_pair2(make_float2(a.x, a.z), make_float2(a.y, a.w), bh, bl,
-                                          nbh, f0, f1);
+        const float2 v = al8_decode_pair2(Ah[j], Al[j], bh, bl, nbh, f0, f1);
         const uint32_t q0 = (uint32_t)(lane + 64 * j);
         if (hmask & 1u) {
             vals[q0] = q0 == 0u ? 0.0f : v.x;
@@ -679,29 +595,7 @@ __device__ __forceinline__ void al8_values_part(float* vals, const float2* tab, 
         }
     }
     if (__builtin_expect(__any_sync(0xFFFFFFFFu, any_fb), 0))
-        al8_values_part_fixup(vals, tab, lmin, delta, j0, nsteps, hmask);
-}
-
-template <int NB>
-__device__ __forceinline__ void al8_build_values(float* vals, float2* tab,
-                                                 const float (&lmin)[NB],
-                                                 const float (&delta)[NB], float kf) {
-    al8_build_tables<NB>(tab, lmin, delta, kf);
-    al8_values_from_tables<NB>(vals, tab, lmin, delta);
-}
-
-// The same for NB >= 2 blocks, their levels two blocks per paired pass.
-template <int NB>
-__device__ __forceinline__ void al8_build_values_paired(float* vals, float2* tab,
-                                                        const float (&lmin)[NB],
-                                                        const float (&delta)[NB], float kf,
-                                                        const Opaque2& k) {
-    static_assert(NB % 2 == 0, "pairs of blocks");
-#pragma unroll
-    for (int b = 0; b < NB; b += 2)
-        al8_build_tables2(tab + 32 * b, tab + 32 * (b + 1), lmin[b], delta[b], lmin[b + 1],
-                          delta[b + 1], kf, k);
-    al8_values_from_tables<NB>(vals, tab, lmin, delta);
+        al8_values_part_fixup_soa(vals, tab, lmin, delta, j0, nsteps, hmask);
 }
 
 // Element decode with the level computed directly in two-float form (any
