@@ -3,14 +3,16 @@
 // the original gradient; rank 256, channel-wise scaling in Sec. 6.1).
 //
 // Launch sequence of one step:
-//   project   R = bf16(G) * P^T on the tensor cores: four converter warps
-//             read 128-channel tiles of G (fp32) and write them as bf16
-//             (round to nearest even) into a 2-stage shared-memory ring in
-//             the 128-byte-swizzled K-major layout, transposing when the
-//             channels are G's columns; TMA loads the matching P tiles; one
-//             thread issues tcgen05.mma (bf16 x bf16 -> fp32) into a
-//             128 x rank accumulator in tensor memory; the epilogue reads it
-//             back with tcgen05.ld and writes R [channels][rank].
+//   project   R = bf16(G) * P^T on the tensor cores, one persistent CTA per
+//             SM over 128-channel tiles: sixteen converter warps read G
+//             (fp32, prefetched into L2 by TMA a few jobs ahead) and write
+//             it as bf16 (round to nearest even) into a 4-stage shared-
+//             memory ring in the 128-byte-swizzled K-major layout,
+//             transposing when the channels are G's columns; TMA loads the
+//             matching P tiles; one thread issues tcgen05.mma (bf16 x bf16 ->
+//             fp32) into one of two 128 x rank accumulators in tensor
+//             memory; four epilogue warps read the other back with
+//             tcgen05.ld and write R [channels][rank].
 //   moments   per channel (one quantization block = rank values): decode
 //             UF8 M^P and AL8 V^P, Adam EMAs with bias correction, channel
 //             norms of Rt and R (exact two-float sums) -> s_j, re-encode.
@@ -35,10 +37,8 @@ namespace alq {
 
 constexpr int kGM = 128;      // UMMA M (rows of A per CTA)
 constexpr int kGK = 64;       // K per stage (64 bf16 = one 128-byte swizzle row)
-constexpr int kStages = 2;  // two CTAs per SM: one drains its accumulator while the other streams
 constexpr int kAStage = kGM * kGK * 2;     // 16 KB
 constexpr int kBStage = 256 * kGK * 2;     // 32 KB (rank <= 256)
-constexpr int kGemmSmem = kStages * (kAStage + kBStage) + 1024 + 256;
 
 // ------------------------------------------------------------ workspace --
 struct ApWs {
@@ -91,6 +91,13 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
         " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
         "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar)
         : "memory");
+}
+
+// L2 prefetch of one box of a tensor map (no shared memory, no barrier).
+__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int x, int y) {
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global [%0, {%1, %2}];" ::"l"((uint64_t)map),
+                 "r"(x), "r"(y)
+                 : "memory");
 }
 
 // Shared-memory matrix descriptor of a K-major operand tile stored in the
@@ -149,23 +156,14 @@ __host__ __device__ constexpr uint32_t umma_idesc_bf16(int M, int N) {
 }
 
 // ---------------------------------------------------------- projection --
-struct GemmArgs {
-    const float* g;  // G [rows][cols] fp32
-    int64_t cols;    // row pitch of G
-    int64_t K;       // short side s: the reduction length
-    float* R;        // [L][rank]
-    int L;           // channels (the long side)
-    int rank;
-    int kblocks;
-    int rows_short;  // channels are G's columns (rows <= cols)
-    int* err;
+struct GemmArgs {     // G as the projection's operand
+    const float* g;   // G [rows][cols] fp32
+    int64_t cols;     // row pitch of G
+    int64_t K;        // short side s: the reduction length
+    int L;            // channels (the long side)
+    int kblocks;      // K blocks of 64
+    int rows_short;   // channels are G's columns (rows <= cols)
 };
-
-// CTA of the projection: warp 0 issues the TMA loads of P, warp 1 the
-// tensor-core MMAs, warps 2..5 convert G to bf16 into the operand stages and
-// then read the accumulator back.
-constexpr int kConvWarps = 4;
-constexpr int kProjThreads = 64 + 32 * kConvWarps;
 
 // bf16 (round to nearest even) of two values, lo in the low half.
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
@@ -173,20 +171,20 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<const uint32_t*>(&b);
 }
 
-// One converter warp's share (64 values per lane) of K block kb of the
-// 128-channel tile at m0. Channels are G's rows (RS false: K contiguous;
-// warp c takes tile rows 32c .. 32c + 31, two rows per load, 16 lanes x 16
-// bytes along K) or G's columns (RS true: K strided; warp c takes K rows
-// 16c .. 16c + 15, lane l the channels l + 32 q, each load a 128-byte row
-// slice). Outside G the values are 0.
-template <bool RS>
+// One converter warp's share (256 / NW values per lane, NW converter
+// warps) of K block kb of the 128-channel tile at m0. Channels are G's rows
+// (RS false: K contiguous; warp c takes tile rows (128 / NW) c onwards, two
+// rows per load, 16 lanes x 16 bytes along K) or G's columns (RS true: K
+// strided; warp c takes K rows (64 / NW) c onwards, lane l the channels
+// l + 32 q, each load a 128-byte row slice). Outside G the values are 0.
+template <bool RS, int NW>
 __device__ __forceinline__ void conv_load(const GemmArgs& a, int m0, int kb, int c, int lane,
-                                          float (&v)[64]) {
+                                          float (&v)[256 / NW]) {
     if constexpr (!RS) {
         const int64_t k = (int64_t)kb * kGK + 4 * (lane & 15);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-            const int64_t j = m0 + 32 * c + 2 * i + (lane >> 4);
+        for (int i = 0; i < 64 / NW; ++i) {
+            const int64_t j = m0 + (128 / NW) * c + 2 * i + (lane >> 4);
             float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
             if (j < a.L && k < a.K) x = __ldcs(reinterpret_cast<const float4*>(a.g + j * a.cols + k));
             v[4 * i] = x.x;
@@ -195,13 +193,14 @@ __device__ __forceinline__ void conv_load(const GemmArgs& a, int m0, int kb, int
             v[4 * i + 3] = x.w;
         }
     } else {
+        constexpr int KR = 64 / NW;  // K rows of a warp
 #pragma unroll
-        for (int kk = 0; kk < 16; ++kk) {
-            const int64_t k = (int64_t)kb * kGK + 16 * c + kk;
+        for (int kk = 0; kk < KR; ++kk) {
+            const int64_t k = (int64_t)kb * kGK + KR * c + kk;
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const int64_t j = m0 + lane + 32 * q;
-                v[16 * q + kk] = (k < a.K && j < a.L) ? __ldcs(a.g + k * a.cols + j) : 0.0f;
+                v[KR * q + kk] = (k < a.K && j < a.L) ? __ldcs(a.g + k * a.cols + j) : 0.0f;
             }
         }
     }
@@ -210,175 +209,43 @@ __device__ __forceinline__ void conv_load(const GemmArgs& a, int m0, int kb, int
 // The same share as bf16 into an operand stage in the layout a 128-byte
 // swizzled TMA load writes (row r of 128 bytes, 16-byte chunk x stored at
 // chunk x ^ (r & 7)): K-major, as the MMA's shared-memory descriptor reads.
-// Each store of a warp covers all 32 banks once per 128 bytes.
-template <bool RS>
-__device__ __forceinline__ void conv_store(uint8_t* sa, int c, int lane, const float (&v)[64]) {
+template <bool RS, int NW>
+__device__ __forceinline__ void conv_store(uint8_t* sa, int c, int lane,
+                                           const float (&v)[256 / NW]) {
     if constexpr (!RS) {
         const int kq = lane & 15;
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-            const int r = 32 * c + 2 * i + (lane >> 4);
+        for (int i = 0; i < 64 / NW; ++i) {
+            const int r = (128 / NW) * c + 2 * i + (lane >> 4);
             const uint2 w = make_uint2(pack_bf16x2(v[4 * i], v[4 * i + 1]),
                                        pack_bf16x2(v[4 * i + 2], v[4 * i + 3]));
             *reinterpret_cast<uint2*>(sa + r * 128 + (((kq >> 1) ^ (r & 7)) << 4) + ((kq & 1) << 3)) = w;
         }
     } else {
+        constexpr int KR = 64 / NW;  // K rows of a warp: 2 KR bytes of each 128-byte row
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
             const int r = lane + 32 * q;
+            const float* x = v + KR * q;
+            if constexpr (KR == 16) {
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const float* x = v + 16 * q + 8 * h;
+                for (int h = 0; h < 2; ++h) {
+                    const float* y = x + 8 * h;
+                    const uint4 w = make_uint4(pack_bf16x2(y[0], y[1]), pack_bf16x2(y[2], y[3]),
+                                               pack_bf16x2(y[4], y[5]), pack_bf16x2(y[6], y[7]));
+                    *reinterpret_cast<uint4*>(sa + r * 128 + (((2 * c + h) ^ (r & 7)) << 4)) = w;
+                }
+            } else if constexpr (KR == 8) {
                 const uint4 w = make_uint4(pack_bf16x2(x[0], x[1]), pack_bf16x2(x[2], x[3]),
                                            pack_bf16x2(x[4], x[5]), pack_bf16x2(x[6], x[7]));
-                *reinterpret_cast<uint4*>(sa + r * 128 + (((2 * c + h) ^ (r & 7)) << 4)) = w;
-            }
-        }
-    }
-}
-
-// Stage kb of a converter warp: wait until the MMAs that read the stage's
-// previous contents retired, write it, make the writes visible to the tensor
-// cores and arrive (one arrival per converter warp).
-template <bool RS>
-__device__ __forceinline__ bool conv_stage(const float (&v)[64], int kb, uint8_t* sA,
-                                           uint32_t afull0, uint32_t empty0, int c, int lane) {
-    const int s = kb % kStages;
-    if (kb >= kStages && !mbar_wait(empty0 + 8 * s, ((kb / kStages) - 1) & 1)) return false;
-    conv_store<RS>(sA + s * kAStage, c, lane, v);
-    fence_proxy_async_smem();
-    __syncwarp();
-    if (lane == 0) mbar_arrive(afull0 + 8 * s);
-    return true;
-}
-
-// All K blocks of a converter warp (the other CTA on the SM keeps the
-// loads flowing while this one converts).
-template <bool RS>
-__device__ __forceinline__ bool conv_all(const GemmArgs& a, int m0, uint8_t* sA, uint32_t afull0,
-                                         uint32_t empty0, int c, int lane) {
-    float va[64];
-    for (int kb = 0; kb < a.kblocks; ++kb) {
-        conv_load<RS>(a, m0, kb, c, lane, va);
-        if (!conv_stage<RS>(va, kb, sA, afull0, empty0, c, lane)) return false;
-    }
-    return true;
-}
-
-// One 128-channel tile of R = bf16(G) * P^T: channels m0 .. m0 + 127
-// against the whole projection, K in a.kblocks steps of 64. G is read once,
-// as fp32, and converted on its way into the operand stages (no bf16 copy
-// in memory). The tensor map of P may live in the kernel's parameters or in
-// global memory.
-__device__ __forceinline__ void project_tile(const CUtensorMap* tmB, const GemmArgs& a, int m0,
-                                             uint8_t* smem_raw) {
-    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    uint8_t* sA = smem;
-    uint8_t* sB = smem + kStages * kAStage;
-    uint64_t* bars = (uint64_t*)(sB + kStages * kBStage);  // bfull, afull, empty per stage; accum
-    uint32_t* tmem_slot = (uint32_t*)(bars + 3 * kStages + 1);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const uint32_t bfull0 = smem_u32(bars), afull0 = smem_u32(bars + kStages);
-    const uint32_t empty0 = smem_u32(bars + 2 * kStages), accum = smem_u32(bars + 3 * kStages);
-    const uint32_t ncols = a.rank <= 128 ? 128u : 256u;
-
-    if (threadIdx.x == 0) {
-        for (int s = 0; s < kStages; ++s) {
-            mbar_init(bfull0 + 8 * s, 1);
-            mbar_init(afull0 + 8 * s, kConvWarps);
-            mbar_init(empty0 + 8 * s, 1);
-        }
-        mbar_init(accum, 1);
-        mbar_init_fence();
-    }
-    if (warp == 0) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                         smem_u32(tmem_slot)),
-                     "r"(ncols)
-                     : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-    }
-    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-    __syncthreads();
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    const uint32_t tmem = *tmem_slot;
-    const uint32_t b_bytes = (uint32_t)a.rank * kGK * 2;
-
-    bool ok = true;
-    if (warp == 0) {
-        if (lane == 0) {
-            // TMA producer of P: stage s is refilled once the MMAs that read
-            // it retire
-            for (int kb = 0; kb < a.kblocks && ok; ++kb) {
-                const int s = kb % kStages;
-                if (kb >= kStages) ok = mbar_wait(empty0 + 8 * s, ((kb / kStages) - 1) & 1);
-                if (!ok) break;
-                mbar_expect_tx(bfull0 + 8 * s, b_bytes);
-                tma_load_2d(smem_u32(sB + s * kBStage), tmB, kb * kGK, 0, bfull0 + 8 * s);
-            }
-        }
-    } else if (warp == 1) {
-        if (lane == 0) {
-            // MMA issuer: four K = 16 steps per stage, 32 bytes apart in the row
-            const uint32_t idesc = umma_idesc_bf16(kGM, a.rank);
-            for (int kb = 0; kb < a.kblocks && ok; ++kb) {
-                const int s = kb % kStages;
-                const uint32_t par = (kb / kStages) & 1;
-                ok = mbar_wait(afull0 + 8 * s, par) && mbar_wait(bfull0 + 8 * s, par);
-                if (!ok) break;
-                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                const uint32_t a0 = smem_u32(sA + s * kAStage), b0 = smem_u32(sB + s * kBStage);
-#pragma unroll
-                for (int k = 0; k < kGK / 16; ++k)
-                    umma_bf16(tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc,
-                              (kb | k) != 0);
-                umma_commit(empty0 + 8 * s);
-            }
-            if (ok) umma_commit(accum);
-        }
-    } else {
-        const int c = warp - 2;
-        ok = a.rows_short ? conv_all<true>(a, m0, sA, afull0, empty0, c, lane)
-                          : conv_all<false>(a, m0, sA, afull0, empty0, c, lane);
-    }
-    if (!ok) atomicExch(a.err, 1);
-
-    if (warp >= 2) {
-        // epilogue: a warp may read TMEM lanes 32 (warp % 4) .. + 31 (tile
-        // rows), 32 columns at a time
-        const int q = warp & 3;
-        const bool have = mbar_wait(accum, 0);
-        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        const int row = m0 + q * 32 + lane;
-        if (!have && lane == 0) atomicExch(a.err, 1);
-        for (int c0 = 0; c0 < a.rank; c0 += 32) {
-            float v[32];
-            if (have) {
-                tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, v);
+                *reinterpret_cast<uint4*>(sa + r * 128 + ((c ^ (r & 7)) << 4)) = w;
             } else {
-#pragma unroll
-                for (int i = 0; i < 32; ++i) v[i] = __int_as_float(0x7FC00000);  // NaN marks a failure
-            }
-            if (row < a.L) {
-                float4* dst = reinterpret_cast<float4*>(a.R + (int64_t)row * a.rank + c0);
-#pragma unroll
-                for (int i = 0; i < 8; ++i)
-                    dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+                static_assert(KR == 4, "4, 8 or 16 converter warps");
+                const uint2 w = make_uint2(pack_bf16x2(x[0], x[1]), pack_bf16x2(x[2], x[3]));
+                *reinterpret_cast<uint2*>(sa + r * 128 + (((c >> 1) ^ (r & 7)) << 4) + ((c & 1) << 3)) = w;
             }
         }
     }
-    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-    __syncthreads();
-    if (warp == 0)
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
-                     "r"(ncols)
-                     : "memory");
-}
-
-__global__ void __launch_bounds__(kProjThreads, 2)
-apollo_project_kernel(const __grid_constant__ CUtensorMap tmB, GemmArgs a) {
-    extern __shared__ uint8_t smem_raw[];
-    project_tile(&tmB, a, blockIdx.x * kGM, smem_raw);
 }
 
 // ------------------------------------------------------------- moments --
@@ -811,6 +678,7 @@ static_assert(sizeof(ApPlanHeader) == 80, "plan header layout");
 
 struct ApEntry {  // aligned as CUtensorMap (at least 64 bytes)
     CUtensorMap tmB;  // bf16 P [rank][s], box [rank][64]
+    CUtensorMap tmG;  // fp32 G, box = one 128-channel x 64-K projection job (L2 prefetch)
     float* p;
     const float* g;
     int8_t* m_codes;
@@ -839,19 +707,289 @@ __device__ __forceinline__ int entry_for(const ApEntry* __restrict__ tab, int nm
     return cur;
 }
 
-__global__ void __launch_bounds__(kProjThreads, 2)
-apollo_project_multi_kernel(const ApEntry* __restrict__ tab, const uint16_t* __restrict__ tile_mat,
-                            int rank, int* err) {
-    extern __shared__ uint8_t smem_raw[];
-    const ApEntry* e = tab + tile_mat[blockIdx.x];
-    if (threadIdx.x == 0) {
-        // the descriptor was written through the generic proxy (a copy to
-        // device memory): make it visible to the tensor-map proxy
-        asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(&e->tmB)
-                     : "memory");
+// ----------------------------------------------------------- projection --
+// R = bf16(G) P^T by a persistent kernel: one CTA per SM walks 128-channel
+// tiles with a stride of the grid. Each tile is kblocks jobs of 64 K; a job
+// is one 4-stage ring slot holding the tile's G slice as bf16 (converted by
+// the converter warps) and P's slice (a TMA load). The ring's stages and
+// phases run on across tiles, and the two accumulators in tensor memory
+// alternate between tiles, so the epilogue of one tile overlaps the operand
+// stream of the next. Warp 0 issues the TMA loads of P and an L2 prefetch of
+// G kPrefetch jobs ahead (so that the converters' loads hit L2), warp 1 the
+// MMAs, warps 2 .. 1 + kPConv convert G, the last kPEpi warps drain the
+// accumulators into R.
+constexpr int kPStages = 4;
+constexpr int kPrefetch = 4;  // G jobs prefetched into L2 ahead of the P loads
+constexpr int kPConv = 16;
+constexpr int kPEpi = 4;
+constexpr int kPThreads = 64 + 32 * (kPConv + kPEpi);
+constexpr int kPSmem = kPStages * (kAStage + kBStage) + 1024 + 256;
+constexpr int kPV = 256 / kPConv;  // values per converter lane and job
+
+// Matrix of tile t: from the plan's tile map, or the one matrix of a
+// single-matrix launch.
+template <bool kOne>
+__device__ __forceinline__ const ApEntry* tile_entry(const ApEntry* tab,
+                                                     const uint16_t* __restrict__ tile_mat,
+                                                     int64_t t) {
+    return kOne ? tab : tab + tile_mat[t];
+}
+
+// One (tile, K block) job of a converter warp's walk.
+struct PJob {
+    GemmArgs a;
+    int m0, kb;
+    bool valid;
+};
+
+template <bool kOne>
+__device__ __forceinline__ PJob pjob_at(const ApEntry* tab, const uint16_t* __restrict__ tile_mat,
+                                        int64_t ntiles, int64_t t) {
+    PJob j;
+    j.valid = t < ntiles;
+    j.kb = 0;
+    j.m0 = 0;
+    if (j.valid) {
+        const ApEntry* e = tile_entry<kOne>(tab, tile_mat, t);
+        j.a = GemmArgs{e->g, e->cols, e->s, (int)e->L, e->kblocks, e->rows_short};
+        j.m0 = (int)(t - e->gemm_t0) * kGM;
     }
-    const GemmArgs a{e->g, e->cols, e->s, e->R, (int)e->L, rank, e->kblocks, e->rows_short, err};
-    project_tile(&e->tmB, a, (int)(blockIdx.x - e->gemm_t0) * kGM, smem_raw);
+    return j;
+}
+
+__device__ __forceinline__ void pjob_load(const PJob& j, int c, int lane, float (&v)[kPV]) {
+    if (j.a.rows_short) conv_load<true, kPConv>(j.a, j.m0, j.kb, c, lane, v);
+    else conv_load<false, kPConv>(j.a, j.m0, j.kb, c, lane, v);
+}
+
+// Job kc of the walk into its ring slot: wait until the MMAs that read the
+// slot's previous contents retired, write it, make the writes visible to the
+// tensor cores and arrive (one arrival per converter warp).
+__device__ __forceinline__ bool pjob_stage(const PJob& j, const float (&v)[kPV], uint32_t kc,
+                                           uint8_t* sA, uint32_t afull0, uint32_t empty0, int c,
+                                           int lane) {
+    const uint32_t s = kc % kPStages;
+    if (kc >= (uint32_t)kPStages && !mbar_wait(empty0 + 8 * s, ((kc / kPStages) - 1) & 1))
+        return false;
+    if (j.a.rows_short) conv_store<true, kPConv>(sA + s * kAStage, c, lane, v);
+    else conv_store<false, kPConv>(sA + s * kAStage, c, lane, v);
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(afull0 + 8 * s);
+    return true;
+}
+
+// A converter warp's walk: the loads of the next job (the next K block, or
+// the first of the next tile) are issued before the current job is stored
+// (two register buffers used in turn).
+template <bool kOne>
+__device__ __forceinline__ bool pconv_walk(const ApEntry* tab, const uint16_t* __restrict__ tile_mat,
+                                           int64_t ntiles, uint8_t* sA, uint32_t afull0,
+                                           uint32_t empty0, int c, int lane) {
+    const int64_t G = gridDim.x;
+    int64_t t = blockIdx.x;
+    PJob ja = pjob_at<kOne>(tab, tile_mat, ntiles, t), jb;
+    float va[kPV], vb[kPV];
+    if (!ja.valid) return true;
+    pjob_load(ja, c, lane, va);
+    uint32_t kc = 0;
+    for (;;) {
+        if (ja.kb + 1 < ja.a.kblocks) {
+            jb = ja;
+            ++jb.kb;
+        } else {
+            t += G;
+            jb = pjob_at<kOne>(tab, tile_mat, ntiles, t);
+        }
+        if (jb.valid) pjob_load(jb, c, lane, vb);
+        if (!pjob_stage(ja, va, kc++, sA, afull0, empty0, c, lane)) return false;
+        if (!jb.valid) return true;
+        if (jb.kb + 1 < jb.a.kblocks) {
+            ja = jb;
+            ++ja.kb;
+        } else {
+            t += G;
+            ja = pjob_at<kOne>(tab, tile_mat, ntiles, t);
+        }
+        if (ja.valid) pjob_load(ja, c, lane, va);
+        if (!pjob_stage(jb, vb, kc++, sA, afull0, empty0, c, lane)) return false;
+        if (!ja.valid) return true;
+    }
+}
+
+// kOne: a single matrix whose descriptor (tensor maps included) is the
+// kernel parameter `one`; otherwise the plan's table `tab` and tile map.
+template <bool kOne>
+__global__ void __launch_bounds__(kPThreads, 1)
+apollo_project_kernel(const ApEntry* __restrict__ plan_tab, const uint16_t* __restrict__ tile_mat,
+                      int64_t ntiles, int rank, int* err, const __grid_constant__ ApEntry one) {
+    extern __shared__ uint8_t smem_raw[];
+    const ApEntry* tab = kOne ? &one : plan_tab;
+    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t* sA = smem;
+    uint8_t* sB = smem + kPStages * kAStage;
+    // bfull, afull, empty per stage; tfull, tempty per accumulator
+    uint64_t* bars = (uint64_t*)(sB + kPStages * kBStage);
+    uint32_t* tmem_slot = (uint32_t*)(bars + 3 * kPStages + 4);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t bfull0 = smem_u32(bars), afull0 = smem_u32(bars + kPStages);
+    const uint32_t empty0 = smem_u32(bars + 2 * kPStages);
+    const uint32_t tfull0 = smem_u32(bars + 3 * kPStages), tempty0 = tfull0 + 16;
+    const uint32_t acc_cols = rank <= 128 ? 128u : 256u;
+    const uint32_t ncols = 2 * acc_cols;
+    const int64_t G = gridDim.x;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kPStages; ++s) {
+            mbar_init(bfull0 + 8 * s, 1);
+            mbar_init(afull0 + 8 * s, kPConv);
+            mbar_init(empty0 + 8 * s, 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(tfull0 + 8 * b, 1);
+            mbar_init(tempty0 + 8 * b, kPEpi);
+        }
+        mbar_init_fence();
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(tmem_slot)),
+                     "r"(ncols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = *tmem_slot;
+    const uint32_t b_bytes = (uint32_t)rank * kGK * 2;
+
+    bool ok = true;
+    if (warp == 0) {
+        if (lane == 0) {
+            // TMA producer of P: stage s is refilled once the MMAs that read
+            // it retire
+            // and L2 prefetcher of G: the job kPrefetch ahead of the one
+            // whose P it loads (tile pt, K block pkb) is fetched into L2, so
+            // that the converter warps' loads of it hit L2
+            uint32_t kc = 0;
+            const ApEntry* last = nullptr;
+            int64_t pt = blockIdx.x;
+            int pkb = 0;
+            const ApEntry* pe = pt < ntiles ? tile_entry<kOne>(tab, tile_mat, pt) : nullptr;
+            const ApEntry* plast = nullptr;
+            auto prefetch_next = [&]() {
+                if (!pe) return;
+                if (!kOne && pe != plast) {
+                    asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(
+                                     &pe->tmG)
+                                 : "memory");
+                    plast = pe;
+                }
+                const int m0 = (int)(pt - pe->gemm_t0) * kGM;
+                if (pe->rows_short) tma_prefetch_2d(&pe->tmG, m0, pkb * kGK);
+                else tma_prefetch_2d(&pe->tmG, pkb * kGK, m0);
+                if (++pkb == pe->kblocks) {
+                    pkb = 0;
+                    pt += G;
+                    pe = pt < ntiles ? tile_entry<kOne>(tab, tile_mat, pt) : nullptr;
+                }
+            };
+            for (int i = 0; i < kPrefetch; ++i) prefetch_next();
+            for (int64_t t = blockIdx.x; t < ntiles && ok; t += G) {
+                const ApEntry* e = tile_entry<kOne>(tab, tile_mat, t);
+                if (!kOne && e != last) {
+                    // a plan's descriptor was written through the generic
+                    // proxy (a copy to device memory): make it visible to the
+                    // tensor-map proxy
+                    asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(
+                                     &e->tmB)
+                                 : "memory");
+                    last = e;
+                }
+                const int kblocks = e->kblocks;
+                for (int kb = 0; kb < kblocks; ++kb, ++kc) {
+                    prefetch_next();
+                    const uint32_t s = kc % kPStages;
+                    if (kc >= (uint32_t)kPStages)
+                        ok = mbar_wait(empty0 + 8 * s, ((kc / kPStages) - 1) & 1);
+                    if (!ok) break;
+                    mbar_expect_tx(bfull0 + 8 * s, b_bytes);
+                    tma_load_2d(smem_u32(sB + s * kBStage), &e->tmB, kb * kGK, 0, bfull0 + 8 * s);
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // MMA issuer: four K = 16 steps per stage, 32 bytes apart in the
+            // row; accumulator it & 1 of tile number it
+            const uint32_t idesc = umma_idesc_bf16(kGM, rank);
+            uint32_t kc = 0, it = 0;
+            for (int64_t t = blockIdx.x; t < ntiles && ok; t += G, ++it) {
+                const int kblocks = tile_entry<kOne>(tab, tile_mat, t)->kblocks;
+                const uint32_t acc = it & 1;
+                if (it >= 2) ok = mbar_wait(tempty0 + 8 * acc, ((it / 2) - 1) & 1);
+                if (!ok) break;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t d = tmem + acc * acc_cols;
+                for (int kb = 0; kb < kblocks; ++kb, ++kc) {
+                    const uint32_t s = kc % kPStages;
+                    const uint32_t par = (kc / kPStages) & 1;
+                    ok = mbar_wait(afull0 + 8 * s, par) && mbar_wait(bfull0 + 8 * s, par);
+                    if (!ok) break;
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                    const uint32_t a0 = smem_u32(sA + s * kAStage), b0 = smem_u32(sB + s * kBStage);
+#pragma unroll
+                    for (int k = 0; k < kGK / 16; ++k)
+                        umma_bf16(d, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc,
+                                  (kb | k) != 0);
+                    umma_commit(empty0 + 8 * s);
+                }
+                if (ok) umma_commit(tfull0 + 8 * acc);
+            }
+        }
+    } else if (warp < 2 + kPConv) {
+        ok = pconv_walk<kOne>(tab, tile_mat, ntiles, sA, afull0, empty0, warp - 2, lane);
+    } else {
+        // epilogue: a warp may read TMEM lanes 32 (warp % 4) .. + 31 (tile
+        // rows), 32 columns at a time
+        const int q = warp & 3;
+        uint32_t it = 0;
+        for (int64_t t = blockIdx.x; t < ntiles && ok; t += G, ++it) {
+            const ApEntry* e = tile_entry<kOne>(tab, tile_mat, t);
+            const uint32_t acc = it & 1;
+            ok = mbar_wait(tfull0 + 8 * acc, (it / 2) & 1);
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const int64_t row = (t - e->gemm_t0) * kGM + q * 32 + lane;
+            float* R = e->R;
+            const int64_t L = e->L;
+            for (int c0 = 0; c0 < rank; c0 += 32) {
+                float v[32];
+                if (ok) {
+                    tmem_ld32(tmem + acc * acc_cols + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, v);
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = __int_as_float(0x7FC00000);  // NaN marks a failure
+                }
+                if (row < L) {
+                    float4* dst = reinterpret_cast<float4*>(R + row * rank + c0);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+                }
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
+        }
+    }
+    if (!ok) atomicExch(err, 1);
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "r"(ncols)
+                     : "memory");
 }
 
 template <int CPB, int VBITS>
@@ -967,22 +1105,43 @@ static bool make_map(CUtensorMap* map, const void* base, uint64_t k, uint64_t ro
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 2-D fp32 tensor map over G [rows][cols] whose box is one projection job:
+// 128 channels by 64 K (channels are G's rows, box [128][64], or its columns,
+// box [64][128]). Used only to prefetch jobs into L2.
+static bool make_gmap(CUtensorMap* map, const float* g, int64_t rows, int64_t cols,
+                      bool rows_short) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)cols * 4};
+    const cuuint32_t box[2] = {rows_short ? (cuuint32_t)kGM : (cuuint32_t)kGK,
+                               rows_short ? (cuuint32_t)kGK : (cuuint32_t)kGM};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(g), dims, strides, box,
+              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 static int launch_project(const float* g, int64_t rows, int64_t cols, const uint16_t* P,
                           int rank, float* R, int* err, cudaStream_t st) {
     const int rows_short = rows <= cols;
-    const int64_t s = rows_short ? rows : cols, L = rows_short ? cols : rows;
-    CUtensorMap mb;
-    if (!make_map(&mb, P, (uint64_t)s, (uint64_t)rank, (uint32_t)rank))
+    ApEntry e;
+    memset(&e, 0, sizeof(e));
+    e.g = g;
+    e.R = R;
+    e.rows = rows;
+    e.cols = cols;
+    e.s = rows_short ? rows : cols;
+    e.L = rows_short ? cols : rows;
+    e.rows_short = rows_short;
+    e.kblocks = (int32_t)blocks_of(e.s, kGK);
+    if (!make_map(&e.tmB, P, (uint64_t)e.s, (uint64_t)rank, (uint32_t)rank) ||
+        !make_gmap(&e.tmG, g, rows, cols, rows_short))
         return record_cuda(cudaErrorInvalidValue);
-    static std::once_flag once;
-    static cudaError_t attr_err = cudaSuccess;
-    std::call_once(once, [] {
-        attr_err = cudaFuncSetAttribute(apollo_project_kernel,
-                                        cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);
-    });
-    if (attr_err != cudaSuccess) return record_cuda(attr_err);
-    GemmArgs a{g, cols, s, R, (int)L, rank, (int)blocks_of(s, kGK), rows_short, err};
-    apollo_project_kernel<<<(unsigned)blocks_of(L, kGM), kProjThreads, kGemmSmem, st>>>(mb, a);
+    const int64_t ntiles = blocks_of(e.L, kGM);
+    apollo_project_kernel<true><<<persistent_grid((const void*)apollo_project_kernel<true>,
+                                                  kPThreads, kPSmem, ntiles),
+                                  kPThreads, kPSmem, st>>>(nullptr, nullptr, ntiles, rank, err, e);
     return check_launch();
 }
 
@@ -1212,7 +1371,8 @@ extern "C" int al_apollo_plan(const al_apollo_matrix* mats, int nmat, int rank, 
         e.mom_t0 = h.mom_tiles;
         e.upd_t0 = h.upd_tiles;
         e.nrm_t0 = h.norm_chunks;
-        if (!make_map(&e.tmB, m.proj, (uint64_t)a.s, (uint64_t)rank, (uint32_t)rank))
+        if (!make_map(&e.tmB, m.proj, (uint64_t)a.s, (uint64_t)rank, (uint32_t)rank) ||
+            !make_gmap(&e.tmG, m.g, m.rows, m.cols, a.rows_short))
             return record_cuda(cudaErrorInvalidValue);
         const int64_t gt = blocks_of(a.L, kGM);
         for (int64_t k = 0; k < gt; ++k) tile_mat[h.gemm_tiles + k] = (uint16_t)i;
@@ -1255,15 +1415,12 @@ extern "C" int al_apollo_step_multi(const void* plan_dev, const al_apollo_info* 
     int* err = (int*)info->workspace;
 
     int rc;
-    static std::once_flag once;
-    static cudaError_t attr_err = cudaSuccess;
-    std::call_once(once, [] {
-        attr_err = cudaFuncSetAttribute(apollo_project_multi_kernel,
-                                        cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);
-    });
-    if (attr_err != cudaSuccess) return record_cuda(attr_err);
-    apollo_project_multi_kernel<<<(unsigned)info->gemm_tiles, kProjThreads, kGemmSmem, st>>>(
-        tab, tile_mat, info->rank, err);
+    ApEntry none;
+    memset(&none, 0, sizeof(none));
+    apollo_project_kernel<false><<<persistent_grid((const void*)apollo_project_kernel<false>,
+                                                   kPThreads, kPSmem, info->gemm_tiles),
+                                   kPThreads, kPSmem, st>>>(tab, tile_mat, info->gemm_tiles,
+                                                            info->rank, err, none);
     rc = check_launch();
     if (rc) return rc;
 
