@@ -843,6 +843,9 @@ def _row_codec(torch, np, wl, B, dev):
                 bytes_note="20 B/element + block constants")
 
 
+HOLD_CYCLES = 525_000  # about 0.25 ms at the 2.1 GHz maximum SM clock
+
+
 class L2Flush:
     """Writes a buffer twice the L2's size between timed steps, so that no
     step starts with the previous step's data in L2."""
@@ -858,8 +861,9 @@ class L2Flush:
 
 def measure_row(name, args, dev, warmup, min_steps, with_cpu, summary):
     """Times one non-headline hot-path row: whole steps (all of the row's
-    launches) with CUDA events around each step and an L2 flush between
-    steps (outside the events), at least min_steps steps and enough to fill
+    launches) with CUDA events around each step and an L2 flush and a
+    short device-side wait between steps (outside the events), at least
+    min_steps steps and enough to fill
     about 0.6 s, with nvidia-smi clock samples over the timed loop; bytes
     per step over time against the measured HBM copy peak; the oracle on a
     bounded sample (its OpenMP build for the multi-matrix rows)."""
@@ -902,6 +906,11 @@ def measure_row(name, args, dev, warmup, min_steps, with_cpu, summary):
     torch.cuda.synchronize(dev)
     for a, b in pairs:
         flush()
+        # a quarter millisecond of device-side wait (outside the events):
+        # the GPU then runs behind the host, so a short step's launches are
+        # all queued before its start event and the events time the device
+        # alone, not the host's launch latency
+        torch.cuda._sleep(HOLD_CYCLES)
         t += 1
         a.record(stream)
         w["step"](t)
@@ -926,7 +935,8 @@ def measure_row(name, args, dev, warmup, min_steps, with_cpu, summary):
             "frac": achieved / peak, "frac_of_8tbs_spec": achieved / 8000.0,
             "traffic": None, "peak_source": f"{peak_src} hbm_gbs",
             "kernel": "whole step (all launches; per-kernel shares in profiles/)"}
-    l2 = "L2 flushed (a write of twice its size) between timed steps, outside the events"
+    l2 = ("L2 flushed (a write of twice its size) and a 0.25 ms device-side wait between "
+          "timed steps, outside the events")
     if summary:
         out = {"workload": w["workload"], "value": w["n"] / (ms_step * 1e-3), "unit": unit,
                "ms_per_step": ms_step, "steps": steps, "warmup": max(3, warmup),
