@@ -629,7 +629,7 @@ def _row_came(torch, np, wl, B, dev):
     (2), absmax and the four factor states; the library's passes read G four
     times and the momentum codes twice (from L2 where a matrix's gradient
     stays there between its passes), which is not counted. Per-matrix steps
-    on three streams by default (see below)."""
+    on eight streams by default (see below)."""
     cfg = wl.CONFIGS["came"]
     rows, cols = cfg["shape"]
     nm = min(cfg["n_mats"], MATS) if MATS else cfg["n_mats"]
@@ -659,9 +659,11 @@ def _row_came(torch, np, wl, B, dev):
                          cc=fac(cols, cb), mc=torch.zeros(n1, dtype=torch.int8, device=dev),
                          ma=torch.zeros((n1 + 255) // 256, dtype=torch.float32, device=dev)))
     # per-matrix steps (al_came_step: eight passes chained by programmatic
-    # dependent launch) on three streams, so that three matrices' gradients
-    # (138 MB) share the L2 while their passes run (1.51 ms against 1.61 ms
-    # for grouped steps over 4 groups on 4 streams, on one box);
+    # dependent launch) dealt over eight streams, so that one matrix's short
+    # factor and scale passes overlap other matrices' streaming passes
+    # (measured on one box: 1.566 ms on 2 streams, 1.515 on 3, 1.494 on 4,
+    # 1.480 on 6, 1.478 on 8, 1.481 on 11, 1.498 on 22; 1.61 ms for grouped
+    # steps over 4 groups on 4 streams);
     # ALQ_BENCH_CAME_SINGLE=0 times grouped steps instead (one launch per
     # pass over a group of matrices, ALQ_BENCH_GROUPS groups on
     # ALQ_BENCH_STREAMS streams; one plan per group and gradient buffer)
@@ -674,7 +676,7 @@ def _row_came(torch, np, wl, B, dev):
              cr_meta=m["cr"][1], cc_codes=m["cc"][0], cc_meta=m["cc"][1], m_codes=m["mc"],
              m_absmax=m["ma"]) for m in grp], 16, vb, 16, cb, 256) for grp in groups]
         for k in range(2)]
-    nstreams = int(os.environ.get("ALQ_BENCH_STREAMS", "3" if single else str(ngroups)))
+    nstreams = int(os.environ.get("ALQ_BENCH_STREAMS", "8" if single else str(ngroups)))
     streams = [torch.cuda.Stream(device=dev) for _ in range(nstreams)]
     wss = ([torch.empty(B.al_workspace_size(B.AL_OP_CAME, rows, cols), dtype=torch.uint8,
                         device=dev) for _ in range(nm)] if single else None)
