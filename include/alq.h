@@ -15,8 +15,12 @@
  *
  * Conventions shared by every entry point
  * ---------------------------------------
- *  - Every array pointer is DEVICE memory owned by the caller, unless the
- *    argument is documented as host memory. The library allocates, frees and
+ *  - Every array pointer is DEVICE-accessible memory owned by the caller,
+ *    unless the argument is documented as host memory: device memory, or
+ *    pinned host memory through its device mapping (the kernels then read
+ *    and write it across the host link; a host-offloaded optimizer can step
+ *    its host-resident arrays in place). Plans themselves live in device
+ *    memory. The library allocates, frees and
  *    synchronises nothing; work is enqueued on `stream` (a cudaStream_t passed
  *    as void*; NULL is the legacy default stream) and the call returns without
  *    waiting for it.
