@@ -137,6 +137,36 @@ def test_adamw_plan_many_tensors(B, v_block):
             pr.compare(f"tensor {i} (n={sizes[i]}) step {t}")
 
 
+def test_adamw_plan_over_pinned_host_buffers(B):
+    """A plan whose parameters, gradients, codes and block constants are
+    pinned host memory (their device mapping): the kernel steps them in
+    place across the host link, as the end-to-end bench does, with the same
+    results as on device buffers (the oracle's, bit for bit for codes and
+    constants)."""
+    import torch
+    sizes = [5, 4097, 2 * 4096 + 511, 64 * 1024]
+    pairs, gens = [], []
+    for i, n in enumerate(sizes):
+        p0 = (wl.rng(60 + i).standard_normal(n) * 0.02).astype(np.float32)
+        pr = Pair(p0, 256, 256, 8)
+        pr.d = {k: v.cpu().pin_memory() for k, v in pr.d.items()}
+        pairs.append(pr)
+        gens.append(lambda t, n=n, i=i: wl.gaussian_grad((n,), 1e-3, 700 + 31 * i + t,
+                                                         wl.zero_mask((n,), 0.1, 57 + i)))
+    ghost = [torch.zeros(n, dtype=torch.float32).pin_memory() for n in sizes]
+    plan = B.AdamWPlan([dict(g=ghost[i], **pr.dev_args()) for i, pr in enumerate(pairs)],
+                       256, 256, 8, device=torch.device("cuda"))
+    for t in range(1, 4):
+        torch.cuda.synchronize()
+        for i, pr in enumerate(pairs):
+            g = gens[i](t)
+            pr.host_step(g, t)
+            ghost[i].copy_(torch.from_numpy(g))
+        plan.step(ADAMW_HP, t)
+        for i, pr in enumerate(pairs):
+            pr.compare(f"host tensor {i} (n={sizes[i]}) step {t}")
+
+
 def test_adamw_tinyllama_full_plan_sampled(B):
     """All 201 TinyLlama-1.1B tensors (1,100,048,384 parameters) in one plan,
     the launch the benchmark times. Blocks are independent in AdamW, so the
