@@ -15,7 +15,8 @@
 //             tcgen05.ld and write R [channels][rank].
 //   moments   per channel (one quantization block = rank values): decode
 //             UF8 M^P and AL8 V^P, Adam EMAs with bias correction, channel
-//             norms of Rt and R (exact two-float sums) -> s_j, re-encode.
+//             norms of Rt and R (fp32 sums: they move p only) -> s_j,
+//             re-encode.
 //   limiter   (optional) ||G s|| and the norm-growth cap: sums of squares
 //             per chunk of kNormChunk update tiles (a partition of each
 //             matrix that does not depend on the grid), summed in chunk
@@ -271,49 +272,12 @@ constexpr int kMCH = 2;
 constexpr int kMSeg = 128 * kMCH;
 constexpr int kMTile = 8 * kMSeg;
 
-// Channel scales waiting for their FP64 evaluation: lane k of a warp holds
-// the two-float norm sums of the warp's k-th pending channel (FP64 runs at a
-// small fraction of the fp32 rate on this part, so the warp evaluates 32
-// channels in one pass instead of one per segment).
-struct PendingScales {
-    float nrh = 0.0f, nrl = 0.0f, ngh = 0.0f, ngl = 0.0f;
-    float* dst = nullptr;
-    int count = 0;
-
-    // s_j = ||Rt_j|| / (||R_j|| + 1e-8) from the sums in double, rounded once
-    __device__ __forceinline__ void flush() {
-        if (dst) {
-            const double nr = (double)nrh + (double)nrl;
-            const double ng = (double)ngh + (double)ngl;
-            *dst = (float)(sqrt(nr) / (sqrt(ng) + 1e-8));
-        }
-        dst = nullptr;
-        count = 0;
-    }
-    // a channel's sums as lane 0 holds them (the butterfly leaves the low
-    // parts of other lanes rounded in another order) go to lane count
-    __device__ __forceinline__ void add(float rh, float rl, float gh, float gl, float* d) {
-        rh = __shfl_sync(0xFFFFFFFFu, rh, 0);
-        rl = __shfl_sync(0xFFFFFFFFu, rl, 0);
-        gh = __shfl_sync(0xFFFFFFFFu, gh, 0);
-        gl = __shfl_sync(0xFFFFFFFFu, gl, 0);
-        if ((int)(threadIdx.x & 31) == count) {
-            nrh = rh;
-            nrl = rl;
-            ngh = gh;
-            ngl = gl;
-            dst = d;
-        }
-        if (++count == 32) flush();
-    }
-};
-
 // One tile of the moments pass. tab and vals are this warp's shared slots
 // for the AL8 decode tables (NB * 32 pairs) and the blocks' 256 decoded
-// values (NB * 256); the channels' norm sums join ps.
+// values (NB * 256); lane 0 writes the blocks' channel scales.
 template <int CPB, int VBITS>
 __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, float2* tab,
-                                             float* vals, PendingScales& ps) {
+                                             float* vals) {
     constexpr int NB = kMCH / CPB;
     constexpr int NE = 4 * kMCH;
     constexpr float Lm2 = VBITS == 8 ? 254.0f : 65534.0f;
@@ -376,23 +340,21 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
     // Moments and channel norms on pairs of elements (paired fp32
     // instructions, each component rounded as the scalar operation; a sum
     // of two rounded products is a fused multiply-add by the opaque one, so
-    // that no product is contracted into it). The norms accumulate the
-    // exact squares (two-float products) in two-float sums, even and odd
-    // elements apart, merged before the warp sum.
+    // that no product is contracted into it). The channel norms, like the
+    // bias-corrected ratio they measure, move only the parameters: fp32
+    // sums of squares (relative error below 2^-19 over a channel).
     const float2 one = make_float2(m.one, m.one);
     const float2 b1 = make_float2(m.beta1, m.beta1), o1 = make_float2(m.omb1, m.omb1);
     const float2 b2 = make_float2(m.beta2, m.beta2), o2 = make_float2(m.omb2, m.omb2);
     const float2 ic1 = make_float2(m.ic1, m.ic1), c2 = make_float2(m.c2, m.c2);
-    const float2 eps = make_float2(m.eps, m.eps), neg = make_float2(-1.0f, -1.0f);
-    const float2 zero = make_float2(m.zero, m.zero);
+    const float2 eps = make_float2(m.eps, m.eps);
     float vf[NE];
     float2 mf2[NE / 2];
     uint32_t cvmin[kMCH], cvmax[kMCH];
     float cmabs[kMCH];
-    float2 nrh[NB], nrl[NB], ngh[NB], ngl[NB];
+    float2 nr2[NB], ng2[NB];
 #pragma unroll
-    for (int b = 0; b < NB; ++b)
-        nrh[b] = nrl[b] = ngh[b] = ngl[b] = make_float2(0.0f, 0.0f);
+    for (int b = 0; b < NB; ++b) nr2[b] = ng2[b] = make_float2(0.0f, 0.0f);
 #pragma unroll
     for (int c = 0; c < kMCH; ++c) {
         const int b = c / CPB;
@@ -419,23 +381,19 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
             mf2[2 * c + i] = mq;
             vf[4 * c + 2 * i] = vq.x;
             vf[4 * c + 2 * i + 1] = vq.y;
-            ff_acc_sq2(nrh[b], nrl[b], rt, neg, zero);
-            ff_acc_sq2(ngh[b], ngl[b], rv, neg, zero);
+            nr2[b] = fma2(rt, rt, nr2[b]);
+            ng2[b] = fma2(rv, rv, ng2[b]);
             const uint32_t vbx = f2u(vq.x), vby = f2u(vq.y);
             cvmin[c] = umix<false>(cvmin[c], umix<false>(vbx - 1u, vby - 1u));
             cvmax[c] = umix<true>(cvmax[c], umix<true>(vbx, vby));
             cmabs[c] = fmaxf(cmabs[c], fmaxf(fabsf(mq.x), fabsf(mq.y)));
         }
     }
-    float nrhs[NB], nrls[NB], nghs[NB], ngls[NB];
+    float nrs[NB], ngs[NB];
 #pragma unroll
     for (int b = 0; b < NB; ++b) {
-        nrhs[b] = nrh[b].x;
-        nrls[b] = nrl[b].x;
-        ff_acc(nrhs[b], nrls[b], nrh[b].y, nrl[b].y);
-        nghs[b] = ngh[b].x;
-        ngls[b] = ngl[b].x;
-        ff_acc(nghs[b], ngls[b], ngh[b].y, ngl[b].y);
+        nrs[b] = nr2[b].x + nr2[b].y;
+        ngs[b] = ng2[b].x + ng2[b].y;
     }
     uint32_t cmabs_u[kMCH];
 #pragma unroll
@@ -445,9 +403,12 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
     warp_blocks_reduce<CPB, true>(cvmax, bvmax);
     warp_blocks_reduce<CPB, true>(cmabs_u, bmabs);
 #pragma unroll
-    for (int b = 0; b < NB; ++b) {
-        ff_warp_sum(nrhs[b], nrls[b]);
-        ff_warp_sum(nghs[b], ngls[b]);
+    for (int k = 16; k >= 1; k >>= 1) {
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            nrs[b] += __shfl_xor_sync(0xFFFFFFFFu, nrs[b], k);
+            ngs[b] += __shfl_xor_sync(0xFFFFFFFFu, ngs[b], k);
+        }
     }
     float vmn[NB], vmx[NB], nlmin[NB], ndelta[NB], ms[NB], sc[NB], inv[NB];
     AlEncConsts ek[NB];
@@ -507,9 +468,12 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
             m.m_absmax[b0 + b] = ms[b];
         }
     }
+    // s_j = ||Rt_j|| / (||R_j|| + 1e-8)
+    if (lane == 0) {
 #pragma unroll
-    for (int b = 0; b < NB; ++b)
-        if (b0 + b < nblk) ps.add(nrhs[b], nrls[b], nghs[b], ngls[b], m.scale + b0 + b);
+        for (int b = 0; b < NB; ++b)
+            if (b0 + b < nblk) m.scale[b0 + b] = sqrtf(nrs[b]) / (sqrtf(ngs[b]) + 1e-8f);
+    }
     __syncwarp();
 }
 
@@ -528,10 +492,8 @@ apollo_moments_kernel(MomentArgs m, int64_t ntiles) {
         s_kLog2Lo[i] = kLog2LoD[i];
     }
     __syncthreads();
-    PendingScales ps;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x)
-        moments_tile<CPB, VBITS>(m, tile, s_tab[warp], s_val[warp], ps);
-    ps.flush();
+        moments_tile<CPB, VBITS>(m, tile, s_tab[warp], s_val[warp]);
 }
 
 // ------------------------------------------------------ limiter, update --
@@ -1008,7 +970,6 @@ apollo_moments_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t n
         s_kLog2Lo[i] = kLog2LoD[i];
     }
     __syncthreads();
-    PendingScales ps;
     int cur = 0;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         cur = entry_for(tab, nmat, tile, cur, &ApEntry::mom_t0);
@@ -1021,9 +982,8 @@ apollo_moments_multi_kernel(const ApEntry* __restrict__ tab, int nmat, int64_t n
         m.v_codes = e.v_codes;
         m.v_meta = e.v_meta;
         m.scale = e.scale;
-        moments_tile<CPB, VBITS>(m, tile - e.mom_t0, s_tab[warp], s_val[warp], ps);
+        moments_tile<CPB, VBITS>(m, tile - e.mom_t0, s_tab[warp], s_val[warp]);
     }
-    ps.flush();
 }
 
 // limited: every matrix's update is scaled by its limiter factor.
