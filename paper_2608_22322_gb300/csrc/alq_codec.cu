@@ -39,11 +39,19 @@ al_encode_kernel(const float* __restrict__ x, int64_t n, int block, float log_fl
     __syncthreads();
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
+        const bool full = seg0 + kSeg <= n;  // warp-uniform: unmasked I/O
         float4 v[4];
         uint32_t cmin[4], cmax[4];
+        if (full) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                v[c] = __ldcs(reinterpret_cast<const float4*>(x + chunk_index(seg0, c, lane)));
+        } else {
+#pragma unroll
+            for (int c = 0; c < 4; ++c) v[c] = load4f(x, chunk_index(seg0, c, lane), n);
+        }
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
-            v[c] = load4f(x, chunk_index(seg0, c, lane), n);
             cmin[c] = 0xFFFFFFFFu;
             cmax[c] = 0u;
 #pragma unroll
@@ -75,15 +83,35 @@ al_encode_kernel(const float* __restrict__ x, int64_t n, int block, float log_fl
         for (int e = 0; e < 16; ++e) xv[e] = f4get(v[e / 4], e % 4);
         uint32_t q[16];
         al_encode_chunks<BITS, CPB, NB, 4>(xv, mn, lmin, delta, ek, q);
+        uint32_t wq[4 * BITS / 8];
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
-            const int64_t idx = chunk_index(seg0, c, lane);
-            if (BITS == 8)
-                store4b((uint8_t*)codes, idx, n,
-                        q[4 * c] | (q[4 * c + 1] << 8) | (q[4 * c + 2] << 16) | (q[4 * c + 3] << 24));
-            else
-                store4h((uint16_t*)codes, idx, n,
-                        make_uint2(q[4 * c] | (q[4 * c + 1] << 16), q[4 * c + 2] | (q[4 * c + 3] << 16)));
+            if constexpr (BITS == 8) {
+                wq[c] = q[4 * c] | (q[4 * c + 1] << 8) | (q[4 * c + 2] << 16) | (q[4 * c + 3] << 24);
+            } else {
+                wq[2 * c] = q[4 * c] | (q[4 * c + 1] << 16);
+                wq[2 * c + 1] = q[4 * c + 2] | (q[4 * c + 3] << 16);
+            }
+        }
+        if (full) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                const int64_t idx = chunk_index(seg0, c, lane);
+                if constexpr (BITS == 8)
+                    __stcs(reinterpret_cast<unsigned int*>((uint8_t*)codes + idx), wq[c]);
+                else
+                    __stcs(reinterpret_cast<uint2*>((uint16_t*)codes + idx),
+                           make_uint2(wq[2 * c], wq[2 * c + 1]));
+            }
+        } else {
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                const int64_t idx = chunk_index(seg0, c, lane);
+                if constexpr (BITS == 8)
+                    store4b((uint8_t*)codes, idx, n, wq[c]);
+                else
+                    store4h((uint16_t*)codes, idx, n, make_uint2(wq[2 * c], wq[2 * c + 1]));
+            }
         }
         if (lane == 0 && (warp % wpb) == 0) {
             const int64_t gb0 = seg0 >> bshift;
@@ -117,14 +145,17 @@ al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta,
     __syncthreads();
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
+        const bool full = seg0 + kSeg <= n;  // warp-uniform: unmasked I/O
         uint32_t w[4 * BITS / 8];
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
             const int64_t idx = chunk_index(seg0, c, lane);
             if (BITS == 8) {
-                w[c] = load4b((const uint8_t*)codes, idx, n);
+                w[c] = full ? __ldcs(reinterpret_cast<const unsigned int*>((const uint8_t*)codes + idx))
+                            : load4b((const uint8_t*)codes, idx, n);
             } else {
-                const uint2 h = load4h((const uint16_t*)codes, idx, n);
+                const uint2 h = full ? __ldcs(reinterpret_cast<const uint2*>((const uint16_t*)codes + idx))
+                                     : load4h((const uint16_t*)codes, idx, n);
                 w[2 * c] = h.x;
                 w[2 * c + 1] = h.y;
             }
@@ -154,6 +185,7 @@ al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta,
             for (int b = 0; b < NB; ++b)
                 al8_values_from_tables_soa(s_val[warp] + 256 * b, ts + 64 * b, lmin[b], delta[b]);
         }
+        float4 r4[4];
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
             const int b = c / CPB;
@@ -166,7 +198,15 @@ al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta,
                 else
                     r[i] = al16_decode(q, lmin[b], delta[b]);
             }
-            store4f(out, chunk_index(seg0, c, lane), n, make_float4(r[0], r[1], r[2], r[3]));
+            r4[c] = make_float4(r[0], r[1], r[2], r[3]);
+        }
+        if (full) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                __stcs(reinterpret_cast<float4*>(out + chunk_index(seg0, c, lane)), r4[c]);
+        } else {
+#pragma unroll
+            for (int c = 0; c < 4; ++c) store4f(out, chunk_index(seg0, c, lane), n, r4[c]);
         }
         __syncwarp();
     }
@@ -185,11 +225,19 @@ uf8_encode_kernel(const float* __restrict__ m, int64_t n, int block, int8_t* __r
     const int bshift = __ffs(block) - 1;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
+        const bool full = seg0 + kSeg <= n;  // warp-uniform: unmasked I/O
         float4 v[4];
         uint32_t ca[4];
+        if (full) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                v[c] = __ldcs(reinterpret_cast<const float4*>(m + chunk_index(seg0, c, lane)));
+        } else {
+#pragma unroll
+            for (int c = 0; c < 4; ++c) v[c] = load4f(m, chunk_index(seg0, c, lane), n);
+        }
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
-            v[c] = load4f(m, chunk_index(seg0, c, lane), n);
             ca[c] = 0u;
 #pragma unroll
             for (int i = 0; i < 4; ++i) ca[c] = umix<true>(ca[c], f2u(f4get(v[c], i)) & 0x7FFFFFFFu);
@@ -205,16 +253,24 @@ uf8_encode_kernel(const float* __restrict__ m, int64_t n, int block, int8_t* __r
             inv[b] = 0.0f;
             if (s[b] > 0.0f) uf8_encode_consts(s[b], sc[b], inv[b]);
         }
+        uint32_t wd[4];
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
             const int b = c / CPB;
-            uint32_t wd = 0;
+            wd[c] = 0;
             if (s[b] > 0.0f) {
 #pragma unroll
                 for (int i = 0; i < 4; ++i)
-                    wd |= ((uint32_t)uf8_quantize(f4get(v[c], i), sc[b], inv[b]) & 0xFFu) << (8 * i);
+                    wd[c] |= ((uint32_t)uf8_quantize(f4get(v[c], i), sc[b], inv[b]) & 0xFFu) << (8 * i);
             }
-            store4b((uint8_t*)codes, chunk_index(seg0, c, lane), n, wd);
+        }
+        if (full) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                __stcs(reinterpret_cast<unsigned int*>((uint8_t*)codes + chunk_index(seg0, c, lane)), wd[c]);
+        } else {
+#pragma unroll
+            for (int c = 0; c < 4; ++c) store4b((uint8_t*)codes, chunk_index(seg0, c, lane), n, wd[c]);
         }
         if (lane == 0 && (warp % wpb) == 0) {
             const int64_t gb0 = seg0 >> bshift;
@@ -241,17 +297,30 @@ uf8_decode_kernel(const int8_t* __restrict__ codes, const float* __restrict__ ab
 #pragma unroll
         for (int b = 0; b < NB; ++b)
             d[b] = (gb0 + b < nblk) ? __ldg(absmax + gb0 + b) / 127.0f : 0.0f;
+        const bool full = seg0 + kSeg <= n;  // warp-uniform: unmasked I/O
+        uint32_t w[4];
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
             const int64_t idx = chunk_index(seg0, c, lane);
-            const uint32_t w = load4b((const uint8_t*)codes, idx, n);
+            w[c] = full ? __ldcs(reinterpret_cast<const unsigned int*>((const uint8_t*)codes + idx))
+                        : load4b((const uint8_t*)codes, idx, n);
+        }
+        float4 r[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
             const int b = c / CPB;
-            float4 r;
-            r.x = s8_to_float(w & 0xFFu) * d[b];
-            r.y = s8_to_float((w >> 8) & 0xFFu) * d[b];
-            r.z = s8_to_float((w >> 16) & 0xFFu) * d[b];
-            r.w = s8_to_float(w >> 24) * d[b];
-            store4f(out, idx, n, r);
+            r[c].x = s8_to_float(w[c] & 0xFFu) * d[b];
+            r[c].y = s8_to_float((w[c] >> 8) & 0xFFu) * d[b];
+            r[c].z = s8_to_float((w[c] >> 16) & 0xFFu) * d[b];
+            r[c].w = s8_to_float(w[c] >> 24) * d[b];
+        }
+        if (full) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                __stcs(reinterpret_cast<float4*>(out + chunk_index(seg0, c, lane)), r[c]);
+        } else {
+#pragma unroll
+            for (int c = 0; c < 4; ++c) store4f(out, chunk_index(seg0, c, lane), n, r[c]);
         }
     }
 }
