@@ -289,17 +289,34 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
     const int64_t b0 = seg0 >> bshift;
     float4 r[kMCH];
     uint32_t mw[kMCH], vw[kMCH * VBITS / 8];
+    const bool full = seg0 + kMSeg <= m.n;  // warp-uniform: unmasked I/O
+    if (full) {
 #pragma unroll
-    for (int c = 0; c < kMCH; ++c) {
-        const int64_t idx = chunk_index(seg0, c, lane);
-        r[c] = load4f(m.R, idx, m.n);
-        mw[c] = load4b((const uint8_t*)m.m_codes, idx, m.n);
-        if constexpr (VBITS == 8) {
-            vw[c] = load4b((const uint8_t*)m.v_codes, idx, m.n);
-        } else {
-            const uint2 h = load4h((const uint16_t*)m.v_codes, idx, m.n);
-            vw[2 * c] = h.x;
-            vw[2 * c + 1] = h.y;
+        for (int c = 0; c < kMCH; ++c) {
+            const int64_t idx = chunk_index(seg0, c, lane);
+            r[c] = __ldcs(reinterpret_cast<const float4*>(m.R + idx));
+            mw[c] = __ldcs(reinterpret_cast<const unsigned int*>((const uint8_t*)m.m_codes + idx));
+            if constexpr (VBITS == 8) {
+                vw[c] = __ldcs(reinterpret_cast<const unsigned int*>((const uint8_t*)m.v_codes + idx));
+            } else {
+                const uint2 h = __ldcs(reinterpret_cast<const uint2*>((const uint16_t*)m.v_codes + idx));
+                vw[2 * c] = h.x;
+                vw[2 * c + 1] = h.y;
+            }
+        }
+    } else {
+#pragma unroll
+        for (int c = 0; c < kMCH; ++c) {
+            const int64_t idx = chunk_index(seg0, c, lane);
+            r[c] = load4f(m.R, idx, m.n);
+            mw[c] = load4b((const uint8_t*)m.m_codes, idx, m.n);
+            if constexpr (VBITS == 8) {
+                vw[c] = load4b((const uint8_t*)m.v_codes, idx, m.n);
+            } else {
+                const uint2 h = load4h((const uint16_t*)m.v_codes, idx, m.n);
+                vw[2 * c] = h.x;
+                vw[2 * c + 1] = h.y;
+            }
         }
     }
     float olmin[NB], odelta[NB], dm[NB];
@@ -452,13 +469,23 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
         }
         const uint32_t qm = __byte_perm(__byte_perm(rb[0], rb[1], 0x0040u),
                                         __byte_perm(rb[2], rb[3], 0x0040u), 0x5410u);
-        store4b((uint8_t*)m.m_codes, idx, m.n, qm);
-        if constexpr (VBITS == 8)
-            store4b((uint8_t*)m.v_codes, idx, m.n,
-                    qv[4 * c] | (qv[4 * c + 1] << 8) | (qv[4 * c + 2] << 16) | (qv[4 * c + 3] << 24));
-        else
-            store4h((uint16_t*)m.v_codes, idx, m.n,
-                    make_uint2(qv[4 * c] | (qv[4 * c + 1] << 16), qv[4 * c + 2] | (qv[4 * c + 3] << 16)));
+        if (full) {
+            __stcs(reinterpret_cast<unsigned int*>((uint8_t*)m.m_codes + idx), qm);
+            if constexpr (VBITS == 8)
+                __stcs(reinterpret_cast<unsigned int*>((uint8_t*)m.v_codes + idx),
+                       qv[4 * c] | (qv[4 * c + 1] << 8) | (qv[4 * c + 2] << 16) | (qv[4 * c + 3] << 24));
+            else
+                __stcs(reinterpret_cast<uint2*>((uint16_t*)m.v_codes + idx),
+                       make_uint2(qv[4 * c] | (qv[4 * c + 1] << 16), qv[4 * c + 2] | (qv[4 * c + 3] << 16)));
+        } else {
+            store4b((uint8_t*)m.m_codes, idx, m.n, qm);
+            if constexpr (VBITS == 8)
+                store4b((uint8_t*)m.v_codes, idx, m.n,
+                        qv[4 * c] | (qv[4 * c + 1] << 8) | (qv[4 * c + 2] << 16) | (qv[4 * c + 3] << 24));
+            else
+                store4h((uint16_t*)m.v_codes, idx, m.n,
+                        make_uint2(qv[4 * c] | (qv[4 * c + 1] << 16), qv[4 * c + 2] | (qv[4 * c + 3] << 16)));
+        }
     }
     if (lane == 0) {
 #pragma unroll
