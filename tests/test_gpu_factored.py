@@ -228,6 +228,49 @@ def test_grouped_factored_step_matches_single(B, op, mom, bits, block):
                 assert bytes_equal(a, b) == 0, (op, t, i, k)
 
 
+def test_came_per_matrix_steps_on_streams_match_sequence(B):
+    """Per-matrix CAME steps dealt over several streams (the benchmark's
+    schedule: each matrix with its own workspace, the passes of different
+    matrices running concurrently) give every matrix exactly the
+    parameters, codes and metadata of the same steps run one after another
+    on one stream."""
+    import torch
+    shapes = [(300, 772), (64, 512), (512, 1024), (130, 516), (257, 2048)]
+    seq = [_fac_states(r, c, 16, 128, True, 60 + i) for i, (r, c) in enumerate(shapes)]
+    da = [{k: _t(v) for k, v in s_.items()} for s_ in seq]
+    db = [{k: _t(v) for k, v in s_.items()} for s_ in seq]
+    grads = [torch.zeros(r * c, dtype=torch.float32, device="cuda") for r, c in shapes]
+
+    def ws():
+        return [torch.empty(B.al_workspace_size(B.AL_OP_CAME, r, c), dtype=torch.uint8,
+                            device="cuda") for r, c in shapes]
+
+    wa, wb = ws(), ws()
+    streams = [torch.cuda.Stream() for _ in range(3)]
+
+    def step(d, i, t, w, stream):
+        r, c = shapes[i]
+        B.al_came_step(d["p"], grads[i], r, c, d["vr_codes"], d["vr_meta"], d["vc_codes"],
+                       d["vc_meta"], 16, 128, d["cr_codes"], d["cr_meta"], d["cc_codes"],
+                       d["cc_meta"], 16, 128, d["m_codes"], d["m_absmax"], 256, CAME_HP, t,
+                       w, stream=stream)
+
+    for t in range(1, 4):
+        for i, (r, c) in enumerate(shapes):
+            grads[i].copy_(torch.from_numpy(
+                wl.student_t_grad((r, c), 1e-3, 3.0, 0.05, 700 + 10 * t + i).ravel()))
+        torch.cuda.synchronize()
+        for i in range(len(shapes)):
+            step(da[i], i, t, wa[i], torch.cuda.current_stream())
+        torch.cuda.synchronize()
+        for i in range(len(shapes)):
+            step(db[i], i, t, wb[i], streams[i % len(streams)])
+        torch.cuda.synchronize()
+        for i in range(len(shapes)):
+            for k in da[i]:
+                assert bytes_equal(da[i][k].cpu().numpy(), db[i][k].cpu().numpy()) == 0, (t, i, k)
+
+
 @pytest.mark.parametrize("op,vb,cb", [("adafactor", 32, 0), ("came", 16, 32), ("came", 32, 32)])
 def test_fp32_factor_roles_match_oracle(B, op, vb, cb):
     """Factors kept unquantized (bits 32, Sec. 4.5): Adafactor with fp32
