@@ -907,6 +907,12 @@ apollo_project_kernel(const ApEntry* __restrict__ plan_tab, const uint16_t* __re
                     tma_load_2d(smem_u32(sB + s * kBStage), &e->tmB, kb * kGK, 0, bfull0 + 8 * s);
                 }
             }
+            if (!ok) {
+                // a wait gave up: let this thread's copies in flight land
+                // (bounded waits) before the CTA releases its shared memory
+                for (uint32_t k = kc > (uint32_t)kPStages ? kc - kPStages : 0u; k < kc; ++k)
+                    mbar_wait(bfull0 + 8 * (k % kPStages), (k / kPStages) & 1);
+            }
         }
     } else if (warp == 1) {
         if (lane == 0) {
@@ -935,6 +941,12 @@ apollo_project_kernel(const ApEntry* __restrict__ plan_tab, const uint16_t* __re
                     umma_commit(empty0 + 8 * s);
                 }
                 if (ok) umma_commit(tfull0 + 8 * acc);
+            }
+            if (!ok && kc > 0) {
+                // a wait gave up: let the MMAs already issued retire
+                // (bounded wait on the last commit) before the tensor memory
+                // is released
+                mbar_wait(empty0 + 8 * ((kc - 1) % kPStages), ((kc - 1) / kPStages) & 1);
             }
         }
     } else if (warp < 2 + kPConv) {
