@@ -31,7 +31,7 @@
  *  - Quantization blocks are consecutive runs of `block` elements of one
  *    tensor; the last block of a tensor may be partial, and elements past the
  *    end never enter a block statistic. `block` must be a power of two in
- *    [128, 4096] (the fused AdamW step: [128, 2048]). The paper's block
+ *    [128, 4096], the fused AdamW step included. The paper's block
  *    sizes (256 and 2048, Sec. 6.2; 128 for the AL16 factors) are all of
  *    this form. The kernels give each lane whole 4-element chunks of 128
  *    consecutive elements per warp and locate blocks by shifts, so a block
@@ -173,7 +173,7 @@ typedef struct {
  *   p        [n] fp32 parameters (read and written).
  *   g        [n] fp32 gradient.
  *   m_codes  [n] int8 UF8 codes, m_absmax [ceil(n/m_block)] fp32.
- *   m_block, v_block  block sizes, powers of two in [128, 2048].
+ *   m_block, v_block  block sizes, powers of two in [128, 4096].
  *   v_codes  [n] uint8 (v_bits = 8) or uint16 (v_bits = 16) AL codes,
  *   v_meta   [2*ceil(n/v_block)] fp32.
  *   v_bits = 32 is the unquantized FP32 role (Sec. 4.5, "AL8, AL16, or

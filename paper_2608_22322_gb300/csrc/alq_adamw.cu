@@ -25,9 +25,10 @@
 
 namespace alq {
 
-// Geometry of this kernel: 2 chunks per lane (8 elements), 256-element
-// segments per warp, 2048-element tiles per CTA; blocks of 128..2048.
-constexpr int kCH = 2;
+// Geometry of this kernel: 4 chunks per lane (16 elements), 512-element
+// segments per warp (two blocks of 256), 4096-element tiles per CTA; blocks
+// of 128..4096.
+constexpr int kCH = 4;
 constexpr int kASeg = 128 * kCH;
 constexpr int kATile = 8 * kASeg;
 
@@ -112,13 +113,15 @@ __device__ __forceinline__ PlanEntry plan_entry(const PlanEntry* table, int nten
     return table[cur];
 }
 
-// Four CTAs per SM (64 registers, no spills): the step is bound by the
-// latency of each warp's dependent chains more than by issue slots, and 32
-// resident warps hide more of it than 24 do.
-// WIDE: AL8 blocks wider than a segment (512 .. 2048 elements), whose value
+// Three CTAs per SM (80 registers, no spills): 16 elements a lane halve
+// the per-segment work of the block constants, plan walk and reductions
+// (two 256-blocks' bounds in one lane pass, their levels in one paired
+// pass); 8 elements a lane at four CTAs per SM ran 0.7% slower at blocks of
+// 256 and 15% slower at blocks of 2048.
+// WIDE: AL8 blocks wider than a segment (1024 .. 4096 elements), whose value
 // table is built once per block by the warps that share it.
 template <int CPBV, int CPBM, int VBITS, bool WIDE = false>
-__global__ void __launch_bounds__(kThreads, 4)
+__global__ void __launch_bounds__(kThreads, 3)
 adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t total_tiles,
                    PlanEntry single, int v_block, int m_block, AdamWPairs s) {
     const int v_shift = __ffs(v_block) - 1, m_shift = __ffs(m_block) - 1;  // powers of two
@@ -266,10 +269,13 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
                                            olmin[0], odelta[0]);
                 tslot ^= 1;
             } else {
-                // two blocks per segment: their levels in one paired pass
+                // two or four blocks per segment: their levels two blocks per
+                // paired pass
                 float* ts = reinterpret_cast<float*>(s_tab[warp][0]);
-                al8_build_tables2_soa(ts, ts + 64, olmin[0], odelta[0], olmin[1], odelta[1], kf,
-                                      ok2);
+#pragma unroll
+                for (int b = 0; b < NBV; b += 2)
+                    al8_build_tables2_soa(ts + 64 * b, ts + 64 * (b + 1), olmin[b], odelta[b],
+                                          olmin[b + 1], odelta[b + 1], kf, ok2);
 #pragma unroll
                 for (int b = 0; b < NBV; ++b)
                     al8_values_from_tables_soa(s_val[warp] + 256 * b, ts + 64 * b, olmin[b],
@@ -529,7 +535,8 @@ static int launch_adamw_v(int cv, int cm, const PlanEntry* table, int ntensors,
     if (cv == A && cm == B)                                                                 \
         return launch_adamw_t<A, B, VBITS>(table, ntensors, total_tiles, single, v_block, \
                                            m_block, s, st);
-    ALQ_CASE(1, 1) ALQ_CASE(1, 2) ALQ_CASE(2, 1) ALQ_CASE(2, 2)
+    ALQ_CASE(1, 1) ALQ_CASE(1, 2) ALQ_CASE(1, 4) ALQ_CASE(2, 1) ALQ_CASE(2, 2) ALQ_CASE(2, 4)
+    ALQ_CASE(4, 1) ALQ_CASE(4, 2) ALQ_CASE(4, 4)
 #undef ALQ_CASE
     return ALQ_ERR_UNSUPPORTED;
 }

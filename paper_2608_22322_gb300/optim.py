@@ -150,7 +150,7 @@ class AdamW(_Base):
     """AdamW (Sec. 3.1, Eq. (1)) with UF8 momentum and AL-coded second moment;
     one fused launch per group and step over every parameter with a gradient
     (al_adamw_step_multi). v_bits 8 or 16 (AL8/AL16 V, UF8 M) or 32 (m and
-    v unquantized fp32), blocks powers of two in [128, 2048]; log_floor
+    v unquantized fp32), blocks powers of two in [128, 4096]; log_floor
     defaults to log2(eps^2)."""
 
     _CODES = {"m_codes": None, "v_codes": "v_bits"}

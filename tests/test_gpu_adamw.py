@@ -98,7 +98,8 @@ def test_adamw_redrawn_mask(B):
 
 @pytest.mark.parametrize("m_block,v_block", [(256, 2048), (128, 128), (512, 1024),
                                              (2048, 256), (128, 2048), (128, 256),
-                                             (256, 128), (2048, 128), (512, 512)])
+                                             (256, 128), (2048, 128), (512, 512),
+                                             (256, 4096), (4096, 128), (4096, 4096)])
 def test_adamw_block_sizes(B, m_block, v_block):
     w = wl.AdamWSingle(shape=(37, 1111))  # 41107 elements: ragged tiles and blocks
     _run_single(B, w, m_block, v_block, 8, 4)
