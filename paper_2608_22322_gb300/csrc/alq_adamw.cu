@@ -105,6 +105,12 @@ static AdamWPairs adamw_pairs(const AdamWScalars& s) {
     return q;
 }
 
+// Barrier of the nwarps warps of a group (named barrier id; a group of
+// every warp of the CTA is the whole CTA).
+__device__ __forceinline__ void group_sync(int id, int nwarps) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(32 * nwarps) : "memory");
+}
+
 __device__ __forceinline__ PlanEntry plan_entry(const PlanEntry* table, int ntensors,
                                                 const PlanEntry& single, int64_t tile,
                                                 int& cur) {
@@ -240,11 +246,11 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
                         }
                     }
                     al8_build_tables_soa(reinterpret_cast<float*>(s_tab[warp][0]), la[0], da[0], kf);
-                    __syncthreads();
+                    group_sync(1 + warp / wpbv, wpbv);
                 }
                 al8_values_part_soa(s_val[g0], reinterpret_cast<const float*>(s_tab[g0 + wit][0]),
                                     olmin[0], odelta[0], r, wpbv);
-                __syncthreads();
+                group_sync(1 + warp / wpbv, wpbv);
                 wit = wit + 1 == wpbv ? 0 : wit + 1;
             } else if constexpr (NBV == 1) {
                 // warps 2k and 2k + 1 hold adjacent blocks of one tensor: the
@@ -364,7 +370,8 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
                 sp[1][warp] = bvmax[0];
                 sp[2][warp] = bmabs[0];
             }
-            __syncthreads();
+            const int gmax = wpbv > wpbm ? wpbv : wpbm;
+            group_sync(5 + warp / gmax, gmax);
             if (wpbv > 1) {
                 const int g0 = (warp / wpbv) * wpbv;
                 uint32_t a = sp[0][g0], b = sp[1][g0];
