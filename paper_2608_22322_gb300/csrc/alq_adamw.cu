@@ -358,7 +358,9 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
 #pragma unroll
         for (int c = 0; c < kCH; ++c) cmabs_u[c] = f2u(cmabs[c]);
         warp_blocks_reduce<CPBM, true>(cmabs_u, bmabs);
-        if (wpbv > 1 || wpbm > 1) {
+        // (only instantiations whose V or M blocks span whole segments can
+        // have blocks wider than a segment)
+        if (((CPBV == kCH) || (CPBM == kCH)) && (wpbv > 1 || wpbm > 1)) {
             // blocks wider than a segment (then one block per warp): one
             // shared round for all three statistics, one barrier; the slots
             // alternate between iterations, so a warp one iteration ahead
