@@ -874,27 +874,37 @@ def _row_codec(torch, np, wl, B, dev):
                 bytes_note="20 B/element + block constants")
 
 
-HOLD_CYCLES = 525_000  # about 0.25 ms at the 2.1 GHz maximum SM clock
+HOLD_HZ = 2.1e9   # cycles per second of a device-side wait (the SM clock's maximum)
+HOLD_BATCH = 64   # timed row steps issued behind one device-side wait, at most
+HOLD_MAX_MS = 50.0  # the longest device-side wait
 
 
 class L2Flush:
-    """Writes a buffer twice the L2's size between timed steps, so that no
-    step starts with the previous step's data in L2."""
+    """Between timed steps: writes a buffer twice the L2's size, so that no
+    step starts with the previous step's data in L2, then reads a second
+    one as large, so that the lines the write left dirty are written back
+    before the next step (outside its events) and the step starts with a
+    clean L2."""
 
     def __init__(self, torch, dev):
         props = torch.cuda.get_device_properties(dev)
         l2 = int(getattr(props, "L2_cache_size", 0) or (129 << 20))
         self.buf = torch.empty(2 * l2 // 4, dtype=torch.float32, device=dev)
+        self.clean = torch.zeros(2 * l2 // 4, dtype=torch.float32, device=dev)
+        self.sink = torch.empty((), dtype=torch.float32, device=dev)
 
     def __call__(self):
         self.buf.zero_()
+        torch_sum = self.clean.sum
+        self.sink.copy_(torch_sum())
 
 
 def measure_row(name, args, dev, warmup, min_steps, with_cpu, summary):
     """Times one non-headline hot-path row: whole steps (all of the row's
-    launches) with CUDA events around each step and an L2 flush and a
-    short device-side wait between steps (outside the events), at least
-    min_steps steps and enough to fill
+    launches) with CUDA events around each step and an L2 flush between
+    steps (outside the events), issued in batches behind a device-side wait
+    so that the host's launch time never shows, at least min_steps steps
+    and enough to fill
     about 0.6 s, with nvidia-smi clock samples over the timed loop; bytes
     per step over time against the measured HBM copy peak; the oracle on a
     bounded sample (its OpenMP build for the multi-matrix rows)."""
@@ -912,15 +922,20 @@ def measure_row(name, args, dev, warmup, min_steps, with_cpu, summary):
     t = 0
     for _ in range(max(3, warmup)):
         t += 1
+        flush()
         w["step"](t)
-    # calibrate the step count to fill about 0.6 s of timed steps
+    # calibrate the step count to fill about 0.6 s of timed steps, and the
+    # host's time to issue one timed iteration
     ev0 = torch.cuda.Event(enable_timing=True)
     ev1 = torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize(dev)
     ev0.record(stream)
+    h0 = time.perf_counter()
     for _ in range(3):
         t += 1
+        flush()
         w["step"](t)
+    host_ms = (time.perf_counter() - h0) * 1e3 / 3
     ev1.record(stream)
     torch.cuda.synchronize(dev)
     est = ev0.elapsed_time(ev1) / 3
@@ -935,17 +950,26 @@ def measure_row(name, args, dev, warmup, min_steps, with_cpu, summary):
     pairs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
              for _ in range(steps)]
     torch.cuda.synchronize(dev)
-    for a, b in pairs:
-        flush()
-        # a quarter millisecond of device-side wait (outside the events):
-        # the GPU then runs behind the host, so a short step's launches are
-        # all queued before its start event and the events time the device
-        # alone, not the host's launch latency
-        torch.cuda._sleep(HOLD_CYCLES)
-        t += 1
-        a.record(stream)
-        w["step"](t)
-        b.record(stream)
+    # The timed steps go in batches, each behind a device-side wait (outside
+    # the events) longer than twice the host's time to issue the batch: the
+    # whole batch is queued before the GPU reaches it, so the events time
+    # the device alone, however slow the host is at launching short steps.
+    # A batch holds at most ~400 queued commands (the launch queue must not
+    # fill, or the host would block behind the wait), and the wait is twice
+    # the calibrated issue time of the batch, at most HOLD_MAX_MS.
+    batch = max(1, min(HOLD_BATCH, 400 // (w["launches"] + 4)))
+    hold_ms = min(HOLD_MAX_MS, max(0.25, 2.0 * batch * host_ms))
+    i = 0
+    while i < steps:
+        nb = min(batch, steps - i)
+        torch.cuda._sleep(int(hold_ms * 1e-3 * HOLD_HZ))
+        for a, b in pairs[i:i + nb]:
+            flush()
+            t += 1
+            a.record(stream)
+            w["step"](t)
+            b.record(stream)
+        i += nb
     torch.cuda.synchronize(dev)
     clocks = sampler.stop()
     ms_step = sum(a.elapsed_time(b) for a, b in pairs) / steps
@@ -966,8 +990,9 @@ def measure_row(name, args, dev, warmup, min_steps, with_cpu, summary):
             "frac": achieved / peak, "frac_of_8tbs_spec": achieved / 8000.0,
             "traffic": None, "peak_source": f"{peak_src} hbm_gbs",
             "kernel": "whole step (all launches; per-kernel shares in profiles/)"}
-    l2 = ("L2 flushed (a write of twice its size) and a 0.25 ms device-side wait between "
-          "timed steps, outside the events")
+    l2 = ("L2 flushed between timed steps, outside the events: a write of twice its "
+          "size, then a read of twice its size (no dirty lines left); the steps issued "
+          "in batches behind a device-side wait")
     if summary:
         out = {"workload": w["workload"], "value": w["n"] / (ms_step * 1e-3), "unit": unit,
                "ms_per_step": ms_step, "steps": steps, "warmup": max(3, warmup),
