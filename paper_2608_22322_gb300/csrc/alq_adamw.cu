@@ -105,6 +105,9 @@ static AdamWPairs adamw_pairs(const AdamWScalars& s) {
     return q;
 }
 
+// log2 of a power of two, at compile time
+__host__ __device__ constexpr int ilog2c(int x) { return x <= 1 ? 0 : 1 + ilog2c(x / 2); }
+
 // Barrier of the nwarps warps of a group (named barrier id; a group of
 // every warp of the CTA is the whole CTA).
 __device__ __forceinline__ void group_sync(int id, int nwarps) {
@@ -130,7 +133,10 @@ template <int CPBV, int CPBM, int VBITS, bool WIDE = false>
 __global__ void __launch_bounds__(kThreads, 3)
 adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t total_tiles,
                    PlanEntry single, int v_block, int m_block, AdamWPairs s) {
-    const int v_shift = __ffs(v_block) - 1, m_shift = __ffs(m_block) - 1;  // powers of two
+    // a block narrower than a segment is 128 CPB elements: its geometry is
+    // the instantiation's (v_block and m_block are then those sizes)
+    const int v_shift = CPBV < kCH ? 7 + ilog2c(CPBV) : __ffs(v_block) - 1;
+    const int m_shift = CPBM < kCH ? 7 + ilog2c(CPBM) : __ffs(m_block) - 1;
     constexpr int NBV = kCH / CPBV;
     constexpr int NBM = kCH / CPBM;
     constexpr int NE = 4 * kCH;
@@ -144,8 +150,8 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
     // is the same for the whole warp, and every branch on the segment's
     // position is a uniform one
     const int warp = __shfl_sync(0xFFFFFFFFu, (int)(threadIdx.x >> 5), 0), lane = threadIdx.x & 31;
-    const int wpbv = v_block > kASeg ? v_block / kASeg : 1;
-    const int wpbm = m_block > kASeg ? m_block / kASeg : 1;
+    const int wpbv = CPBV == kCH && v_block > kASeg ? v_block / kASeg : 1;
+    const int wpbm = CPBM == kCH && m_block > kASeg ? m_block / kASeg : 1;
     const float kf = al8_table_k(lane);
     const Opaque2 ok2{s.one, s.zero};
     const int G = gridDim.x;
@@ -206,7 +212,7 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
         }
 
         // ---- previous block constants
-        const int64_t nvb = (n + v_block - 1) >> v_shift, nmb = (n + m_block - 1) >> m_shift;
+        const int64_t nvb = (n + (1 << v_shift) - 1) >> v_shift, nmb = (n + (1 << m_shift) - 1) >> m_shift;
         const int64_t vb0 = seg0 >> v_shift, mb0 = seg0 >> m_shift;
         float olmin[NBV], odelta[NBV], dm[NBM];
 #pragma unroll
