@@ -105,9 +105,6 @@ static AdamWPairs adamw_pairs(const AdamWScalars& s) {
     return q;
 }
 
-// log2 of a power of two, at compile time
-__host__ __device__ constexpr int ilog2c(int x) { return x <= 1 ? 0 : 1 + ilog2c(x / 2); }
-
 // Barrier of the nwarps warps of a group (named barrier id; a group of
 // every warp of the CTA is the whole CTA).
 __device__ __forceinline__ void group_sync(int id, int nwarps) {

@@ -285,8 +285,8 @@ __device__ __forceinline__ void moments_tile(const MomentArgs& m, int64_t tile, 
     constexpr float Lm2 = VBITS == 8 ? 254.0f : 65534.0f;
     const int warp = __shfl_sync(0xFFFFFFFFu, (int)(threadIdx.x >> 5), 0), lane = threadIdx.x & 31;
     const float kf = al8_table_k(lane);
-    const int64_t nblk = blocks_of_dev(m.n, m.block);
-    const int bshift = __ffs(m.block) - 1;
+    const int bshift = block_shift<CPB, kMCH>(m.block);  // rank = 128 CPB
+    const int64_t nblk = (m.n + (1 << bshift) - 1) >> bshift;
     const int64_t seg0 = tile * kMTile + (int64_t)warp * kMSeg;
     const int64_t b0 = seg0 >> bshift;
     float4 r[kMCH];

@@ -26,9 +26,9 @@ al_encode_kernel(const float* __restrict__ x, int64_t n, int block, float log_fl
     constexpr float Lm2 = BITS == 8 ? 254.0f : 65534.0f;
     __shared__ uint32_t s_part[2][kThreads / 32];
     const int warp = __shfl_sync(0xFFFFFFFFu, (int)(threadIdx.x >> 5), 0), lane = threadIdx.x & 31;
-    const int wpb = block > kSeg ? block / kSeg : 1;
-    const int64_t nblk = blocks_of_dev(n, block);
-    const int bshift = __ffs(block) - 1;
+    const int wpb = CPB == 4 && block > kSeg ? block / kSeg : 1;
+    const int bshift = block_shift<CPB, 4>(block);
+    const int64_t nblk = (n + (1 << bshift) - 1) >> bshift;
     for (int i = threadIdx.x; i < 1024; i += kThreads) {
         s_kExp2Hi[i] = kExp2HiD[i];
         s_kExp2Lo[i] = kExp2LoD[i];
@@ -133,8 +133,8 @@ al_decode_kernel(const void* __restrict__ codes, const float* __restrict__ meta,
     __shared__ float s_val[kThreads / 32][BITS == 8 ? NB * 256 : 1];
     const int warp = __shfl_sync(0xFFFFFFFFu, (int)(threadIdx.x >> 5), 0), lane = threadIdx.x & 31;
     const float kf = al8_table_k(lane);
-    const int64_t nblk = blocks_of_dev(n, block);
-    const int bshift = __ffs(block) - 1;
+    const int bshift = block_shift<CPB, 4>(block);
+    const int64_t nblk = (n + (1 << bshift) - 1) >> bshift;
     for (int i = threadIdx.x; i < 1024; i += kThreads) {
         s_kExp2Hi[i] = kExp2HiD[i];
         s_kExp2Lo[i] = kExp2LoD[i];
@@ -220,9 +220,9 @@ uf8_encode_kernel(const float* __restrict__ m, int64_t n, int block, int8_t* __r
     constexpr int NB = 4 / CPB;
     __shared__ uint32_t s_part[kThreads / 32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int wpb = block > kSeg ? block / kSeg : 1;
-    const int64_t nblk = blocks_of_dev(n, block);
-    const int bshift = __ffs(block) - 1;
+    const int wpb = CPB == 4 && block > kSeg ? block / kSeg : 1;
+    const int bshift = block_shift<CPB, 4>(block);
+    const int64_t nblk = (n + (1 << bshift) - 1) >> bshift;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
         const bool full = seg0 + kSeg <= n;  // warp-uniform: unmasked I/O
@@ -288,8 +288,8 @@ uf8_decode_kernel(const int8_t* __restrict__ codes, const float* __restrict__ ab
                   int block, float* __restrict__ out, int64_t ntiles) {
     constexpr int NB = 4 / CPB;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t nblk = blocks_of_dev(n, block);
-    const int bshift = __ffs(block) - 1;
+    const int bshift = block_shift<CPB, 4>(block);
+    const int64_t nblk = (n + (1 << bshift) - 1) >> bshift;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
         float d[NB];

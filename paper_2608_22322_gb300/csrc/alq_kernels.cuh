@@ -77,6 +77,17 @@ __device__ __forceinline__ float rcp_approx(float x) {
     return r;
 }
 
+// log2 of a power of two, at compile time
+__host__ __device__ constexpr int ilog2c(int x) { return x <= 1 ? 0 : 1 + ilog2c(x / 2); }
+
+// Shift of a kernel's block size: a block narrower than a segment of CH
+// chunks is 128 CPB elements, known when the kernel is instantiated;
+// otherwise the runtime size.
+template <int CPB, int CH>
+__device__ __forceinline__ int block_shift(int block) {
+    return CPB < CH ? 7 + ilog2c(CPB) : __ffs(block) - 1;
+}
+
 __device__ __forceinline__ int64_t blocks_of_dev(int64_t n, int block) {
     return (n + block - 1) / block;
 }
