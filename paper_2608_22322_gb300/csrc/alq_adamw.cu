@@ -124,15 +124,19 @@ __device__ __forceinline__ PlanEntry plan_entry(const PlanEntry* table, int nten
 // (two 256-blocks' bounds in one lane pass, their levels in one paired
 // pass); 8 elements a lane at four CTAs per SM ran 0.7% slower at blocks of
 // 256 and 15% slower at blocks of 2048.
-// WIDE: AL8 blocks wider than a segment (1024 .. 4096 elements), whose value
-// table is built once per block by the warps that share it.
-template <int CPBV, int CPBM, int VBITS, bool WIDE = false>
+// WIDE (AL8, WPBV > 1): blocks wider than a segment (1024 .. 4096
+// elements), whose value table is built once per block by the warps that
+// share it.
+// WPBV: warps per V block (v_block / 512 for blocks of at least a segment,
+// else 1), a compile-time constant of each instantiation.
+template <int CPBV, int CPBM, int VBITS, int WPBV = 1>
 __global__ void __launch_bounds__(kThreads, 3)
 adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t total_tiles,
                    PlanEntry single, int v_block, int m_block, AdamWPairs s) {
     // a block narrower than a segment is 128 CPB elements: its geometry is
     // the instantiation's (v_block and m_block are then those sizes)
-    const int v_shift = CPBV < kCH ? 7 + ilog2c(CPBV) : __ffs(v_block) - 1;
+    constexpr bool WIDE = VBITS == 8 && WPBV > 1;
+    const int v_shift = CPBV < kCH ? 7 + ilog2c(CPBV) : 7 + ilog2c(kCH) + ilog2c(WPBV);
     const int m_shift = CPBM < kCH ? 7 + ilog2c(CPBM) : __ffs(m_block) - 1;
     constexpr int NBV = kCH / CPBV;
     constexpr int NBM = kCH / CPBM;
@@ -147,7 +151,7 @@ adamw_fused_kernel(const PlanEntry* __restrict__ table, int ntensors, int64_t to
     // is the same for the whole warp, and every branch on the segment's
     // position is a uniform one
     const int warp = __shfl_sync(0xFFFFFFFFu, (int)(threadIdx.x >> 5), 0), lane = threadIdx.x & 31;
-    const int wpbv = CPBV == kCH && v_block > kASeg ? v_block / kASeg : 1;
+    constexpr int wpbv = WPBV;
     const int wpbm = CPBM == kCH && m_block > kASeg ? m_block / kASeg : 1;
     const float kf = al8_table_k(lane);
     const Opaque2 ok2{s.one, s.zero};
@@ -530,9 +534,12 @@ template <int CPBV, int CPBM, int VBITS>
 static int launch_adamw_t(const PlanEntry* table, int ntensors, int64_t total_tiles,
                           const PlanEntry& single, int v_block, int m_block,
                           const AdamWScalars& s, cudaStream_t stream) {
-    constexpr bool kWideOk = VBITS == 8 && CPBV == kCH;
-    auto k = kWideOk && v_block > kASeg ? adamw_fused_kernel<CPBV, CPBM, VBITS, kWideOk>
-                                        : adamw_fused_kernel<CPBV, CPBM, VBITS, false>;
+    auto k = adamw_fused_kernel<CPBV, CPBM, VBITS, 1>;
+    if constexpr (CPBV == kCH) {
+        if (v_block == 2 * kASeg) k = adamw_fused_kernel<CPBV, CPBM, VBITS, 2>;
+        if (v_block == 4 * kASeg) k = adamw_fused_kernel<CPBV, CPBM, VBITS, 4>;
+        if (v_block == 8 * kASeg) k = adamw_fused_kernel<CPBV, CPBM, VBITS, 8>;
+    }
     const int grid = persistent_grid((const void*)k, kThreads, 0, total_tiles);
     k<<<grid, kThreads, 0, stream>>>(table, ntensors, total_tiles, single, v_block, m_block,
                                      adamw_pairs(s));
