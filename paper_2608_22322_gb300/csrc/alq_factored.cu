@@ -633,10 +633,10 @@ template <int MODE, int CPBM>
 __device__ __forceinline__ void update_tile(const UpdateArgs& u, int64_t tile, uint32_t* s_part) {
     constexpr int NBM = 4 / CPBM;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int wpbm = u.m_block > kSeg ? u.m_block / kSeg : 1;
+    const int wpbm = CPBM == 4 && u.m_block > kSeg ? u.m_block / kSeg : 1;
     const float icf = __ldg(u.scal);
-    const int64_t nmb = blocks_of_dev(u.n, u.m_block);
-    const int mshift = __ffs(u.m_block) - 1;
+    const int mshift = block_shift<CPBM, 4>(u.m_block);
+    const int64_t nmb = (u.n + (1 << mshift) - 1) >> mshift;
     {
         const int64_t seg0 = tile * kTile + (int64_t)warp * kSeg;
         const int64_t mb0 = seg0 >> mshift;
