@@ -334,6 +334,19 @@ def run_ours(args):
     peak = float(peaks.get("hbm_gbs", 6800.0))
     traffic = recorded_traffic() if not args.tensors and args.v_block == 256 else None
 
+    # The other rows next, before the end-to-end and CPU legs (so that no
+    # host-side work of those legs is still settling while short steps are
+    # timed); single-GPU measurements of their own workloads.
+    rows = None
+    if rank == 0 and world == 1 and not args.no_rows and not args.tensors:
+        import gc
+        rows = {}
+        for name in ("adafactor", "came", "apollo", "codec"):
+            rows[name] = measure_row(name, args, dev, warmup=5, min_steps=20,
+                                     with_cpu=not args.no_cpu, summary=True)
+            gc.collect()
+            torch.cuda.empty_cache()
+
     e2e = None
     if not args.no_e2e:
         e2e = run_e2e(torch, B, arrs, hp, t, args.e2e_steps, n_params, dev)
@@ -350,19 +363,6 @@ def run_ours(args):
         import oracle as ora
         cpu = cpu_baseline(torch, ora, arrs, hp, t + 1, v_block=args.v_block)
 
-    rows = None
-    if rank == 0 and world == 1 and not args.no_rows and not args.tensors:
-        # the other rows are single-GPU measurements of their own workloads
-        del arrs, plans
-        import gc
-        gc.collect()
-        torch.cuda.empty_cache()
-        rows = {}
-        for name in ("adafactor", "came", "apollo", "codec"):
-            rows[name] = measure_row(name, args, dev, warmup=5, min_steps=20,
-                                     with_cpu=not args.no_cpu, summary=True)
-            gc.collect()
-            torch.cuda.empty_cache()
 
     if world > 1:
         dist.destroy_process_group()
