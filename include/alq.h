@@ -218,7 +218,7 @@ typedef struct {
     int32_t m_block;
     int32_t v_block;
     int32_t v_bits;
-    int64_t total_tiles; /* work items of the fused kernel          */
+    int64_t total_tiles; /* 4096-element tiles of the fused kernel  */
     int64_t total_elems; /* sum of n over the tensors               */
 } al_multi_info;
 
@@ -406,7 +406,7 @@ typedef struct {
     int32_t v_bits, v_block, c_bits, c_block, m_block;
     int32_t has_momentum;
     int64_t total_params;
-    int64_t sumsq_tiles;  /* 64 x 512 tiles of the sums passes               */
+    int64_t sumsq_tiles;  /* 64 x 256 tiles of the sums passes               */
     int64_t factor_tiles; /* factor blocks (rows and columns) of V           */
     int64_t factor2_tiles;/* factor blocks of CAME's confidence (else 0)     */
     int64_t scale_tiles;  /* 256-entry tiles of the scale passes             */
@@ -481,9 +481,9 @@ int al_apollo_step(float* p, const float* g, int64_t rows, int64_t cols,
 
 /* ---------------------------------------------------- grouped APOLLO step -- */
 /*
- * One APOLLO step over many matrices in three launches (one projection
- * launch whose grid covers every matrix's 128-channel tiles, one moments
- * launch, one update launch) instead of three launches per matrix. Each matrix gets exactly the arithmetic of al_apollo_step (the
+ * One APOLLO step over many matrices in three launches (one persistent
+ * projection launch whose CTAs walk every matrix's 128-channel tiles, one
+ * moments launch, one update launch) instead of three launches per matrix. Each matrix gets exactly the arithmetic of al_apollo_step (the
  * results are bit-identical). This grouping is the library's; the paper
  * applies the method matrix by matrix.
  *
@@ -520,7 +520,7 @@ typedef struct {
     int64_t total_params;   /* sum of rows * cols                            */
     int64_t total_channels; /* sum of max(rows, cols)                        */
     int64_t gemm_tiles;     /* 128-channel tiles of the grouped projection   */
-    int64_t mom_tiles;      /* 2048-value tiles of the moments pass          */
+    int64_t mom_tiles;      /* 4096-value tiles of the moments pass          */
     int64_t upd_tiles;      /* 4096-parameter tiles of the update pass       */
     void* workspace;        /* the workspace the plan is bound to            */
     int64_t norm_chunks;    /* limiter partial sums (8 update tiles each)    */

@@ -3,7 +3,7 @@
 // factored confidence states tracking a residual) and UF8 momentum.
 //
 // Launch sequence of one step (all on the caller's stream, no host sync):
-//   sumsq      G read once: per 64-row x 512-column tile, exact float-float
+//   sumsq      G read once: per 64-row x 256-column tile, exact float-float
 //              sums of g^2 per row (over the tile's columns) and per column
 //              (over its rows) -> fp64 partials in the workspace.
 //   factor     one CTA per factor block: finish r_i / c_j (fp64, fixed order),
